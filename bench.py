@@ -1,0 +1,483 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused PBB decode step (ring append + attention over A(t)).
+
+Default workload (the steady-state throughput point with the largest rings):
+batch 512, Hq 32, Hkv 8, d 128, B 4096, bf16, every sequence at its own
+position t0 ~ U[B, 2^20) so the phase r is random and the bridge exists.
+Rings: 2 x 4.3 GB, far larger than L2, so every step streams from HBM.
+
+A step is one pbb_decode_step over the whole batch plus the device-side
+position advance. Prints one JSON line (rank 0):
+  value      decode-core tokens*heads/s = batch * Hq * steps / time, summed over ranks
+  roofline   algorithmic bytes per launch / mean kernel time vs measured HBM copy bandwidth
+  e2e        the same metric through the host-memory entry (H2D of q/k/v, D2H of out per step)
+  cpu_baseline  the fp64 oracle timed on the host cores on a bounded sample
+
+--impl reference times the fp64 CPU oracle (the only reference this method has)
+on a bounded sample per step. --sweep prints one line per throughput-sweep point.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "PBB decode-core tokens*heads/s"
+UNIT = "tokens*heads/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=400)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--batch", type=int, default=512)
+    ap.add_argument("--block", type=int, default=4096)
+    ap.add_argument("--sweep", action="store_true", help="one line per throughput-sweep point")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--chunk", type=int, default=0, help="keys per CTA (0 = library plan)")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------ clocks --
+
+_REASONS = {0x1: "gpu_idle", 0x2: "applications_clocks_setting", 0x4: "sw_power_cap",
+            0x8: "hw_slowdown", 0x10: "sync_boost", 0x20: "sw_thermal_slowdown",
+            0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown",
+            0x100: "display_clock_setting"}
+
+
+class ClockSampler:
+    """Samples SM clock and clock-event reasons of one GPU through NVML (read only)."""
+
+    def __init__(self, uuid: str | None, period_s: float = 0.01):
+        self.period = period_s
+        self.samples = []
+        self.max_mhz = None
+        self._stop = threading.Event()
+        self._thread = None
+        self._nvml = None
+        self._h = None
+        try:
+            nv = ctypes.CDLL("libnvidia-ml.so.1")
+            if nv.nvmlInit_v2() != 0:
+                return
+            h = ctypes.c_void_p()
+            rc = -1
+            if uuid:
+                rc = nv.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h))
+            if rc != 0:
+                idx = int(os.environ.get("CUDA_VISIBLE_DEVICES", "0").split(",")[0] or 0)
+                rc = nv.nvmlDeviceGetHandleByIndex_v2(idx, ctypes.byref(h))
+            if rc != 0:
+                return
+            self._nvml, self._h = nv, h
+            mx = ctypes.c_uint()
+            if nv.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+                self.max_mhz = mx.value
+        except OSError:
+            pass
+
+    def _run(self):
+        nv, h = self._nvml, self._h
+        clk, rs = ctypes.c_uint(), ctypes.c_ulonglong()
+        get_reasons = getattr(nv, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            nv.nvmlDeviceGetCurrentClocksThrottleReasons
+        while not self._stop.is_set():
+            if nv.nvmlDeviceGetClockInfo(h, 1, ctypes.byref(clk)) == 0 and \
+                    get_reasons(h, ctypes.byref(rs)) == 0:
+                self.samples.append((clk.value, rs.value))
+            time.sleep(self.period)
+
+    def __enter__(self):
+        if self._nvml is not None:
+            self._thread = threading.Thread(target=self._run, daemon=True)
+            self._thread.start()
+        return self
+
+    def __exit__(self, *exc):
+        self._stop.set()
+        if self._thread:
+            self._thread.join()
+
+    def summary(self):
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": [], "samples": 0,
+                    "source": "nvml unavailable" if self._nvml is None else "no samples"}
+        reasons = set()
+        for _, r in self.samples:
+            for bit, name in _REASONS.items():
+                if r & bit and name != "gpu_idle":
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(c for c, _ in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(reasons), "samples": len(self.samples), "source": "nvml"}
+
+
+# ------------------------------------------------------------------- peaks --
+
+def hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_sha() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2606_02680_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload_key: str, launch_bytes: float):
+    """DRAM traffic per launch from the committed ncu record, if it was taken on
+    the current kernel source (else None). Scaled from the captured case by
+    algorithmic bytes, which grow in proportion with the batch."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    if rec.get("kernel_source_sha") != kernel_source_sha():
+        return None
+    entry = rec.get("workloads", {}).get(workload_key)
+    if not entry:
+        return None
+    return entry["dram_bytes_per_launch"] / entry["algorithmic_bytes_per_launch"] * launch_bytes
+
+
+# --------------------------------------------------------------- workload --
+
+def describe(w):
+    return (f"{w.name}: batch {w.batch}, Hq {w.Hq}, Hkv {w.Hkv}, d {w.d}, B {w.B}, {w.dtype}, "
+            f"t0 ~ U[{w.t0_lo}, {w.t0_hi})")
+
+
+def setup_device_workload(w, dev, pool: int):
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import inputs
+
+    t0 = inputs.start_positions(w)
+    pos = t0.to(torch.int32).to(dev)
+    dt = inputs.torch_dtype(w)
+    k_ring = torch.empty((w.batch, w.Hkv, w.B, w.d), dtype=dt, device=dev)
+    v_ring = torch.empty_like(k_ring)
+    hk, hv = inputs.history_window(w, t0, device=dev)
+    pbb.ring_prefill(hk, hv, pos, k_ring, v_ring)
+    torch.cuda.synchronize()
+    del hk, hv
+    torch.cuda.empty_cache()
+    steps_in = [inputs.step_inputs(w, i, device=dev) for i in range(pool)]
+    return t0, pos, k_ring, v_ring, steps_in
+
+
+def time_device(w, dev, steps, warmup, dist=None):
+    """Device-timed loop; returns dict of timings."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import bytemodel
+
+    pool = 8
+    t0, pos, k_ring, v_ring, steps_in = setup_device_workload(w, dev, pool)
+    out = torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32, device=dev)
+    pbb.reserve_workspace(w.batch, w.Hq, w.Hkv, w.d, w.B)
+    stream = torch.cuda.current_stream()
+    for i in range(warmup):
+        q, k, v = steps_in[i % pool]
+        pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+        pbb.advance_positions(pos)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:  # noqa: BLE001
+        pass
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clocks:
+        start.record(stream)
+        for i in range(steps):
+            q, k, v = steps_in[(warmup + i) % pool]
+            ev[2 * i].record(stream)
+            pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+            ev[2 * i + 1].record(stream)
+            pbb.advance_positions(pos)
+        end.record(stream)
+        torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    status = pbb.get_device_status()
+    if status != pbb.PBB_OK:
+        raise RuntimeError(f"device status {status} after the timed loop")
+    total_ms = start.elapsed_time(end)
+    kern_ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
+    t_np = t0.numpy()
+    launch_bytes = [bytemodel.step_bytes(t_np + warmup + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes)
+                    for i in range(steps)]
+    res = {
+        "total_ms": total_ms,
+        "kernel_ms_mean": sum(kern_ms) / steps,
+        "kernel_ms_median": statistics.median(kern_ms),
+        "launch_bytes_mean": sum(launch_bytes) / steps,
+        "clocks": clocks.summary(),
+        "ring_bytes": 2 * k_ring.numel() * k_ring.element_size(),
+        "state": (t0, pos, k_ring, v_ring, steps_in, out),
+    }
+    return res
+
+
+def time_e2e(w, dev, steps, state):
+    """Same step through the host-memory entry: pinned inputs copied in, output copied out."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+
+    t0, pos, k_ring, v_ring, steps_in, _ = state
+    pool = len(steps_in)
+    host = [tuple(x.cpu().pin_memory() for x in s) for s in steps_in]
+    out_h = [torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32).pin_memory() for _ in range(2)]
+    staging = pbb.HostStep(w.batch, w.Hq, w.Hkv, w.d, k_ring.dtype, dev)
+    stream = torch.cuda.current_stream()
+    for i in range(3):
+        q, k, v = host[i % pool]
+        pbb.decode_step_host(q, k, v, k_ring, v_ring, pos, out_h[i % 2], staging)
+        pbb.advance_positions(pos)
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for i in range(steps):
+        q, k, v = host[i % pool]
+        pbb.decode_step_host(q, k, v, k_ring, v_ring, pos, out_h[i % 2], staging)
+        pbb.advance_positions(pos)
+    end.record(stream)
+    torch.cuda.synchronize()
+    ms = start.elapsed_time(end)
+    q, k, v = host[0]
+    h2d = sum(x.numel() * x.element_size() for x in (q, k, v))
+    d2h = out_h[0].numel() * out_h[0].element_size()
+    return {"value": w.batch * w.Hq * steps / (ms / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms / steps}
+
+
+def oracle_sample(w, seconds: float, seqs_per_call: int = 8, max_calls: int | None = None):
+    """Time the fp64 oracle on sequences of workload w (inputs of the same recipe,
+    generated on the host outside the timed region) until `seconds` have passed."""
+    import oracle
+    from paper_2606_02680_gb300 import inputs
+
+    oracle.build()
+    sub = w.with_(batch=seqs_per_call)
+    t0 = inputs.start_positions(sub)
+    hk, hv = inputs.history_window(sub, t0)
+    q, k, v = inputs.step_inputs(sub, 0)
+    hk = hk.clone()
+    hv = hv.clone()
+    # window of B+1 rows ending at the current token t0: rows t0-B .. t0
+    import torch
+
+    wk = torch.cat([hk, k.unsqueeze(2)], dim=2)[:, :, 1:]
+    wv = torch.cat([hv, v.unsqueeze(2)], dim=2)[:, :, 1:]
+    done = 0
+    calls = 0
+    elapsed = 0.0
+    while elapsed < seconds and (max_calls is None or calls < max_calls):
+        t_start = time.perf_counter()
+        oracle.attend(q, wk, wv, s0=(t0 - w.B + 1).numpy(), t=t0.numpy(), b=w.B)
+        elapsed += time.perf_counter() - t_start
+        done += seqs_per_call
+        calls += 1
+    return {"value": done * w.Hq / elapsed, "unit": UNIT, "cores": oracle.max_threads(),
+            "kind": "oracle", "seconds": elapsed,
+            "sample": f"{done} sequence-steps of {w.name} ({seqs_per_call} sequences per call, "
+                      f"fp64 brute force over every position up to t)"}
+
+
+# ------------------------------------------------------------------- arms --
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if world <= 1:
+        return None, 0, 1, 0
+    import torch
+    import torch.distributed as dist
+
+    rank = int(os.environ["RANK"])
+    local = int(os.environ.get("LOCAL_RANK", rank))
+    backend = "nccl" if torch.cuda.is_available() else "gloo"
+    if torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    dist.init_process_group(backend=backend)
+    return dist, rank, world, local
+
+
+def shard_batch(batch: int, rank: int, world: int, scaling: str = "weak"):
+    """Sequences of one rank: weak scaling keeps `batch` per rank; strong splits it."""
+    if scaling == "weak":
+        return batch
+    base, rem = divmod(batch, world)
+    return base + (1 if rank < rem else 0)
+
+
+def max_over_ranks(dist, x: float) -> float:
+    if dist is None:
+        return x
+    import torch
+
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(dist, x: float) -> float:
+    if dist is None:
+        return x
+    import torch
+
+    dev = torch.device("cuda", torch.cuda.current_device()) if torch.cuda.is_available() else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def run_ours(args):
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import build as nvbuild
+    from paper_2606_02680_gb300 import inputs
+
+    dist, rank, world, local = dist_setup()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a GPU (no CPU fallback)")
+    if rank == 0 or dist is None:
+        nvbuild.build()
+    if dist is not None:
+        dist.barrier()
+    dev = torch.device("cuda", local if dist is not None else 0)
+    torch.cuda.set_device(dev)
+    pbb.set_chunk_keys(args.chunk)
+
+    points = [(args.batch, args.block)]
+    if args.sweep:
+        points = [(b, B) for b in inputs.SWEEP_BATCHES for B in inputs.SWEEP_BLOCKS]
+    peak, peak_kind = hbm_peak()
+    for batch, B in points:
+        w = inputs.sweep_workload(shard_batch(batch, rank, world), B)
+        res = time_device(w, dev, args.steps, args.warmup, dist)
+        total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
+        units = sum_over_ranks(dist, w.batch * w.Hq * args.steps)
+        value = units / total_s
+        achieved = res["launch_bytes_mean"] / (res["kernel_ms_mean"] / 1e3) / 1e9
+        key = f"sweep_b{batch}_B{B}"
+        traffic = recorded_traffic(key, res["launch_bytes_mean"])
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
+            "data": "synthetic (seeded N(0,1) K/V/q; rings prefilled consistent with each t0)",
+            "config": {"workload": describe(w), "batch_per_gpu": w.batch, "Hq": w.Hq, "Hkv": w.Hkv,
+                       "head_dim": w.d, "block": w.B,
+                       "keys_per_cta": pbb.plan_chunk_keys(w.batch, w.Hq, w.Hkv, w.d, w.B),
+                       "l2": ("inputs larger than L2: rings %.2f GB" % (res["ring_bytes"] / 1e9))
+                       if res["ring_bytes"] > L2_BYTES else
+                       "rings fit in L2 (%.1f MB): latency/L2-bound point, not an HBM claim" % (res["ring_bytes"] / 1e6),
+                       "parallelism": f"dp{world} (independent sequences, no collective)"},
+            "hbm_gbs": achieved,
+            "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": traffic,
+                         "kernel": "decode_kernel<2,128,4>", "peak_kind": peak_kind,
+                         "algorithmic_bytes_per_launch": res["launch_bytes_mean"],
+                         "kernel_ms_mean": res["kernel_ms_mean"],
+                         "kernel_ms_median": res["kernel_ms_median"]},
+            "clocks": res["clocks"],
+            "gpu_launches": 2 * args.steps,
+        }
+        if not args.no_e2e and not args.sweep:
+            line["e2e"] = time_e2e(w, dev, args.steps, res["state"])
+        res.pop("state")
+        torch.cuda.empty_cache()
+        if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep:
+            line["cpu_baseline"] = oracle_sample(w, args.cpu_seconds)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def run_reference(args):
+    """The fp64 oracle on the host cores; each step is a bounded sample of the workload."""
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if rank != 0:
+        return
+    from paper_2606_02680_gb300 import inputs
+
+    w = inputs.sweep_workload(args.batch, args.block)
+    seqs = 4
+    for _ in range(args.warmup):
+        oracle_sample(w, 0.0, seqs_per_call=seqs, max_calls=1)
+    times = []
+    for _ in range(args.steps):
+        s = oracle_sample(w, 0.0, seqs_per_call=seqs, max_calls=1)
+        times.append(s["seconds"])
+        cores = s["cores"]
+    total = sum(times)
+    value = seqs * w.Hq * args.steps / total
+    sample = (f"each step: {seqs} sequences of {w.name} (fp64 brute force over every "
+              f"position up to t), not the whole batch")
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total * 1e3 / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": describe(w), "batch_per_gpu": w.batch, "Hq": w.Hq, "Hkv": w.Hkv,
+                   "head_dim": w.d, "block": w.B},
+        "impl": "reference",
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,167 @@
+/*
+ * libpbb: fused decode step of Post-Boundary Bridge (PBB) local attention on
+ * one GPU (sm_103a).
+ *
+ * The operation (Sec. 3, Eq. (pbb) and Eq. (attention); Appendix F.1):
+ * a sequence whose current token sits at absolute position t, with block size
+ * B = 2h, block start p = B*floor(t/B) and phase r = t - p, reads the support
+ *
+ *     A(t) = {p, ..., t}  U  {p-h, ..., p-1} if p > 0 and r < h,
+ *
+ * which is the interval [a(t), t], a(t) = max(0, h(floor(t/h) - 1))
+ * (Eq. pbb_relay). Each query head j of the sequence returns
+ *
+ *     o_j = sum_{s in A(t)} exp(z_s) v_s / sum_{s in A(t)} exp(z_s),
+ *     z_s = q_j . k_s / sqrt(d),
+ *
+ * where K/V come from KV head j / (Hq/Hkv) (contiguous GQA grouping). K/V of
+ * every KV head live in a fixed ring of B slots: position s is stored in slot
+ * s mod B and no retained entry is ever moved (Appendix F.1, Proposition
+ * "Relocation-free PBB cache"). One decode step writes the new token's K/V
+ * into slot r and attends over the ring; the slot written is never one read.
+ *
+ * Conventions shared by every call below.
+ *   - Layouts are dense, row-major, in this order:
+ *       q      [batch][Hq][d]        query of the current token (already rotated)
+ *       k_new  [batch][Hkv][d]       K of the current token
+ *       v_new  [batch][Hkv][d]       V of the current token
+ *       ring   [batch][Hkv][B][d]    one K ring and one V ring
+ *       pos    [batch] int32         absolute position t of the current token
+ *       out    [batch][Hq][d] fp32   attention output
+ *     Element type: bf16 for pbb_decode_step, fp32 for pbb_decode_step_f32;
+ *     the output is fp32 in both.
+ *   - Every tensor pointer is a DEVICE pointer, owned by the caller, 16-byte
+ *     aligned (pos: 4-byte aligned). Rings are either caller memory with the
+ *     layout above or come from pbb_ring_alloc.
+ *   - Calls are asynchronous on `stream` (0 = the legacy default stream) and
+ *     never synchronise. Sizes: batch >= 0, Hq % Hkv == 0 with
+ *     Hq/Hkv in {1, 2, 4, 8}, d in {64, 128}, B even and 2 <= B <= 2^20.
+ *   - Return value: PBB_OK or a negative PBB_ERR_* code; nothing is launched
+ *     when argument checking fails. Faults the device finds (a negative
+ *     position, a wait that ran out) are kept in a device-side status word
+ *     read by pbb_get_device_status.
+ */
+#ifndef PBB_H_
+#define PBB_H_
+
+#include <stddef.h>
+#include <stdint.h>
+#include <cuda_runtime_api.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { PBB_BF16 = 0, PBB_F32 = 1 } pbb_dtype;
+
+enum {
+    PBB_OK = 0,
+    PBB_ERR_INVALID_ARG = -1,    /* null or misaligned pointer, negative size */
+    PBB_ERR_UNSUPPORTED = -2,    /* B odd/out of range, Hq % Hkv != 0, group or d not supported */
+    PBB_ERR_CUDA = -3,           /* a CUDA runtime call or a launch failed */
+    PBB_ERR_DEVICE_TIMEOUT = -4, /* a kernel's bounded wait on a bulk copy ran out */
+    PBB_ERR_WORKSPACE = -5,      /* workspace too small while the stream is being captured */
+    PBB_ERR_DEVICE_POSITION = -6 /* a kernel saw pos[b] < 0; that sequence was skipped */
+};
+
+/*
+ * Bytes of ONE ring (K or V): batch * Hkv * B * d * element size. The pair is
+ * twice this: 2 * batch * B * Hkv * d * u, Appendix F.1 (65,536 bytes at
+ * batch 1, B 128, Hkv 2, d 64, bf16). Returns 0 for invalid sizes. Host only.
+ */
+size_t pbb_ring_bytes(int batch, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
+ * Allocate a zero-filled K ring and V ring (cudaMallocAsync on `stream`,
+ * zeroed on the same stream). The caller owns both and frees them with
+ * pbb_ring_free. On error nothing stays allocated and *k_ring, *v_ring are
+ * set to NULL.
+ */
+int pbb_ring_alloc(void** k_ring, void** v_ring, int batch, int Hkv, int d, int B,
+                   pbb_dtype dtype, cudaStream_t stream);
+
+/* Free rings from pbb_ring_alloc (cudaFreeAsync on `stream`). NULL is ignored. */
+int pbb_ring_free(void* k_ring, void* v_ring, cudaStream_t stream);
+
+/*
+ * Load the ring of a sequence that resumes at position t = pos[b] from its
+ * history (Appendix F.1: position s goes to slot s mod B).
+ *   k_hist, v_hist [batch][Hkv][B][d]: row j holds position t - B + j.
+ * Every slot is written: rows whose position is negative (before the start of
+ * the sequence) write zeros. The result is the ring that t sequential decode
+ * steps from a zeroed ring would have left, so the next pbb_decode_step at
+ * position t continues it exactly. Sequences with pos[b] < 0 are skipped and
+ * flagged (PBB_ERR_DEVICE_POSITION). Bit copy; same element type as the ring.
+ */
+int pbb_ring_prefill(const void* k_hist, const void* v_hist, const int32_t* pos, void* k_ring,
+                     void* v_ring, int batch, int Hkv, int d, int B, pbb_dtype dtype,
+                     cudaStream_t stream);
+
+/*
+ * Make sure the library's workspace on the current device holds the split
+ * partials of a step of this shape (and of every smaller batch). The
+ * workspace (per device, owned by the library, freed at exit) holds the
+ * per-split partial (max, sum, output) of Eq. (lse) and one counter per
+ * (sequence, KV head); a decode step grows it on demand, which allocates, so
+ * call this first when decode steps are to be captured in a CUDA graph.
+ */
+int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
+ * One PBB decode step for every sequence (bf16 q/k/v/ring, fp32 out).
+ * For each sequence b with t = pos[b]: writes k_new/v_new[b] into slot
+ * t mod B of its rings (bit copy), then computes out[b] as defined above over
+ * A(t), the new token included (read from k_new/v_new, not back from the
+ * ring). Precondition (Appendix F.1, sequential single-token decoding): the
+ * rings hold positions t-B .. t-1 of the sequence in their slots, which holds
+ * after pbb_ring_prefill at t, or after steps at t-1, t-2, ... starting from a
+ * zeroed ring at t = 0. pos is read on the device and never by the host.
+ * Deterministic: the same inputs give bitwise the same out and rings.
+ */
+int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
+                    void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
+                    int d, int B, cudaStream_t stream);
+
+/* Same as pbb_decode_step with fp32 q, k_new, v_new and rings. */
+int pbb_decode_step_f32(const float* q, const float* k_new, const float* v_new, float* k_ring,
+                        float* v_ring, const int32_t* pos, float* out, int batch, int Hq,
+                        int Hkv, int d, int B, cudaStream_t stream);
+
+/* pos[b] += 1 for every sequence, on the device (advances a decode loop, e.g. in a graph). */
+int pbb_advance_positions(int32_t* pos, int batch, cudaStream_t stream);
+
+/*
+ * Synchronise `stream`, then return and clear the device status word of the
+ * current device: PBB_OK, PBB_ERR_DEVICE_TIMEOUT or PBB_ERR_DEVICE_POSITION
+ * (first fault recorded since the last call). Clearing also resets the split
+ * counters in the workspace, which an aborted step can leave behind.
+ */
+int pbb_get_device_status(cudaStream_t stream);
+
+/*
+ * Limit, in nanoseconds, of every wait of a decode kernel on a bulk copy
+ * (default 1e9). A wait that runs out sets PBB_ERR_DEVICE_TIMEOUT, the CTA
+ * drains its copies and returns without writing its output. A limit of 0
+ * makes a wait give up as soon as its data has not yet landed (for tests).
+ */
+int pbb_set_wait_timeout_ns(unsigned long long ns);
+
+/*
+ * Keys of the support each CTA handles (the split of the support across CTAs
+ * whose partials are fused with Eq. (lse)). 0 = automatic (default): chosen
+ * from the batch, Hkv, B, d and the device's SM count. A positive value is
+ * rounded up to a whole number of tiles. Returns the previous setting.
+ */
+int pbb_set_chunk_keys(int keys);
+
+/* Keys per CTA a decode step of this shape would use on the current device (0 on error). */
+int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/* Static description of an error code. */
+const char* pbb_error_string(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PBB_H_ */

@@ -1,0 +1,277 @@
+"""Python binding of libpbb, the GB300 decode step of Post-Boundary Bridge attention.
+
+Argument marshalling only: every step of the computation runs in the CUDA
+kernels of ``libpbb.so`` (built in-tree by ``build.py``), reached through the
+C ABI of ``include/pbb.h`` with ctypes. PyTorch provides device memory and
+streams. There is no CPU fallback: if the library is missing or no GPU is
+visible, the calls raise.
+
+Names follow the C ABI:
+
+* ``ring_bytes``, ``ring_alloc`` / ``Rings``   the B-slot K/V rings (Appendix F.1)
+* ``ring_prefill``                             load a ring from a history window
+* ``decode_step``                              append + attention over A(t) (Sec. 3)
+* ``decode_step_host``                         the same with host-resident inputs/outputs
+* ``advance_positions``, ``get_device_status``, ``reserve_workspace``,
+  ``set_wait_timeout_ns``, ``set_chunk_keys``, ``plan_chunk_keys``
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+__all__ = [
+    "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
+    "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION", "PbbError",
+    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step",
+    "decode_step_host", "advance_positions", "get_device_status", "reserve_workspace",
+    "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "error_string", "EXPORTS",
+]
+
+PBB_OK = 0
+PBB_ERR_INVALID_ARG = -1
+PBB_ERR_UNSUPPORTED = -2
+PBB_ERR_CUDA = -3
+PBB_ERR_DEVICE_TIMEOUT = -4
+PBB_ERR_WORKSPACE = -5
+PBB_ERR_DEVICE_POSITION = -6
+
+PBB_BF16 = 0
+PBB_F32 = 1
+
+# Every symbol include/pbb.h declares, with its ctypes signature.
+_P, _I, _SZ, _ULL = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t, ctypes.c_ulonglong
+EXPORTS = {
+    "pbb_ring_bytes": (_SZ, [_I, _I, _I, _I, _I]),
+    "pbb_ring_alloc": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _I, _I, _I, _I, _P]),
+    "pbb_ring_free": (_I, [_P, _P, _P]),
+    "pbb_ring_prefill": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_reserve_workspace": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_advance_positions": (_I, [_P, _I, _P]),
+    "pbb_get_device_status": (_I, [_P]),
+    "pbb_set_wait_timeout_ns": (_I, [_ULL]),
+    "pbb_set_chunk_keys": (_I, [_I]),
+    "pbb_plan_chunk_keys": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_error_string": (ctypes.c_char_p, [_I]),
+}
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+lib_path = os.path.join(_HERE, "libpbb.so")
+_lib = None
+_lock = threading.Lock()
+
+
+class PbbError(RuntimeError):
+    def __init__(self, code: int, what: str = ""):
+        self.code = code
+        super().__init__(f"{what}: {error_string(code)} ({code})" if what else error_string(code))
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libpbb.so (raises if it has not been built)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(lib_path):
+                raise RuntimeError(f"libpbb.so not built at {lib_path}; run __graft_entry__.build()")
+            handle = ctypes.CDLL(lib_path)
+            for name, (res, args) in EXPORTS.items():
+                fn = getattr(handle, name)
+                fn.restype = res
+                fn.argtypes = args
+            _lib = handle
+        return _lib
+
+
+def error_string(code: int) -> str:
+    try:
+        return lib().pbb_error_string(code).decode()
+    except Exception:  # noqa: BLE001 - library not loadable: still describe the code
+        return f"pbb error {code}"
+
+
+def _check(rc: int, what: str) -> None:
+    if rc != PBB_OK:
+        raise PbbError(rc, what)
+
+
+def _dt(dtype: torch.dtype) -> int:
+    if dtype == torch.bfloat16:
+        return PBB_BF16
+    if dtype == torch.float32:
+        return PBB_F32
+    raise TypeError(f"unsupported element type {dtype} (bf16 or fp32)")
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None) -> int:
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    return t.data_ptr()
+
+
+def ring_bytes(batch: int, Hkv: int, d: int, B: int, dtype: torch.dtype = torch.bfloat16) -> int:
+    """Bytes of one ring (K or V); the pair is twice this (Appendix F.1)."""
+    return int(lib().pbb_ring_bytes(batch, Hkv, d, B, _dt(dtype)))
+
+
+class _CudaArray:
+    """Minimal __cuda_array_interface__ view of library-owned device memory."""
+
+    def __init__(self, ptr: int, shape, typestr: str):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": typestr,
+                                         "data": (ptr, False), "version": 3, "strides": None}
+
+
+class Rings:
+    """K and V rings allocated by pbb_ring_alloc; freed with ``free()`` or at collection."""
+
+    def __init__(self, batch: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16, stream=None):
+        k, v = ctypes.c_void_p(), ctypes.c_void_p()
+        self._stream = stream
+        _check(lib().pbb_ring_alloc(ctypes.byref(k), ctypes.byref(v), batch, Hkv, d, B, _dt(dtype),
+                                    _stream(stream)), "pbb_ring_alloc")
+        self.k_ptr, self.v_ptr = k.value, v.value
+        self.shape = (batch, Hkv, B, d)
+        self.dtype = dtype
+        typestr = "<i2" if dtype == torch.bfloat16 else "<f4"
+        dev = torch.cuda.current_device()
+
+        def view(ptr):
+            t = torch.as_tensor(_CudaArray(ptr, self.shape, typestr), device=f"cuda:{dev}")
+            return t.view(torch.bfloat16) if dtype == torch.bfloat16 else t
+
+        self.k = view(self.k_ptr)
+        self.v = view(self.v_ptr)
+
+    def free(self) -> None:
+        if getattr(self, "k_ptr", None):
+            self.k = self.v = None
+            _check(lib().pbb_ring_free(self.k_ptr, self.v_ptr, _stream(self._stream)), "pbb_ring_free")
+            self.k_ptr = self.v_ptr = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:  # noqa: BLE001 - interpreter shutdown
+            pass
+
+
+def ring_alloc(batch: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16, stream=None) -> Rings:
+    return Rings(batch, Hkv, d, B, dtype, stream)
+
+
+def ring_prefill(k_hist: torch.Tensor, v_hist: torch.Tensor, pos: torch.Tensor,
+                 k_ring: torch.Tensor, v_ring: torch.Tensor, stream=None) -> None:
+    """Ring of sequences resuming at pos[b] from the B positions before it ([batch, Hkv, B, d])."""
+    batch, Hkv, B, d = k_ring.shape
+    dtype = k_ring.dtype
+    for name, t in (("k_hist", k_hist), ("v_hist", v_hist), ("v_ring", v_ring)):
+        if tuple(t.shape) != (batch, Hkv, B, d):
+            raise ValueError(f"{name} must have shape {(batch, Hkv, B, d)}")
+    if pos.numel() != batch:
+        raise ValueError("pos must have batch entries")
+    _check(lib().pbb_ring_prefill(_dev(k_hist, "k_hist", dtype), _dev(v_hist, "v_hist", dtype),
+                                  _dev(pos, "pos", torch.int32), _dev(k_ring, "k_ring", dtype),
+                                  _dev(v_ring, "v_ring", dtype), batch, Hkv, d, B, _dt(dtype),
+                                  _stream(stream)), "pbb_ring_prefill")
+
+
+def decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_ring: torch.Tensor,
+                v_ring: torch.Tensor, pos: torch.Tensor, out: torch.Tensor | None = None,
+                stream=None) -> torch.Tensor:
+    """One PBB decode step (include/pbb.h: pbb_decode_step / pbb_decode_step_f32).
+
+    q [batch, Hq, d], k_new/v_new [batch, Hkv, d], rings [batch, Hkv, B, d] (bf16 or
+    fp32, all the same), pos [batch] int32 on the device, out [batch, Hq, d] fp32.
+    """
+    batch, Hq, d = q.shape
+    _, Hkv, B, d2 = k_ring.shape
+    dtype = q.dtype
+    if d2 != d or k_ring.shape[0] != batch or tuple(v_ring.shape) != tuple(k_ring.shape):
+        raise ValueError("ring shape must be [batch, Hkv, B, d]")
+    if tuple(k_new.shape) != (batch, Hkv, d) or tuple(v_new.shape) != (batch, Hkv, d):
+        raise ValueError("k_new/v_new must be [batch, Hkv, d]")
+    if pos.numel() != batch:
+        raise ValueError("pos must have batch entries")
+    if out is None:
+        out = torch.empty((batch, Hq, d), dtype=torch.float32, device=q.device)
+    elif tuple(out.shape) != (batch, Hq, d):
+        raise ValueError("out must be [batch, Hq, d]")
+    fn = lib().pbb_decode_step if _dt(dtype) == PBB_BF16 else lib().pbb_decode_step_f32
+    _check(fn(_dev(q, "q", dtype), _dev(k_new, "k_new", dtype), _dev(v_new, "v_new", dtype),
+              _dev(k_ring, "k_ring", dtype), _dev(v_ring, "v_ring", dtype),
+              _dev(pos, "pos", torch.int32), _dev(out, "out", torch.float32), batch, Hq, Hkv, d, B,
+              _stream(stream)), "pbb_decode_step")
+    return out
+
+
+class HostStep:
+    """Device staging for ``decode_step_host`` (reused across calls of the same shape)."""
+
+    def __init__(self, batch: int, Hq: int, Hkv: int, d: int, dtype, device):
+        self.q = torch.empty((batch, Hq, d), dtype=dtype, device=device)
+        self.k = torch.empty((batch, Hkv, d), dtype=dtype, device=device)
+        self.v = torch.empty((batch, Hkv, d), dtype=dtype, device=device)
+        self.out = torch.empty((batch, Hq, d), dtype=torch.float32, device=device)
+
+
+def decode_step_host(q_h: torch.Tensor, k_h: torch.Tensor, v_h: torch.Tensor, k_ring: torch.Tensor,
+                     v_ring: torch.Tensor, pos: torch.Tensor, out_h: torch.Tensor,
+                     staging: HostStep, stream=None) -> None:
+    """decode_step with the step's inputs and output in (pinned) host memory.
+
+    Copies q/k/v host -> device, runs the step, copies out device -> host, all
+    enqueued on the stream; the caller synchronises before reading out_h.
+    """
+    s = torch.cuda.current_stream() if stream is None else stream
+    with torch.cuda.stream(s):
+        staging.q.copy_(q_h, non_blocking=True)
+        staging.k.copy_(k_h, non_blocking=True)
+        staging.v.copy_(v_h, non_blocking=True)
+        decode_step(staging.q, staging.k, staging.v, k_ring, v_ring, pos, staging.out, stream=s)
+        out_h.copy_(staging.out, non_blocking=True)
+
+
+def advance_positions(pos: torch.Tensor, stream=None) -> None:
+    """pos += 1 on the device."""
+    _check(lib().pbb_advance_positions(_dev(pos, "pos", torch.int32), pos.numel(), _stream(stream)),
+           "pbb_advance_positions")
+
+
+def get_device_status(stream=None) -> int:
+    """Synchronise and return (and clear) the device status word (PBB_OK or a PBB_ERR_DEVICE_* code)."""
+    return int(lib().pbb_get_device_status(_stream(stream)))
+
+
+def reserve_workspace(max_batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> None:
+    _check(lib().pbb_reserve_workspace(max_batch, Hq, Hkv, d, B, _dt(dtype)), "pbb_reserve_workspace")
+
+
+def set_wait_timeout_ns(ns: int) -> None:
+    _check(lib().pbb_set_wait_timeout_ns(int(ns)), "pbb_set_wait_timeout_ns")
+
+
+def set_chunk_keys(keys: int) -> int:
+    """Override the keys per CTA (0 = automatic); returns the previous setting."""
+    prev = int(lib().pbb_set_chunk_keys(int(keys)))
+    if prev < 0:
+        raise PbbError(prev, "pbb_set_chunk_keys")
+    return prev
+
+
+def plan_chunk_keys(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> int:
+    return int(lib().pbb_plan_chunk_keys(batch, Hq, Hkv, d, B, _dt(dtype)))

@@ -1,0 +1,49 @@
+// Internal interface between the C-ABI layer (pbb_api.cu) and the kernels
+// (pbb_decode.cu). Not installed; the public interface is include/pbb.h.
+#pragma once
+
+#include <cuda_runtime_api.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace pbb {
+
+// Device status codes (the word read by pbb_get_device_status).
+enum DeviceStatus : int { kDevOk = 0, kDevTimeout = 1, kDevBadPosition = 2 };
+
+struct DecodeArgs {
+    const void* q;       // [batch][Hq][d]
+    const void* k_new;   // [batch][Hkv][d]
+    const void* v_new;   // [batch][Hkv][d]
+    void* k_ring;        // [batch][Hkv][B][d]
+    void* v_ring;        // [batch][Hkv][B][d]
+    const int32_t* pos;  // [batch]
+    float* out;          // [batch][Hq][d]
+    float* part_o;       // [batch][Hkv][nchunk][G][d]   split partials (unnormalised output)
+    float* part_ml;      // [batch][Hkv][nchunk][G][2]   split partials (max, sum), log2 domain
+    int* counters;       // [batch][Hkv]                 arrivals per (sequence, KV head)
+    int batch, Hq, Hkv, d, B;
+    int chunk;           // keys of the support per CTA (multiple of the tile)
+    int nchunk;          // CTAs per (sequence, KV head) in the grid = ceil((B-1)/chunk)
+    unsigned long long timeout_ns;
+};
+
+// Keys per shared-memory tile of a kernel instance (rows of K and of V).
+int tile_keys(int elem_bytes, int d);
+
+// Resident CTAs per SM of the decode kernel for this instance (0 if unsupported).
+int decode_ctas_per_sm(int elem_bytes, int d, int group);
+
+// Launch the fused append + split attention + combine kernel. elem_bytes: 2 (bf16) or 4 (fp32).
+cudaError_t launch_decode(const DecodeArgs& a, int elem_bytes, cudaStream_t stream);
+
+cudaError_t launch_prefill(const void* k_hist, const void* v_hist, const int32_t* pos, void* k_ring,
+                           void* v_ring, int batch, int Hkv, int B, int row_bytes,
+                           cudaStream_t stream);
+
+cudaError_t launch_advance(int32_t* pos, int batch, cudaStream_t stream);
+
+// Read (and clear) the device status word of the current device.
+cudaError_t read_and_clear_status(int* status, cudaStream_t stream);
+
+}  // namespace pbb
