@@ -308,12 +308,14 @@ def oracle_sample(w, seconds: float, seqs_per_call: int = 8, max_calls: int | No
     done = 0
     calls = 0
     elapsed = 0.0
-    while elapsed < seconds and (max_calls is None or calls < max_calls):
+    while True:  # at least one call
         t_start = time.perf_counter()
         oracle.attend(q, wk, wv, s0=(t0 - w.B + 1).numpy(), t=t0.numpy(), b=w.B)
         elapsed += time.perf_counter() - t_start
         done += seqs_per_call
         calls += 1
+        if elapsed >= seconds or (max_calls is not None and calls >= max_calls):
+            break
     return {"value": done * w.Hq / elapsed, "unit": UNIT, "cores": oracle.max_threads(),
             "kind": "oracle", "seconds": elapsed,
             "sample": f"{done} sequence-steps of {w.name} ({seqs_per_call} sequences per call, "

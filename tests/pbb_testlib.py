@@ -87,11 +87,67 @@ class SequentialRun:
         i = self.step_i - 1
         # window of B+1 rows ending at the current token: positions t-B .. t
         lo = i  # history row of position t - B
-        hk = self.hk[seqs][:, :, lo:w.B + i + 1]
-        hv = self.hv[seqs][:, :, lo:w.B + i + 1]
+        sel = torch.as_tensor(seqs)
+        hk = self.hk[:, :, lo:w.B + i + 1].index_select(0, sel)
+        hv = self.hv[:, :, lo:w.B + i + 1].index_select(0, sel)
         t = self.t_now()[seqs]
         return oracle.attend(self.q_last[seqs], hk, hv, s0=t - w.B, t=t, b=w.B)
 
     def check_rings(self) -> None:
         assert np.array_equal(ring_bytes_np(self.k_ring), self.sim.k), "K ring differs from the oracle's"
         assert np.array_equal(ring_bytes_np(self.v_ring), self.sim.v), "V ring differs from the oracle's"
+
+
+class DeviceRun:
+    """Full-size run: inputs generated on the GPU (same recipe), rings prefilled
+    on the GPU; the oracle checks a sample of sequences, whose history rows and
+    step inputs are copied back to the host."""
+
+    def __init__(self, w: inputs.Workload, sample, device="cuda"):
+        self.w = w
+        self.dev = torch.device(device)
+        self.dtype = inputs.torch_dtype(w)
+        self.sample = np.asarray(sample)
+        self.t0 = inputs.start_positions(w)
+        self.pos = self.t0.to(torch.int32).to(self.dev)
+        self.k_ring = torch.empty((w.batch, w.Hkv, w.B, w.d), dtype=self.dtype, device=self.dev)
+        self.v_ring = torch.empty_like(self.k_ring)
+        wk, wv = inputs.history_window(w, self.t0, device=self.dev)
+        pbb.ring_prefill(wk, wv, self.pos, self.k_ring, self.v_ring)
+        idx = torch.as_tensor(self.sample, device=self.dev)
+        # host history of the sampled sequences: window then one row per step
+        self.hk = [wk.index_select(0, idx).cpu()]
+        self.hv = [wv.index_select(0, idx).cpu()]
+        del wk, wv
+        torch.cuda.empty_cache()
+        n = len(self.sample)
+        self.sim = oracle.RingSim(n, w.Hkv, w.d, w.B, w.elem_bytes)
+        self.sim.replay(self.hk[0], self.hv[0], (self.t0[self.sample] - w.B).numpy())
+        self.step_i = 0
+        self.q_last = None
+
+    def step(self):
+        w, i = self.w, self.step_i
+        q, k, v = inputs.step_inputs(w, i, device=self.dev)
+        out = pbb.decode_step(q, k, v, self.k_ring, self.v_ring, self.pos)
+        pbb.advance_positions(self.pos)
+        idx = torch.as_tensor(self.sample, device=self.dev)
+        ks, vs = k.index_select(0, idx).cpu(), v.index_select(0, idx).cpu()
+        self.hk.append(ks.unsqueeze(2))
+        self.hv.append(vs.unsqueeze(2))
+        self.q_last = q.index_select(0, idx).cpu()
+        self.sim.append(ks, vs, (self.t0[self.sample] + i).numpy())
+        self.step_i += 1
+        return out.index_select(0, idx).cpu()
+
+    def oracle_out(self) -> np.ndarray:
+        w, i = self.w, self.step_i - 1
+        hk = torch.cat(self.hk, dim=2)[:, :, i:w.B + i + 1]
+        hv = torch.cat(self.hv, dim=2)[:, :, i:w.B + i + 1]
+        t = (self.t0[self.sample] + i).numpy()
+        return oracle.attend(self.q_last, hk, hv, s0=t - w.B, t=t, b=w.B)
+
+    def check_rings(self) -> None:
+        idx = torch.as_tensor(self.sample, device=self.dev)
+        assert np.array_equal(ring_bytes_np(self.k_ring.index_select(0, idx)), self.sim.k)
+        assert np.array_equal(ring_bytes_np(self.v_ring.index_select(0, idx)), self.sim.v)
