@@ -61,7 +61,9 @@ enum {
     PBB_ERR_CUDA = -3,           /* a CUDA runtime call or a launch failed */
     PBB_ERR_DEVICE_TIMEOUT = -4, /* a kernel's bounded wait on a bulk copy ran out */
     PBB_ERR_WORKSPACE = -5,      /* workspace too small while the stream is being captured */
-    PBB_ERR_DEVICE_POSITION = -6 /* a kernel saw pos[b] < 0; that sequence was skipped */
+    PBB_ERR_DEVICE_POSITION = -6, /* a kernel saw pos[b] < 0; that sequence was skipped */
+    PBB_ERR_SCRATCH_LIMIT = -7    /* pbb_decode_step_noalloc: the step needs more scratch than
+                                     PBB_NOALLOC_SCRATCH_BYTES */
 };
 
 /*
@@ -156,6 +158,36 @@ int pbb_set_chunk_keys(int keys);
 
 /* Keys per CTA a decode step of this shape would use on the current device (0 on error). */
 int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
+ * No counterpart in the paper: a library-usage variant for callers that cannot
+ * allocate device memory while they decode (a runtime that owns all of HBM
+ * through its own pool and forbids other allocations, code inside a CUDA
+ * stream capture, loops that cannot afford cudaMalloc's implicit device
+ * synchronisation).
+ *
+ * Same arguments, layouts and result as pbb_decode_step (bf16), but the split
+ * scratch (per-(sequence, KV head) arrival counters and split partials) lives
+ * in a fixed array of PBB_NOALLOC_SCRATCH_BYTES compiled into the library;
+ * every GPU that loads the library holds that array until the process exits.
+ * The call never allocates or frees memory. A step whose split needs more than
+ * the array holds (more than 65,536 (sequence, KV head) pairs, or partials
+ * beyond the rest of the array) returns PBB_ERR_SCRATCH_LIMIT without
+ * launching; pbb_decode_step handles those shapes. Bounded waits use the
+ * default limit of one second (pbb_set_wait_timeout_ns does not apply here).
+ *   - The first call on each device, with that device current, looks up the
+ *     array's device address (cudaGetSymbolAddress) and caches it; make that
+ *     first call before any stream capture.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents; each call zeroes the counters it uses (an asynchronous memset
+ *     on `stream`) before its kernel. Calls whose execution overlaps on the GPU
+ *     (different streams, or concurrent host threads) race on the array: the
+ *     caller must order them.
+ */
+#define PBB_NOALLOC_SCRATCH_BYTES (16u << 20)
+int pbb_decode_step_noalloc(const void* q, const void* k_new, const void* v_new, void* k_ring,
+                            void* v_ring, const int32_t* pos, float* out, int batch, int Hq,
+                            int Hkv, int d, int B, cudaStream_t stream);
 
 /* Static description of an error code. */
 const char* pbb_error_string(int code);

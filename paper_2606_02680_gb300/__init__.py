@@ -25,7 +25,8 @@ import torch
 
 __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
-    "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION", "PbbError",
+    "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
+    "PBB_ERR_SCRATCH_LIMIT", "PbbError",
     "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step",
     "decode_step_host", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "error_string", "EXPORTS",
@@ -38,6 +39,7 @@ PBB_ERR_CUDA = -3
 PBB_ERR_DEVICE_TIMEOUT = -4
 PBB_ERR_WORKSPACE = -5
 PBB_ERR_DEVICE_POSITION = -6
+PBB_ERR_SCRATCH_LIMIT = -7
 
 PBB_BF16 = 0
 PBB_F32 = 1
@@ -52,6 +54,7 @@ EXPORTS = {
     "pbb_reserve_workspace": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_decode_step_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
     "pbb_get_device_status": (_I, [_P]),
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),

@@ -362,6 +362,7 @@ const char* pbb_error_string(int code)
         case PBB_ERR_DEVICE_TIMEOUT: return "a kernel's bounded wait on a bulk copy ran out";
         case PBB_ERR_WORKSPACE: return "workspace too small while the stream is captured; call pbb_reserve_workspace first";
         case PBB_ERR_DEVICE_POSITION: return "a kernel saw a negative position; that sequence was skipped";
+        case PBB_ERR_SCRATCH_LIMIT: return "the step needs more scratch than pbb_decode_step_noalloc's fixed array holds; use pbb_decode_step";
         default: return "unknown error code";
     }
 }

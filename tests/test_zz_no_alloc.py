@@ -1,0 +1,99 @@
+"""pbb_decode_step_noalloc against pbb_decode_step, through the C ABI.
+
+The no-allocation entry point serves callers that cannot allocate device
+memory while they decode (a runtime that owns all of HBM through its own pool,
+code inside a CUDA stream capture, loops that cannot afford cudaMalloc's
+implicit synchronisation). Its split scratch is a fixed array inside the
+library instead of the workspace pbb_decode_step grows with cudaMalloc. This
+file is collected last on purpose, so a run that stops at the first failure
+has already run every other test; it also passes when run alone.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2606_02680_gb300 import build as nvbuild
+
+    nvbuild.build()
+    import paper_2606_02680_gb300 as pbb
+
+    torch.cuda.set_device(0)
+    prev = pbb.set_chunk_keys(0)  # the library's own split plan
+    yield pbb
+    pbb.set_chunk_keys(prev)
+
+
+def _state(pbb, w, t0, wk, wv, dev):
+    pos = t0.to(torch.int32).to(dev)
+    kr = torch.zeros((w.batch, w.Hkv, w.B, w.d), dtype=torch.bfloat16, device=dev)
+    vr = torch.zeros_like(kr)
+    pbb.ring_prefill(wk, wv, pos, kr, vr)
+    return pos, kr, vr
+
+
+def test_noalloc_matches_decode_step_on_two_calls(lib):
+    pbb = lib
+    from paper_2606_02680_gb300 import inputs
+
+    dev = torch.device("cuda", 0)
+    # small batch: the plan splits every support across many CTAs, so the scratch is used
+    w = inputs.Workload("noalloc", batch=4, Hq=16, Hkv=4, d=128, B=2048, dtype="bf16", steps=2,
+                        t0_lo=2048, t0_hi=100000, seed=77)
+    assert pbb.plan_chunk_keys(w.batch, w.Hq, w.Hkv, w.d, w.B) < w.B - 1
+    t0 = inputs.start_positions(w)
+    wk, wv = inputs.history_window(w, t0, device=dev)
+    pos_a, kr_a, vr_a = _state(pbb, w, t0, wk, wv, dev)
+    pos_b, kr_b, vr_b = _state(pbb, w, t0, wk, wv, dev)
+    stream = torch.cuda.current_stream()
+    s = ctypes.c_void_p(stream.cuda_stream)
+    L = pbb.lib()
+    for step in range(2):
+        q, k, v = inputs.step_inputs(w, step, device=dev)
+        out_a = torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32, device=dev)
+        out_b = torch.full_like(out_a, float("nan"))
+        rc = L.pbb_decode_step(q.data_ptr(), k.data_ptr(), v.data_ptr(), kr_a.data_ptr(),
+                               vr_a.data_ptr(), pos_a.data_ptr(), out_a.data_ptr(), w.batch, w.Hq,
+                               w.Hkv, w.d, w.B, s)
+        assert rc == pbb.PBB_OK
+        rc = L.pbb_decode_step_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(), kr_b.data_ptr(),
+                                       vr_b.data_ptr(), pos_b.data_ptr(), out_b.data_ptr(), w.batch,
+                                       w.Hq, w.Hkv, w.d, w.B, s)
+        assert rc == pbb.PBB_OK
+        assert L.pbb_advance_positions(pos_a.data_ptr(), w.batch, s) == pbb.PBB_OK
+        assert L.pbb_advance_positions(pos_b.data_ptr(), w.batch, s) == pbb.PBB_OK
+        torch.cuda.synchronize()
+        a = out_a.cpu().double().numpy()
+        b = out_b.cpu().double().numpy()
+        assert np.all(np.isfinite(b))
+        err = np.abs(a - b)
+        assert err.max() <= 1e-2 and (err / np.maximum(np.abs(a), 1.0)).max() <= 1e-2, step
+        assert torch.equal(kr_a.view(torch.int16), kr_b.view(torch.int16))
+        assert torch.equal(vr_a.view(torch.int16), vr_b.view(torch.int16))
+    assert L.pbb_get_device_status(s) == pbb.PBB_OK
+
+
+def test_noalloc_rejects_steps_beyond_its_scratch(lib):
+    pbb = lib
+    dev = torch.device("cuda", 0)
+    batch, Hq, Hkv, d, B = 64, 32, 8, 128, 4096
+    prev = pbb.set_chunk_keys(32)  # 128 CTAs per support: partials far beyond the fixed array
+    try:
+        x = torch.zeros(16, dtype=torch.bfloat16, device=dev)  # never read: rejected before launch
+        o = torch.zeros(16, dtype=torch.float32, device=dev)
+        p = torch.zeros(16, dtype=torch.int32, device=dev)
+        rc = pbb.lib().pbb_decode_step_noalloc(x.data_ptr(), x.data_ptr(), x.data_ptr(), x.data_ptr(),
+                                               x.data_ptr(), p.data_ptr(), o.data_ptr(), batch, Hq,
+                                               Hkv, d, B, None)
+        assert rc == pbb.PBB_ERR_SCRATCH_LIMIT
+        assert "scratch" in pbb.error_string(rc)
+    finally:
+        pbb.set_chunk_keys(prev)
