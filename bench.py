@@ -49,6 +49,8 @@ def parse_args():
     ap.add_argument("--batch", type=int, default=512)
     ap.add_argument("--block", type=int, default=4096)
     ap.add_argument("--sweep", action="store_true", help="one line per throughput-sweep point")
+    ap.add_argument("--workload", default="", help="a named workload of paper_2606_02680_gb300.inputs "
+                    "(default: the throughput point given by --batch/--block)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -141,12 +143,12 @@ def hbm_peak():
 
 
 def kernel_source_sha() -> str:
+    """Hash of the decode kernel's source (the file the ncu traffic record depends on)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_02680_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
-        if name.endswith((".cu", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+    for name in ("pbb_decode.cu", "pbb_internal.h"):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()[:16]
 
 
@@ -388,18 +390,23 @@ def run_ours(args):
     torch.cuda.set_device(dev)
     pbb.set_chunk_keys(args.chunk)
 
-    points = [(args.batch, args.block)]
-    if args.sweep:
-        points = [(b, B) for b in inputs.SWEEP_BATCHES for B in inputs.SWEEP_BLOCKS]
+    if args.workload:
+        base = inputs.WORKLOADS[args.workload]
+        points = [base.with_(batch=shard_batch(base.batch, rank, world))]
+    elif args.sweep:
+        points = [inputs.sweep_workload(shard_batch(b, rank, world), B)
+                  for b in inputs.SWEEP_BATCHES for B in inputs.SWEEP_BLOCKS]
+    else:
+        points = [inputs.sweep_workload(shard_batch(args.batch, rank, world), args.block)]
     peak, peak_kind = hbm_peak()
-    for batch, B in points:
-        w = inputs.sweep_workload(shard_batch(batch, rank, world), B)
+    for w in points:
+        batch, B = w.batch, w.B
         res = time_device(w, dev, args.steps, args.warmup, dist)
         total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
         units = sum_over_ranks(dist, w.batch * w.Hq * args.steps)
         value = units / total_s
         achieved = res["launch_bytes_mean"] / (res["kernel_ms_mean"] / 1e3) / 1e9
-        key = f"sweep_b{batch}_B{B}"
+        key = w.name
         traffic = recorded_traffic(key, res["launch_bytes_mean"])
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -417,7 +424,8 @@ def run_ours(args):
             "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
-                         "kernel": "decode_kernel<2,128,4>", "peak_kind": peak_kind,
+                         "kernel": "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group),
+                         "peak_kind": peak_kind,
                          "algorithmic_bytes_per_launch": res["launch_bytes_mean"],
                          "kernel_ms_mean": res["kernel_ms_mean"],
                          "kernel_ms_median": res["kernel_ms_median"]},

@@ -34,19 +34,28 @@ def up_to_date() -> bool:
     return all(os.path.getmtime(f) <= t for f in _inputs())
 
 
-def build(force: bool = False, verbose: bool = False) -> str:
-    """Build paper_2606_02680_gb300/libpbb.so if any source is newer; return its path."""
-    if not force and up_to_date():
+def build(force: bool = False, verbose: bool = False, out: str | None = None,
+          defines: dict | None = None) -> str:
+    """Build paper_2606_02680_gb300/libpbb.so if any source is newer; return its path.
+
+    `out` and `defines` (-D macros, e.g. the kernel's launch-shape knobs) build a
+    variant elsewhere, always from scratch.
+    """
+    lib = out or LIB
+    if out is None and not force and not defines and up_to_date():
         return LIB
-    os.makedirs(OBJ_DIR, exist_ok=True)
+    obj_dir = OBJ_DIR if out is None else os.path.splitext(out)[0] + "_obj"
+    os.makedirs(obj_dir, exist_ok=True)
     nvcc = _nvcc()
     common = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE,
                      "-I", CSRC]
+    for k, v in (defines or {}).items():
+        common.append(f"-D{k}={v}")
     if verbose:
         common += ["-Xptxas", "-v"]
 
     def compile_one(src):
-        obj = os.path.join(OBJ_DIR, os.path.splitext(src)[0] + ".o")
+        obj = os.path.join(obj_dir, os.path.splitext(src)[0] + ".o")
         cmd = [nvcc] + common + ["-c", os.path.join(CSRC, src), "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -58,13 +67,13 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if verbose:
         for _, log in results:
             print(log)
-    tmp = LIB + f".tmp{os.getpid()}"
+    tmp = lib + f".tmp{os.getpid()}"
     cmd = [nvcc] + ARCH + ["-shared", "-cudart", "shared", "-o", tmp] + [o for o, _ in results]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
-    return LIB
+    os.replace(tmp, lib)
+    return lib
 
 
 if __name__ == "__main__":

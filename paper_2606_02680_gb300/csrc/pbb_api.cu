@@ -15,11 +15,12 @@ namespace {
 constexpr int kMaxDevices = 64;
 constexpr int kMaxBlock = 1 << 20;
 
-// Library-owned scratch of one device: one arrival counter per (sequence, KV
-// head), which must read zero between steps, and the split partials.
+// Library-owned scratch of one device: the work-queue control words and one
+// counter per (sequence, KV head), all of which read zero between steps, and
+// the split partials.
 struct Workspace {
-    int* counters = nullptr;
-    size_t counter_cap = 0;  // counters allocated (pairs)
+    int* counters = nullptr;  // [0, 2): queue control; then one per (sequence, KV head)
+    size_t counter_cap = 0;   // ints allocated
     float* parts = nullptr;
     size_t parts_bytes = 0;
 };
@@ -79,7 +80,7 @@ int sm_count(int dev)
 // over (at least kWaves waves of resident CTAs); large batches run unsplit.
 int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
 {
-    const int tile = pbb::tile_keys(elem, d);
+    const int tile = pbb::tile_keys(elem, d, group);
     const int max_keys = B - 1;
     int chunk;
     const int over = g_chunk_override.load();
@@ -135,7 +136,7 @@ int grow_workspace(int dev, size_t pairs, size_t pbytes, cudaStream_t stream, bo
         ws.counters = c;
         ws.counter_cap = pairs;
     }
-    if (ws.parts_bytes < pbytes) {
+    if (pbytes > 0 && ws.parts_bytes < pbytes) {
         void* p = nullptr;
         if (cudaMalloc(&p, pbytes) != cudaSuccess) return PBB_ERR_CUDA;
         cudaFree(ws.parts);
@@ -182,17 +183,22 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     if (a.nchunk < 1) a.nchunk = 1;
     a.timeout_ns = g_timeout_ns.load();
     if (a.nchunk > 65535) return PBB_ERR_UNSUPPORTED;
-    if (a.nchunk > 1) {
-        const size_t pairs = static_cast<size_t>(batch) * Hkv;
-        const size_t pbytes = parts_bytes(batch, Hkv, d, group, a.nchunk);
+    const size_t pairs = static_cast<size_t>(batch) * Hkv;
+    a.total_items = static_cast<int>(pairs * a.nchunk);
+    if (pairs * a.nchunk > static_cast<size_t>(INT_MAX)) return PBB_ERR_UNSUPPORTED;
+    {
+        const size_t pbytes = a.nchunk > 1 ? parts_bytes(batch, Hkv, d, group, a.nchunk) : 0;
         std::lock_guard<std::mutex> lock(g_mutex);
-        rc = grow_workspace(dev, pairs, pbytes, stream, true);
+        rc = grow_workspace(dev, pairs + 2, pbytes, stream, true);
         if (rc != PBB_OK) return rc;
         const size_t parts = pairs * a.nchunk * group;
-        a.counters = g_ws[dev].counters;
-        a.part_o = g_ws[dev].parts;
-        a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(g_ws[dev].parts) +
-                                             round_up(parts * d * sizeof(float), 256));
+        a.ctl = g_ws[dev].counters;
+        a.counters = g_ws[dev].counters + 2;
+        if (a.nchunk > 1) {
+            a.part_o = g_ws[dev].parts;
+            a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(g_ws[dev].parts) +
+                                                 round_up(parts * d * sizeof(float), 256));
+        }
     }
     return pbb::launch_decode(a, elem, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
@@ -274,18 +280,15 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
     const int group = Hq / Hkv;
     // Every batch up to max_batch: the plan's split shrinks as the batch grows.
     size_t need = 0;
-    size_t pairs_need = 0;
     for (int bsz = 1; bsz <= max_batch; ++bsz) {
         const int chunk = plan_chunk(bsz, Hkv, d, B, elem, group, dev);
         const int nchunk = (B - 1 + chunk - 1) / chunk;
         if (nchunk <= 1) continue;
         const size_t w = parts_bytes(bsz, Hkv, d, group, nchunk);
         if (w > need) need = w;
-        pairs_need = static_cast<size_t>(bsz) * Hkv;
     }
-    if (need == 0) return PBB_OK;
     std::lock_guard<std::mutex> lock(g_mutex);
-    return grow_workspace(dev, pairs_need, need, nullptr, false);
+    return grow_workspace(dev, static_cast<size_t>(max_batch) * Hkv + 2, need, nullptr, false);
 }
 
 int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,

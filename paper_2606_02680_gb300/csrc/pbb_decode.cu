@@ -1,41 +1,52 @@
 // Kernels of the PBB decode step for sm_103a.
 //
-// Work decomposition. The support of a sequence at position t = p + r is the
-// interval [a(t), t] (Eq. pbb_relay). Apart from the current token, which
-// comes from k_new/v_new, it occupies at most two contiguous runs of ring
-// slots (Appendix F.1): bridge phases (p > 0, r < h) read slots h..B-1 (the
-// previous block's tail, positions p-h..p-1) and then 0..r-1; the other phases
-// read 0..r-1. Counting those n keys in position order, logical key i lives in
-// slot (base + i) mod B with base = h for a bridge phase and 0 otherwise.
+// The support. For a sequence whose current token is at t = p + r (block
+// start p, phase r, B = 2h) the support is the interval [a(t), t]
+// (Eq. pbb_relay). Apart from the current token, which comes from
+// k_new/v_new, it occupies at most two contiguous runs of ring slots
+// (Appendix F.1): a bridge phase (p > 0, r < h) reads slots h..B-1 (the
+// previous block's tail, positions p-h..p-1) and then 0..r-1; the other
+// phases read 0..r-1. In position order, ring key i of the support lives in
+// slot (base + i) mod B, base = h for a bridge phase and 0 otherwise.
 //
-// The grid is (chunk, KV head, sequence). CTA `chunk` takes logical keys
-// [chunk*C, chunk*C + C) of its (sequence, KV head), serves all G = Hq/Hkv
-// query heads of the group (each K/V byte is read from HBM once per step),
-// and CTAs past the end of a short support exit at once. Chunk 0 also appends
-// the new K/V to slot r and folds the current token into its softmax state;
-// slot r is never in the read set, so the append and the reads do not race.
+// Work items. Item (sequence, KV head, chunk) covers ring keys
+// [chunk*C, chunk*C + C) of one support, for all G = Hq/Hkv query heads of the
+// group, so each K/V byte is read from HBM once per step. Chunk 0 of every
+// (sequence, KV head) also carries the current token: it appends k_new/v_new
+// to slot r (never a slot that is read) and folds the token into its softmax.
+// Items past the end of a short support are empty and skipped.
 //
-// Inside a CTA one thread streams K/V tiles of TK keys into a 4-stage shared
-// memory ring with 1-D bulk copies (cp.async.bulk, completion on an mbarrier);
-// a tile that straddles the ring's end is fetched as two copies. Each of the 4
-// warps owns a quarter of every tile and keeps its own fp32 online softmax in
-// the base-2 domain (the scale log2(e)/sqrt(d) is folded into q):
-//   scores: 8 lanes per key, 4 keys per warp step; a lane holds q for d/8 dims
-//           of all G heads in registers and the partial dot products are
-//           combined with a reduce-scatter over the 8 lanes, so each lane ends
-//           with the score of one (key, head);
-//   P.V:    the warp walks its keys; every lane owns d/32 output dims of all G
-//           heads and reads the weights of a key as a broadcast from shared
-//           memory.
-// The warps' states are merged in shared memory. A single-CTA support writes
-// `out` directly; otherwise each CTA stores its partial (max, sum, output) and
-// the last CTA of the (sequence, KV head) to arrive (an atomic counter, no
-// spinning) fuses them in chunk order with Eq. (lse) and resets the counter,
-// so the result does not depend on CTA scheduling.
+// Persistent CTAs, one per SM. A producer lane takes items from a device-wide
+// queue (an atomic counter) and streams them without a break: every item
+// becomes tiles of TK keys, and each tile lands in one stage of a 3-stage
+// shared-memory ring through 1-D bulk copies (cp.async.bulk, completion
+// counted in bytes on the stage's "full" mbarrier). The first tile of an item
+// also brings the item's G query rows and, for chunk 0, the new K/V rows; a
+// tile that straddles the end of the ring is fetched as two copies. The
+// producer writes a small descriptor per stage (item, keys, first/last flags)
+// before arming the barrier, so consumers learn item boundaries in order.
 //
-// Every wait on an mbarrier is bounded (globaltimer); when it runs out the CTA
-// records kDevTimeout, waits (bounded) for its own copies still in flight and
-// returns without writing its output.
+// Eight consumer warps share every tile (KW = TK/8 keys each) and keep
+// independent fp32 online-softmax states in the base-2 domain (the scale
+// log2(e)/sqrt(d) is folded into q), releasing the stage through its "empty"
+// mbarrier:
+//   scores: KL lanes per key (8, or 16 for G = 8 so the query registers fit);
+//           a lane holds the queries of d/KL dims of all G heads and the
+//           partial dot products are combined by a reduce-scatter over the
+//           KL lanes, so each lane ends with the score of one (key, head);
+//           products are packed fp32x2 FMAs;
+//   P.V:    each lane owns d/32 output dims of all G heads and reads a key's
+//           weights from shared memory as ready fp32x2 pairs.
+// At an item's last tile the consumer warps merge their states in shared
+// memory (Eq. lse). A single-item support writes `out`; otherwise the item
+// stores its partial (max, sum, output) and the last item of the (sequence,
+// KV head) to finish (an atomic counter, no spinning) fuses all partials in
+// chunk order with Eq. (lse) and resets the counter, so results do not depend
+// on scheduling. The last CTA to finish resets the queue.
+//
+// No wait can hang: waits on mbarriers and the consumers' software barrier are
+// bounded by the global timer. A wait that runs out records kDevTimeout; the
+// CTA then stops, waits (bounded) for the copies it issued and returns.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -48,11 +59,40 @@ __device__ int g_status;  // first device-side fault recorded, kDevOk if none
 
 namespace {
 
-constexpr int kWarps = 4;
-constexpr int kThreads = kWarps * 32;
-constexpr int kStages = 4;
-constexpr int kTileBytes = 8192;  // bytes of K (and of V) per stage
+// Launch shape. Chosen by measurement on GB300 (a sweep of consumer warps,
+// tile bytes, stages and resident CTAs per SM); the macros let a build try
+// other shapes without editing the kernel.
+#ifndef PBB_CONSUMER_WARPS
+#define PBB_CONSUMER_WARPS 4
+#endif
+#ifndef PBB_STAGES
+#define PBB_STAGES 3
+#endif
+#ifndef PBB_TILE_BYTES
+#define PBB_TILE_BYTES 8192
+#endif
+#ifndef PBB_TILE_BYTES_G8
+#define PBB_TILE_BYTES_G8 8192
+#endif
+#ifndef PBB_MIN_CTAS
+#define PBB_MIN_CTAS 3
+#endif
+#ifndef PBB_MIN_CTAS_G8
+#define PBB_MIN_CTAS_G8 2
+#endif
+constexpr int kConsumers = PBB_CONSUMER_WARPS;   // warps that compute
+constexpr int kThreads = (kConsumers + 1) * 32;  // plus one producer warp
+constexpr int kStages = PBB_STAGES;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken GPU can exceed
+
+enum : int { kFirst = 1, kLast = 2, kCurrent = 4, kEnd = 8 };
+
+// Descriptor of the tile in one stage, written by the producer before it arms the stage.
+struct __align__(16) TileMeta {
+    int b, kvh, chunk, nk;  // item and ring keys in this tile
+    int nch, r, flags, pad; // chunks of the support, phase, kFirst/kLast/kCurrent/kEnd
+};
 
 // ---------------------------------------------------------------- PTX ----
 
@@ -211,36 +251,6 @@ __device__ __forceinline__ void load_elems(const unsigned char* p, float* f)
 
 // --------------------------------------------------------- reductions ----
 
-// Within each aligned group of 8 lanes, every lane holds G partial sums (one
-// per head). Afterwards lane `sub` (0..7) holds the group's full sum for head
-// sub >> (3 - log2 G): each exchange step halves the values a lane keeps and
-// the steps left over once one value remains are plain butterfly sums.
-template <int G>
-__device__ __forceinline__ float reduce_scatter8(const float (&acc)[G], int sub)
-{
-    float v[G];
-#pragma unroll
-    for (int i = 0; i < G; ++i) v[i] = acc[i];
-    int cnt = G;
-#pragma unroll
-    for (int lvl = 4; lvl >= 1; lvl >>= 1) {
-        if (cnt > 1) {
-            const int half = cnt / 2;
-            const bool up = (sub & lvl) != 0;
-#pragma unroll
-            for (int i = 0; i < half; ++i) {
-                const float send = up ? v[i] : v[i + half];
-                const float keep = up ? v[i + half] : v[i];
-                v[i] = keep + __shfl_xor_sync(kFull, send, lvl);
-            }
-            cnt = half;
-        } else {
-            v[0] += __shfl_xor_sync(kFull, v[0], lvl);
-        }
-    }
-    return v[0];
-}
-
 template <int N>
 struct Log2 {
     static constexpr int value = (N <= 1) ? 0 : 1 + Log2<N / 2>::value;
@@ -250,309 +260,517 @@ struct Log2<1> {
     static constexpr int value = 0;
 };
 
+// Within each aligned group of KL lanes, every lane holds G partial sums, one
+// per head, in a lane-specific order: position p holds head (myhead ^ p), where
+// myhead = sub >> (log2 KL - log2 G). Each exchange step then keeps the first
+// half of the positions and sends the second half, which are exactly the
+// partner lane's first half, so no lane needs a select. Once a lane keeps one
+// value the remaining steps are butterfly sums. Afterwards every lane holds the
+// group's full sum for its own head.
+template <int G, int KL>
+__device__ __forceinline__ float reduce_scatter(float (&v)[G])
+{
+    int cnt = G;
+#pragma unroll
+    for (int lvl = KL / 2; lvl >= 1; lvl >>= 1) {
+        if (cnt > 1) {
+            const int half = cnt / 2;
+#pragma unroll
+            for (int i = 0; i < half; ++i) v[i] += __shfl_xor_sync(kFull, v[i + half], lvl);
+            cnt = half;
+        } else {
+            v[0] += __shfl_xor_sync(kFull, v[0], lvl);
+        }
+    }
+    return v[0];
+}
+
+// 2^x with the SFU instruction (flushes subnormal results to zero; 2^-inf = 0).
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+// Barrier of the consumer warps through a shared-memory counter, bounded by
+// `limit_ns` (a hardware named barrier could not be bounded). All lanes of all
+// consumer warps call it; returns false if it gave up.
+__device__ __forceinline__ bool consumer_barrier(unsigned* count, volatile unsigned* gen, int lane,
+                                                 unsigned long long limit_ns)
+{
+    bool ok = true;
+    __syncwarp();
+    if (lane == 0) {
+        const unsigned g = *gen;
+        __threadfence_block();
+        if (atomicAdd(count, 1u) == kConsumers - 1) {
+            *count = 0;
+            __threadfence_block();
+            *gen = g + 1;
+        } else {
+            const unsigned long long t0 = global_ns();
+            while (*gen == g) {
+                if (global_ns() - t0 > limit_ns) {
+                    ok = false;
+                    break;
+                }
+            }
+        }
+        __threadfence_block();
+    }
+    return __shfl_sync(kFull, ok ? 1 : 0, 0) != 0;
+}
+
 // ------------------------------------------------------------ config ----
 
 template <int ELEM, int D, int G>
 struct Cfg {
-    static constexpr int ROW = D * ELEM;            // bytes of one K or V row
-    static constexpr int TK = kTileBytes / ROW;     // keys per tile
-    static constexpr int KW = TK / kWarps;          // keys per warp per tile
-    static constexpr int STEPS = KW / 4;            // score steps (4 keys each) per tile
-    static constexpr int VPL = ROW / 128;           // 16-byte vectors per lane (score phase)
-    static constexpr int EPV = 16 / ELEM;           // elements per 16-byte vector
-    static constexpr int DPL = D / 8;               // dims per lane (score phase)
-    static constexpr int PVD = D / 32;              // dims per lane (P.V phase)
-    static constexpr int REP = 3 - Log2<G>::value;  // lanes per (key, head) = 2^REP
-    static constexpr int STAGE = 2 * TK * ROW;      // K tile + V tile
-    static constexpr int SMEM = kStages * STAGE;
-    static_assert(KW % 4 == 0 && KW >= 4, "a warp needs whole score steps");
-    static_assert(VPL * EPV == DPL, "score-phase slice");
-    static_assert(kWarps * G * D * 4 <= SMEM, "merge buffer must fit in the stages");
+    // resident CTAs per SM the registers and shared memory must allow
+    static constexpr int MIN_CTAS = (G == 8) ? PBB_MIN_CTAS_G8 : PBB_MIN_CTAS;
+    static constexpr int ROW = D * ELEM;                            // bytes of one K or V row
+    static constexpr int KL = (G == 8 && ROW >= 256) ? 16 : 8;      // lanes per key, score phase
+    static constexpr int KPS = 32 / KL;                             // keys per warp step
+    static constexpr int MERGE = kConsumers * G * D * 4;            // per-warp outputs at a merge
+    static constexpr int BUDGET = 218 * 1024 / MIN_CTAS;            // dynamic shared memory per CTA
+    static constexpr int stage_bytes(int tile)
+    {
+        return (2 * tile + (G + 2) * ROW + 127) / 128 * 128;
+    }
+    // The requested K (and V) bytes per stage, halved until the stages and the
+    // merge buffer fit the budget (fp32 rows are twice as wide).
+    static constexpr int fit_tile(int tile)
+    {
+        while (kStages * stage_bytes(tile) + MERGE > BUDGET && tile > ROW * kConsumers * KPS) tile /= 2;
+        return tile;
+    }
+    static constexpr int TILE_BYTES = fit_tile((G == 8) ? PBB_TILE_BYTES_G8 : PBB_TILE_BYTES);
+    static constexpr int TK = TILE_BYTES / ROW;                     // keys per tile
+    static constexpr int KW = TK / kConsumers;                      // keys per consumer warp per tile
+    static constexpr int STEPS = KW / KPS;                          // score steps per tile
+    static constexpr int VPL = ROW / (KL * 16);                     // 16-byte vectors per lane, score phase
+    static constexpr int EPV = 16 / ELEM;                           // elements per 16-byte vector
+    static constexpr int DPL = D / KL;                              // dims per lane, score phase
+    static constexpr int PVD = D / 32;                              // dims per lane, P.V phase
+    static constexpr int REP = Log2<KL>::value - Log2<G>::value;    // lanes per (key, head) = 2^REP
+    static constexpr int KV = 2 * TK * ROW;                         // K tile then V tile
+    static constexpr int Q_OFF = KV;                                // the item's G query rows
+    static constexpr int KN_OFF = Q_OFF + G * ROW;                  // k_new row (chunk 0)
+    static constexpr int VN_OFF = KN_OFF + ROW;                     // v_new row (chunk 0)
+    static constexpr int STAGE = (VN_OFF + ROW + 127) / 128 * 128;
+    static constexpr int SMEM = kStages * STAGE + MERGE;
+    static_assert(KW % KPS == 0 && STEPS >= 1, "a warp needs whole score steps");
+    static_assert(VPL >= 1 && VPL * EPV == DPL && (EPV % 2) == 0 && (PVD % 2) == 0, "lane slices");
+    static_assert(REP >= 0, "group larger than the lanes of a key");
+    static_assert(SMEM <= BUDGET, "shared memory budget (dynamic; the static part is a few KiB)");
 };
 
 // ------------------------------------------------------------ kernel ----
 
 template <int ELEM, int D, int G>
-__global__ void __launch_bounds__(kThreads) decode_kernel(const DecodeArgs a)
+__global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_kernel(const DecodeArgs a)
 {
     using C = Cfg<ELEM, D, G>;
     extern __shared__ __align__(128) unsigned char dsmem[];
     __shared__ __align__(8) uint64_t full_bar[kStages];
-    __shared__ __align__(16) float q_s[G * D];
-    __shared__ __align__(16) float p_s[kWarps][C::KW][G];
-    __shared__ __align__(16) float alpha_s[kWarps][G];
-    __shared__ float2 ml_s[kWarps][G];
+    __shared__ __align__(8) uint64_t empty_bar[kStages];
+    __shared__ TileMeta meta_s[kStages];
+    __shared__ __align__(16) float p_s[kConsumers][C::KW][G];  // softmax weights of a tile
+    __shared__ __align__(16) float alpha_s[kConsumers][G];     // rescale factors of a tile
+    __shared__ float2 ml_s[kConsumers][G];
+    __shared__ unsigned sbar_count;
+    __shared__ volatile unsigned sbar_gen;
+    __shared__ volatile int abort_s;
     __shared__ int last_s;
+    __shared__ int issued_s;
 
-    const int chunk = blockIdx.x, kvh = blockIdx.y, b = blockIdx.z;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int t = __ldg(a.pos + b);
-    if (t < 0) {
-        if (chunk == 0 && kvh == 0 && tid == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
-        return;
-    }
-    const int B = a.B, h = B >> 1;
-    const int blk = t / B;
-    const int r = t - blk * B;
-    const bool bridge = (blk > 0) && (r < h);
-    const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
-    const int base = bridge ? h : 0;   // slot of logical key 0
-    const int nch = n > 0 ? (n + a.chunk - 1) / a.chunk : 1;
-    if (chunk >= nch) return;
-    const int i0 = chunk * a.chunk;
-    const int i1 = min(i0 + a.chunk, n);
-    const int ntiles = i1 > i0 ? (i1 - i0 + C::TK - 1) / C::TK : 0;
-
-    const size_t head = static_cast<size_t>(b) * a.Hkv + kvh;
-    const unsigned char* kring = static_cast<const unsigned char*>(a.k_ring) + head * B * C::ROW;
-    const unsigned char* vring = static_cast<const unsigned char*>(a.v_ring) + head * B * C::ROW;
-
     if (tid == 0) {
 #pragma unroll
-        for (int s = 0; s < kStages; ++s) mbar_init(&full_bar[s], 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], kConsumers);
+        }
         fence_mbar_init();
-    }
-    // Scaled queries of the group, fp32: q_s[j][c] = q[b][kvh*G + j][c] * log2(e)/sqrt(d).
-    {
-        const float scale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
-        const unsigned char* qg = static_cast<const unsigned char*>(a.q) +
-                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * C::ROW;
-        for (int e = tid; e < G * D; e += kThreads) q_s[e] = Elem<ELEM>::to_float(qg + e * ELEM) * scale;
+        sbar_count = 0;
+        sbar_gen = 0;
+        abort_s = 0;
+        issued_s = 0;
     }
     __syncthreads();
 
-    auto issue = [&](int it) {
-        const int s = it % kStages;
-        const int k0 = i0 + it * C::TK;
-        const int nk = min(C::TK, i1 - k0);
-        int slot = base + k0;
-        if (slot >= B) slot -= B;
-        const int len1 = min(nk, B - slot);
-        unsigned char* sK = dsmem + s * C::STAGE;
-        unsigned char* sV = sK + C::TK * C::ROW;
-        mbar_expect_tx(&full_bar[s], static_cast<uint32_t>(2 * nk * C::ROW));
-        bulk_g2s(sK, kring + static_cast<size_t>(slot) * C::ROW, len1 * C::ROW, &full_bar[s]);
-        bulk_g2s(sV, vring + static_cast<size_t>(slot) * C::ROW, len1 * C::ROW, &full_bar[s]);
-        if (len1 < nk) {  // wrapped past slot B-1: the rest starts at slot 0
-            bulk_g2s(sK + len1 * C::ROW, kring, (nk - len1) * C::ROW, &full_bar[s]);
-            bulk_g2s(sV + len1 * C::ROW, vring, (nk - len1) * C::ROW, &full_bar[s]);
-        }
-    };
-    if (tid == 0) {
-        const int pro = min(kStages, ntiles);
-        for (int it = 0; it < pro; ++it) issue(it);
-    }
-
-    // Queries of this lane's score-phase slice: vector m covers dims (sub + 8m)*EPV ...
-    const int sub = lane & 7, kq = lane >> 3;
-    float qr[G][C::DPL];
-#pragma unroll
-    for (int j = 0; j < G; ++j)
-#pragma unroll
-        for (int m = 0; m < C::VPL; ++m)
-#pragma unroll
-            for (int x = 0; x < C::EPV; ++x)
-                qr[j][m * C::EPV + x] = q_s[j * D + (sub + 8 * m) * C::EPV + x];
-
-    const int myhead = sub >> C::REP;
-    const bool primary = (sub & ((1 << C::REP) - 1)) == 0;
-    float m_run = -INFINITY;  // running max of this lane's head (log2 domain)
-    float l_run = 0.f;        // this lane's share of the running sum (primary lanes only)
-    float o[G][C::PVD];
-#pragma unroll
-    for (int j = 0; j < G; ++j)
-#pragma unroll
-        for (int x = 0; x < C::PVD; ++x) o[j][x] = 0.f;
-
-    if (chunk == 0) {
-        // Append: slot r of both rings <- the new token's rows (bit copy).
-        const uint4* kn = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(a.k_new) + head * C::ROW);
-        const uint4* vn = reinterpret_cast<const uint4*>(static_cast<const unsigned char*>(a.v_new) + head * C::ROW);
-        uint4* kd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.k_ring) + (head * B + r) * C::ROW);
-        uint4* vd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.v_ring) + (head * B + r) * C::ROW);
-        for (int x = tid; x < C::ROW / 16; x += kThreads) {
-            kd[x] = __ldg(kn + x);
-            vd[x] = __ldg(vn + x);
-        }
-        if (warp == 0) {  // the current token seeds warp 0's softmax state
-            float kc[C::PVD], vc[C::PVD];
-            const unsigned char* knb = static_cast<const unsigned char*>(a.k_new) + head * C::ROW;
-            const unsigned char* vnb = static_cast<const unsigned char*>(a.v_new) + head * C::ROW;
-            load_elems<ELEM, C::PVD>(knb + lane * C::PVD * ELEM, kc);
-            load_elems<ELEM, C::PVD>(vnb + lane * C::PVD * ELEM, vc);
-            float zc[G];
-#pragma unroll
-            for (int j = 0; j < G; ++j) {
-                float acc = 0.f;
-#pragma unroll
-                for (int x = 0; x < C::PVD; ++x) acc = fmaf(q_s[j * D + lane * C::PVD + x], kc[x], acc);
-#pragma unroll
-                for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
-                zc[j] = acc;
+    if (warp == kConsumers) {
+        // ================= producer: one lane =================
+        if (lane == 0) {
+            int seq = 0;  // tiles issued so far (stage seq % kStages)
+            bool ok = true;
+            while (ok) {
+                const int item = atomicAdd(a.ctl, 1);
+                if (item >= a.total_items) break;
+                const int chunk = item % a.nchunk;
+                const int pair = item / a.nchunk;
+                const int kvh = pair % a.Hkv, b = pair / a.Hkv;
+                const int t = __ldg(a.pos + b);
+                if (t < 0) {
+                    if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
+                    continue;
+                }
+                const int B = a.B, h = B >> 1;
+                const int blk = t / B;
+                const int r = t - blk * B;
+                const bool bridge = (blk > 0) && (r < h);
+                const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
+                const int base = bridge ? h : 0;   // slot of ring key 0
+                const int nch = n > 0 ? (n + a.chunk - 1) / a.chunk : 1;
+                if (chunk >= nch) continue;
+                const int i0 = chunk * a.chunk;
+                const int i1 = min(i0 + a.chunk, n);
+                const int nkeys = max(i1 - i0, 0);
+                const int ntiles = nkeys > 0 ? (nkeys + C::TK - 1) / C::TK : 1;
+                const size_t head = static_cast<size_t>(b) * a.Hkv + kvh;
+                const unsigned char* kring = static_cast<const unsigned char*>(a.k_ring) + head * B * C::ROW;
+                const unsigned char* vring = static_cast<const unsigned char*>(a.v_ring) + head * B * C::ROW;
+                for (int it = 0; it < ntiles; ++it, ++seq) {
+                    const int s = seq % kStages;
+                    if (seq >= kStages &&
+                        !mbar_wait(&empty_bar[s], static_cast<uint32_t>((seq / kStages - 1) & 1), kGuardNs)) {
+                        ok = false;
+                        break;
+                    }
+                    if (abort_s) {
+                        ok = false;
+                        break;
+                    }
+                    const int k0 = i0 + it * C::TK;
+                    const int nk = max(min(C::TK, i1 - k0), 0);
+                    const bool first = it == 0;
+                    const bool current = first && chunk == 0;
+                    TileMeta mt;
+                    mt.b = b;
+                    mt.kvh = kvh;
+                    mt.chunk = chunk;
+                    mt.nk = nk;
+                    mt.nch = nch;
+                    mt.r = r;
+                    mt.flags = (first ? kFirst : 0) | (it == ntiles - 1 ? kLast : 0) | (current ? kCurrent : 0);
+                    mt.pad = 0;
+                    meta_s[s] = mt;
+                    unsigned char* st = dsmem + s * C::STAGE;
+                    const uint32_t bytes = static_cast<uint32_t>(2 * nk * C::ROW + (first ? G * C::ROW : 0) +
+                                                                 (current ? 2 * C::ROW : 0));
+                    fence_proxy_async();
+                    mbar_expect_tx(&full_bar[s], bytes);  // arrives (release): the descriptor is visible
+                    if (nk > 0) {
+                        int slot = base + k0;
+                        if (slot >= B) slot -= B;
+                        const int len1 = min(nk, B - slot);
+                        bulk_g2s(st, kring + static_cast<size_t>(slot) * C::ROW, len1 * C::ROW, &full_bar[s]);
+                        bulk_g2s(st + C::TK * C::ROW, vring + static_cast<size_t>(slot) * C::ROW,
+                                 len1 * C::ROW, &full_bar[s]);
+                        if (len1 < nk) {  // wrapped past slot B-1: the rest starts at slot 0
+                            bulk_g2s(st + len1 * C::ROW, kring, (nk - len1) * C::ROW, &full_bar[s]);
+                            bulk_g2s(st + (C::TK + len1) * C::ROW, vring, (nk - len1) * C::ROW, &full_bar[s]);
+                        }
+                    }
+                    if (first) {
+                        const unsigned char* qg = static_cast<const unsigned char*>(a.q) +
+                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * C::ROW;
+                        bulk_g2s(st + C::Q_OFF, qg, G * C::ROW, &full_bar[s]);
+                    }
+                    if (current) {
+                        bulk_g2s(st + C::KN_OFF, static_cast<const unsigned char*>(a.k_new) + head * C::ROW,
+                                 C::ROW, &full_bar[s]);
+                        bulk_g2s(st + C::VN_OFF, static_cast<const unsigned char*>(a.v_new) + head * C::ROW,
+                                 C::ROW, &full_bar[s]);
+                    }
+                }
             }
-            m_run = zc[0];
-#pragma unroll
-            for (int j = 1; j < G; ++j)
-                if (myhead == j) m_run = zc[j];
-            l_run = (primary && kq == 0) ? 1.f : 0.f;
-#pragma unroll
-            for (int j = 0; j < G; ++j)
-#pragma unroll
-                for (int x = 0; x < C::PVD; ++x) o[j][x] = vc[x];
+            if (ok) {  // end-of-work descriptor: a plain arrival completes the stage's phase
+                const int s = seq % kStages;
+                if (seq >= kStages &&
+                    !mbar_wait(&empty_bar[s], static_cast<uint32_t>((seq / kStages - 1) & 1), kGuardNs)) {
+                    ok = false;
+                } else {
+                    TileMeta mt{};
+                    mt.flags = kEnd;
+                    meta_s[s] = mt;
+                    mbar_arrive(&full_bar[s]);
+                    ++seq;
+                }
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+            }
+            issued_s = seq;
         }
-    }
+    } else {
+        // ================= consumers =================
+        const int sub = lane & (C::KL - 1), kq = lane / C::KL;
+        const int myhead = sub >> C::REP;
+        const bool primary = (sub & ((1 << C::REP) - 1)) == 0;
+        const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
+        float* merge_o = reinterpret_cast<float*>(dsmem + kStages * C::STAGE);  // [kConsumers][G][D]
+        float2 qr[G][C::DPL / 2];  // this lane's query slice, scaled, as pairs
+        float m_run = -INFINITY;   // running max of this lane's head (log2 domain)
+        float l_run = 0.f;         // this lane's share of the running sum (primary lanes only)
+        float2 o[G][C::PVD / 2];   // output dims lane*PVD .. +PVD of every head
+#pragma unroll
+        for (int j = 0; j < G; ++j)
+#pragma unroll
+            for (int x = 0; x < C::DPL / 2; ++x) qr[j][x] = make_float2(0.f, 0.f);
 
-    int it = 0;
-    bool failed = false;
-    for (; it < ntiles; ++it) {
-        const int s = it % kStages;
-        const bool ok = mbar_wait(&full_bar[s], static_cast<uint32_t>((it / kStages) & 1), a.timeout_ns);
-        const int k0 = i0 + it * C::TK;
-        const int nk = min(C::TK, i1 - k0);
-        const int nkw = ok ? min(max(nk - warp * C::KW, 0), C::KW) : 0;
-        if (nkw > 0) {
-            const unsigned char* sK = dsmem + s * C::STAGE + warp * C::KW * C::ROW;
-            const unsigned char* sV = dsmem + s * C::STAGE + C::TK * C::ROW + warp * C::KW * C::ROW;
-            float zs[C::STEPS];
-            float mx = -INFINITY;
+        for (int seq = 0;; ++seq) {
+            const int s = seq % kStages;
+            if (!mbar_wait(&full_bar[s], static_cast<uint32_t>((seq / kStages) & 1), a.timeout_ns)) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+                break;
+            }
+            const TileMeta mt = meta_s[s];
+            if (mt.flags & kEnd) break;
+            if (abort_s) break;
+            const unsigned char* st = dsmem + s * C::STAGE;
+            const size_t head = static_cast<size_t>(mt.b) * a.Hkv + mt.kvh;
+
+            if (mt.flags & kFirst) {
+                // the item's queries: position p of this lane holds head (myhead ^ p), the
+                // order reduce_scatter expects; vector m covers dims (sub + KL*m)*EPV ...
 #pragma unroll
-            for (int st = 0; st < C::STEPS; ++st) {
-                const int key = st * 4 + kq;
-                float z = -INFINITY;
-                if (st * 4 < nkw) {  // warp-uniform
-                    float acc[G];
-#pragma unroll
-                    for (int j = 0; j < G; ++j) acc[j] = 0.f;
+                for (int p = 0; p < G; ++p)
 #pragma unroll
                     for (int m = 0; m < C::VPL; ++m) {
-                        float kf[C::EPV];
-                        const uint4 u = *reinterpret_cast<const uint4*>(sK + key * C::ROW + (sub + 8 * m) * 16);
-                        Elem<ELEM>::vec16(u, kf);
+                        float qf[C::EPV];
+                        const uint4 u = *reinterpret_cast<const uint4*>(st + C::Q_OFF + (myhead ^ p) * C::ROW +
+                                                                        (sub + C::KL * m) * 16);
+                        Elem<ELEM>::vec16(u, qf);
 #pragma unroll
-                        for (int j = 0; j < G; ++j)
-#pragma unroll
-                            for (int x = 0; x < C::EPV; ++x)
-                                acc[j] = fmaf(qr[j][m * C::EPV + x], kf[x], acc[j]);
+                        for (int x = 0; x < C::EPV / 2; ++x)
+                            qr[p][m * (C::EPV / 2) + x] = make_float2(qf[2 * x] * qscale, qf[2 * x + 1] * qscale);
                     }
-                    const float zz = reduce_scatter8<G>(acc, sub);
-                    z = key < nkw ? zz : -INFINITY;
-                }
-                zs[st] = z;
-                mx = fmaxf(mx, z);
-            }
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 8));
-            mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 16));
-            const float m_new = fmaxf(m_run, mx);
-            const float alpha = exp2f(m_run - m_new);
-            float lsum = 0.f;
-#pragma unroll
-            for (int st = 0; st < C::STEPS; ++st) {
-                const float pz = exp2f(zs[st] - m_new);
-                if (st * 4 < nkw && primary) p_s[warp][st * 4 + kq][myhead] = pz;
-                lsum += pz;
-            }
-            l_run = l_run * alpha + (primary ? lsum : 0.f);
-            m_run = m_new;
-            if (primary && kq == 0) alpha_s[warp][myhead] = alpha;
-            __syncwarp();
-#pragma unroll
-            for (int j = 0; j < G; ++j) {
-                const float al = alpha_s[warp][j];
-#pragma unroll
-                for (int x = 0; x < C::PVD; ++x) o[j][x] *= al;
-            }
-#pragma unroll 4
-            for (int k = 0; k < nkw; ++k) {
-                float pv[G];
-#pragma unroll
-                for (int j = 0; j < G; ++j) pv[j] = p_s[warp][k][j];
-                float vf[C::PVD];
-                load_elems<ELEM, C::PVD>(sV + k * C::ROW + lane * C::PVD * ELEM, vf);
+                m_run = -INFINITY;
+                l_run = 0.f;
 #pragma unroll
                 for (int j = 0; j < G; ++j)
 #pragma unroll
-                    for (int x = 0; x < C::PVD; ++x) o[j][x] = fmaf(pv[j], vf[x], o[j][x]);
+                    for (int x = 0; x < C::PVD / 2; ++x) o[j][x] = make_float2(0.f, 0.f);
+                if (mt.flags & kCurrent) {
+                    if (warp == 0) {  // the current token seeds warp 0's softmax state
+                        float kc[C::PVD], vc[C::PVD];
+                        load_elems<ELEM, C::PVD>(st + C::KN_OFF + lane * C::PVD * ELEM, kc);
+                        load_elems<ELEM, C::PVD>(st + C::VN_OFF + lane * C::PVD * ELEM, vc);
+                        float zc[G];
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            float qf[C::PVD];
+                            load_elems<ELEM, C::PVD>(st + C::Q_OFF + j * C::ROW + lane * C::PVD * ELEM, qf);
+                            float acc = 0.f;
+#pragma unroll
+                            for (int x = 0; x < C::PVD; ++x) acc = fmaf(qf[x] * qscale, kc[x], acc);
+#pragma unroll
+                            for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
+                            zc[j] = acc;
+                        }
+                        m_run = zc[0];
+#pragma unroll
+                        for (int j = 1; j < G; ++j)
+                            if (myhead == j) m_run = zc[j];
+                        l_run = (primary && kq == 0) ? 1.f : 0.f;
+#pragma unroll
+                        for (int j = 0; j < G; ++j)
+#pragma unroll
+                            for (int x = 0; x < C::PVD / 2; ++x) o[j][x] = make_float2(vc[2 * x], vc[2 * x + 1]);
+                    }
+                    if (warp == kConsumers - 1) {  // append: slot r of both rings <- the new rows
+                        uint4* kd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.k_ring) +
+                                                             (head * a.B + mt.r) * C::ROW);
+                        uint4* vd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.v_ring) +
+                                                             (head * a.B + mt.r) * C::ROW);
+                        for (int x = lane; x < C::ROW / 16; x += 32) {
+                            kd[x] = *reinterpret_cast<const uint4*>(st + C::KN_OFF + x * 16);
+                            vd[x] = *reinterpret_cast<const uint4*>(st + C::VN_OFF + x * 16);
+                        }
+                    }
+                }
+            }
+
+            const int nkw = min(max(mt.nk - warp * C::KW, 0), C::KW);
+            if (nkw > 0) {
+                const unsigned char* sK = st + warp * C::KW * C::ROW;
+                const unsigned char* sV = st + (C::TK + warp * C::KW) * C::ROW;
+                float zs[C::STEPS];
+                float mx = -INFINITY;
+#pragma unroll
+                for (int stp = 0; stp < C::STEPS; ++stp) {
+                    const int key = stp * C::KPS + kq;
+                    float z = -INFINITY;
+                    if (stp * C::KPS < nkw) {  // warp-uniform
+                        float2 acc[G];
+#pragma unroll
+                        for (int j = 0; j < G; ++j) acc[j] = make_float2(0.f, 0.f);
+#pragma unroll
+                        for (int m = 0; m < C::VPL; ++m) {
+                            float kf[C::EPV];
+                            const uint4 u = *reinterpret_cast<const uint4*>(sK + key * C::ROW + (sub + C::KL * m) * 16);
+                            Elem<ELEM>::vec16(u, kf);
+#pragma unroll
+                            for (int x = 0; x < C::EPV / 2; ++x) {
+                                const float2 k2 = make_float2(kf[2 * x], kf[2 * x + 1]);
+#pragma unroll
+                                for (int j = 0; j < G; ++j)
+                                    acc[j] = __ffma2_rn(qr[j][m * (C::EPV / 2) + x], k2, acc[j]);
+                            }
+                        }
+                        float part[G];
+#pragma unroll
+                        for (int j = 0; j < G; ++j) part[j] = acc[j].x + acc[j].y;
+                        const float zz = reduce_scatter<G, C::KL>(part);
+                        z = key < nkw ? zz : -INFINITY;
+                    }
+                    zs[stp] = z;
+                    mx = fmaxf(mx, z);
+                }
+#pragma unroll
+                for (int off = C::KL; off < 32; off <<= 1) mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, off));
+                const float m_new = fmaxf(m_run, mx);
+                float lsum = 0.f;
+#pragma unroll
+                for (int stp = 0; stp < C::STEPS; ++stp) {
+                    const float pz = fast_exp2(zs[stp] - m_new);
+                    if (stp * C::KPS < nkw && primary) p_s[warp][stp * C::KPS + kq][myhead] = pz;
+                    lsum += pz;
+                }
+                // rescale only when some head's running max moved (rare once it settles)
+                const bool grew = m_new > m_run;
+                if (__any_sync(kFull, grew)) {
+                    const float alpha = fast_exp2(m_run - m_new);  // 2^-inf = 0 on the first keys
+                    l_run *= alpha;
+                    if (primary && kq == 0) alpha_s[warp][myhead] = alpha;
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < G; ++j) {
+                        const float al = alpha_s[warp][j];
+#pragma unroll
+                        for (int x = 0; x < C::PVD / 2; ++x) o[j][x] = __fmul2_rn(o[j][x], make_float2(al, al));
+                    }
+                }
+                l_run += primary ? lsum : 0.f;
+                m_run = m_new;
+                __syncwarp();
+#pragma unroll 4
+                for (int k = 0; k < nkw; ++k) {
+                    float vf[C::PVD];
+                    load_elems<ELEM, C::PVD>(sV + k * C::ROW + lane * C::PVD * ELEM, vf);
+                    float pv[G];
+#pragma unroll
+                    for (int j = 0; j < G; ++j) pv[j] = p_s[warp][k][j];
+#pragma unroll
+                    for (int j = 0; j < G; ++j)
+#pragma unroll
+                        for (int x = 0; x < C::PVD / 2; ++x)
+                            o[j][x] = __ffma2_rn(make_float2(pv[j], pv[j]), make_float2(vf[2 * x], vf[2 * x + 1]), o[j][x]);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty_bar[s]);
+            if (!(mt.flags & kLast)) continue;
+
+            // ---- end of the item: merge the consumer warps' states (Eq. lse)
+            {
+                float l = l_run;
+#pragma unroll
+                for (int off = C::KL; off < 32; off <<= 1) l += __shfl_xor_sync(kFull, l, off);
+#pragma unroll
+                for (int x = 1; x < (1 << C::REP); x <<= 1) l += __shfl_xor_sync(kFull, l, x);
+                if (lane == (myhead << C::REP)) ml_s[warp][myhead] = make_float2(m_run, l);
+            }
+#pragma unroll
+            for (int j = 0; j < G; ++j)
+#pragma unroll
+                for (int x = 0; x < C::PVD / 2; ++x)
+                    *reinterpret_cast<float2*>(&merge_o[(warp * G + j) * D + lane * C::PVD + 2 * x]) = o[j][x];
+            bool ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
+            const int ctid = tid;  // 0 .. 32*kConsumers-1
+            const size_t part = head * a.nchunk + mt.chunk;
+            if (ok) {
+                for (int e = ctid; e < G * D; e += kConsumers * 32) {
+                    const int j = e / D;
+                    float M = -INFINITY;
+#pragma unroll
+                    for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, ml_s[w][j].x);
+                    float L = 0.f, O = 0.f;
+#pragma unroll
+                    for (int w = 0; w < kConsumers; ++w) {
+                        const float sc = exp2f(ml_s[w][j].x - M);
+                        L = fmaf(ml_s[w][j].y, sc, L);
+                        O = fmaf(merge_o[(w * G) * D + e], sc, O);
+                    }
+                    if (mt.nch == 1) {
+                        a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
+                    } else {
+                        a.part_o[part * G * D + e] = O;
+                        if ((e % D) == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
+                    }
+                }
+            }
+            if (ok && mt.nch > 1) {
+                // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
+                __threadfence();
+                ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
+                if (ok && ctid == 0) last_s = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
+                ok = ok && consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
+                if (ok && last_s) {
+                    __threadfence();
+                    const float* po = a.part_o + head * a.nchunk * G * D;
+                    const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
+                    for (int e = ctid; e < G * D; e += kConsumers * 32) {
+                        const int j = e / D;
+                        float M = -INFINITY;
+                        for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+                        float L = 0.f, O = 0.f;
+                        for (int c = 0; c < mt.nch; ++c) {
+                            const float2 ml = __ldcg(&pml[c * G + j]);
+                            const float sc = exp2f(ml.x - M);
+                            L = fmaf(ml.y, sc, L);
+                            O = fmaf(__ldcg(po + c * G * D + e), sc, O);
+                        }
+                        a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
+                    }
+                    if (ctid == 0) a.counters[head] = 0;
+                }
+            }
+            ok = ok && consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);  // merge buffers free again
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+                break;
             }
         }
-        failed = __syncthreads_or(!ok) != 0;
-        if (failed) break;
-        if (tid == 0 && it + kStages < ntiles) {
-            fence_proxy_async();
-            issue(it + kStages);
-        }
     }
-    if (failed) {
+    __syncthreads();
+    if (abort_s) {
         if (tid == 0) {
-            atomicCAS(&g_status, kDevOk, kDevTimeout);
-            const int issued = min(ntiles, it + kStages);
-            for (int j = it; j < issued; ++j)
-                mbar_wait(&full_bar[j % kStages], static_cast<uint32_t>((j / kStages) & 1), 1000000000ull);
+            // wait (bounded) for the last copy issued into each stage
+            const int issued = issued_s;
+            for (int s = 0; s < kStages && s < issued; ++s) {
+                const int j = s + kStages * ((issued - 1 - s) / kStages);
+                mbar_wait(&full_bar[s], static_cast<uint32_t>((j / kStages) & 1), kGuardNs);
+            }
         }
         __syncthreads();
-        return;
     }
-
-    // ---- merge the warps' states (all copies have landed: the stages are free)
-    {
-        float l = l_run;
-        l += __shfl_xor_sync(kFull, l, 8);
-        l += __shfl_xor_sync(kFull, l, 16);
-#pragma unroll
-        for (int x = 1; x < (1 << C::REP); x <<= 1) l += __shfl_xor_sync(kFull, l, x);
-        if (lane == (myhead << C::REP)) ml_s[warp][myhead] = make_float2(m_run, l);
-    }
-    float* o_s = reinterpret_cast<float*>(dsmem);  // [kWarps][G][D]
-#pragma unroll
-    for (int j = 0; j < G; ++j)
-#pragma unroll
-        for (int x = 0; x < C::PVD; ++x) o_s[(warp * G + j) * D + lane * C::PVD + x] = o[j][x];
-    __syncthreads();
-
-    const size_t part = head * a.nchunk + chunk;
-    for (int e = tid; e < G * D; e += kThreads) {
-        const int j = e / D;
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, ml_s[w][j].x);
-        float L = 0.f, O = 0.f;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
-            const float sc = exp2f(ml_s[w][j].x - M);
-            L = fmaf(ml_s[w][j].y, sc, L);
-            O = fmaf(o_s[(w * G) * D + e], sc, O);
-        }
-        if (nch == 1) {
-            a.out[(static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * D + e] = O / L;
-        } else {
-            a.part_o[part * G * D + e] = O;
-            if ((e % D) == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
+    if (tid == 0) {  // the last CTA to finish resets the work queue for the next launch
+        __threadfence();
+        if (atomicAdd(a.ctl + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+            atomicExch(a.ctl, 0);
+            atomicExch(a.ctl + 1, 0);
         }
     }
-    if (nch == 1) return;
-
-    // ---- split combine (Eq. lse): the last CTA of this (sequence, KV head) fuses all partials
-    __threadfence();
-    __syncthreads();
-    if (tid == 0) last_s = (atomicAdd(a.counters + head, 1) == nch - 1);
-    __syncthreads();
-    if (!last_s) return;
-    __threadfence();
-    const float* po = a.part_o + head * a.nchunk * G * D;
-    const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
-    for (int e = tid; e < G * D; e += kThreads) {
-        const int j = e / D;
-        float M = -INFINITY;
-        for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
-        float L = 0.f, O = 0.f;
-        for (int c = 0; c < nch; ++c) {
-            const float2 ml = __ldcg(&pml[c * G + j]);
-            const float sc = exp2f(ml.x - M);
-            L = fmaf(ml.y, sc, L);
-            O = fmaf(__ldcg(po + c * G * D + e), sc, O);
-        }
-        a.out[(static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * D + e] = O / L;
-    }
-    if (tid == 0) a.counters[head] = 0;
 }
 
 // --------------------------------------------------- prefill / advance ----
@@ -606,12 +824,35 @@ cudaError_t ensure_smem_attr()
 }
 
 template <int ELEM, int D, int G>
+int occupancy_t()
+{
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 0;
+    if (ensure_smem_attr<ELEM, D, G>() != cudaSuccess) return 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<ELEM, D, G>, kThreads,
+                                                      Cfg<ELEM, D, G>::SMEM) != cudaSuccess)
+        return 0;
+    if (dev < 64) cache[dev] = n;
+    return n;
+}
+
+template <int ELEM, int D, int G>
 cudaError_t launch_t(const DecodeArgs& a, cudaStream_t stream)
 {
     using C = Cfg<ELEM, D, G>;
     cudaError_t err = ensure_smem_attr<ELEM, D, G>();
     if (err != cudaSuccess) return err;
-    const dim3 grid(a.nchunk, a.Hkv, a.batch);
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    int per_sm = occupancy_t<ELEM, D, G>();
+    if (per_sm < 1) per_sm = 1;
+    const long long ctas = static_cast<long long>(sms) * per_sm;
+    const int grid = static_cast<int>(a.total_items < ctas ? a.total_items : ctas);
+    if (grid < 1) return cudaSuccess;
     decode_kernel<ELEM, D, G><<<grid, kThreads, C::SMEM, stream>>>(a);
     return cudaGetLastError();
 }
@@ -628,22 +869,6 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t stream)
     }
 }
 
-template <int ELEM, int D, int G>
-int occupancy_t()
-{
-    static int cache[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev < 64 && cache[dev] > 0) return cache[dev];
-    int n = 0;
-    if (ensure_smem_attr<ELEM, D, G>() != cudaSuccess) return 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<ELEM, D, G>, kThreads,
-                                                      Cfg<ELEM, D, G>::SMEM) != cudaSuccess)
-        return 0;
-    if (dev < 64) cache[dev] = n;
-    return n;
-}
-
 template <int ELEM, int D>
 int occupancy_g(int group)
 {
@@ -656,9 +881,28 @@ int occupancy_g(int group)
     }
 }
 
+template <int ELEM, int D>
+int tile_g(int group)
+{
+    switch (group) {
+        case 1: return Cfg<ELEM, D, 1>::TK;
+        case 2: return Cfg<ELEM, D, 2>::TK;
+        case 4: return Cfg<ELEM, D, 4>::TK;
+        case 8: return Cfg<ELEM, D, 8>::TK;
+        default: return 0;
+    }
+}
+
 }  // namespace
 
-int tile_keys(int elem_bytes, int d) { return kTileBytes / (elem_bytes * d); }
+int tile_keys(int elem_bytes, int d, int group)
+{
+    if (elem_bytes == 2 && d == 64) return tile_g<2, 64>(group);
+    if (elem_bytes == 2 && d == 128) return tile_g<2, 128>(group);
+    if (elem_bytes == 4 && d == 64) return tile_g<4, 64>(group);
+    if (elem_bytes == 4 && d == 128) return tile_g<4, 128>(group);
+    return 0;
+}
 
 int decode_ctas_per_sm(int elem_bytes, int d, int group)
 {

@@ -21,20 +21,23 @@ struct DecodeArgs {
     float* out;          // [batch][Hq][d]
     float* part_o;       // [batch][Hkv][nchunk][G][d]   split partials (unnormalised output)
     float* part_ml;      // [batch][Hkv][nchunk][G][2]   split partials (max, sum), log2 domain
-    int* counters;       // [batch][Hkv]                 arrivals per (sequence, KV head)
+    int* counters;       // [batch][Hkv]                 finished chunks per (sequence, KV head)
+    int* ctl;            // [2] work-queue head and finished CTAs; zero between launches
     int batch, Hq, Hkv, d, B;
-    int chunk;           // keys of the support per CTA (multiple of the tile)
-    int nchunk;          // CTAs per (sequence, KV head) in the grid = ceil((B-1)/chunk)
+    int chunk;           // ring keys of the support per work item (a multiple of the tile)
+    int nchunk;          // work items per (sequence, KV head) = ceil((B-1)/chunk)
+    int total_items;     // batch * Hkv * nchunk
     unsigned long long timeout_ns;
 };
 
 // Keys per shared-memory tile of a kernel instance (rows of K and of V).
-int tile_keys(int elem_bytes, int d);
+int tile_keys(int elem_bytes, int d, int group);
 
 // Resident CTAs per SM of the decode kernel for this instance (0 if unsupported).
 int decode_ctas_per_sm(int elem_bytes, int d, int group);
 
-// Launch the fused append + split attention + combine kernel. elem_bytes: 2 (bf16) or 4 (fp32).
+// Launch the fused append + attention + combine kernel (persistent grid of at
+// most SMs x resident CTAs). elem_bytes: 2 (bf16) or 4 (fp32).
 cudaError_t launch_decode(const DecodeArgs& a, int elem_bytes, cudaStream_t stream);
 
 cudaError_t launch_prefill(const void* k_hist, const void* v_hist, const int32_t* pos, void* k_ring,

@@ -29,10 +29,11 @@
 namespace {
 
 constexpr size_t kNoallocScratchBytes = PBB_NOALLOC_SCRATCH_BYTES;
-constexpr size_t kCounterBytes = 256 * 1024;  // arrival counters: up to 65,536 (sequence, KV head) pairs
+constexpr size_t kCounterBytes = 256 * 1024;  // queue words and counters: up to 65,534 (sequence, KV head) pairs
 constexpr int kMaxDevices = 64;
 
-// Split scratch: [0, kCounterBytes) counters, then split partials.
+// Scratch: [0, kCounterBytes) the work-queue words and the per-(sequence, KV
+// head) counters, then the split partials.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
 std::mutex g_setup_mutex;
@@ -99,22 +100,24 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     if (a.nchunk > 65535) return PBB_ERR_UNSUPPORTED;
     a.timeout_ns = 1000000000ull;
 
+    const size_t pairs = static_cast<size_t>(batch) * Hkv;
+    const size_t parts = a.nchunk > 1 ? pairs * a.nchunk * group : 0;
+    const size_t o_bytes = round_up(parts * d * sizeof(float), 256);
+    const size_t need = kCounterBytes + o_bytes + parts * 2 * sizeof(float);
+    if ((pairs + 2) * sizeof(int) > kCounterBytes || need > kNoallocScratchBytes)
+        return PBB_ERR_SCRATCH_LIMIT;
+    a.total_items = static_cast<int>(pairs * a.nchunk);
+    unsigned char* base = nullptr;
+    const int rc = scratch_address(dev, &base);
+    if (rc != PBB_OK) return rc;
+    a.ctl = reinterpret_cast<int*>(base);
+    a.counters = reinterpret_cast<int*>(base) + 2;
     if (a.nchunk > 1) {
-        const size_t pairs = static_cast<size_t>(batch) * Hkv;
-        const size_t parts = pairs * a.nchunk * group;
-        const size_t o_bytes = round_up(parts * d * sizeof(float), 256);
-        const size_t need = kCounterBytes + o_bytes + parts * 2 * sizeof(float);
-        if (pairs * sizeof(int) > kCounterBytes || need > kNoallocScratchBytes)
-            return PBB_ERR_SCRATCH_LIMIT;
-        unsigned char* base = nullptr;
-        const int rc = scratch_address(dev, &base);
-        if (rc != PBB_OK) return rc;
-        a.counters = reinterpret_cast<int*>(base);
         a.part_o = reinterpret_cast<float*>(base + kCounterBytes);
         a.part_ml = reinterpret_cast<float*>(base + kCounterBytes + o_bytes);
-        // The array keeps whatever the previous call left: the counters must start at zero.
-        if (cudaMemsetAsync(a.counters, 0, pairs * sizeof(int), stream) != cudaSuccess)
-            return PBB_ERR_CUDA;
     }
+    // The array keeps whatever the previous call left: the queue words and the
+    // counters must start at zero.
+    if (cudaMemsetAsync(a.ctl, 0, (pairs + 2) * sizeof(int), stream) != cudaSuccess) return PBB_ERR_CUDA;
     return pbb::launch_decode(a, 2, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
