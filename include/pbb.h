@@ -171,7 +171,7 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
  * in a fixed array of PBB_NOALLOC_SCRATCH_BYTES compiled into the library;
  * every GPU that loads the library holds that array until the process exits.
  * The call never allocates or frees memory. A step whose split needs more than
- * the array holds (more than 65,536 (sequence, KV head) pairs, or partials
+ * the array holds (more than 65,534 (sequence, KV head) pairs, or partials
  * beyond the rest of the array) returns PBB_ERR_SCRATCH_LIMIT without
  * launching; pbb_decode_step handles those shapes. Bounded waits use the
  * default limit of one second (pbb_set_wait_timeout_ns does not apply here).
