@@ -74,10 +74,12 @@ int sm_count(int dev)
     return g_sms[dev];
 }
 
-// Keys of the support per CTA. The support of a (sequence, KV head) has at
-// most B-1 ring keys besides the current token. Without an override the plan
-// splits it only as far as needed for the grid to fill the GPU several times
-// over (at least kWaves waves of resident CTAs); large batches run unsplit.
+// Ring keys of the support per work item. The support of a (sequence, KV
+// head) has at most B-1 ring keys besides the current token. Without an
+// override the plan splits it only as far as needed for the items to fill the
+// GPU several times over (kWaves waves of resident CTAs), and never into
+// chunks of less than kMinChunkBytes of K+V, below which the combine would cost
+// more than the parallel streaming saves; large batches run unsplit.
 int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
 {
     const int tile = pbb::tile_keys(elem, d, group);
@@ -88,12 +90,15 @@ int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
         chunk = over;
     } else {
         constexpr int kWaves = 4;
+        constexpr int kMinChunkBytes = 64 * 1024;
         const long long pairs = static_cast<long long>(batch) * Hkv;
         int per_sm = pbb::decode_ctas_per_sm(elem, d, group);
         if (per_sm <= 0) per_sm = 1;
         const long long want = static_cast<long long>(kWaves) * sm_count(dev) * per_sm;
         long long split = pairs > 0 ? (want + pairs - 1) / pairs : 1;
-        const long long max_split = (max_keys + tile - 1) / tile;
+        int min_keys = kMinChunkBytes / (2 * d * elem);
+        if (min_keys < tile) min_keys = tile;
+        const long long max_split = (max_keys + min_keys - 1) / min_keys;
         if (split > max_split) split = max_split;
         if (split < 1) split = 1;
         chunk = static_cast<int>((max_keys + split - 1) / split);

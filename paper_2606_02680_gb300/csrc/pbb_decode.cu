@@ -409,9 +409,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
         if (lane == 0) {
             int seq = 0;  // tiles issued so far (stage seq % kStages)
             bool ok = true;
-            while (ok) {
-                const int item = atomicAdd(a.ctl, 1);
-                if (item >= a.total_items) break;
+            // the first item of a CTA is its index (no queue round trip before the first
+            // tile); later ones come from the queue, which hands out items grid, grid+1, ...
+            for (int item = blockIdx.x; ok && item < a.total_items;
+                 item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
                 const int chunk = item % a.nchunk;
                 const int pair = item / a.nchunk;
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
@@ -728,18 +729,53 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     __threadfence();
                     const float* po = a.part_o + head * a.nchunk * G * D;
                     const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
-                    for (int e = ctid; e < G * D; e += kConsumers * 32) {
-                        const int j = e / D;
-                        float M = -INFINITY;
-                        for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
-                        float L = 0.f, O = 0.f;
-                        for (int c = 0; c < mt.nch; ++c) {
-                            const float2 ml = __ldcg(&pml[c * G + j]);
-                            const float sc = exp2f(ml.x - M);
-                            L = fmaf(ml.y, sc, L);
-                            O = fmaf(__ldcg(po + c * G * D + e), sc, O);
+                    float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D;
+                    if (mt.nch <= kConsumers * D) {
+                        // weight of every (chunk, head) in shared memory: e^(m_c - M) / L, with M and
+                        // L reduced across the chunks by one warp per head
+                        float* wgt = merge_o;  // [nch][G], free after the barrier above
+                        for (int j = warp; j < G; j += kConsumers) {
+                            float M = -INFINITY;
+                            for (int c = lane; c < mt.nch; c += 32) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+#pragma unroll
+                            for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
+                            float L = 0.f;
+                            for (int c = lane; c < mt.nch; c += 32) {
+                                const float2 ml = __ldcg(&pml[c * G + j]);
+                                const float e = fast_exp2(ml.x - M);
+                                wgt[c * G + j] = e;
+                                L = fmaf(ml.y, e, L);
+                            }
+#pragma unroll
+                            for (int off = 16; off >= 1; off >>= 1) L += __shfl_xor_sync(kFull, L, off);
+                            const float inv = 1.f / L;
+                            __syncwarp();
+                            for (int c = lane; c < mt.nch; c += 32) wgt[c * G + j] *= inv;
                         }
-                        a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
+                        ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
+                        if (ok) {
+                            for (int e = ctid; e < G * D; e += kConsumers * 32) {
+                                const int j = e / D;
+                                float O = 0.f;
+#pragma unroll 8
+                                for (int c = 0; c < mt.nch; ++c) O = fmaf(__ldcg(po + c * G * D + e), wgt[c * G + j], O);
+                                out_g[e] = O;
+                            }
+                        }
+                    } else {
+                        for (int e = ctid; e < G * D; e += kConsumers * 32) {
+                            const int j = e / D;
+                            float M = -INFINITY;
+                            for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+                            float L = 0.f, O = 0.f;
+                            for (int c = 0; c < mt.nch; ++c) {
+                                const float2 ml = __ldcg(&pml[c * G + j]);
+                                const float sc = fast_exp2(ml.x - M);
+                                L = fmaf(ml.y, sc, L);
+                                O = fmaf(__ldcg(po + c * G * D + e), sc, O);
+                            }
+                            out_g[e] = O / L;
+                        }
                     }
                     if (ctid == 0) a.counters[head] = 0;
                 }
