@@ -474,7 +474,10 @@ def run_ours(args):
             "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
-                         "kernel": "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group),
+                         "kernel": ("decode_kernel_tc<%d>" % w.d
+                                    if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w))
+                                    == "tensor_cores" else
+                                    "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group)),
                          "peak_kind": peak_kind,
                          "algorithmic_bytes_per_launch": res["launch_bytes_mean"],
                          "kernel_ms_mean": res["kernel_ms_mean"],

@@ -160,6 +160,15 @@ int pbb_set_chunk_keys(int keys);
 int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
 
 /*
+ * Which kernel a decode step of this shape runs on the current device:
+ * PBB_KERNEL_CUDA_CORES (packed fp32 FMAs; every shape) or PBB_KERNEL_TENSOR_CORES
+ * (bf16 with Hq/Hkv = 8, where the scores of a 16-key block against the 8 query
+ * heads form a dense mma tile; needs B a multiple of 64). Negative on error.
+ */
+enum { PBB_KERNEL_CUDA_CORES = 0, PBB_KERNEL_TENSOR_CORES = 1 };
+int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
  * No counterpart in the paper: a library-usage variant for callers that cannot
  * allocate device memory while they decode (a runtime that owns all of HBM
  * through its own pool and forbids other allocations, code inside a CUDA

@@ -29,7 +29,7 @@ __all__ = [
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
     "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step",
     "decode_step_host", "advance_positions", "get_device_status", "reserve_workspace",
-    "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "error_string", "EXPORTS",
+    "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
 
 PBB_OK = 0
@@ -60,6 +60,7 @@ EXPORTS = {
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),
     "pbb_set_chunk_keys": (_I, [_I]),
     "pbb_plan_chunk_keys": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_plan_kernel": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_error_string": (ctypes.c_char_p, [_I]),
 }
 
@@ -278,3 +279,15 @@ def set_chunk_keys(keys: int) -> int:
 
 def plan_chunk_keys(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> int:
     return int(lib().pbb_plan_chunk_keys(batch, Hq, Hkv, d, B, _dt(dtype)))
+
+
+PBB_KERNEL_CUDA_CORES = 0
+PBB_KERNEL_TENSOR_CORES = 1
+
+
+def plan_kernel(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> str:
+    """'cuda_cores' or 'tensor_cores': the kernel a step of this shape runs."""
+    rc = int(lib().pbb_plan_kernel(batch, Hq, Hkv, d, B, _dt(dtype)))
+    if rc < 0:
+        raise PbbError(rc, "pbb_plan_kernel")
+    return "tensor_cores" if rc == PBB_KERNEL_TENSOR_CORES else "cuda_cores"

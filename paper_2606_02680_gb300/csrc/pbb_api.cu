@@ -360,6 +360,25 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
     return plan_chunk(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, dev);
 }
 
+int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
+{
+    int rc = check_shape(batch, Hkv, d, B, dtype);
+    if (rc != PBB_OK) return rc;
+    rc = check_group(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    pbb::DecodeArgs a{};
+    a.batch = batch;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.d = d;
+    a.B = B;
+    a.chunk = plan_chunk(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, dev);
+    return pbb::use_tensor_cores(a, elem_size(dtype)) ? PBB_KERNEL_TENSOR_CORES : PBB_KERNEL_CUDA_CORES;
+}
+
 const char* pbb_error_string(int code)
 {
     switch (code) {

@@ -47,8 +47,10 @@
 // No wait can hang: waits on mbarriers and the consumers' software barrier are
 // bounded by the global timer. A wait that runs out records kDevTimeout; the
 // CTA then stops, waits (bounded) for the copies it issued and returns.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
+#include <cudaTypedefs.h>
 #include <stdint.h>
 
 #include "pbb_internal.h"
@@ -180,6 +182,58 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
         : "memory");
 }
 
+// 2-D tiled TMA load of one box at (x = column, y = row) of a tensor map, completion on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
+            "r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(addr));
+}
+
+// Transpose of an 8x8 b16 matrix held in the m8n8 fragment layout.
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x)
+{
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
+}
+
+// d += a (16x16, row) * b (16x8, col), bf16 inputs, fp32 accumulation.
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
+{
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// Two floats -> bf16x2 (round to nearest even): lo in the low half, hi in the high half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
 // ---------------------------------------------------------- elements ----
 
 template <int ELEM>
@@ -301,6 +355,7 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar)
 // Barrier of the consumer warps through a shared-memory counter, bounded by
 // `limit_ns` (a hardware named barrier could not be bounded). All lanes of all
 // consumer warps call it; returns false if it gave up.
+template <int NC>
 __device__ __forceinline__ bool consumer_barrier(unsigned* count, volatile unsigned* gen, int lane,
                                                  unsigned long long limit_ns)
 {
@@ -309,7 +364,7 @@ __device__ __forceinline__ bool consumer_barrier(unsigned* count, volatile unsig
     if (lane == 0) {
         const unsigned g = *gen;
         __threadfence_block();
-        if (atomicAdd(count, 1u) == kConsumers - 1) {
+        if (atomicAdd(count, 1u) == NC - 1) {
             *count = 0;
             __threadfence_block();
             *gen = g + 1;
@@ -369,6 +424,107 @@ struct Cfg {
     static_assert(REP >= 0, "group larger than the lanes of a key");
     static_assert(SMEM <= BUDGET, "shared memory budget (dynamic; the static part is a few KiB)");
 };
+
+// ----------------------------------------------------------- item end ----
+
+// End of a work item, run by all consumer threads: merge the consumer warps'
+// (max, sum, output) states of the item (Eq. lse) from ml_s [NC][G] and
+// merge_o [NC][G][D]; write `out` for an unsplit support, else the item's
+// partial, and let the last item of the (sequence, KV head) to finish fuse all
+// partials in chunk order. Returns false if a bounded barrier gave up.
+template <int G, int D, int NC>
+__device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta& mt, size_t head, const float2* ml_s,
+                                         float* merge_o, unsigned* sbar_count, volatile unsigned* sbar_gen,
+                                         int* last_s, int tid, int lane, int warp)
+{
+    bool ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
+    const int ctid = tid;  // 0 .. 32*NC-1 (consumer threads)
+    const size_t part = head * a.nchunk + mt.chunk;
+    if (ok) {
+        for (int e = ctid; e < G * D; e += NC * 32) {
+            const int j = e / D;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < NC; ++w) M = fmaxf(M, ml_s[w * G + j].x);
+            float L = 0.f, O = 0.f;
+#pragma unroll
+            for (int w = 0; w < NC; ++w) {
+                const float sc = exp2f(ml_s[w * G + j].x - M);
+                L = fmaf(ml_s[w * G + j].y, sc, L);
+                O = fmaf(merge_o[(w * G) * D + e], sc, O);
+            }
+            if (mt.nch == 1) {
+                a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
+            } else {
+                a.part_o[part * G * D + e] = O;
+                if ((e % D) == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
+            }
+        }
+    }
+    if (ok && mt.nch > 1) {
+        // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
+        __threadfence();
+        ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
+        if (ok && ctid == 0) *last_s = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
+        ok = ok && consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
+        if (ok && *last_s) {
+            __threadfence();
+            const float* po = a.part_o + head * a.nchunk * G * D;
+            const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
+            float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D;
+            if (mt.nch <= NC * D) {
+                // weight of every (chunk, head) in shared memory: e^(m_c - M) / L, with M and
+                // L reduced across the chunks by one warp per head
+                float* wgt = merge_o;  // [nch][G], free after the barrier above
+                for (int j = warp; j < G; j += NC) {
+                    float M = -INFINITY;
+                    for (int c = lane; c < mt.nch; c += 32) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+#pragma unroll
+                    for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
+                    float L = 0.f;
+                    for (int c = lane; c < mt.nch; c += 32) {
+                        const float2 ml = __ldcg(&pml[c * G + j]);
+                        const float e = fast_exp2(ml.x - M);
+                        wgt[c * G + j] = e;
+                        L = fmaf(ml.y, e, L);
+                    }
+#pragma unroll
+                    for (int off = 16; off >= 1; off >>= 1) L += __shfl_xor_sync(kFull, L, off);
+                    const float inv = 1.f / L;
+                    __syncwarp();
+                    for (int c = lane; c < mt.nch; c += 32) wgt[c * G + j] *= inv;
+                }
+                ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
+                if (ok) {
+                    for (int e = ctid; e < G * D; e += NC * 32) {
+                        const int j = e / D;
+                        float O = 0.f;
+#pragma unroll 8
+                        for (int c = 0; c < mt.nch; ++c) O = fmaf(__ldcg(po + c * G * D + e), wgt[c * G + j], O);
+                        out_g[e] = O;
+                    }
+                }
+            } else {
+                for (int e = ctid; e < G * D; e += NC * 32) {
+                    const int j = e / D;
+                    float M = -INFINITY;
+                    for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+                    float L = 0.f, O = 0.f;
+                    for (int c = 0; c < mt.nch; ++c) {
+                        const float2 ml = __ldcg(&pml[c * G + j]);
+                        const float sc = fast_exp2(ml.x - M);
+                        L = fmaf(ml.y, sc, L);
+                        O = fmaf(__ldcg(po + c * G * D + e), sc, O);
+                    }
+                    out_g[e] = O / L;
+                }
+            }
+            if (ctid == 0) a.counters[head] = 0;
+        }
+    }
+    ok = ok && consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);  // merge buffers free again
+    return ok;
+}
 
 // ------------------------------------------------------------ kernel ----
 
@@ -695,92 +851,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
 #pragma unroll
                 for (int x = 0; x < C::PVD / 2; ++x)
                     *reinterpret_cast<float2*>(&merge_o[(warp * G + j) * D + lane * C::PVD + 2 * x]) = o[j][x];
-            bool ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
-            const int ctid = tid;  // 0 .. 32*kConsumers-1
-            const size_t part = head * a.nchunk + mt.chunk;
-            if (ok) {
-                for (int e = ctid; e < G * D; e += kConsumers * 32) {
-                    const int j = e / D;
-                    float M = -INFINITY;
-#pragma unroll
-                    for (int w = 0; w < kConsumers; ++w) M = fmaxf(M, ml_s[w][j].x);
-                    float L = 0.f, O = 0.f;
-#pragma unroll
-                    for (int w = 0; w < kConsumers; ++w) {
-                        const float sc = exp2f(ml_s[w][j].x - M);
-                        L = fmaf(ml_s[w][j].y, sc, L);
-                        O = fmaf(merge_o[(w * G) * D + e], sc, O);
-                    }
-                    if (mt.nch == 1) {
-                        a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
-                    } else {
-                        a.part_o[part * G * D + e] = O;
-                        if ((e % D) == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
-                    }
-                }
-            }
-            if (ok && mt.nch > 1) {
-                // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
-                __threadfence();
-                ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
-                if (ok && ctid == 0) last_s = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
-                ok = ok && consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
-                if (ok && last_s) {
-                    __threadfence();
-                    const float* po = a.part_o + head * a.nchunk * G * D;
-                    const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
-                    float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D;
-                    if (mt.nch <= kConsumers * D) {
-                        // weight of every (chunk, head) in shared memory: e^(m_c - M) / L, with M and
-                        // L reduced across the chunks by one warp per head
-                        float* wgt = merge_o;  // [nch][G], free after the barrier above
-                        for (int j = warp; j < G; j += kConsumers) {
-                            float M = -INFINITY;
-                            for (int c = lane; c < mt.nch; c += 32) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
-#pragma unroll
-                            for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
-                            float L = 0.f;
-                            for (int c = lane; c < mt.nch; c += 32) {
-                                const float2 ml = __ldcg(&pml[c * G + j]);
-                                const float e = fast_exp2(ml.x - M);
-                                wgt[c * G + j] = e;
-                                L = fmaf(ml.y, e, L);
-                            }
-#pragma unroll
-                            for (int off = 16; off >= 1; off >>= 1) L += __shfl_xor_sync(kFull, L, off);
-                            const float inv = 1.f / L;
-                            __syncwarp();
-                            for (int c = lane; c < mt.nch; c += 32) wgt[c * G + j] *= inv;
-                        }
-                        ok = consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);
-                        if (ok) {
-                            for (int e = ctid; e < G * D; e += kConsumers * 32) {
-                                const int j = e / D;
-                                float O = 0.f;
-#pragma unroll 8
-                                for (int c = 0; c < mt.nch; ++c) O = fmaf(__ldcg(po + c * G * D + e), wgt[c * G + j], O);
-                                out_g[e] = O;
-                            }
-                        }
-                    } else {
-                        for (int e = ctid; e < G * D; e += kConsumers * 32) {
-                            const int j = e / D;
-                            float M = -INFINITY;
-                            for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
-                            float L = 0.f, O = 0.f;
-                            for (int c = 0; c < mt.nch; ++c) {
-                                const float2 ml = __ldcg(&pml[c * G + j]);
-                                const float sc = fast_exp2(ml.x - M);
-                                L = fmaf(ml.y, sc, L);
-                                O = fmaf(__ldcg(po + c * G * D + e), sc, O);
-                            }
-                            out_g[e] = O / L;
-                        }
-                    }
-                    if (ctid == 0) a.counters[head] = 0;
-                }
-            }
-            ok = ok && consumer_barrier(&sbar_count, &sbar_gen, lane, kGuardNs);  // merge buffers free again
+            bool ok = finish_item<G, D, kConsumers>(a, mt, head, &ml_s[0][0], merge_o, &sbar_count, &sbar_gen,
+                                                    &last_s, tid, lane, warp);
             if (!ok) {
                 abort_s = 1;
                 atomicCAS(&g_status, kDevOk, kDevTimeout);
@@ -796,6 +868,410 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
             for (int s = 0; s < kStages && s < issued; ++s) {
                 const int j = s + kStages * ((issued - 1 - s) / kStages);
                 mbar_wait(&full_bar[s], static_cast<uint32_t>((j / kStages) & 1), kGuardNs);
+            }
+        }
+        __syncthreads();
+    }
+    if (tid == 0) {  // the last CTA to finish resets the work queue for the next launch
+        __threadfence();
+        if (atomicAdd(a.ctl + 1, 1) == static_cast<int>(gridDim.x) - 1) {
+            atomicExch(a.ctl, 0);
+            atomicExch(a.ctl + 1, 0);
+        }
+    }
+}
+
+// ------------------------------------------------- tensor-core kernel ----
+//
+// GQA group 8 makes the score product a dense tile: for a block of 16 keys,
+// S^T [16 keys x 8 heads] = K [16 x d] . Q^T [d x 8] is an mma.m16n8k16 chain
+// over d, and the output O^T [d x 8 heads] += V^T [d x 16 keys] . P^T
+// [16 keys x 8 heads] is one mma per 16 output dims. This kernel serves
+// bf16, G = 8 and block sizes that are multiples of twice the tile, so that no
+// tile straddles the end of a ring. It keeps the persistent producer /
+// consumer structure, work queue, merge and combine of decode_kernel; what
+// changes is how a consumer warp handles its 16 keys of a tile:
+//   - K and V tiles arrive by 2-D TMA copies with the 128-byte swizzle, one
+//     box per 64 columns, so ldmatrix reads them without bank conflicts;
+//   - A operands come from ldmatrix (K) and ldmatrix.trans (V^T), the Q^T
+//     operand from registers loaded once per item;
+//   - the scores (fp32) go through the same online softmax; the weights P are
+//     split into a bf16 high part and a bf16 low part (p = hi + lo to about
+//     2^-16) and both are multiplied, so P.V keeps fp32-level accuracy; the
+//     C fragment of S^T becomes the B fragment of P^T by an 8x8 movmatrix
+//     transpose.
+#ifndef PBB_TC_CONSUMER_WARPS
+#define PBB_TC_CONSUMER_WARPS 2
+#endif
+#ifndef PBB_TC_STAGES
+#define PBB_TC_STAGES 3
+#endif
+#ifndef PBB_TC_MIN_CTAS
+#define PBB_TC_MIN_CTAS 3
+#endif
+constexpr int kTcConsumers = PBB_TC_CONSUMER_WARPS;
+constexpr int kTcThreads = (kTcConsumers + 1) * 32;
+constexpr int kTcStages = PBB_TC_STAGES;
+
+template <int D>
+struct TcCfg {
+    static constexpr int G = 8;
+    static constexpr int ROW = D * 2;                      // bf16 row bytes
+    static constexpr int BOXES = D / 64;                   // 64-column (128-byte) boxes per row
+    static constexpr int TK = 16 * kTcConsumers;           // keys per tile: one m16 block per warp
+    static constexpr int BOX_BYTES = TK * 128;             // one swizzled [TK rows x 128 B] box
+    static constexpr int K_OFF = 0;
+    static constexpr int V_OFF = BOXES * BOX_BYTES;
+    static constexpr int Q_OFF = 2 * BOXES * BOX_BYTES;    // the item's 8 query rows (plain)
+    static constexpr int KN_OFF = Q_OFF + G * ROW;         // k_new row (chunk 0)
+    static constexpr int VN_OFF = KN_OFF + ROW;            // v_new row (chunk 0)
+    static constexpr int STAGE = (VN_OFF + ROW + 1023) / 1024 * 1024;  // boxes stay 1024-aligned
+    static constexpr int MERGE = kTcConsumers * G * D * 4;
+    static constexpr int SMEM = kTcStages * STAGE + MERGE + 1024;      // + alignment slack
+    static constexpr int KSTEPS = D / 16;                  // k-steps of the score chain
+    static constexpr int MTILES = D / 16;                  // 16-dim tiles of the output
+    static constexpr int PVD = D / 32;                     // dims per lane for the current token
+    static_assert(BOX_BYTES % 1024 == 0, "swizzle atoms");
+};
+
+// Byte offset of 16-byte chunk `c` (0..7) of row `r` in a box written with the 128-byte swizzle.
+__device__ __forceinline__ uint32_t swz(int r, int c) { return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4)); }
+
+template <int D>
+__global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
+    decode_kernel_tc(const DecodeArgs a, const __grid_constant__ CUtensorMap kmap,
+                     const __grid_constant__ CUtensorMap vmap)
+{
+    using C = TcCfg<D>;
+    constexpr int G = C::G;
+    extern __shared__ unsigned char dsmem_raw[];
+    __shared__ __align__(8) uint64_t full_bar[kTcStages];
+    __shared__ __align__(8) uint64_t empty_bar[kTcStages];
+    __shared__ TileMeta meta_s[kTcStages];
+    __shared__ float2 ml_s[kTcConsumers][G];
+    __shared__ unsigned sbar_count;
+    __shared__ volatile unsigned sbar_gen;
+    __shared__ volatile int abort_s;
+    __shared__ int last_s;
+    __shared__ int issued_s;
+    unsigned char* dsmem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) {
+#pragma unroll
+        for (int s = 0; s < kTcStages; ++s) {
+            mbar_init(&full_bar[s], 1);
+            mbar_init(&empty_bar[s], kTcConsumers);
+        }
+        fence_mbar_init();
+        sbar_count = 0;
+        sbar_gen = 0;
+        abort_s = 0;
+        issued_s = 0;
+    }
+    __syncthreads();
+
+    if (warp == kTcConsumers) {
+        // ================= producer: one lane =================
+        if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&kmap)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
+            int seq = 0;
+            bool ok = true;
+            for (int item = blockIdx.x; ok && item < a.total_items;
+                 item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
+                const int chunk = item % a.nchunk;
+                const int pair = item / a.nchunk;
+                const int kvh = pair % a.Hkv, b = pair / a.Hkv;
+                const int t = __ldg(a.pos + b);
+                if (t < 0) {
+                    if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
+                    continue;
+                }
+                const int B = a.B, h = B >> 1;
+                const int blk = t / B;
+                const int r = t - blk * B;
+                const bool bridge = (blk > 0) && (r < h);
+                const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
+                const int base = bridge ? h : 0;   // slot of ring key 0
+                const int nch = n > 0 ? (n + a.chunk - 1) / a.chunk : 1;
+                if (chunk >= nch) continue;
+                const int i0 = chunk * a.chunk;
+                const int i1 = min(i0 + a.chunk, n);
+                const int nkeys = max(i1 - i0, 0);
+                const int ntiles = nkeys > 0 ? (nkeys + C::TK - 1) / C::TK : 1;
+                const int head = b * a.Hkv + kvh;
+                for (int it = 0; it < ntiles; ++it, ++seq) {
+                    const int s = seq % kTcStages;
+                    if (seq >= kTcStages &&
+                        !mbar_wait(&empty_bar[s], static_cast<uint32_t>((seq / kTcStages - 1) & 1), kGuardNs)) {
+                        ok = false;
+                        break;
+                    }
+                    if (abort_s) {
+                        ok = false;
+                        break;
+                    }
+                    const int k0 = i0 + it * C::TK;
+                    const int nk = max(min(C::TK, i1 - k0), 0);
+                    const bool first = it == 0;
+                    const bool current = first && chunk == 0;
+                    TileMeta mt;
+                    mt.b = b;
+                    mt.kvh = kvh;
+                    mt.chunk = chunk;
+                    mt.nk = nk;
+                    mt.nch = nch;
+                    mt.r = r;
+                    mt.flags = (first ? kFirst : 0) | (it == ntiles - 1 ? kLast : 0) | (current ? kCurrent : 0);
+                    mt.pad = 0;
+                    meta_s[s] = mt;
+                    unsigned char* st = dsmem + s * C::STAGE;
+                    const uint32_t bytes = static_cast<uint32_t>((nk > 0 ? 2 * C::BOXES * C::BOX_BYTES : 0) +
+                                                                 (first ? G * C::ROW : 0) + (current ? 2 * C::ROW : 0));
+                    fence_proxy_async();
+                    mbar_expect_tx(&full_bar[s], bytes);
+                    if (nk > 0) {
+                        // whole boxes of TK rows: the tile never crosses slot B-1 (B is a multiple of
+                        // 2*TK and tiles start at multiples of TK), rows past the support are masked
+                        int slot = base + k0;
+                        if (slot >= B) slot -= B;
+                        const int y = head * B + slot;
+#pragma unroll
+                        for (int bx = 0; bx < C::BOXES; ++bx) {
+                            tma_load_2d(st + C::K_OFF + bx * C::BOX_BYTES, &kmap, bx * 64, y, &full_bar[s]);
+                            tma_load_2d(st + C::V_OFF + bx * C::BOX_BYTES, &vmap, bx * 64, y, &full_bar[s]);
+                        }
+                    }
+                    if (first) {
+                        const unsigned char* qg = static_cast<const unsigned char*>(a.q) +
+                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * C::ROW;
+                        bulk_g2s(st + C::Q_OFF, qg, G * C::ROW, &full_bar[s]);
+                    }
+                    if (current) {
+                        bulk_g2s(st + C::KN_OFF, static_cast<const unsigned char*>(a.k_new) + static_cast<size_t>(head) * C::ROW,
+                                 C::ROW, &full_bar[s]);
+                        bulk_g2s(st + C::VN_OFF, static_cast<const unsigned char*>(a.v_new) + static_cast<size_t>(head) * C::ROW,
+                                 C::ROW, &full_bar[s]);
+                    }
+                }
+            }
+            if (ok) {  // end-of-work descriptor
+                const int s = seq % kTcStages;
+                if (seq >= kTcStages &&
+                    !mbar_wait(&empty_bar[s], static_cast<uint32_t>((seq / kTcStages - 1) & 1), kGuardNs)) {
+                    ok = false;
+                } else {
+                    TileMeta mt{};
+                    mt.flags = kEnd;
+                    meta_s[s] = mt;
+                    mbar_arrive(&full_bar[s]);
+                    ++seq;
+                }
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+            }
+            issued_s = seq;
+        }
+    } else {
+        // ================= consumers =================
+        const int g = lane >> 2, tig = lane & 3;  // fragment row group and thread in group
+        const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
+        float* merge_o = reinterpret_cast<float*>(dsmem + kTcStages * C::STAGE);  // [kTcConsumers][G][D]
+        uint32_t qb[C::KSTEPS][2];  // Q^T B fragments: head g, dims 16kk + 2tig (+8)
+        float o[C::MTILES][4];      // O^T C fragments: dims 16mt + g (+8), heads 2tig, 2tig+1
+        float m0 = -INFINITY, m1 = -INFINITY;  // running max of heads 2tig, 2tig+1 (log2 domain)
+        float l0 = 0.f, l1 = 0.f;               // this lane's share of their running sums
+#pragma unroll
+        for (int kk = 0; kk < C::KSTEPS; ++kk) qb[kk][0] = qb[kk][1] = 0u;
+#pragma unroll
+        for (int mt_ = 0; mt_ < C::MTILES; ++mt_)
+#pragma unroll
+            for (int x = 0; x < 4; ++x) o[mt_][x] = 0.f;
+        // lane's ldmatrix row within a 16-row block and its chunk offset, for both operand orders
+        const int lm = lane >> 3;                     // which 8x8 matrix this lane addresses
+        const int rowA = 8 * (lm & 1) + (lane & 7);   // K (non-transposed): matrices (rows, +8) x (chunk, +1)
+        const int chA = lm >> 1;
+        const int rowV = 8 * (lm >> 1) + (lane & 7);  // V^T (transposed): matrices (chunk, +1) x (rows, +8)
+        const int chV = lm & 1;
+
+        for (int seq = 0;; ++seq) {
+            const int s = seq % kTcStages;
+            if (!mbar_wait(&full_bar[s], static_cast<uint32_t>((seq / kTcStages) & 1), a.timeout_ns)) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+                break;
+            }
+            const TileMeta mt = meta_s[s];
+            if (mt.flags & kEnd) break;
+            if (abort_s) break;
+            const unsigned char* st = dsmem + s * C::STAGE;
+            const size_t head = static_cast<size_t>(mt.b) * a.Hkv + mt.kvh;
+
+            if (mt.flags & kFirst) {
+#pragma unroll
+                for (int kk = 0; kk < C::KSTEPS; ++kk) {
+                    qb[kk][0] = *reinterpret_cast<const uint32_t*>(st + C::Q_OFF + g * C::ROW + (16 * kk + 2 * tig) * 2);
+                    qb[kk][1] = *reinterpret_cast<const uint32_t*>(st + C::Q_OFF + g * C::ROW + (16 * kk + 2 * tig + 8) * 2);
+                }
+                m0 = m1 = -INFINITY;
+                l0 = l1 = 0.f;
+#pragma unroll
+                for (int mt_ = 0; mt_ < C::MTILES; ++mt_)
+#pragma unroll
+                    for (int x = 0; x < 4; ++x) o[mt_][x] = 0.f;
+                if (mt.flags & kCurrent) {
+                    if (warp == 0) {  // the current token seeds warp 0's state (weight 1 at its own max)
+                        float kc[C::PVD];
+                        load_elems<2, C::PVD>(st + C::KN_OFF + lane * C::PVD * 2, kc);
+                        float zc[G];
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            float qf[C::PVD];
+                            load_elems<2, C::PVD>(st + C::Q_OFF + j * C::ROW + lane * C::PVD * 2, qf);
+                            float acc = 0.f;
+#pragma unroll
+                            for (int x = 0; x < C::PVD; ++x) acc = fmaf(qf[x], kc[x], acc);
+#pragma unroll
+                            for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
+                            zc[j] = acc * qscale;
+                        }
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            if (j == 2 * tig) m0 = zc[j];
+                            if (j == 2 * tig + 1) m1 = zc[j];
+                        }
+                        l0 = l1 = (g == 0) ? 1.f : 0.f;
+                        const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(st + C::VN_OFF);
+#pragma unroll
+                        for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
+                            const float va = __bfloat162float(vn[16 * mt_ + g]);
+                            const float vb = __bfloat162float(vn[16 * mt_ + g + 8]);
+                            o[mt_][0] = va;
+                            o[mt_][1] = va;
+                            o[mt_][2] = vb;
+                            o[mt_][3] = vb;
+                        }
+                    }
+                    if (warp == kTcConsumers - 1) {  // append: slot r of both rings <- the new rows
+                        uint4* kd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.k_ring) +
+                                                             (head * a.B + mt.r) * C::ROW);
+                        uint4* vd = reinterpret_cast<uint4*>(static_cast<unsigned char*>(a.v_ring) +
+                                                             (head * a.B + mt.r) * C::ROW);
+                        for (int x = lane; x < C::ROW / 16; x += 32) {
+                            kd[x] = *reinterpret_cast<const uint4*>(st + C::KN_OFF + x * 16);
+                            vd[x] = *reinterpret_cast<const uint4*>(st + C::VN_OFF + x * 16);
+                        }
+                    }
+                }
+            }
+
+            const int nkw = min(max(mt.nk - warp * 16, 0), 16);  // this warp's keys: rows 16*warp ..
+            if (nkw > 0) {
+                const uint32_t kbase = smem_addr(st + C::K_OFF);
+                const uint32_t vbase = smem_addr(st + C::V_OFF);
+                // ---- scores S^T [16 keys x 8 heads]
+                float c[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int kk = 0; kk < C::KSTEPS; ++kk) {
+                    const int chunk16 = 2 * kk + chA;  // 16-byte chunk of the 256-byte (or 128-byte) row
+                    const int row = 16 * warp + rowA;
+                    uint32_t af[4];
+                    ldmatrix_x4(af, kbase + (chunk16 >> 3) * C::BOX_BYTES + swz(row, chunk16 & 7));
+                    mma_bf16_16816(c, af, qb[kk][0], qb[kk][1]);
+                }
+                // keys g and g+8 of this warp's block; heads 2tig and 2tig+1
+                const bool va = g < nkw, vb = g + 8 < nkw;
+                const float z0 = va ? c[0] * qscale : -INFINITY;
+                const float z1 = va ? c[1] * qscale : -INFINITY;
+                const float z2 = vb ? c[2] * qscale : -INFINITY;
+                const float z3 = vb ? c[3] * qscale : -INFINITY;
+                float mx0 = fmaxf(z0, z2), mx1 = fmaxf(z1, z3);
+#pragma unroll
+                for (int off = 4; off < 32; off <<= 1) {
+                    mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, off));
+                    mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, off));
+                }
+                const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
+                if (__any_sync(kFull, (mn0 > m0) || (mn1 > m1))) {
+                    const float al0 = fast_exp2(m0 - mn0), al1 = fast_exp2(m1 - mn1);
+                    l0 *= al0;
+                    l1 *= al1;
+#pragma unroll
+                    for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
+                        o[mt_][0] *= al0;
+                        o[mt_][1] *= al1;
+                        o[mt_][2] *= al0;
+                        o[mt_][3] *= al1;
+                    }
+                }
+                m0 = mn0;
+                m1 = mn1;
+                const float p0 = fast_exp2(z0 - mn0), p1 = fast_exp2(z1 - mn1);
+                const float p2 = fast_exp2(z2 - mn0), p3 = fast_exp2(z3 - mn1);
+                l0 += p0 + p2;
+                l1 += p1 + p3;
+                // P^T B fragments: high and low bf16 parts, transposed from the S^T C layout
+                const uint32_t h01 = pack_bf16x2(p0, p1), h23 = pack_bf16x2(p2, p3);
+                const uint32_t r01 = pack_bf16x2(p0 - bf16_lo(h01), p1 - bf16_hi(h01));
+                const uint32_t r23 = pack_bf16x2(p2 - bf16_lo(h23), p3 - bf16_hi(h23));
+                const uint32_t bh0 = movmatrix_trans(h01), bh1 = movmatrix_trans(h23);
+                const uint32_t bl0 = movmatrix_trans(r01), bl1 = movmatrix_trans(r23);
+                // ---- O^T [d x 8 heads] += V^T [d x 16 keys] . P^T
+#pragma unroll
+                for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
+                    const int chunk16 = 2 * mt_ + chV;
+                    const int row = 16 * warp + rowV;
+                    uint32_t af[4];
+                    ldmatrix_x4_trans(af, vbase + (chunk16 >> 3) * C::BOX_BYTES + swz(row, chunk16 & 7));
+                    mma_bf16_16816(o[mt_], af, bh0, bh1);
+                    mma_bf16_16816(o[mt_], af, bl0, bl1);
+                }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty_bar[s]);
+            if (!(mt.flags & kLast)) continue;
+
+            // ---- end of the item: this warp's (max, sum, output) into the merge buffers
+            {
+                float s0 = l0, s1 = l1;
+#pragma unroll
+                for (int off = 4; off < 32; off <<= 1) {
+                    s0 += __shfl_xor_sync(kFull, s0, off);
+                    s1 += __shfl_xor_sync(kFull, s1, off);
+                }
+                if (g == 0) {
+                    ml_s[warp][2 * tig] = make_float2(m0, s0);
+                    ml_s[warp][2 * tig + 1] = make_float2(m1, s1);
+                }
+            }
+#pragma unroll
+            for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
+                float* ow = merge_o + (warp * G) * D;
+                ow[(2 * tig) * D + 16 * mt_ + g] = o[mt_][0];
+                ow[(2 * tig + 1) * D + 16 * mt_ + g] = o[mt_][1];
+                ow[(2 * tig) * D + 16 * mt_ + g + 8] = o[mt_][2];
+                ow[(2 * tig + 1) * D + 16 * mt_ + g + 8] = o[mt_][3];
+            }
+            const bool ok = finish_item<G, D, kTcConsumers>(a, mt, head, &ml_s[0][0], merge_o, &sbar_count,
+                                                            &sbar_gen, &last_s, tid, lane, warp);
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_status, kDevOk, kDevTimeout);
+                break;
+            }
+        }
+    }
+    __syncthreads();
+    if (abort_s) {
+        if (tid == 0) {
+            const int issued = issued_s;
+            for (int s = 0; s < kTcStages && s < issued; ++s) {
+                const int j = s + kTcStages * ((issued - 1 - s) / kTcStages);
+                mbar_wait(&full_bar[s], static_cast<uint32_t>((j / kTcStages) & 1), kGuardNs);
             }
         }
         __syncthreads();
@@ -893,6 +1369,108 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t stream)
     return cudaGetLastError();
 }
 
+// ---- tensor-core path: TMA tensor maps over the rings and the launch
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+// Map a ring [rows][d] bf16 as a 2-D tensor read in boxes of 64 columns x box_rows
+// rows with the 128-byte swizzle. Caches the last maps built (rings rarely move).
+bool ring_tensor_map(CUtensorMap* map, void* ring, unsigned long long rows, int d, int box_rows)
+{
+    struct Entry {
+        void* ring;
+        unsigned long long rows;
+        int d, box_rows;
+        CUtensorMap map;
+    };
+    static Entry cache[8];
+    static int next = 0;
+    for (auto& e : cache)
+        if (e.ring == ring && e.rows == rows && e.d == d && e.box_rows == box_rows) {
+            *map = e.map;
+            return true;
+        }
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (enc == nullptr) return false;
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+    const cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * 2};
+    const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
+    const cuuint32_t estr[2] = {1, 1};
+    CUtensorMap m;
+    if (enc(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ring, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+            CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
+        CUDA_SUCCESS)
+        return false;
+    cache[next] = Entry{ring, rows, d, box_rows, m};
+    next = (next + 1) % 8;
+    *map = m;
+    return true;
+}
+
+template <int D>
+int occupancy_tc()
+{
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev < 64 && cache[dev] > 0) return cache[dev];
+    if (cudaFuncSetAttribute(decode_kernel_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<D>::SMEM) !=
+        cudaSuccess)
+        return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel_tc<D>, kTcThreads, TcCfg<D>::SMEM) !=
+        cudaSuccess)
+        return 0;
+    if (dev < 64) cache[dev] = n;
+    return n;
+}
+
+// Whether a step takes the tensor-core path: bf16, GQA group 8, block a multiple
+// of two tiles (no tile straddles the ring end), chunks whole tiles, row
+// coordinates within int32.
+bool tc_eligible(const DecodeArgs& a, int elem_bytes)
+{
+    if (elem_bytes != 2 || a.Hq != 8 * a.Hkv || (a.d != 64 && a.d != 128)) return false;
+    constexpr int tk = 16 * kTcConsumers;
+    if (a.B % (2 * tk) != 0 || a.chunk % tk != 0) return false;
+    const unsigned long long rows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.B;
+    return rows < (1ull << 31) && tensor_map_encoder() != nullptr;
+}
+
+template <int D>
+cudaError_t launch_tc(const DecodeArgs& a, cudaStream_t stream)
+{
+    using C = TcCfg<D>;
+    const int per_sm = occupancy_tc<D>();
+    if (per_sm < 1) return cudaErrorInvalidConfiguration;
+    const unsigned long long rows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.B;
+    CUtensorMap kmap, vmap;
+    if (!ring_tensor_map(&kmap, a.k_ring, rows, D, C::TK) || !ring_tensor_map(&vmap, a.v_ring, rows, D, C::TK))
+        return cudaErrorInvalidValue;
+    int dev = 0, sms = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const long long ctas = static_cast<long long>(sms) * per_sm;
+    const int grid = static_cast<int>(a.total_items < ctas ? a.total_items : ctas);
+    if (grid < 1) return cudaSuccess;
+    decode_kernel_tc<D><<<grid, kTcThreads, C::SMEM, stream>>>(a, kmap, vmap);
+    return cudaGetLastError();
+}
+
 template <int ELEM, int D>
 cudaError_t launch_g(const DecodeArgs& a, cudaStream_t stream)
 {
@@ -949,8 +1527,11 @@ int decode_ctas_per_sm(int elem_bytes, int d, int group)
     return 0;
 }
 
+bool use_tensor_cores(const DecodeArgs& a, int elem_bytes) { return tc_eligible(a, elem_bytes); }
+
 cudaError_t launch_decode(const DecodeArgs& a, int elem_bytes, cudaStream_t stream)
 {
+    if (tc_eligible(a, elem_bytes)) return a.d == 64 ? launch_tc<64>(a, stream) : launch_tc<128>(a, stream);
     if (elem_bytes == 2 && a.d == 64) return launch_g<2, 64>(a, stream);
     if (elem_bytes == 2 && a.d == 128) return launch_g<2, 128>(a, stream);
     if (elem_bytes == 4 && a.d == 64) return launch_g<4, 64>(a, stream);

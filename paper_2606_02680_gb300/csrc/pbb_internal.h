@@ -36,6 +36,9 @@ int tile_keys(int elem_bytes, int d, int group);
 // Resident CTAs per SM of the decode kernel for this instance (0 if unsupported).
 int decode_ctas_per_sm(int elem_bytes, int d, int group);
 
+// Whether launch_decode would run the tensor-core kernel for these arguments.
+bool use_tensor_cores(const DecodeArgs& a, int elem_bytes);
+
 // Launch the fused append + attention + combine kernel (persistent grid of at
 // most SMs x resident CTAs). elem_bytes: 2 (bf16) or 4 (fp32).
 cudaError_t launch_decode(const DecodeArgs& a, int elem_bytes, cudaStream_t stream);

@@ -69,9 +69,12 @@ def test_fp32_one_layer_split(chunk_keys):
 @pytest.mark.parametrize("chunk", [0, 32])
 def test_bf16_groups_and_dims(chunk_keys, group, d, chunk):
     """bf16, every supported GQA group and head size, B = 96 (not a power of two,
-    tiles straddle the ring end), 3 blocks from t = 0, batch 3."""
+    tiles straddle the ring end; CUDA-core kernel for every group), 3 blocks from
+    t = 0, batch 3."""
     w = inputs.Workload(f"g{group}_d{d}", batch=3, Hq=2 * group, Hkv=2, d=d, B=96, dtype="bf16",
                         steps=3 * 96 + 5, t0_lo=0, t0_hi=1, seed=100 + group + d)
+    chunk_keys(chunk)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "cuda_cores"
     run_and_check(w, chunk_keys, chunk=chunk, check_every=1)
 
 
@@ -278,3 +281,27 @@ def test_large_block(chunk_keys):
     w = inputs.Workload("bigB", batch=1, Hq=4, Hkv=1, d=128, B=1 << 16, dtype="bf16", steps=3,
                         t0_lo=(1 << 16) * 3 + 100, t0_hi=(1 << 16) * 4, seed=61)
     run_and_check(w, chunk_keys, chunk=0)
+
+
+@pytest.mark.parametrize("B", [64, 128, 256])
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("chunk", [0, 64])
+def test_bf16_group8_tensor_core_path(chunk_keys, B, d, chunk):
+    """bf16 with GQA group 8 and B a multiple of 64 runs the tensor-core kernel
+    (TMA-swizzled tiles, mma.sync for Q.K^T and P.V): every step of 3 blocks from
+    t = 0 (first-block, bridge and partial tiles), batch 3, against the oracle."""
+    w = inputs.Workload(f"tc_B{B}_d{d}", batch=3, Hq=16, Hkv=2, d=d, B=B, dtype="bf16",
+                        steps=3 * B + 3, t0_lo=0, t0_hi=1, seed=300 + B + d)
+    chunk_keys(chunk)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
+    run_and_check(w, chunk_keys, chunk=chunk)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_bf16_group8_tensor_core_ragged_outliers(chunk_keys, d):
+    """Tensor-core path with ragged prefilled rings and x20 outliers (large logits)."""
+    w = inputs.Workload("tc_outlier", batch=6, Hq=8, Hkv=1, d=d, B=512, dtype="bf16", steps=80,
+                        t0_lo=0, t0_hi=20000, outlier_frac=0.01, outlier_scale=20.0, seed=77 + d)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
+    run_and_check(w, chunk_keys, chunk=0)
+    run_and_check(w, chunk_keys, chunk=128)
