@@ -48,6 +48,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--batch", type=int, default=512)
     ap.add_argument("--block", type=int, default=4096)
+    ap.add_argument("--hq", type=int, default=0, help="query heads of the throughput point (default 32)")
+    ap.add_argument("--hkv", type=int, default=0, help="KV heads of the throughput point (default 8)")
     ap.add_argument("--sweep", action="store_true", help="one line per throughput-sweep point")
     ap.add_argument("--workload", default="", help="a named workload of paper_2606_02680_gb300.inputs "
                     "(default: the throughput point given by --batch/--block)")
@@ -447,7 +449,11 @@ def run_ours(args):
         points = [inputs.sweep_workload(shard_batch(b, rank, world), B)
                   for b in inputs.SWEEP_BATCHES for B in inputs.SWEEP_BLOCKS]
     else:
-        points = [inputs.sweep_workload(shard_batch(args.batch, rank, world), args.block)]
+        w0 = inputs.sweep_workload(shard_batch(args.batch, rank, world), args.block)
+        if args.hq or args.hkv:
+            hq, hkv = args.hq or w0.Hq, args.hkv or w0.Hkv
+            w0 = w0.with_(Hq=hq, Hkv=hkv, name=f"{w0.name}_Hq{hq}_Hkv{hkv}")
+        points = [w0]
     peak, peak_kind = hbm_peak()
     for w in points:
         batch, B = w.batch, w.B

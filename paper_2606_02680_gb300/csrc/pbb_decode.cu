@@ -1127,7 +1127,6 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     if (warp == 0) {  // the current token seeds warp 0's state (weight 1 at its own max)
                         float kc[C::PVD];
                         load_elems<2, C::PVD>(st + C::KN_OFF + lane * C::PVD * 2, kc);
-                        float zc[G];
 #pragma unroll
                         for (int j = 0; j < G; ++j) {
                             float qf[C::PVD];
@@ -1137,12 +1136,9 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                             for (int x = 0; x < C::PVD; ++x) acc = fmaf(qf[x], kc[x], acc);
 #pragma unroll
                             for (int off = 16; off >= 1; off >>= 1) acc += __shfl_xor_sync(kFull, acc, off);
-                            zc[j] = acc * qscale;
-                        }
-#pragma unroll
-                        for (int j = 0; j < G; ++j) {
-                            if (j == 2 * tig) m0 = zc[j];
-                            if (j == 2 * tig + 1) m1 = zc[j];
+                            const float zj = acc * qscale;
+                            m0 = (j == 2 * tig) ? zj : m0;
+                            m1 = (j == 2 * tig + 1) ? zj : m1;
                         }
                         l0 = l1 = (g == 0) ? 1.f : 0.f;
                         const __nv_bfloat16* vn = reinterpret_cast<const __nv_bfloat16*>(st + C::VN_OFF);
@@ -1173,16 +1169,23 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             if (nkw > 0) {
                 const uint32_t kbase = smem_addr(st + C::K_OFF);
                 const uint32_t vbase = smem_addr(st + C::V_OFF);
-                // ---- scores S^T [16 keys x 8 heads]
+                // ---- scores S^T [16 keys x 8 heads]: two independent mma chains (even and odd
+                // k-steps) halve the dependent latency
                 float c[4] = {0.f, 0.f, 0.f, 0.f};
+                float c2[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int kk = 0; kk < C::KSTEPS; ++kk) {
                     const int chunk16 = 2 * kk + chA;  // 16-byte chunk of the 256-byte (or 128-byte) row
                     const int row = 16 * warp + rowA;
                     uint32_t af[4];
                     ldmatrix_x4(af, kbase + (chunk16 >> 3) * C::BOX_BYTES + swz(row, chunk16 & 7));
-                    mma_bf16_16816(c, af, qb[kk][0], qb[kk][1]);
+                    if (kk & 1)
+                        mma_bf16_16816(c2, af, qb[kk][0], qb[kk][1]);
+                    else
+                        mma_bf16_16816(c, af, qb[kk][0], qb[kk][1]);
                 }
+#pragma unroll
+                for (int x = 0; x < 4; ++x) c[x] += c2[x];
                 // keys g and g+8 of this warp's block; heads 2tig and 2tig+1
                 const bool va = g < nkw, vb = g + 8 < nkw;
                 const float z0 = va ? c[0] * qscale : -INFINITY;
