@@ -11,7 +11,8 @@ Names follow the C ABI:
 * ``ring_bytes``, ``ring_alloc`` / ``Rings``   the B-slot K/V rings (Appendix F.1)
 * ``ring_prefill``                             load a ring from a history window
 * ``decode_step``                              append + attention over A(t) (Sec. 3)
-* ``decode_step_host``                         the same with host-resident inputs/outputs
+* ``decode_step_host``, ``HostPipeline``       the same with host-resident inputs/outputs
+                                               (one at a time / overlapped across steps)
 * ``advance_positions``, ``get_device_status``, ``reserve_workspace``,
   ``set_wait_timeout_ns``, ``set_chunk_keys``, ``plan_chunk_keys``
 """
@@ -28,7 +29,7 @@ __all__ = [
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
     "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step",
-    "decode_step_host", "advance_positions", "get_device_status", "reserve_workspace",
+    "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
 
@@ -248,6 +249,61 @@ def decode_step_host(q_h: torch.Tensor, k_h: torch.Tensor, v_h: torch.Tensor, k_
         staging.v.copy_(v_h, non_blocking=True)
         decode_step(staging.q, staging.k, staging.v, k_ring, v_ring, pos, staging.out, stream=s)
         out_h.copy_(staging.out, non_blocking=True)
+
+
+class HostPipeline:
+    """Decode steps whose inputs and outputs live in (pinned) host memory, with the
+    transfers overlapped with the device work of neighbouring steps.
+
+    Two device staging sets alternate between steps. Step i copies its q/k/v in on
+    an input-copy stream while the compute stream may still run step i-1; the
+    compute stream waits for those copies, runs the decode step and advances the
+    positions; an output-copy stream then copies the output back. Events keep a
+    staging set from being overwritten before its previous step is done with it.
+    Call ``synchronize()`` before reading the host outputs.
+    """
+
+    def __init__(self, batch: int, Hq: int, Hkv: int, d: int, dtype, device, compute_stream=None):
+        self.compute = torch.cuda.current_stream(device) if compute_stream is None else compute_stream
+        self.copy_in = torch.cuda.Stream(device=device)
+        self.copy_out = torch.cuda.Stream(device=device)
+        self.sets = [HostStep(batch, Hq, Hkv, d, dtype, device) for _ in range(2)]
+        self.inputs_ready = [torch.cuda.Event() for _ in range(2)]
+        self.inputs_used = [torch.cuda.Event() for _ in range(2)]
+        self.output_ready = [torch.cuda.Event() for _ in range(2)]
+        self.output_sent = [torch.cuda.Event() for _ in range(2)]
+        self.i = 0
+
+    def step(self, q_h, k_h, v_h, k_ring, v_ring, pos, out_h) -> None:
+        j = self.i % 2
+        st = self.sets[j]
+        if self.i >= 2:
+            self.copy_in.wait_event(self.inputs_used[j])   # step i-2 has read these inputs
+            self.compute.wait_event(self.output_sent[j])   # and its output has left this buffer
+        with torch.cuda.stream(self.copy_in):
+            st.q.copy_(q_h, non_blocking=True)
+            st.k.copy_(k_h, non_blocking=True)
+            st.v.copy_(v_h, non_blocking=True)
+            self.inputs_ready[j].record(self.copy_in)
+        self.compute.wait_event(self.inputs_ready[j])
+        decode_step(st.q, st.k, st.v, k_ring, v_ring, pos, st.out, stream=self.compute)
+        self.inputs_used[j].record(self.compute)
+        self.output_ready[j].record(self.compute)
+        advance_positions(pos, stream=self.compute)
+        self.copy_out.wait_event(self.output_ready[j])
+        with torch.cuda.stream(self.copy_out):
+            out_h.copy_(st.out, non_blocking=True)
+            self.output_sent[j].record(self.copy_out)
+        self.i += 1
+
+    def last_output_event(self) -> torch.cuda.Event:
+        """Event recorded after the output copy of the latest step."""
+        return self.output_sent[(self.i - 1) % 2]
+
+    def synchronize(self) -> None:
+        self.copy_in.synchronize()
+        self.compute.synchronize()
+        self.copy_out.synchronize()
 
 
 def advance_positions(pos: torch.Tensor, stream=None) -> None:

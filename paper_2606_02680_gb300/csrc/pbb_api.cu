@@ -76,10 +76,13 @@ int sm_count(int dev)
 
 // Ring keys of the support per work item. The support of a (sequence, KV
 // head) has at most B-1 ring keys besides the current token. Without an
-// override the plan splits it only as far as needed for the items to fill the
-// GPU several times over (kWaves waves of resident CTAs), and never into
+// override the plan splits supports only when there are fewer of them than
+// resident CTAs, into at most as many items as there are CTAs, and never into
 // chunks of less than kMinChunkBytes of K+V, below which the combine would cost
-// more than the parallel streaming saves; large batches run unsplit.
+// more than the parallel streaming saves. Measured on GB300 at 512 supports
+// (batch 64 x 8 KV heads, or 256 x 2) on 456 resident CTAs, splitting into 2-4
+// chunks was 5-25 % slower than running them whole (the per-item merge and the
+// cross-CTA combine cost more than the shorter tail saves).
 int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
 {
     const int tile = pbb::tile_keys(elem, d, group);
@@ -89,10 +92,10 @@ int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
     if (over > 0) {
         chunk = over;
     } else {
-        constexpr int kWaves = 4;
+        constexpr int kWaves = 1;
         constexpr int kMinChunkBytes = 64 * 1024;
         const long long pairs = static_cast<long long>(batch) * Hkv;
-        int per_sm = pbb::decode_ctas_per_sm(elem, d, group);
+        int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B);
         if (per_sm <= 0) per_sm = 1;
         const long long want = static_cast<long long>(kWaves) * sm_count(dev) * per_sm;
         long long split = pairs > 0 ? (want + pairs - 1) / pairs : 1;

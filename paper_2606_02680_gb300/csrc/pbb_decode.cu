@@ -569,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
             // tile); later ones come from the queue, which hands out items grid, grid+1, ...
             for (int item = blockIdx.x; ok && item < a.total_items;
                  item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
-                const int chunk = item % a.nchunk;
+                const int chunk = item % a.nchunk;  // a support's chunks are consecutive items
                 const int pair = item / a.nchunk;
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
                 const int t = __ldg(a.pos + b);
@@ -981,7 +981,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             bool ok = true;
             for (int item = blockIdx.x; ok && item < a.total_items;
                  item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
-                const int chunk = item % a.nchunk;
+                const int chunk = item % a.nchunk;  // a support's chunks are consecutive items
                 const int pair = item / a.nchunk;
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
                 const int t = __ldg(a.pos + b);
@@ -1521,8 +1521,11 @@ int tile_keys(int elem_bytes, int d, int group)
     return 0;
 }
 
-int decode_ctas_per_sm(int elem_bytes, int d, int group)
+int decode_ctas_per_sm(int elem_bytes, int d, int group, int B)
 {
+    if (elem_bytes == 2 && group == 8 && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
+        tensor_map_encoder() != nullptr)
+        return d == 64 ? occupancy_tc<64>() : occupancy_tc<128>();
     if (elem_bytes == 2 && d == 64) return occupancy_g<2, 64>(group);
     if (elem_bytes == 2 && d == 128) return occupancy_g<2, 128>(group);
     if (elem_bytes == 4 && d == 64) return occupancy_g<4, 64>(group);

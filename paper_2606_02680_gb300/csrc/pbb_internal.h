@@ -33,8 +33,8 @@ struct DecodeArgs {
 // Keys per shared-memory tile of a kernel instance (rows of K and of V).
 int tile_keys(int elem_bytes, int d, int group);
 
-// Resident CTAs per SM of the decode kernel for this instance (0 if unsupported).
-int decode_ctas_per_sm(int elem_bytes, int d, int group);
+// Resident CTAs per SM of the decode kernel a step of this shape runs (0 if unsupported).
+int decode_ctas_per_sm(int elem_bytes, int d, int group, int B);
 
 // Whether launch_decode would run the tensor-core kernel for these arguments.
 bool use_tensor_cores(const DecodeArgs& a, int elem_bytes);

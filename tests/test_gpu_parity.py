@@ -305,3 +305,38 @@ def test_bf16_group8_tensor_core_ragged_outliers(chunk_keys, d):
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
     run_and_check(w, chunk_keys, chunk=0)
     run_and_check(w, chunk_keys, chunk=128)
+
+
+def test_host_pipeline_matches_device_steps():
+    """HostPipeline (host-resident inputs and outputs, copies overlapped across
+    steps) gives bitwise the outputs and rings of plain device steps."""
+    w = inputs.Workload("pipe", batch=4, Hq=16, Hkv=4, d=128, B=256, dtype="bf16", steps=6,
+                        t0_lo=300, t0_hi=5000, seed=91)
+    dev = torch.device("cuda")
+    t0 = inputs.start_positions(w)
+    wk, wv = inputs.history_window(w, t0)
+    steps = [inputs.step_inputs(w, i) for i in range(w.steps)]
+    results = []
+    for mode in ("device", "pipeline"):
+        pos = t0.to(torch.int32).to(dev)
+        kr = torch.zeros((w.batch, w.Hkv, w.B, w.d), dtype=torch.bfloat16, device=dev)
+        vr = torch.zeros_like(kr)
+        pbb.ring_prefill(wk.to(dev), wv.to(dev), pos, kr, vr)
+        outs = []
+        if mode == "device":
+            for q, k, v in steps:
+                outs.append(pbb.decode_step(q.to(dev), k.to(dev), v.to(dev), kr, vr, pos).cpu())
+                pbb.advance_positions(pos)
+        else:
+            pipe = pbb.HostPipeline(w.batch, w.Hq, w.Hkv, w.d, torch.bfloat16, dev)
+            host_out = [torch.empty((w.batch, w.Hq, w.d)).pin_memory() for _ in steps]
+            for (q, k, v), o in zip(steps, host_out):
+                pipe.step(q.pin_memory(), k.pin_memory(), v.pin_memory(), kr, vr, pos, o)
+            pipe.synchronize()
+            outs = [o.clone() for o in host_out]
+        torch.cuda.synchronize()
+        results.append((outs, kr.cpu(), pos.cpu()))
+    for a, b in zip(results[0][0], results[1][0]):
+        assert torch.equal(a, b)
+    assert torch.equal(results[0][1].view(torch.int16), results[1][1].view(torch.int16))
+    assert torch.equal(results[0][2], results[1][2])
