@@ -74,48 +74,93 @@ int sm_count(int dev)
     return g_sms[dev];
 }
 
-// Ring keys of the support per work item. The support of a (sequence, KV
-// head) has at most B-1 ring keys besides the current token. Without an
-// override the plan splits supports only when there are fewer of them than
-// resident CTAs, into at most as many items as there are CTAs, and never into
-// chunks of less than kMinChunkBytes of K+V, below which the combine would cost
-// more than the parallel streaming saves. Measured on GB300 at 512 supports
-// (batch 64 x 8 KV heads, or 256 x 2) on 456 resident CTAs, splitting into 2-4
-// chunks was 5-25 % slower than running them whole (the per-item merge and the
-// cross-CTA combine cost more than the shorter tail saves).
-int plan_chunk(int batch, int Hkv, int d, int B, int elem, int group, int dev)
+// The split plan. Whole supports are the cheapest work items (no cross-CTA
+// combine), but a batch of P supports on G resident CTAs leaves P mod G
+// supports for a last round; when that round would leave more than half the
+// CTAs idle, those last supports are split into about G / (P mod G) chunks
+// each, so the step ends on small items. A batch with fewer supports than CTAs
+// splits every support so that there are about G items. Chunks never hold less
+// than kMinChunkBytes of K+V (below that the combine costs more than the
+// parallel streaming saves). Measured on GB300 at 512 supports on 456 CTAs,
+// splitting every support into 2-4 chunks was 5-25 % slower than running them
+// whole, while splitting only the last round's supports paid for long supports
+// (see below); a positive pbb_set_chunk_keys override splits every support
+// into chunks of that many keys.
+int min_split_keys(int d, int elem, int tile)
 {
-    const int tile = pbb::tile_keys(elem, d, group);
-    const int max_keys = B - 1;
-    int chunk;
-    const int over = g_chunk_override.load();
-    if (over > 0) {
-        chunk = over;
-    } else {
-        constexpr int kWaves = 1;
-        constexpr int kMinChunkBytes = 64 * 1024;
-        const long long pairs = static_cast<long long>(batch) * Hkv;
-        int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B);
-        if (per_sm <= 0) per_sm = 1;
-        const long long want = static_cast<long long>(kWaves) * sm_count(dev) * per_sm;
-        long long split = pairs > 0 ? (want + pairs - 1) / pairs : 1;
-        int min_keys = kMinChunkBytes / (2 * d * elem);
-        if (min_keys < tile) min_keys = tile;
-        const long long max_split = (max_keys + min_keys - 1) / min_keys;
-        if (split > max_split) split = max_split;
-        if (split < 1) split = 1;
-        chunk = static_cast<int>((max_keys + split - 1) / split);
-    }
-    chunk = static_cast<int>(round_up(static_cast<size_t>(chunk), static_cast<size_t>(tile)));
-    if (chunk < tile) chunk = tile;
-    return chunk;
+    constexpr int kMinChunkBytes = 64 * 1024;
+    const int k = kMinChunkBytes / (2 * d * elem);
+    return k < tile ? tile : k;
 }
 
-// Bytes of split partials for a step: per (sequence, KV head, chunk, head)
-// d floats of unnormalised output, then 2 floats (max, sum).
-size_t parts_bytes(int batch, int Hkv, int d, int group, int nchunk)
+}  // namespace
+
+namespace pbb {
+
+SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group)
 {
-    const size_t parts = static_cast<size_t>(batch) * Hkv * nchunk * group;
+    SplitPlan sp{0, 0, 1};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) dev = 0;
+    const int tile = pbb::tile_keys(elem, d, group);
+    const int max_keys = B - 1 > 0 ? B - 1 : 1;
+    const long long pairs = static_cast<long long>(batch) * Hkv;
+    auto finish = [&](long long split) {
+        const long long max_split = (max_keys + min_split_keys(d, elem, tile) - 1) / min_split_keys(d, elem, tile);
+        if (split > max_split) split = max_split;
+        if (split < 1) split = 1;
+        int chunk = static_cast<int>((max_keys + split - 1) / split);
+        chunk = static_cast<int>(round_up(static_cast<size_t>(chunk), static_cast<size_t>(tile)));
+        sp.chunk = chunk;
+        sp.nchunk = (max_keys + chunk - 1) / chunk;
+        if (sp.nchunk <= 1) {  // nothing to split
+            sp.whole = static_cast<int>(pairs);
+            sp.nchunk = 1;
+        }
+    };
+    const int over = g_chunk_override.load();
+    if (over > 0) {
+        sp.whole = 0;
+        int chunk = static_cast<int>(round_up(static_cast<size_t>(over), static_cast<size_t>(tile)));
+        sp.chunk = chunk;
+        sp.nchunk = (max_keys + chunk - 1) / chunk;
+        return sp;
+    }
+    int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B);
+    if (per_sm <= 0) per_sm = 1;
+    const long long G = static_cast<long long>(sm_count(dev)) * per_sm;
+    if (pairs >= G) {
+        const long long R = pairs % G;
+        // Splitting the last round pays only for long supports on the CUDA-core kernel
+        // (measured: +29 % at B 4096 and +6 % at B 2048, but -12 to -15 % at B <= 1024 and
+        // -19 % for the tensor-core kernel, whose two consumer warps combine slowly).
+        const bool long_supports = max_keys >= 2047 && pbb::tile_keys(elem, d, group) == tile &&
+                                   !(elem == 2 && group == 8 && B % 64 == 0);
+        if (R == 0 || 2 * R > G || !long_supports) {  // no split
+            sp.whole = static_cast<int>(pairs);
+            sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
+            sp.nchunk = 1;
+            return sp;
+        }
+        sp.whole = static_cast<int>(pairs - R);
+        finish((G + R - 1) / R);
+    } else {
+        sp.whole = 0;
+        finish(pairs > 0 ? (G + pairs - 1) / pairs : 1);
+    }
+    return sp;
+}
+
+}  // namespace pbb
+
+namespace {
+
+// Bytes of split partials for a step: per (split support, chunk, head) d floats
+// of unnormalised output, then 2 floats (max, sum).
+size_t parts_bytes(int batch, int Hkv, int d, int group, const pbb::SplitPlan& sp)
+{
+    const size_t split_pairs = static_cast<size_t>(batch) * Hkv - static_cast<size_t>(sp.whole);
+    const size_t parts = split_pairs * sp.nchunk * group;
     return round_up(parts * d * sizeof(float), 256) + parts * 2 * sizeof(float);
 }
 
@@ -186,23 +231,25 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
-    a.chunk = plan_chunk(batch, Hkv, d, B, elem, group, dev);
-    a.nchunk = (B - 1 + a.chunk - 1) / a.chunk;
-    if (a.nchunk < 1) a.nchunk = 1;
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, group);
+    a.whole = sp.whole;
+    a.chunk = sp.chunk;
+    a.nchunk = sp.nchunk;
     a.timeout_ns = g_timeout_ns.load();
     if (a.nchunk > 65535) return PBB_ERR_UNSUPPORTED;
     const size_t pairs = static_cast<size_t>(batch) * Hkv;
-    a.total_items = static_cast<int>(pairs * a.nchunk);
-    if (pairs * a.nchunk > static_cast<size_t>(INT_MAX)) return PBB_ERR_UNSUPPORTED;
+    const size_t items = static_cast<size_t>(sp.whole) + (pairs - static_cast<size_t>(sp.whole)) * sp.nchunk;
+    if (items > static_cast<size_t>(INT_MAX)) return PBB_ERR_UNSUPPORTED;
+    a.total_items = static_cast<int>(items);
     {
-        const size_t pbytes = a.nchunk > 1 ? parts_bytes(batch, Hkv, d, group, a.nchunk) : 0;
+        const size_t pbytes = static_cast<size_t>(sp.whole) < pairs ? parts_bytes(batch, Hkv, d, group, sp) : 0;
         std::lock_guard<std::mutex> lock(g_mutex);
         rc = grow_workspace(dev, pairs + 2, pbytes, stream, true);
         if (rc != PBB_OK) return rc;
-        const size_t parts = pairs * a.nchunk * group;
+        const size_t parts = (pairs - static_cast<size_t>(sp.whole)) * a.nchunk * group;
         a.ctl = g_ws[dev].counters;
         a.counters = g_ws[dev].counters + 2;
-        if (a.nchunk > 1) {
+        if (pbytes > 0) {
             a.part_o = g_ws[dev].parts;
             a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(g_ws[dev].parts) +
                                                  round_up(parts * d * sizeof(float), 256));
@@ -286,13 +333,12 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
     if (rc != PBB_OK) return rc;
     const int elem = elem_size(dtype);
     const int group = Hq / Hkv;
-    // Every batch up to max_batch: the plan's split shrinks as the batch grows.
+    // Every batch up to max_batch: the plan's split depends on the batch.
     size_t need = 0;
     for (int bsz = 1; bsz <= max_batch; ++bsz) {
-        const int chunk = plan_chunk(bsz, Hkv, d, B, elem, group, dev);
-        const int nchunk = (B - 1 + chunk - 1) / chunk;
-        if (nchunk <= 1) continue;
-        const size_t w = parts_bytes(bsz, Hkv, d, group, nchunk);
+        const pbb::SplitPlan sp = pbb::plan_split(bsz, Hkv, d, B, elem, group);
+        if (static_cast<size_t>(sp.whole) >= static_cast<size_t>(bsz) * Hkv) continue;
+        const size_t w = parts_bytes(bsz, Hkv, d, group, sp);
         if (w > need) need = w;
     }
     std::lock_guard<std::mutex> lock(g_mutex);
@@ -360,7 +406,7 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
     if (check_shape(batch, Hkv, d, B, dtype) != PBB_OK || check_group(Hq, Hkv) != PBB_OK) return 0;
     int dev = 0;
     if (current_device(&dev) != PBB_OK) return 0;
-    return plan_chunk(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, dev);
+    return pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv).chunk;
 }
 
 int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
@@ -378,7 +424,8 @@ int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
-    a.chunk = plan_chunk(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, dev);
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv);
+    a.chunk = sp.chunk;
     return pbb::use_tensor_cores(a, elem_size(dtype)) ? PBB_KERNEL_TENSOR_CORES : PBB_KERNEL_CUDA_CORES;
 }
 

@@ -9,12 +9,14 @@
 // phases read 0..r-1. In position order, ring key i of the support lives in
 // slot (base + i) mod B, base = h for a bridge phase and 0 otherwise.
 //
-// Work items. Item (sequence, KV head, chunk) covers ring keys
-// [chunk*C, chunk*C + C) of one support, for all G = Hq/Hkv query heads of the
-// group, so each K/V byte is read from HBM once per step. Chunk 0 of every
-// (sequence, KV head) also carries the current token: it appends k_new/v_new
-// to slot r (never a slot that is read) and folds the token into its softmax.
-// Items past the end of a short support are empty and skipped.
+// Work items. An item covers one (sequence, KV head) support, or a chunk of C
+// ring keys of one, for all G = Hq/Hkv query heads of the group, so each K/V
+// byte is read from HBM once per step. The first `whole` supports are items of
+// their own; each later support is split into chunks (the plan splits only
+// the supports of a last, partly filled round, or all supports of a batch too
+// small to fill the GPU). Chunk 0 of a support also carries the current token:
+// it appends k_new/v_new to slot r (never a slot that is read) and folds the
+// token into its softmax. Chunks past the end of a short support are skipped.
 //
 // Persistent CTAs, one per SM. A producer lane takes items from a device-wide
 // queue (an atomic counter) and streams them without a break: every item
@@ -439,7 +441,7 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
 {
     bool ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
     const int ctid = tid;  // 0 .. 32*NC-1 (consumer threads)
-    const size_t part = head * a.nchunk + mt.chunk;
+    const size_t part = (head - a.whole) * a.nchunk + mt.chunk;  // only split supports have partials
     if (ok) {
         for (int e = ctid; e < G * D; e += NC * 32) {
             const int j = e / D;
@@ -469,8 +471,8 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
         ok = ok && consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
         if (ok && *last_s) {
             __threadfence();
-            const float* po = a.part_o + head * a.nchunk * G * D;
-            const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + head * a.nchunk * G;
+            const float* po = a.part_o + (head - a.whole) * a.nchunk * G * D;
+            const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + (head - a.whole) * a.nchunk * G;
             float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D;
             if (mt.nch <= NC * D) {
                 // weight of every (chunk, head) in shared memory: e^(m_c - M) / L, with M and
@@ -569,8 +571,16 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
             // tile); later ones come from the queue, which hands out items grid, grid+1, ...
             for (int item = blockIdx.x; ok && item < a.total_items;
                  item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
-                const int chunk = item % a.nchunk;  // a support's chunks are consecutive items
-                const int pair = item / a.nchunk;
+                // items [0, whole): whole supports; then nchunk chunks of each later support
+                int pair, chunk;
+                if (item < a.whole) {
+                    pair = item;
+                    chunk = 0;
+                } else {
+                    const int j = item - a.whole;
+                    pair = a.whole + j / a.nchunk;
+                    chunk = j % a.nchunk;
+                }
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
                 const int t = __ldg(a.pos + b);
                 if (t < 0) {
@@ -583,10 +593,12 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                 const bool bridge = (blk > 0) && (r < h);
                 const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
                 const int base = bridge ? h : 0;   // slot of ring key 0
-                const int nch = n > 0 ? (n + a.chunk - 1) / a.chunk : 1;
+                const bool whole = pair < a.whole;
+                const int csize = whole ? max(n, 1) : a.chunk;  // keys per chunk of this support
+                const int nch = n > 0 ? (n + csize - 1) / csize : 1;
                 if (chunk >= nch) continue;
-                const int i0 = chunk * a.chunk;
-                const int i1 = min(i0 + a.chunk, n);
+                const int i0 = chunk * csize;
+                const int i1 = min(i0 + csize, n);
                 const int nkeys = max(i1 - i0, 0);
                 const int ntiles = nkeys > 0 ? (nkeys + C::TK - 1) / C::TK : 1;
                 const size_t head = static_cast<size_t>(b) * a.Hkv + kvh;
@@ -981,8 +993,16 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             bool ok = true;
             for (int item = blockIdx.x; ok && item < a.total_items;
                  item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
-                const int chunk = item % a.nchunk;  // a support's chunks are consecutive items
-                const int pair = item / a.nchunk;
+                // items [0, whole): whole supports; then nchunk chunks of each later support
+                int pair, chunk;
+                if (item < a.whole) {
+                    pair = item;
+                    chunk = 0;
+                } else {
+                    const int j = item - a.whole;
+                    pair = a.whole + j / a.nchunk;
+                    chunk = j % a.nchunk;
+                }
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
                 const int t = __ldg(a.pos + b);
                 if (t < 0) {
@@ -995,10 +1015,12 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                 const bool bridge = (blk > 0) && (r < h);
                 const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
                 const int base = bridge ? h : 0;   // slot of ring key 0
-                const int nch = n > 0 ? (n + a.chunk - 1) / a.chunk : 1;
+                const bool whole = pair < a.whole;
+                const int csize = whole ? max(n, 1) : a.chunk;  // keys per chunk of this support
+                const int nch = n > 0 ? (n + csize - 1) / csize : 1;
                 if (chunk >= nch) continue;
-                const int i0 = chunk * a.chunk;
-                const int i1 = min(i0 + a.chunk, n);
+                const int i0 = chunk * csize;
+                const int i1 = min(i0 + csize, n);
                 const int nkeys = max(i1 - i0, 0);
                 const int ntiles = nkeys > 0 ? (nkeys + C::TK - 1) / C::TK : 1;
                 const int head = b * a.Hkv + kvh;

@@ -19,14 +19,15 @@ struct DecodeArgs {
     void* v_ring;        // [batch][Hkv][B][d]
     const int32_t* pos;  // [batch]
     float* out;          // [batch][Hq][d]
-    float* part_o;       // [batch][Hkv][nchunk][G][d]   split partials (unnormalised output)
-    float* part_ml;      // [batch][Hkv][nchunk][G][2]   split partials (max, sum), log2 domain
+    float* part_o;       // [batch*Hkv - whole][nchunk][G][d]   split partials (unnormalised output)
+    float* part_ml;      // [batch*Hkv - whole][nchunk][G][2]   split partials (max, sum), log2 domain
     int* counters;       // [batch][Hkv]                 finished chunks per (sequence, KV head)
     int* ctl;            // [2] work-queue head and finished CTAs; zero between launches
     int batch, Hq, Hkv, d, B;
-    int chunk;           // ring keys of the support per work item (a multiple of the tile)
-    int nchunk;          // work items per (sequence, KV head) = ceil((B-1)/chunk)
-    int total_items;     // batch * Hkv * nchunk
+    int whole;           // supports [0, whole) are one work item each
+    int chunk;           // ring keys per work item of the later supports (a multiple of the tile)
+    int nchunk;          // work items per later support = ceil((B-1)/chunk)
+    int total_items;     // whole + (batch * Hkv - whole) * nchunk
     unsigned long long timeout_ns;
 };
 
@@ -35,6 +36,13 @@ int tile_keys(int elem_bytes, int d, int group);
 
 // Resident CTAs per SM of the decode kernel a step of this shape runs (0 if unsupported).
 int decode_ctas_per_sm(int elem_bytes, int d, int group, int B);
+
+// The split plan of a step (see plan_split in pbb_api.cu): supports [0, whole)
+// run whole, every later one in nchunk chunks of `chunk` ring keys.
+struct SplitPlan {
+    int whole, chunk, nchunk;
+};
+SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem_bytes, int group);
 
 // Whether launch_decode would run the tensor-core kernel for these arguments.
 bool use_tensor_cores(const DecodeArgs& a, int elem_bytes);

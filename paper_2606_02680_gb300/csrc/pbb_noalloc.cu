@@ -93,26 +93,27 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
-    a.chunk = pbb_plan_chunk_keys(batch, Hq, Hkv, d, B, PBB_BF16);  // the same split as pbb_decode_step
-    if (a.chunk <= 0) return PBB_ERR_CUDA;
-    a.nchunk = (B - 1 + a.chunk - 1) / a.chunk;
-    if (a.nchunk < 1) a.nchunk = 1;
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, 2, group);  // the same plan as pbb_decode_step
+    if (sp.chunk <= 0) return PBB_ERR_CUDA;
+    a.whole = sp.whole;
+    a.chunk = sp.chunk;
+    a.nchunk = sp.nchunk;
     if (a.nchunk > 65535) return PBB_ERR_UNSUPPORTED;
     a.timeout_ns = 1000000000ull;
 
     const size_t pairs = static_cast<size_t>(batch) * Hkv;
-    const size_t parts = a.nchunk > 1 ? pairs * a.nchunk * group : 0;
+    const size_t parts = (pairs - static_cast<size_t>(sp.whole)) * a.nchunk * group;
     const size_t o_bytes = round_up(parts * d * sizeof(float), 256);
     const size_t need = kCounterBytes + o_bytes + parts * 2 * sizeof(float);
     if ((pairs + 2) * sizeof(int) > kCounterBytes || need > kNoallocScratchBytes)
         return PBB_ERR_SCRATCH_LIMIT;
-    a.total_items = static_cast<int>(pairs * a.nchunk);
+    a.total_items = static_cast<int>(static_cast<size_t>(sp.whole) + (pairs - static_cast<size_t>(sp.whole)) * a.nchunk);
     unsigned char* base = nullptr;
     const int rc = scratch_address(dev, &base);
     if (rc != PBB_OK) return rc;
     a.ctl = reinterpret_cast<int*>(base);
     a.counters = reinterpret_cast<int*>(base) + 2;
-    if (a.nchunk > 1) {
+    if (parts > 0) {
         a.part_o = reinterpret_cast<float*>(base + kCounterBytes);
         a.part_ml = reinterpret_cast<float*>(base + kCounterBytes + o_bytes);
     }
