@@ -14,6 +14,8 @@ arrays. What each function computes is stated in the C file and below:
 * ``attend``           Eq. (attention), brute force over a history window.
 * ``RingSim``          the relocation-free ring of Appendix F.1 (slot s mod b)
                        and a ring-indexed second evaluation over [a(t), t].
+* ``in_window``, ``window_count``, ``attend_window``
+                       sliding-window attention (Sec. 2.3), the comparison pattern.
 """
 from __future__ import annotations
 
@@ -72,6 +74,12 @@ def _load():
         lib.pbb_oracle_ring_replay.restype = None
         lib.pbb_oracle_attend_ring.argtypes = [P, P, P, P, I, P, I, I, I, I, L, P, I]
         lib.pbb_oracle_attend_ring.restype = I
+        lib.pbb_oracle_in_window.argtypes = [L, L, L]
+        lib.pbb_oracle_in_window.restype = I
+        lib.pbb_oracle_window_count.argtypes = [L, L]
+        lib.pbb_oracle_window_count.restype = L
+        lib.pbb_oracle_attend_window.argtypes = [P, P, P, P, P, L, I, I, I, I, L, P, I]
+        lib.pbb_oracle_attend_window.restype = I
         lib.pbb_oracle_max_threads.argtypes = []
         lib.pbb_oracle_max_threads.restype = I
         _lib = lib
@@ -141,6 +149,34 @@ def attend(q, hist_k, hist_v, s0, t, b: int, n_threads: int = 0) -> np.ndarray:
                                    batch, Hq, Hkv, d, b, _ptr(out), n_threads)
     if rc != ORACLE_OK:
         raise OracleError(f"pbb_oracle_attend returned {rc}")
+    return out
+
+
+def in_window(t: int, s: int, w: int) -> bool:
+    """Sliding window (Sec. 2.3): s in {max(0, t-w+1), ..., t}."""
+    return bool(_load().pbb_oracle_in_window(t, s, w))
+
+
+def window_count(t: int, w: int) -> int:
+    return int(_load().pbb_oracle_window_count(t, w))
+
+
+def attend_window(q, hist_k, hist_v, s0, t, w: int, n_threads: int = 0) -> np.ndarray:
+    """Brute-force sliding-window attention (window w, current position included);
+    same arguments and layout as ``attend``."""
+    q = _f64(q)
+    hk = _f64(hist_k)
+    hv = _f64(hist_v)
+    batch, Hq, d = q.shape
+    _, Hkv, n_hist, d2 = hk.shape
+    assert d2 == d and hv.shape == hk.shape and hk.shape[0] == batch
+    s0a = np.ascontiguousarray(np.broadcast_to(np.asarray(s0, dtype=np.int64), (batch,)))
+    ta = np.ascontiguousarray(np.broadcast_to(np.asarray(t, dtype=np.int64), (batch,)))
+    out = np.zeros((batch, Hq, d), dtype=np.float64)
+    rc = _load().pbb_oracle_attend_window(_ptr(q), _ptr(hk), _ptr(hv), _ptr(s0a), _ptr(ta), n_hist,
+                                          batch, Hq, Hkv, d, w, _ptr(out), n_threads)
+    if rc != ORACLE_OK:
+        raise OracleError(f"pbb_oracle_attend_window returned {rc}")
     return out
 
 

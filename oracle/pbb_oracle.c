@@ -16,7 +16,9 @@
  *   - the relocation-free ring of Appendix F.1 (Proposition "Relocation-free
  *     PBB cache"): position s is stored in slot s mod b; and a second,
  *     ring-indexed evaluation of the same attention over the interval form
- *     [a(t), t], a(t) = max(0, h(floor(t/h) - 1)) (Eq. pbb_relay, App. A.3).
+ *     [a(t), t], a(t) = max(0, h(floor(t/h) - 1)) (Eq. pbb_relay, App. A.3);
+ *   - sliding-window attention over {t-w+1, ..., t} (Sec. 2.3), the pattern
+ *     the paper compares PBB with, for the window-ring decode control.
  *
  * The brute-force evaluation visits every s in [0, t] and tests the support
  * predicate in its block/bridge form; it never uses the interval form, so the
@@ -126,6 +128,76 @@ int pbb_oracle_attend(const double* q, const double* hist_k, const double* hist_
         for (long s = 0; s <= tb && !bad; ++s) {
             if (!pbb_oracle_in_support(tb, s, b)) continue;
             if (s < s0[bi] || s >= s0[bi] + n_hist || n >= b + 1) { bad = 1; break; }
+            src[n++] = s;
+        }
+        if (bad) {
+#pragma omp critical
+            status = ORACLE_ERR_WINDOW;
+            free(src);
+            continue;
+        }
+        const double** kr = (const double**)malloc(sizeof(double*) * (size_t)n);
+        const double** vr = (const double**)malloc(sizeof(double*) * (size_t)n);
+        double* z = (double*)malloc(sizeof(double) * (size_t)n);
+        for (int j = 0; j < Hq; ++j) {
+            const int kv = j / group;
+            const size_t head = ((size_t)bi * Hkv + kv) * (size_t)n_hist;
+            for (long i = 0; i < n; ++i) {
+                const size_t row = head + (size_t)(src[i] - s0[bi]);
+                kr[i] = hist_k + row * d;
+                vr[i] = hist_v + row * d;
+            }
+            softmax_attend(q + ((size_t)bi * Hq + j) * d, kr, vr, n, d, z,
+                           out + ((size_t)bi * Hq + j) * d);
+        }
+        free(z);
+        free(vr);
+        free(kr);
+        free(src);
+    }
+    return status;
+}
+
+/*
+ * Sliding-window attention, the comparison pattern of the paper (Sec. 2.3,
+ * Proposition "Sliding-window relay"): A_SWA(t) = {max(0, t-w+1), ..., t}, the
+ * window w counting the current position. Same brute-force evaluation as
+ * pbb_oracle_attend (predicate at every s in [0, t], fp64, two passes).
+ */
+int pbb_oracle_in_window(long t, long s, long w)
+{
+    return s >= 0 && s <= t && s >= t - w + 1;
+}
+
+long pbb_oracle_window_count(long t, long w)
+{
+    long n = 0;
+    for (long s = 0; s <= t; ++s) n += pbb_oracle_in_window(t, s, w);
+    return n;
+}
+
+int pbb_oracle_attend_window(const double* q, const double* hist_k, const double* hist_v,
+                             const long* s0, const long* t, long n_hist, int batch, int Hq,
+                             int Hkv, int d, long w, double* out, int n_threads)
+{
+    if (batch < 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || w < 1 || (Hq % Hkv) || n_hist <= 0)
+        return ORACLE_ERR_ARG;
+    const int group = Hq / Hkv;
+    int status = ORACLE_OK;
+#ifdef _OPENMP
+    if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+    (void)n_threads;
+#endif
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int bi = 0; bi < batch; ++bi) {
+        const long tb = t[bi];
+        long* src = (long*)malloc(sizeof(long) * (size_t)(w + 1));
+        long n = 0;
+        int bad = (tb < 0);
+        for (long s = 0; s <= tb && !bad; ++s) {
+            if (!pbb_oracle_in_window(tb, s, w)) continue;
+            if (s < s0[bi] || s >= s0[bi] + n_hist || n >= w + 1) { bad = 1; break; }
             src[n++] = s;
         }
         if (bad) {

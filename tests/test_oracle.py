@@ -369,3 +369,63 @@ def test_ring_detects_missing_source(oracle_mod):
             ring.append(one, one, t)
     with pytest.raises(oracle_mod.OracleError):
         ring.attend(np.zeros((1, 1, 2)), 9)
+
+
+# ---------------------------------------------------------- sliding window --
+
+
+def test_window_score_count_at_8192(oracle_mod):
+    """Sec. 3 / App. A.5: SWA-128 uses 1,040,448 scores at n = 8192 (counted by brute force)."""
+    g = load("paper_counts.json")
+    n, w = g["n"], 128
+    assert sum(oracle_mod.window_count(t, w) for t in range(n)) == g["E_SWA"]
+
+
+@pytest.mark.parametrize("w", [1, 2, 5, 16])
+def test_window_predicate(oracle_mod, w):
+    for t in range(40):
+        for s in range(-2, t + 3):
+            assert oracle_mod.in_window(t, s, w) == (max(0, t - w + 1) <= s <= t)
+
+
+def test_pbb_support_inside_the_window(oracle_mod):
+    """App. A.4: with w = b = 2h every PBB source is an SWA source."""
+    b = 16
+    for t in range(8 * b):
+        for s in range(t + 1):
+            if oracle_mod.in_support(t, s, b):
+                assert oracle_mod.in_window(t, s, b)
+
+
+def test_window_attention_matches_scipy(oracle_mod):
+    from scipy.special import softmax
+
+    rng = np.random.default_rng(21)
+    batch, Hq, Hkv, d, w, n = 2, 4, 2, 8, 6, 30
+    q, k, v = _rand_problem(rng, batch, Hq, Hkv, d, n)
+    ts = np.array([3, 29])
+    o = oracle_mod.attend_window(q, k, v, s0=0, t=ts, w=w)
+    for bi in range(batch):
+        t = int(ts[bi])
+        lo = max(0, t - w + 1)
+        for j in range(Hq):
+            kv = j // (Hq // Hkv)
+            z = k[bi, kv, lo:t + 1] @ q[bi, j] / math.sqrt(d)
+            ref = softmax(z) @ v[bi, kv, lo:t + 1]
+            assert np.allclose(o[bi, j], ref, rtol=1e-13, atol=1e-13)
+
+
+def test_window_hand_values(oracle_mod):
+    """w = 4 at the Fig. 1 size: uniform weights give the mean of the last 4 positions;
+    at t = 4 SWA reads {1,2,3,4} (mean 5/2) where PBB reads {2,3,4} (mean 3)."""
+    T = 8
+    s = np.arange(T, dtype=np.float64)
+    v = s.reshape(1, 1, T, 1)
+    k = np.zeros_like(v)
+    q = np.zeros((1, 1, 1))
+    for t in range(T):
+        o = oracle_mod.attend_window(q, k, v, s0=0, t=t, w=4)
+        lo = max(0, t - 3)
+        assert abs(o[0, 0, 0] - (lo + t) / 2) < 1e-12
+    assert abs(oracle_mod.attend_window(q, k, v, s0=0, t=4, w=4)[0, 0, 0] - 2.5) < 1e-12
+    assert abs(oracle_mod.attend(q, k, v, s0=0, t=4, b=4)[0, 0, 0] - 3.0) < 1e-12
