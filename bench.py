@@ -15,6 +15,9 @@ position advance. Prints one JSON line (rank 0):
 
 --impl reference times the fp64 CPU oracle (the only reference this method has)
 on a bounded sample per step. --sweep prints one line per throughput-sweep point.
+--pattern swa times the sliding-window control (window B, same rings and
+kernel family) instead, --pattern both prints the PBB line and then the
+control's; the control lines carry their own metric name.
 """
 from __future__ import annotations
 
@@ -34,6 +37,7 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "PBB decode-core tokens*heads/s"
+METRIC_SWA = "SWA-B decode-core tokens*heads/s (control: window = B over the same ring)"
 UNIT = "tokens*heads/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
@@ -57,6 +61,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--chunk", type=int, default=0, help="keys per CTA (0 = library plan)")
+    ap.add_argument("--pattern", choices=["pbb", "swa", "both"], default="pbb",
+                    help="attention pattern: PBB (default), the sliding-window control with window B, or both")
     ap.add_argument("--graph", choices=["auto", "on", "off"], default="auto",
                     help="replay the timed steps as one CUDA graph (auto: when a step is under 100 us, "
                          "where host launch overhead would otherwise dominate)")
@@ -167,10 +173,8 @@ def recorded_traffic(workload_key: str, launch_bytes: float):
             rec = json.load(f)
     except (OSError, ValueError):
         return None
-    if rec.get("kernel_source_sha") != kernel_source_sha():
-        return None
     entry = rec.get("workloads", {}).get(workload_key)
-    if not entry:
+    if not entry or entry.get("kernel_source_sha") != kernel_source_sha():
         return None
     return entry["dram_bytes_per_launch"] / entry["algorithmic_bytes_per_launch"] * launch_bytes
 
@@ -202,7 +206,16 @@ def setup_device_workload(w, dev, pool: int):
     return t0, pos, k_ring, v_ring, steps_in
 
 
-def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
+def stepper(window):
+    """The decode call of a pattern: PBB (window None) or the sliding window."""
+    import paper_2606_02680_gb300 as pbb
+
+    if window is None:
+        return pbb.decode_step
+    return lambda q, k, v, kr, vr, pos, out: pbb.swa_decode_step(q, k, v, kr, vr, pos, out, window=window)
+
+
+def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None):
     """Device-timed loop; returns dict of timings.
 
     Eager mode records a CUDA event pair around every decode launch inside the
@@ -216,13 +229,14 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
     from paper_2606_02680_gb300 import bytemodel
 
     pool = 8
+    decode = stepper(window)
     t0, pos, k_ring, v_ring, steps_in = setup_device_workload(w, dev, pool)
     out = torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32, device=dev)
     pbb.reserve_workspace(w.batch, w.Hq, w.Hkv, w.d, w.B)
     stream = torch.cuda.current_stream()
     for i in range(warmup):
         q, k, v = steps_in[i % pool]
-        pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+        decode(q, k, v, k_ring, v_ring, pos, out)
         pbb.advance_positions(pos)
     torch.cuda.synchronize()
     if graph == "auto":  # a short eager probe decides
@@ -230,7 +244,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
         e0.record(stream)
         for i in range(3):
             q, k, v = steps_in[i % pool]
-            pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+            decode(q, k, v, k_ring, v_ring, pos, out)
             pbb.advance_positions(pos)
         e1.record(stream)
         torch.cuda.synchronize()
@@ -247,7 +261,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
         with torch.cuda.graph(g, stream=cap):
             for i in range(steps):
                 q, k, v = steps_in[(warmup + i) % pool]
-                pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+                decode(q, k, v, k_ring, v_ring, pos, out)
                 pbb.advance_positions(pos)
         stream.wait_stream(cap)
         torch.cuda.synchronize()
@@ -267,7 +281,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
             for i in range(steps):
                 q, k, v = steps_in[(warmup + i) % pool]
                 ev[2 * i].record(stream)
-                pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+                decode(q, k, v, k_ring, v_ring, pos, out)
                 ev[2 * i + 1].record(stream)
                 pbb.advance_positions(pos)
         end.record(stream)
@@ -286,12 +300,12 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
         for i in range(steps):
             q, k, v = steps_in[(first + i) % pool]
             ev[2 * i].record(stream)
-            pbb.decode_step(q, k, v, k_ring, v_ring, pos, out)
+            decode(q, k, v, k_ring, v_ring, pos, out)
             ev[2 * i + 1].record(stream)
             pbb.advance_positions(pos)
         torch.cuda.synchronize()
     kern_ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
-    launch_bytes = [bytemodel.step_bytes(t_np + first + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes)
+    launch_bytes = [bytemodel.step_bytes(t_np + first + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes, window)
                     for i in range(steps)]
     res = {
         "total_ms": total_ms,
@@ -308,7 +322,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto"):
     return res
 
 
-def time_e2e(w, dev, steps, state):
+def time_e2e(w, dev, steps, state, window=None):
     """Same steps through the host-memory API: every step copies its q/k/v in from
     pinned host memory and its output back, inside the timed region; the
     transfers of a step overlap the kernels of its neighbours (HostPipeline)."""
@@ -321,7 +335,8 @@ def time_e2e(w, dev, steps, state):
     host = [tuple(x.cpu().pin_memory() for x in s) for s in steps_in]
     out_h = [torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32).pin_memory() for _ in range(4)]
     stream = torch.cuda.current_stream()
-    pipe = pbb.HostPipeline(w.batch, w.Hq, w.Hkv, w.d, k_ring.dtype, dev, compute_stream=stream)
+    pipe = pbb.HostPipeline(w.batch, w.Hq, w.Hkv, w.d, k_ring.dtype, dev, compute_stream=stream,
+                            window=window)
     for i in range(3):
         q, k, v = host[i % pool]
         pipe.step(q, k, v, k_ring, v_ring, pos, out_h[i % 4])
@@ -458,17 +473,24 @@ def run_ours(args):
             w0 = w0.with_(Hq=hq, Hkv=hkv, name=f"{w0.name}_Hq{hq}_Hkv{hkv}")
         points = [w0]
     peak, peak_kind = hbm_peak()
-    for w in points:
-        batch, B = w.batch, w.B
-        res = time_device(w, dev, args.steps, args.warmup, dist, args.graph)
+    patterns = {"pbb": ["pbb"], "swa": ["swa"], "both": ["pbb", "swa"]}[args.pattern]
+    for w, pattern in [(w, p) for w in points for p in patterns]:
+        window = w.B if pattern == "swa" else None
+        res = time_device(w, dev, args.steps, args.warmup, dist, args.graph, window)
         total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
         units = sum_over_ranks(dist, w.batch * w.Hq * args.steps)
         value = units / total_s
         achieved = res["launch_bytes_mean"] / (res["kernel_ms_mean"] / 1e3) / 1e9
-        key = w.name
+        key = w.name if window is None else f"{w.name}_swa"
         traffic = recorded_traffic(key, res["launch_bytes_mean"])
+        if window is None:
+            kernel = ("decode_kernel_tc<%d>" % w.d
+                      if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w)) == "tensor_cores"
+                      else "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group))
+        else:
+            kernel = "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group)
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "metric": METRIC if window is None else METRIC_SWA, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": w.dtype,
             "data": "synthetic (seeded N(0,1) K/V/q; rings prefilled consistent with each t0)",
@@ -483,10 +505,7 @@ def run_ours(args):
             "frac_of_8tbs": achieved / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": traffic,
-                         "kernel": ("decode_kernel_tc<%d>" % w.d
-                                    if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w))
-                                    == "tensor_cores" else
-                                    "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group)),
+                         "kernel": kernel,
                          "peak_kind": peak_kind,
                          "algorithmic_bytes_per_launch": res["launch_bytes_mean"],
                          "kernel_ms_mean": res["kernel_ms_mean"],
@@ -496,10 +515,12 @@ def run_ours(args):
             "gpu_launches": 2 * args.steps,
         }
         if not args.no_e2e and not args.sweep:
-            line["e2e"] = time_e2e(w, dev, args.steps, res["state"])
+            line["e2e"] = time_e2e(w, dev, args.steps, res["state"], window)
         res.pop("state")
         torch.cuda.empty_cache()
-        if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep:
+        if window is not None:
+            line["config"]["window"] = window
+        if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep and window is None:
             line["cpu_baseline"] = oracle_sample(w, args.cpu_seconds)
         if rank == 0:
             print(json.dumps(line), flush=True)

@@ -56,7 +56,7 @@ typedef enum { PBB_BF16 = 0, PBB_F32 = 1 } pbb_dtype;
 
 enum {
     PBB_OK = 0,
-    PBB_ERR_INVALID_ARG = -1,    /* null or misaligned pointer, negative size */
+    PBB_ERR_INVALID_ARG = -1,    /* null or misaligned pointer, negative size, window outside [1, B] */
     PBB_ERR_UNSUPPORTED = -2,    /* B odd/out of range, Hq % Hkv != 0, group or d not supported */
     PBB_ERR_CUDA = -3,           /* a CUDA runtime call or a launch failed */
     PBB_ERR_DEVICE_TIMEOUT = -4, /* a kernel's bounded wait on a bulk copy ran out */
@@ -129,6 +129,26 @@ int pbb_decode_step_f32(const float* q, const float* k_new, const float* v_new, 
                         float* v_ring, const int32_t* pos, float* out, int batch, int Hq,
                         int Hkv, int d, int B, cudaStream_t stream);
 
+/*
+ * Sliding-window attention decode step over the same rings: the control the
+ * paper compares PBB with (Sec. 2.3; Sec. 3 notes that SWA with w = B can also
+ * live in a B-slot ring). Identical to pbb_decode_step / pbb_decode_step_f32
+ * (element type `dtype`) except for the support, which is the window
+ *
+ *     A_SWA(t) = {max(0, t-w+1), ..., t},   w = window, 1 <= w <= B,
+ *
+ * the current token included. Same ring contents and precondition: the step
+ * writes k_new/v_new into slot t mod B, which holds position t-B, outside the
+ * window. A ring can be switched between the two kinds of step at any
+ * position. Runs on the CUDA-core kernel for every group size. Returns
+ * PBB_ERR_INVALID_ARG for a window outside [1, B]. pbb_reserve_workspace
+ * covers window steps with window = B; for a smaller window make one step
+ * outside any stream capture first.
+ */
+int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
+                        void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
+                        int d, int B, int window, pbb_dtype dtype, cudaStream_t stream);
+
 /* pos[b] += 1 for every sequence, on the device (advances a decode loop, e.g. in a graph). */
 int pbb_advance_positions(int32_t* pos, int batch, cudaStream_t stream);
 
@@ -156,7 +176,7 @@ int pbb_set_wait_timeout_ns(unsigned long long ns);
  */
 int pbb_set_chunk_keys(int keys);
 
-/* Keys per CTA a decode step of this shape would use on the current device (0 on error). */
+/* Keys per CTA a PBB decode step of this shape would use on the current device (0 on error). */
 int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
 
 /*

@@ -11,6 +11,7 @@ Names follow the C ABI:
 * ``ring_bytes``, ``ring_alloc`` / ``Rings``   the B-slot K/V rings (Appendix F.1)
 * ``ring_prefill``                             load a ring from a history window
 * ``decode_step``                              append + attention over A(t) (Sec. 3)
+* ``swa_decode_step``                          the sliding-window control over the same rings
 * ``decode_step_host``, ``HostPipeline``       the same with host-resident inputs/outputs
                                                (one at a time / overlapped across steps)
 * ``advance_positions``, ``get_device_status``, ``reserve_workspace``,
@@ -28,7 +29,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step",
+    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -56,6 +57,7 @@ EXPORTS = {
     "pbb_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_swa_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
     "pbb_get_device_status": (_I, [_P]),
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),
@@ -195,14 +197,7 @@ def ring_prefill(k_hist: torch.Tensor, v_hist: torch.Tensor, pos: torch.Tensor,
                                   _stream(stream)), "pbb_ring_prefill")
 
 
-def decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_ring: torch.Tensor,
-                v_ring: torch.Tensor, pos: torch.Tensor, out: torch.Tensor | None = None,
-                stream=None) -> torch.Tensor:
-    """One PBB decode step (include/pbb.h: pbb_decode_step / pbb_decode_step_f32).
-
-    q [batch, Hq, d], k_new/v_new [batch, Hkv, d], rings [batch, Hkv, B, d] (bf16 or
-    fp32, all the same), pos [batch] int32 on the device, out [batch, Hq, d] fp32.
-    """
+def _step_shapes(q, k_new, v_new, k_ring, v_ring, pos, out):
     batch, Hq, d = q.shape
     _, Hkv, B, d2 = k_ring.shape
     dtype = q.dtype
@@ -216,11 +211,38 @@ def decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_rin
         out = torch.empty((batch, Hq, d), dtype=torch.float32, device=q.device)
     elif tuple(out.shape) != (batch, Hq, d):
         raise ValueError("out must be [batch, Hq, d]")
+    return batch, Hq, Hkv, d, B, dtype, out
+
+
+def decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_ring: torch.Tensor,
+                v_ring: torch.Tensor, pos: torch.Tensor, out: torch.Tensor | None = None,
+                stream=None) -> torch.Tensor:
+    """One PBB decode step (include/pbb.h: pbb_decode_step / pbb_decode_step_f32).
+
+    q [batch, Hq, d], k_new/v_new [batch, Hkv, d], rings [batch, Hkv, B, d] (bf16 or
+    fp32, all the same), pos [batch] int32 on the device, out [batch, Hq, d] fp32.
+    """
+    batch, Hq, Hkv, d, B, dtype, out = _step_shapes(q, k_new, v_new, k_ring, v_ring, pos, out)
     fn = lib().pbb_decode_step if _dt(dtype) == PBB_BF16 else lib().pbb_decode_step_f32
     _check(fn(_dev(q, "q", dtype), _dev(k_new, "k_new", dtype), _dev(v_new, "v_new", dtype),
               _dev(k_ring, "k_ring", dtype), _dev(v_ring, "v_ring", dtype),
               _dev(pos, "pos", torch.int32), _dev(out, "out", torch.float32), batch, Hq, Hkv, d, B,
               _stream(stream)), "pbb_decode_step")
+    return out
+
+
+def swa_decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_ring: torch.Tensor,
+                    v_ring: torch.Tensor, pos: torch.Tensor, out: torch.Tensor | None = None,
+                    window: int | None = None, stream=None) -> torch.Tensor:
+    """Sliding-window decode step over the same rings (pbb_swa_decode_step): the
+    support is {t-w+1, ..., t}, w = window (default B). Arguments as ``decode_step``."""
+    batch, Hq, Hkv, d, B, dtype, out = _step_shapes(q, k_new, v_new, k_ring, v_ring, pos, out)
+    w = B if window is None else int(window)
+    _check(lib().pbb_swa_decode_step(_dev(q, "q", dtype), _dev(k_new, "k_new", dtype),
+                                     _dev(v_new, "v_new", dtype), _dev(k_ring, "k_ring", dtype),
+                                     _dev(v_ring, "v_ring", dtype), _dev(pos, "pos", torch.int32),
+                                     _dev(out, "out", torch.float32), batch, Hq, Hkv, d, B, w,
+                                     _dt(dtype), _stream(stream)), "pbb_swa_decode_step")
     return out
 
 
@@ -263,7 +285,9 @@ class HostPipeline:
     Call ``synchronize()`` before reading the host outputs.
     """
 
-    def __init__(self, batch: int, Hq: int, Hkv: int, d: int, dtype, device, compute_stream=None):
+    def __init__(self, batch: int, Hq: int, Hkv: int, d: int, dtype, device, compute_stream=None,
+                 window: int | None = None):
+        self.window = window  # None: PBB steps; an integer: sliding-window steps of that window
         self.compute = torch.cuda.current_stream(device) if compute_stream is None else compute_stream
         self.copy_in = torch.cuda.Stream(device=device)
         self.copy_out = torch.cuda.Stream(device=device)
@@ -286,7 +310,11 @@ class HostPipeline:
             st.v.copy_(v_h, non_blocking=True)
             self.inputs_ready[j].record(self.copy_in)
         self.compute.wait_event(self.inputs_ready[j])
-        decode_step(st.q, st.k, st.v, k_ring, v_ring, pos, st.out, stream=self.compute)
+        if self.window is None:
+            decode_step(st.q, st.k, st.v, k_ring, v_ring, pos, st.out, stream=self.compute)
+        else:
+            swa_decode_step(st.q, st.k, st.v, k_ring, v_ring, pos, st.out, window=self.window,
+                            stream=self.compute)
         self.inputs_used[j].record(self.compute)
         self.output_ready[j].record(self.compute)
         advance_positions(pos, stream=self.compute)

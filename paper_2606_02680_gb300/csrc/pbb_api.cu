@@ -97,13 +97,15 @@ int min_split_keys(int d, int elem, int tile)
 
 namespace pbb {
 
-SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group)
+SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int window)
 {
     SplitPlan sp{0, 0, 1};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) dev = 0;
     const int tile = pbb::tile_keys(elem, d, group);
-    const int max_keys = B - 1 > 0 ? B - 1 : 1;
+    // ring keys of the longest support: B-1 for PBB (phase B-1), w-1 for a window of w
+    const int span = window > 0 ? window - 1 : B - 1;
+    const int max_keys = span > 0 ? span : 1;
     const long long pairs = static_cast<long long>(batch) * Hkv;
     auto finish = [&](long long split) {
         const long long max_split = (max_keys + min_split_keys(d, elem, tile) - 1) / min_split_keys(d, elem, tile);
@@ -126,7 +128,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group)
         sp.nchunk = (max_keys + chunk - 1) / chunk;
         return sp;
     }
-    int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B);
+    int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B, window);
     if (per_sm <= 0) per_sm = 1;
     const long long G = static_cast<long long>(sm_count(dev)) * per_sm;
     if (pairs >= G) {
@@ -135,7 +137,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group)
         // (measured: +29 % at B 4096 and +6 % at B 2048, but -12 to -15 % at B <= 1024 and
         // -19 % for the tensor-core kernel, whose two consumer warps combine slowly).
         const bool long_supports = max_keys >= 2047 && pbb::tile_keys(elem, d, group) == tile &&
-                                   !(elem == 2 && group == 8 && B % 64 == 0);
+                                   !(window == 0 && elem == 2 && group == 8 && B % 64 == 0);
         if (R == 0 || 2 * R > G || !long_supports) {  // no split
             sp.whole = static_cast<int>(pairs);
             sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
@@ -201,10 +203,11 @@ int grow_workspace(int dev, size_t pairs, size_t pbytes, cudaStream_t stream, bo
 
 int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_ring, void* v_ring,
                 const int32_t* pos, float* out, int batch, int Hq, int Hkv, int d, int B,
-                pbb_dtype dt, cudaStream_t stream)
+                int window, pbb_dtype dt, cudaStream_t stream)
 {
     int rc = check_shape(batch, Hkv, d, B, dt);
     if (rc != PBB_OK) return rc;
+    if (window < 0 || window > B) return PBB_ERR_INVALID_ARG;
     rc = check_group(Hq, Hkv);
     if (rc != PBB_OK) return rc;
     if (batch == 0) return PBB_OK;
@@ -231,7 +234,8 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
-    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, group);
+    a.window = window;
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, group, window);
     a.whole = sp.whole;
     a.chunk = sp.chunk;
     a.nchunk = sp.nchunk;
@@ -333,13 +337,16 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
     if (rc != PBB_OK) return rc;
     const int elem = elem_size(dtype);
     const int group = Hq / Hkv;
-    // Every batch up to max_batch: the plan's split depends on the batch.
+    // Every batch up to max_batch (the plan's split depends on the batch), for
+    // PBB steps and for window steps with window = B.
     size_t need = 0;
     for (int bsz = 1; bsz <= max_batch; ++bsz) {
-        const pbb::SplitPlan sp = pbb::plan_split(bsz, Hkv, d, B, elem, group);
-        if (static_cast<size_t>(sp.whole) >= static_cast<size_t>(bsz) * Hkv) continue;
-        const size_t w = parts_bytes(bsz, Hkv, d, group, sp);
-        if (w > need) need = w;
+        for (int window : {0, B}) {
+            const pbb::SplitPlan sp = pbb::plan_split(bsz, Hkv, d, B, elem, group, window);
+            if (static_cast<size_t>(sp.whole) >= static_cast<size_t>(bsz) * Hkv) continue;
+            const size_t w = parts_bytes(bsz, Hkv, d, group, sp);
+            if (w > need) need = w;
+        }
     }
     std::lock_guard<std::mutex> lock(g_mutex);
     return grow_workspace(dev, static_cast<size_t>(max_batch) * Hkv + 2, need, nullptr, false);
@@ -349,7 +356,7 @@ int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k
                     void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
                     int d, int B, cudaStream_t stream)
 {
-    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, PBB_BF16,
+    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, 0, PBB_BF16,
                        stream);
 }
 
@@ -357,8 +364,17 @@ int pbb_decode_step_f32(const float* q, const float* k_new, const float* v_new, 
                         float* v_ring, const int32_t* pos, float* out, int batch, int Hq,
                         int Hkv, int d, int B, cudaStream_t stream)
 {
-    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, PBB_F32,
+    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, 0, PBB_F32,
                        stream);
+}
+
+int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
+                        void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
+                        int d, int B, int window, pbb_dtype dtype, cudaStream_t stream)
+{
+    if (window < 1) return PBB_ERR_INVALID_ARG;
+    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, window,
+                       dtype, stream);
 }
 
 int pbb_advance_positions(int32_t* pos, int batch, cudaStream_t stream)
@@ -406,7 +422,7 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
     if (check_shape(batch, Hkv, d, B, dtype) != PBB_OK || check_group(Hq, Hkv) != PBB_OK) return 0;
     int dev = 0;
     if (current_device(&dev) != PBB_OK) return 0;
-    return pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv).chunk;
+    return pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, 0).chunk;
 }
 
 int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
@@ -424,7 +440,7 @@ int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
-    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv);
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, 0);
     a.chunk = sp.chunk;
     return pbb::use_tensor_cores(a, elem_size(dtype)) ? PBB_KERNEL_TENSOR_CORES : PBB_KERNEL_CUDA_CORES;
 }
@@ -433,7 +449,7 @@ const char* pbb_error_string(int code)
 {
     switch (code) {
         case PBB_OK: return "ok";
-        case PBB_ERR_INVALID_ARG: return "invalid argument (null or misaligned pointer, negative size)";
+        case PBB_ERR_INVALID_ARG: return "invalid argument (null or misaligned pointer, negative size, window outside [1, B])";
         case PBB_ERR_UNSUPPORTED: return "unsupported shape (B odd or out of range, Hq % Hkv != 0, group or d not supported)";
         case PBB_ERR_CUDA: return "CUDA runtime error";
         case PBB_ERR_DEVICE_TIMEOUT: return "a kernel's bounded wait on a bulk copy ran out";

@@ -341,6 +341,31 @@ __device__ __forceinline__ float reduce_scatter(float (&v)[G])
     return v[0];
 }
 
+// The ring keys of a support, i.e. all of it but the current token t (which
+// comes from k_new/v_new). r = t mod B is the slot the step writes.
+//   window == 0, PBB (Eq. pbb_relay, Appendix F.1): positions a(t) .. t-1,
+//     n = h + r keys from slot h in a bridge phase (p > 0, r < h), else the r
+//     keys of slots 0 .. r-1.
+//   window == w in [1, B], the sliding window {t-w+1, ..., t} (Sec. 2.3):
+//     n = min(t, w-1) keys from slot (t-n) mod B; the run may wrap past slot
+//     B-1. Slot r holds position t-B <= t-w, outside the window.
+// In both cases ring key i (position t-n+i) lives in slot (base + i) mod B.
+__device__ __forceinline__ void support_keys(int t, int B, int window, int& r, int& n, int& base)
+{
+    const int blk = t / B;
+    r = t - blk * B;
+    if (window > 0) {
+        n = min(t, window - 1);
+        base = r - n;
+        if (base < 0) base += B;
+    } else {
+        const int h = B >> 1;
+        const bool bridge = (blk > 0) && (r < h);
+        n = bridge ? h + r : r;
+        base = bridge ? h : 0;
+    }
+}
+
 // 2^x with the SFU instruction (flushes subnormal results to zero; 2^-inf = 0).
 __device__ __forceinline__ float fast_exp2(float x)
 {
@@ -587,12 +612,9 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
                     continue;
                 }
-                const int B = a.B, h = B >> 1;
-                const int blk = t / B;
-                const int r = t - blk * B;
-                const bool bridge = (blk > 0) && (r < h);
-                const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
-                const int base = bridge ? h : 0;   // slot of ring key 0
+                const int B = a.B;
+                int r, n, base;  // slot of t; ring keys of the support (positions t-n .. t-1); slot of key 0
+                support_keys(t, B, a.window, r, n, base);
                 const bool whole = pair < a.whole;
                 const int csize = whole ? max(n, 1) : a.chunk;  // keys per chunk of this support
                 const int nch = n > 0 ? (n + csize - 1) / csize : 1;
@@ -1469,7 +1491,9 @@ int occupancy_tc()
 // coordinates within int32.
 bool tc_eligible(const DecodeArgs& a, int elem_bytes)
 {
-    if (elem_bytes != 2 || a.Hq != 8 * a.Hkv || (a.d != 64 && a.d != 128)) return false;
+    // PBB only: its tiles start at multiples of the tile in slot order (slots 0 and
+    // h), which whole TMA boxes need; a window's run starts at any slot.
+    if (a.window != 0 || elem_bytes != 2 || a.Hq != 8 * a.Hkv || (a.d != 64 && a.d != 128)) return false;
     constexpr int tk = 16 * kTcConsumers;
     if (a.B % (2 * tk) != 0 || a.chunk % tk != 0) return false;
     const unsigned long long rows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.B;
@@ -1543,9 +1567,9 @@ int tile_keys(int elem_bytes, int d, int group)
     return 0;
 }
 
-int decode_ctas_per_sm(int elem_bytes, int d, int group, int B)
+int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window)
 {
-    if (elem_bytes == 2 && group == 8 && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
+    if (window == 0 && elem_bytes == 2 && group == 8 && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
         tensor_map_encoder() != nullptr)
         return d == 64 ? occupancy_tc<64>() : occupancy_tc<128>();
     if (elem_bytes == 2 && d == 64) return occupancy_g<2, 64>(group);

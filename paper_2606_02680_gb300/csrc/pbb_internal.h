@@ -24,6 +24,7 @@ struct DecodeArgs {
     int* counters;       // [batch][Hkv]                 finished chunks per (sequence, KV head)
     int* ctl;            // [2] work-queue head and finished CTAs; zero between launches
     int batch, Hq, Hkv, d, B;
+    int window;          // 0: the PBB support [a(t), t]; w in [1, B]: the sliding window {t-w+1, ..., t}
     int whole;           // supports [0, whole) are one work item each
     int chunk;           // ring keys per work item of the later supports (a multiple of the tile)
     int nchunk;          // work items per later support = ceil((B-1)/chunk)
@@ -35,14 +36,15 @@ struct DecodeArgs {
 int tile_keys(int elem_bytes, int d, int group);
 
 // Resident CTAs per SM of the decode kernel a step of this shape runs (0 if unsupported).
-int decode_ctas_per_sm(int elem_bytes, int d, int group, int B);
+int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window);
 
 // The split plan of a step (see plan_split in pbb_api.cu): supports [0, whole)
-// run whole, every later one in nchunk chunks of `chunk` ring keys.
+// run whole, every later one in nchunk chunks of `chunk` ring keys. window as
+// in DecodeArgs (0 = PBB).
 struct SplitPlan {
     int whole, chunk, nchunk;
 };
-SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem_bytes, int group);
+SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem_bytes, int group, int window);
 
 // Whether launch_decode would run the tensor-core kernel for these arguments.
 bool use_tensor_cores(const DecodeArgs& a, int elem_bytes);

@@ -37,12 +37,31 @@ def ring_bytes_np(t: torch.Tensor) -> np.ndarray:
     return iv.numpy().view(np.uint8).reshape(*t.shape[:-1], -1)
 
 
+def _decode(q, k, v, k_ring, v_ring, pos, window):
+    """PBB step (window None) or sliding-window step of `window` positions."""
+    if window is None:
+        return pbb.decode_step(q, k, v, k_ring, v_ring, pos)
+    return pbb.swa_decode_step(q, k, v, k_ring, v_ring, pos, window=window)
+
+
+def _expected(q, hk, hv, t, B, window):
+    """Oracle output over history rows of positions t-B .. t (PBB or window)."""
+    if window is None:
+        return oracle.attend(q, hk, hv, s0=t - B, t=t, b=B)
+    return oracle.attend_window(q, hk, hv, s0=t - B, t=t, w=window)
+
+
 class SequentialRun:
     """Drive the GPU decode step over consecutive steps of a workload and keep the
-    host copy of the history the oracle needs (start window + every new token)."""
+    host copy of the history the oracle needs (start window + every new token).
+    window=None runs PBB steps, an integer runs sliding-window steps of that
+    window; ``step(window=...)`` overrides it for one step."""
 
-    def __init__(self, w: inputs.Workload, device="cuda", prefill: bool = True, gen_device="cpu"):
+    def __init__(self, w: inputs.Workload, device="cuda", prefill: bool = True, gen_device="cpu",
+                 window=None):
         self.w = w
+        self.window = window
+        self.last_window = window
         self.dev = torch.device(device)
         self.dtype = inputs.torch_dtype(w)
         self.t0 = inputs.start_positions(w)
@@ -62,14 +81,16 @@ class SequentialRun:
         self.step_i = 0
         self.q_last = None
 
-    def step(self, gen_device="cpu"):
+    def step(self, gen_device="cpu", window="default"):
         w, i = self.w, self.step_i
+        win = self.window if window == "default" else window
         q, k, v = inputs.step_inputs(w, i, device=gen_device)
         q, k, v = q.cpu(), k.cpu(), v.cpu()
         self.hk[:, :, w.B + i] = k
         self.hv[:, :, w.B + i] = v
-        out = pbb.decode_step(q.to(self.dev), k.to(self.dev), v.to(self.dev), self.k_ring,
-                              self.v_ring, self.pos)
+        out = _decode(q.to(self.dev), k.to(self.dev), v.to(self.dev), self.k_ring, self.v_ring,
+                      self.pos, win)
+        self.last_window = win
         pbb.advance_positions(self.pos)
         self.sim.append(k, v, (self.t0 + i).numpy())
         self.q_last = q
@@ -91,7 +112,7 @@ class SequentialRun:
         hk = self.hk[:, :, lo:w.B + i + 1].index_select(0, sel)
         hv = self.hv[:, :, lo:w.B + i + 1].index_select(0, sel)
         t = self.t_now()[seqs]
-        return oracle.attend(self.q_last[seqs], hk, hv, s0=t - w.B, t=t, b=w.B)
+        return _expected(self.q_last[seqs], hk, hv, t, w.B, self.last_window)
 
     def check_rings(self) -> None:
         assert np.array_equal(ring_bytes_np(self.k_ring), self.sim.k), "K ring differs from the oracle's"
@@ -103,8 +124,9 @@ class DeviceRun:
     on the GPU; the oracle checks a sample of sequences, whose history rows and
     step inputs are copied back to the host."""
 
-    def __init__(self, w: inputs.Workload, sample, device="cuda"):
+    def __init__(self, w: inputs.Workload, sample, device="cuda", window=None):
         self.w = w
+        self.window = window
         self.dev = torch.device(device)
         self.dtype = inputs.torch_dtype(w)
         self.sample = np.asarray(sample)
@@ -129,7 +151,7 @@ class DeviceRun:
     def step(self):
         w, i = self.w, self.step_i
         q, k, v = inputs.step_inputs(w, i, device=self.dev)
-        out = pbb.decode_step(q, k, v, self.k_ring, self.v_ring, self.pos)
+        out = _decode(q, k, v, self.k_ring, self.v_ring, self.pos, self.window)
         pbb.advance_positions(self.pos)
         idx = torch.as_tensor(self.sample, device=self.dev)
         ks, vs = k.index_select(0, idx).cpu(), v.index_select(0, idx).cpu()
@@ -145,7 +167,7 @@ class DeviceRun:
         hk = torch.cat(self.hk, dim=2)[:, :, i:w.B + i + 1]
         hv = torch.cat(self.hv, dim=2)[:, :, i:w.B + i + 1]
         t = (self.t0[self.sample] + i).numpy()
-        return oracle.attend(self.q_last, hk, hv, s0=t - w.B, t=t, b=w.B)
+        return _expected(self.q_last, hk, hv, t, w.B, self.window)
 
     def check_rings(self) -> None:
         idx = torch.as_tensor(self.sample, device=self.dev)

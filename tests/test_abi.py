@@ -113,3 +113,13 @@ def test_product_path_does_not_use_the_oracle():
                 text = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in text and "from oracle" not in text, f
                 assert "pbb_oracle" not in text, f
+
+
+def test_window_checked_before_launch(pbb):
+    """pbb_swa_decode_step: a window outside [1, B] is refused before anything
+    else; batch 0 with a valid window is a no-op (no device work)."""
+    lib = pbb.lib()
+    for window, code in ((0, -1), (-1, -1), (129, -1), (1, 0), (128, 0)):
+        rc = lib.pbb_swa_decode_step(None, None, None, None, None, None, None, 0, 8, 2, 128, 128,
+                                     window, 0, None)
+        assert rc == code, (window, rc)
