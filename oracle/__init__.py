@@ -1,4 +1,5 @@
-"""fp64 CPU oracle for the Post-Boundary Bridge (PBB) decode step.
+"""fp64 CPU oracle for Post-Boundary Bridge (PBB) attention: the decode step and
+the whole-sequence forward.
 
 TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
 benchmark's CPU-baseline leg may import this package; the product path
@@ -16,6 +17,8 @@ arrays. What each function computes is stated in the C file and below:
                        and a ring-indexed second evaluation over [a(t), t].
 * ``in_window``, ``window_count``, ``attend_window``
                        sliding-window attention (Sec. 2.3), the comparison pattern.
+* ``forward``          PBB attention for every position of whole sequences (the
+                       forward pass / prefill), with the log-partition of Eq. (lse).
 """
 from __future__ import annotations
 
@@ -80,6 +83,8 @@ def _load():
         lib.pbb_oracle_window_count.restype = L
         lib.pbb_oracle_attend_window.argtypes = [P, P, P, P, P, L, I, I, I, I, L, P, I]
         lib.pbb_oracle_attend_window.restype = I
+        lib.pbb_oracle_forward_rows.argtypes = [P, P, P, I, I, I, L, I, L, P, L, P, P, I]
+        lib.pbb_oracle_forward_rows.restype = I
         lib.pbb_oracle_max_threads.argtypes = []
         lib.pbb_oracle_max_threads.restype = I
         _lib = lib
@@ -178,6 +183,36 @@ def attend_window(q, hist_k, hist_v, s0, t, w: int, n_threads: int = 0) -> np.nd
     if rc != ORACLE_OK:
         raise OracleError(f"pbb_oracle_attend_window returned {rc}")
     return out
+
+
+def forward(q, k, v, b: int, rows=None, n_threads: int = 0):
+    """PBB attention for whole sequences (Sec. 3, Eq. attention over A_PBB(t) for every t).
+
+    q: [batch, Hq, n, d]; k, v: [batch, Hkv, n, d] (row s = position s). rows: None for every
+    (sequence, head, position), else an int array [n_rows, 3] of (sequence, query head, t).
+    Returns (out, lse): out [batch, Hq, n, d] and lse [batch, Hq, n] for rows=None, else
+    [n_rows, d] and [n_rows]; lse = ln sum_{s in A(t)} exp(z_ts) (natural log).
+    """
+    q = _f64(q)
+    kk = _f64(k)
+    vv = _f64(v)
+    batch, Hq, n, d = q.shape
+    _, Hkv, n2, d2 = kk.shape
+    assert n2 == n and d2 == d and vv.shape == kk.shape and kk.shape[0] == batch
+    full = rows is None
+    if full:
+        bi, j, t = np.meshgrid(np.arange(batch), np.arange(Hq), np.arange(n), indexing="ij")
+        rows = np.stack([bi.ravel(), j.ravel(), t.ravel()], axis=1)
+    rows = np.ascontiguousarray(np.asarray(rows, dtype=np.int64).reshape(-1, 3))
+    out = np.zeros((rows.shape[0], d), dtype=np.float64)
+    lse = np.zeros(rows.shape[0], dtype=np.float64)
+    rc = _load().pbb_oracle_forward_rows(_ptr(q), _ptr(kk), _ptr(vv), batch, Hq, Hkv, n, d, b,
+                                         _ptr(rows), rows.shape[0], _ptr(out), _ptr(lse), n_threads)
+    if rc != ORACLE_OK:
+        raise OracleError(f"pbb_oracle_forward_rows returned {rc}")
+    if full:
+        return out.reshape(batch, Hq, n, d), lse.reshape(batch, Hq, n)
+    return out, lse
 
 
 class RingSim:

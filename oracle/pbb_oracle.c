@@ -1,5 +1,6 @@
 /*
- * Post-Boundary Bridge (PBB) decode step: plain fp64 CPU oracle.
+ * Post-Boundary Bridge (PBB) attention (decode step and whole-sequence
+ * forward): plain fp64 CPU oracle.
  *
  * TEST INFRASTRUCTURE ONLY. Nothing on the product path may link, load or call
  * this file: only the tests, the smoke check and the benchmark's CPU-baseline
@@ -18,7 +19,9 @@
  *     ring-indexed evaluation of the same attention over the interval form
  *     [a(t), t], a(t) = max(0, h(floor(t/h) - 1)) (Eq. pbb_relay, App. A.3);
  *   - sliding-window attention over {t-w+1, ..., t} (Sec. 2.3), the pattern
- *     the paper compares PBB with, for the window-ring decode control.
+ *     the paper compares PBB with, for the window-ring decode control;
+ *   - PBB attention for every position of whole sequences (the forward pass /
+ *     prefill of Sec. 3) with its log-partition ln sum exp(z) (Eq. lse).
  *
  * The brute-force evaluation visits every s in [0, t] and tests the support
  * predicate in its block/bridge form; it never uses the interval form, so the
@@ -71,7 +74,7 @@ long pbb_oracle_support_count(long t, long b)
  */
 static void softmax_attend(const double* q, const double* const* k_rows,
                            const double* const* v_rows, long n, int d,
-                           double* z, double* out)
+                           double* z, double* out, double* lse)
 {
     const double scale = 1.0 / sqrt((double)d);
     double m = -INFINITY;
@@ -89,6 +92,7 @@ static void softmax_attend(const double* q, const double* const* k_rows,
         for (int c = 0; c < d; ++c) out[c] += w * v_rows[i][c];
     }
     for (int c = 0; c < d; ++c) out[c] /= den;
+    if (lse) *lse = m + log(den); /* ln sum_s exp(z_s), the log-partition of Eq. (lse) */
 }
 
 /*
@@ -148,7 +152,7 @@ int pbb_oracle_attend(const double* q, const double* hist_k, const double* hist_
                 vr[i] = hist_v + row * d;
             }
             softmax_attend(q + ((size_t)bi * Hq + j) * d, kr, vr, n, d, z,
-                           out + ((size_t)bi * Hq + j) * d);
+                           out + ((size_t)bi * Hq + j) * d, NULL);
         }
         free(z);
         free(vr);
@@ -156,6 +160,68 @@ int pbb_oracle_attend(const double* q, const double* hist_k, const double* hist_
         free(src);
     }
     return status;
+}
+
+/*
+ * PBB attention over whole sequences (Sec. 3): every position t of a sequence
+ * attends to A_PBB(t) among that sequence's positions 0..n-1 with the single
+ * softmax of Eq. (attention). This is what the paper's fused forward kernel
+ * computes for all t at once (the training forward, and the prefill that
+ * precedes decoding); here it is evaluated one requested output row at a time.
+ *
+ *   q     [batch][Hq][n][d]   row t is the query of position t
+ *   k, v  [batch][Hkv][n][d]  row s is the key / value of position s
+ *   rows  [n_rows][3]         (sequence, query head, position t) of each row
+ *   out   [n_rows][d]
+ *   lse   [n_rows]            ln sum_{s in A(t)} exp(z_ts), the log-partition a
+ *                             backward pass reuses (Eq. lse); NULL to skip
+ *
+ * Query head j reads KV head j / (Hq/Hkv). The predicate is tested at every
+ * s in [0, t] (block/bridge form), as in pbb_oracle_attend.
+ */
+int pbb_oracle_forward_rows(const double* q, const double* k, const double* v, int batch, int Hq,
+                            int Hkv, long n, int d, long b, const long* rows, long n_rows,
+                            double* out, double* lse, int n_threads)
+{
+    if (batch < 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || n <= 0 || b < 2 || (b % 2) || (Hq % Hkv) ||
+        n_rows < 0)
+        return ORACLE_ERR_ARG;
+    for (long i = 0; i < n_rows; ++i) {
+        const long* rw = rows + 3 * i;
+        if (rw[0] < 0 || rw[0] >= batch || rw[1] < 0 || rw[1] >= Hq || rw[2] < 0 || rw[2] >= n)
+            return ORACLE_ERR_ARG;
+    }
+    const int group = Hq / Hkv;
+#ifdef _OPENMP
+    if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+    (void)n_threads;
+#endif
+#pragma omp parallel for schedule(dynamic, 16)
+    for (long i = 0; i < n_rows; ++i) {
+        const long bi = rows[3 * i], j = rows[3 * i + 1], t = rows[3 * i + 2];
+        const long kv = j / group;
+        const double** kr = (const double**)malloc(sizeof(double*) * (size_t)(b + 1));
+        const double** vr = (const double**)malloc(sizeof(double*) * (size_t)(b + 1));
+        double* z = (double*)malloc(sizeof(double) * (size_t)(b + 1));
+        const size_t head = ((size_t)bi * Hkv + (size_t)kv) * (size_t)n;
+        long m = 0;
+        for (long s = 0; s <= t; ++s) {
+            if (!pbb_oracle_in_support(t, s, b)) continue;
+            if (m < b + 1) { /* |A(t)| <= b always (Eq. pbb_cache_support) */
+                kr[m] = k + (head + (size_t)s) * d;
+                vr[m] = v + (head + (size_t)s) * d;
+            }
+            ++m;
+        }
+        if (m > b) m = b + 1; /* cannot happen; keeps the buffers in bounds */
+        softmax_attend(q + (((size_t)bi * Hq + (size_t)j) * (size_t)n + (size_t)t) * d, kr, vr, m, d, z,
+                       out + (size_t)i * d, lse ? lse + i : NULL);
+        free(z);
+        free(vr);
+        free(kr);
+    }
+    return ORACLE_OK;
 }
 
 /*
@@ -218,7 +284,7 @@ int pbb_oracle_attend_window(const double* q, const double* hist_k, const double
                 vr[i] = hist_v + row * d;
             }
             softmax_attend(q + ((size_t)bi * Hq + j) * d, kr, vr, n, d, z,
-                           out + ((size_t)bi * Hq + j) * d);
+                           out + ((size_t)bi * Hq + j) * d, NULL);
         }
         free(z);
         free(vr);
@@ -346,7 +412,7 @@ int pbb_oracle_attend_ring(const double* q, const uint8_t* ring_k, const uint8_t
             for (int g = 0; g < group; ++g) {
                 const int j = kv * group + g;
                 softmax_attend(q + ((size_t)bi * Hq + j) * d, kr, vr, n, d, z,
-                               out + ((size_t)bi * Hq + j) * d);
+                               out + ((size_t)bi * Hq + j) * d, NULL);
             }
         }
         free(z);

@@ -429,3 +429,93 @@ def test_window_hand_values(oracle_mod):
         assert abs(o[0, 0, 0] - (lo + t) / 2) < 1e-12
     assert abs(oracle_mod.attend_window(q, k, v, s0=0, t=4, w=4)[0, 0, 0] - 2.5) < 1e-12
     assert abs(oracle_mod.attend(q, k, v, s0=0, t=4, b=4)[0, 0, 0] - 3.0) < 1e-12
+
+
+# ------------------------------------------------ whole-sequence forward --
+
+
+def test_forward_equals_decode_oracle_at_every_position(oracle_mod):
+    """The forward at position t is the decode step at t over the same history
+    (attend, pinned above): same support, same softmax."""
+    rng = np.random.default_rng(31)
+    batch, Hq, Hkv, d, b, n = 2, 4, 2, 8, 8, 40
+    q = rng.standard_normal((batch, Hq, n, d))
+    k = rng.standard_normal((batch, Hkv, n, d))
+    v = rng.standard_normal((batch, Hkv, n, d))
+    out, _ = oracle_mod.forward(q, k, v, b)
+    for t in range(n):
+        ref = oracle_mod.attend(q[:, :, t], k[:, :, :t + 1], v[:, :, :t + 1], s0=0, t=t, b=b)
+        assert np.array_equal(out[:, :, t], ref), t
+
+
+def test_forward_matches_scipy_with_log_partition(oracle_mod):
+    """scipy softmax and logsumexp over the interval form [a(t), t] (Eq. pbb_relay)."""
+    from scipy.special import logsumexp, softmax
+
+    rng = np.random.default_rng(32)
+    batch, Hq, Hkv, d, b, n = 1, 6, 3, 4, 6, 31
+    q = rng.standard_normal((batch, Hq, n, d))
+    k = rng.standard_normal((batch, Hkv, n, d))
+    v = rng.standard_normal((batch, Hkv, n, d))
+    out, lse = oracle_mod.forward(q, k, v, b)
+    for j in range(Hq):
+        kv = j // (Hq // Hkv)
+        for t in range(n):
+            a = interval_start(t, b)
+            z = k[0, kv, a:t + 1] @ q[0, j, t] / math.sqrt(d)
+            assert np.allclose(out[0, j, t], softmax(z) @ v[0, kv, a:t + 1], rtol=1e-13, atol=1e-13)
+            assert abs(lse[0, j, t] - logsumexp(z)) < 1e-12
+
+
+def test_forward_zero_query_closed_form(oracle_mod):
+    """q = 0: every weight is equal, so lse = ln |A(t)| with |A(t)| = h + 1 + (t mod h)
+    after the first block (Eq. pbb_cache_support), and out is the support's mean of V."""
+    rng = np.random.default_rng(33)
+    b, d, n = 16, 3, 100
+    h = b // 2
+    k = rng.standard_normal((1, 1, n, d))
+    v = rng.standard_normal((1, 1, n, d))
+    out, lse = oracle_mod.forward(np.zeros((1, 1, n, d)), k, v, b)
+    for t in range(n):
+        size = t + 1 if t < b else h + 1 + t % h
+        assert abs(lse[0, 0, t] - math.log(size)) < 1e-12
+        assert np.allclose(out[0, 0, t], v[0, 0, interval_start(t, b):t + 1].mean(axis=0), atol=1e-13)
+
+
+def test_forward_hand_values(oracle_mod):
+    """Hand-derived outputs of the Fig. 1 size (b = 4) for every position of one sequence."""
+    g = load("hand_b4.json")
+    b, T = g["b"], 12
+    s = np.arange(T, dtype=np.float64)
+    v = s.reshape(1, 1, T, 1)
+    for case, (qv, kv) in {"uniform weights": (0.0, np.zeros_like(s)),
+                           "weights 3 and 1": (1.0, np.where(s % 2 == 0, math.log(3.0), 0.0))}.items():
+        c = next(c for c in g["cases"] if c["name"] == case)
+        out, _ = oracle_mod.forward(np.full((1, 1, T, 1), qv), kv.reshape(1, 1, T, 1), v, b)
+        for t in range(T):
+            assert abs(out[0, 0, t, 0] - _frac(c["out"][t])) < 1e-12, (case, t)
+
+
+def test_forward_first_position(oracle_mod):
+    """t = 0: the support is {0}: out = v_0 exactly and lse = z_00 = q_0.k_0/sqrt(d)."""
+    rng = np.random.default_rng(34)
+    q = rng.standard_normal((2, 4, 5, 16))
+    k = rng.standard_normal((2, 2, 5, 16))
+    v = rng.standard_normal((2, 2, 5, 16))
+    out, lse = oracle_mod.forward(q, k, v, 4)
+    for j in range(4):
+        assert np.array_equal(out[:, j, 0], v[:, j // 2, 0])
+        assert np.allclose(lse[:, j, 0], (q[:, j, 0] * k[:, j // 2, 0]).sum(-1) / 4.0, atol=1e-14)
+
+
+def test_forward_rows_subset(oracle_mod):
+    """Requested rows equal the same rows of the full evaluation."""
+    rng = np.random.default_rng(35)
+    q = rng.standard_normal((2, 4, 20, 8))
+    k = rng.standard_normal((2, 1, 20, 8))
+    v = rng.standard_normal((2, 1, 20, 8))
+    out, lse = oracle_mod.forward(q, k, v, 8)
+    rows = np.array([[0, 0, 0], [1, 3, 19], [0, 2, 7], [1, 1, 8]])
+    o2, l2 = oracle_mod.forward(q, k, v, 8, rows=rows)
+    for i, (bi, j, t) in enumerate(rows):
+        assert np.array_equal(o2[i], out[bi, j, t]) and l2[i] == lse[bi, j, t]
