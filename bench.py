@@ -17,7 +17,9 @@ position advance. Prints one JSON line (rank 0):
 on a bounded sample per step. --sweep prints one line per throughput-sweep point.
 --pattern swa times the sliding-window control (window B, same rings and
 kernel family) instead, --pattern both prints the PBB line and then the
-control's; the control lines carry their own metric name.
+control's; the control lines carry their own metric name. --forward times the
+whole-sequence forward (prefill) workloads, one line each, with a roofline
+against HBM or the tensor cores, whichever bounds the workload.
 """
 from __future__ import annotations
 
@@ -38,6 +40,7 @@ if ROOT not in sys.path:
 
 METRIC = "PBB decode-core tokens*heads/s"
 METRIC_SWA = "SWA-B decode-core tokens*heads/s (control: window = B over the same ring)"
+METRIC_FWD = "PBB forward tokens*heads/s"
 UNIT = "tokens*heads/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
@@ -63,6 +66,9 @@ def parse_args():
     ap.add_argument("--chunk", type=int, default=0, help="keys per CTA (0 = library plan)")
     ap.add_argument("--pattern", choices=["pbb", "swa", "both"], default="pbb",
                     help="attention pattern: PBB (default), the sliding-window control with window B, or both")
+    ap.add_argument("--forward", action="store_true",
+                    help="time the whole-sequence forward (prefill) workloads instead of the decode step")
+    ap.add_argument("--fwd-workload", default="", help="one forward workload (default: all)")
     ap.add_argument("--graph", choices=["auto", "on", "off"], default="auto",
                     help="replay the timed steps as one CUDA graph (auto: when a step is under 100 us, "
                          "where host launch overhead would otherwise dominate)")
@@ -154,10 +160,10 @@ def hbm_peak():
 
 
 def kernel_source_sha() -> str:
-    """Hash of the decode kernel's source (the file the ncu traffic record depends on)."""
+    """Hash of the decode kernel's source (the files the ncu traffic record depends on)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2606_02680_gb300", "csrc")
-    for name in ("pbb_decode.cu", "pbb_internal.h"):
+    for name in ("pbb_decode.cu", "pbb_device.cuh", "pbb_internal.h"):
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode() + b"\0" + f.read())
     return h.hexdigest()[:16]
@@ -396,6 +402,184 @@ def oracle_sample(w, seconds: float, seqs_per_call: int = 8, max_calls: int | No
 
 # ------------------------------------------------------------------- arms --
 
+def forward_flops_bytes(w):
+    """Algorithmic FLOPs (4 d |A(t)| per query head and position: q.k and p.v, App. A.5)
+    and bytes (q, k, v read once; bf16 out and fp32 lse written once) of one forward."""
+    import numpy as np
+
+    from paper_2606_02680_gb300 import bytemodel
+
+    sizes = bytemodel.support_size(np.arange(w.n), w.B)
+    flops = 4 * w.d * w.batch * w.Hq * int(sizes.sum())
+    bytes_ = 2 * w.d * w.n * w.batch * (2 * w.Hq + 2 * w.Hkv) + 4 * w.batch * w.Hq * w.n
+    return flops, bytes_
+
+
+def tensor_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"]), "measured (cuBLAS bf16 burst)"
+    except (OSError, KeyError, ValueError):
+        return 1900.0, "fallback"
+
+
+def time_forward(w, dev, steps, warmup, dist=None):
+    """Eager forward launches with CUDA events around each; inputs resident in HBM."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import inputs
+
+    q, k, v = inputs.sequence_inputs(w, device=dev)
+    out = torch.empty((w.batch, w.Hq, w.n, w.d), dtype=torch.bfloat16, device=dev)
+    lse = torch.empty((w.batch, w.Hq, w.n), dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        pbb.forward(q, k, v, w.B, out=out, lse=lse)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:  # noqa: BLE001
+        pass
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clocks:
+        start.record(stream)
+        for i in range(steps):
+            ev[2 * i].record(stream)
+            pbb.forward(q, k, v, w.B, out=out, lse=lse)
+            ev[2 * i + 1].record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    if pbb.get_device_status() != pbb.PBB_OK:
+        raise RuntimeError("device status after the timed forward loop")
+    kern = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
+    return {"total_ms": start.elapsed_time(end), "kernel_ms_mean": sum(kern) / steps,
+            "kernel_ms_median": statistics.median(kern), "clocks": clocks.summary(),
+            "state": (q, k, v, out, lse)}
+
+
+def time_forward_e2e(w, dev, steps, state):
+    """Through the public API with host-resident inputs: each step copies q/k/v in from
+    pinned host memory, runs the forward and copies out/lse back (all on one stream)."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+
+    q, k, v, out, lse = state
+    hq, hk, hv = (x.cpu().pin_memory() for x in (q, k, v))
+    ho = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    hl = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    stream = torch.cuda.current_stream()
+
+    def step():
+        q.copy_(hq, non_blocking=True)
+        k.copy_(hk, non_blocking=True)
+        v.copy_(hv, non_blocking=True)
+        pbb.forward(q, k, v, w.B, out=out, lse=lse)
+        ho.copy_(out, non_blocking=True)
+        hl.copy_(lse, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        step()
+    end.record(stream)
+    end.synchronize()
+    ms = start.elapsed_time(end)
+    return {"value": w.batch * w.Hq * w.n * steps / (ms / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": sum(x.numel() * x.element_size() for x in (hq, hk, hv)),
+            "d2h_bytes_per_step": ho.numel() * ho.element_size() + hl.numel() * hl.element_size(),
+            "ms_per_step": ms / steps,
+            "api": "paper_2606_02680_gb300.forward (pinned host q/k/v in, out/lse back, one stream)"}
+
+
+def oracle_forward_sample(w, seconds: float, rows_per_call: int = 64):
+    """The fp64 oracle forward on sampled rows of the workload (one sequence, one KV head)."""
+    import numpy as np
+
+    import oracle
+    from paper_2606_02680_gb300 import inputs
+
+    oracle.build()
+    sub = w.with_(batch=1, Hq=w.group, Hkv=1)
+    q, k, v = inputs.sequence_inputs(sub)
+    rng = np.random.default_rng(0)
+    done, elapsed = 0, 0.0
+    while True:
+        rows = np.stack([np.zeros(rows_per_call, dtype=np.int64), rng.integers(0, sub.Hq, rows_per_call),
+                         rng.integers(0, w.n, rows_per_call)], axis=1)
+        t_start = time.perf_counter()
+        oracle.forward(q, k, v, w.B, rows=rows)
+        elapsed += time.perf_counter() - t_start
+        done += rows_per_call
+        if elapsed >= seconds:
+            break
+    return {"value": done / elapsed, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "seconds": elapsed,
+            "sample": f"{done} output rows (position, head) of {w.name}, uniform positions, fp64 brute "
+                      f"force over every position up to t (includes widening the slice to fp64)"}
+
+
+def run_forward(args, dist, rank, world, dev):
+    import torch
+
+    from paper_2606_02680_gb300 import inputs
+
+    names = [args.fwd_workload] if args.fwd_workload else list(inputs.FORWARD_WORKLOADS)
+    hbm, hbm_kind = hbm_peak()
+    tpk, tpk_kind = tensor_peak()
+    for name in names:
+        w = inputs.FORWARD_WORKLOADS[name]
+        w = w.with_(batch=shard_batch(w.batch, rank, world))
+        res = time_forward(w, dev, args.steps, args.warmup, dist)
+        total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
+        units = sum_over_ranks(dist, w.batch * w.Hq * w.n * args.steps)
+        flops, bytes_ = forward_flops_bytes(w)
+        kern_s = res["kernel_ms_mean"] / 1e3
+        t_hbm, t_tc = bytes_ / (hbm * 1e9), flops / (tpk * 1e12)
+        if t_tc >= t_hbm:
+            roof = {"bound": "tensor", "achieved": flops / kern_s / 1e12, "peak": tpk, "unit": "TFLOP/s",
+                    "peak_kind": tpk_kind}
+        else:
+            roof = {"bound": "hbm", "achieved": bytes_ / kern_s / 1e9, "peak": hbm, "unit": "GB/s",
+                    "peak_kind": hbm_kind}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        roof.update({"traffic": None, "kernel": "forward_kernel<%d,%d>" % (w.d, w.group),
+                     "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,
+                     "hbm_gbs": bytes_ / kern_s / 1e9, "tflops": flops / kern_s / 1e12,
+                     "kernel_ms_mean": res["kernel_ms_mean"], "kernel_ms_median": res["kernel_ms_median"]})
+        line = {
+            "metric": METRIC_FWD, "value": units / total_s, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,1) q/k/v)",
+            "config": {"workload": f"{w.name}: batch {w.batch}, Hq {w.Hq}, Hkv {w.Hkv}, d {w.d}, B {w.B}, n {w.n}, bf16 out + fp32 lse",
+                       "batch_per_gpu": w.batch, "Hq": w.Hq, "Hkv": w.Hkv, "head_dim": w.d, "block": w.B,
+                       "n": w.n, "l2": "inputs larger than L2: q/k/v/out %.2f GB" % (bytes_ / 1e9),
+                       "parallelism": f"dp{world} (independent sequences, no collective)"},
+            "roofline": roof, "clocks": res["clocks"],
+            "timing": "eager launches; CUDA events around every forward launch",
+            "gpu_launches": args.steps,
+        }
+        if not args.no_e2e:
+            line["e2e"] = time_forward_e2e(w, dev, min(args.steps, 10), res["state"])
+        res.pop("state")
+        torch.cuda.empty_cache()
+        if rank == 0 and world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = oracle_forward_sample(w, args.cpu_seconds)
+        if rank == 0:
+            print(json.dumps(line), flush=True)
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     if world <= 1:
@@ -460,6 +644,12 @@ def run_ours(args):
     torch.cuda.set_device(dev)
     pbb.set_chunk_keys(args.chunk)
 
+    if args.forward:
+        run_forward(args, dist, rank, world, dev)
+        if dist is not None:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
     if args.workload:
         base = inputs.WORKLOADS[args.workload]
         points = [base.with_(batch=shard_batch(base.batch, rank, world))]

@@ -1,6 +1,7 @@
 /*
  * libpbb: fused decode step of Post-Boundary Bridge (PBB) local attention on
- * one GPU (sm_103a).
+ * one GPU (sm_103a), with the sliding-window control and the whole-sequence
+ * forward (prefill) over the same support.
  *
  * The operation (Sec. 3, Eq. (pbb) and Eq. (attention); Appendix F.1):
  * a sequence whose current token sits at absolute position t, with block size
@@ -149,13 +150,45 @@ int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, voi
                         void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
                         int d, int B, int window, pbb_dtype dtype, cudaStream_t stream);
 
+/*
+ * PBB attention over whole sequences: the forward pass of the paper's fused
+ * training kernel and the prefill before decoding (Sec. 3, Eq. (attention) over
+ * A(t) for every position t; Appendix "exact union and numerical checks": block
+ * tiles and bridge rectangles under one softmax, native GQA, no dense mask).
+ * Every position t in [0, n) of a sequence attends to [a(t), t] of the same
+ * sequence, a(t) = max(0, h(floor(t/h) - 1)); positions start at 0.
+ *   q    [batch][Hq][n][d]   bf16, row t = query of position t (already rotated)
+ *   k, v [batch][Hkv][n][d]  bf16, row s = key / value of position s
+ *   out  [batch][Hq][n][d]   out_dtype (PBB_BF16 or PBB_F32)
+ *   lse  [batch][Hq][n]      fp32 ln sum_{s in A(t)} exp(q_t.k_s/sqrt(d)), the
+ *                            log-partition of Eq. (lse) a backward pass reuses;
+ *                            NULL to skip
+ * Device pointers owned by the caller; q, k, v, out 16-byte aligned. Same
+ * group and head-size rules as the decode step; batch*Hq*n < 2^31. Runs on the
+ * tensor cores (mma.sync, bf16 operands, fp32 accumulation; the softmax weights
+ * are rounded to bf16 before P.V). Asynchronous on `stream`; a bounded wait that
+ * runs out is reported by pbb_get_device_status as PBB_ERR_DEVICE_TIMEOUT.
+ */
+int pbb_forward(const void* q, const void* k, const void* v, void* out, float* lse, int batch, int Hq,
+                int Hkv, int n, int d, int B, pbb_dtype out_dtype, cudaStream_t stream);
+
+/*
+ * Load the decode rings of sequences whose first n positions went through
+ * pbb_forward (the cache-populating prefill, Appendix F.1): slot j of each ring
+ * receives the position s in [n-B, n-1] with s = j (mod B), zeros where s < 0.
+ * k, v [batch][Hkv][n][d] as for pbb_forward (may be NULL when n = 0). The next
+ * decode step is at position n. Bit copy; element type `dtype`.
+ */
+int pbb_ring_from_sequence(const void* k, const void* v, int n, void* k_ring, void* v_ring, int batch,
+                           int Hkv, int d, int B, pbb_dtype dtype, cudaStream_t stream);
+
 /* pos[b] += 1 for every sequence, on the device (advances a decode loop, e.g. in a graph). */
 int pbb_advance_positions(int32_t* pos, int batch, cudaStream_t stream);
 
 /*
- * Synchronise `stream`, then return and clear the device status word of the
- * current device: PBB_OK, PBB_ERR_DEVICE_TIMEOUT or PBB_ERR_DEVICE_POSITION
- * (first fault recorded since the last call). Clearing also resets the split
+ * Synchronise `stream`, then return and clear the device status words (decode
+ * and forward kernels) of the current device: PBB_OK, PBB_ERR_DEVICE_TIMEOUT or
+ * PBB_ERR_DEVICE_POSITION (first fault recorded since the last call). Clearing also resets the split
  * counters in the workspace, which an aborted step can leave behind.
  */
 int pbb_get_device_status(cudaStream_t stream);

@@ -12,6 +12,8 @@ Names follow the C ABI:
 * ``ring_prefill``                             load a ring from a history window
 * ``decode_step``                              append + attention over A(t) (Sec. 3)
 * ``swa_decode_step``                          the sliding-window control over the same rings
+* ``forward``, ``ring_from_sequence``          whole-sequence PBB attention (prefill / training
+                                               forward) and the rings it leaves for decoding
 * ``decode_step_host``, ``HostPipeline``       the same with host-resident inputs/outputs
                                                (one at a time / overlapped across steps)
 * ``advance_positions``, ``get_device_status``, ``reserve_workspace``,
@@ -29,7 +31,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step",
+    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step", "forward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -58,6 +60,8 @@ EXPORTS = {
     "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_swa_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
+    "pbb_forward": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
+    "pbb_ring_from_sequence": (_I, [_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
     "pbb_get_device_status": (_I, [_P]),
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),
@@ -332,6 +336,50 @@ class HostPipeline:
         self.copy_in.synchronize()
         self.compute.synchronize()
         self.copy_out.synchronize()
+
+
+def forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, B: int, out: torch.Tensor | None = None,
+            lse: torch.Tensor | bool | None = True, out_dtype=torch.bfloat16, stream=None):
+    """PBB attention for every position of whole sequences (pbb_forward).
+
+    q [batch, Hq, n, d], k/v [batch, Hkv, n, d] bf16 on the device; B the block size.
+    Returns (out [batch, Hq, n, d] out_dtype, lse [batch, Hq, n] fp32 or None).
+    lse: True allocates it, a tensor receives it, None/False skips it.
+    """
+    batch, Hq, n, d = q.shape
+    Hkv = k.shape[1]
+    if tuple(k.shape) != (batch, Hkv, n, d) or tuple(v.shape) != tuple(k.shape):
+        raise ValueError("k/v must be [batch, Hkv, n, d] with q's batch, n and d")
+    if out is None:
+        out = torch.empty((batch, Hq, n, d), dtype=out_dtype, device=q.device)
+    elif tuple(out.shape) != (batch, Hq, n, d):
+        raise ValueError("out must be [batch, Hq, n, d]")
+    if lse is True:
+        lse = torch.empty((batch, Hq, n), dtype=torch.float32, device=q.device)
+    elif lse is False:
+        lse = None
+    if lse is not None and tuple(lse.shape) != (batch, Hq, n):
+        raise ValueError("lse must be [batch, Hq, n]")
+    _check(lib().pbb_forward(_dev(q, "q", torch.bfloat16), _dev(k, "k", torch.bfloat16),
+                             _dev(v, "v", torch.bfloat16), _dev(out, "out", out.dtype),
+                             _dev(lse, "lse", torch.float32) if lse is not None else None,
+                             batch, Hq, Hkv, n, d, B, _dt(out.dtype), _stream(stream)), "pbb_forward")
+    return out, lse
+
+
+def ring_from_sequence(k: torch.Tensor, v: torch.Tensor, k_ring: torch.Tensor, v_ring: torch.Tensor,
+                       stream=None) -> None:
+    """Rings [batch, Hkv, B, d] of sequences whose positions 0..n-1 are k/v [batch, Hkv, n, d]
+    (pbb_ring_from_sequence); the next decode step is at position n."""
+    batch, Hkv, B, d = k_ring.shape
+    n = k.shape[2]
+    dtype = k_ring.dtype
+    if tuple(k.shape) != (batch, Hkv, n, d) or tuple(v.shape) != tuple(k.shape):
+        raise ValueError("k/v must be [batch, Hkv, n, d] matching the rings")
+    _check(lib().pbb_ring_from_sequence(_dev(k, "k", dtype), _dev(v, "v", dtype), n,
+                                        _dev(k_ring, "k_ring", dtype), _dev(v_ring, "v_ring", dtype),
+                                        batch, Hkv, d, B, _dt(dtype), _stream(stream)),
+           "pbb_ring_from_sequence")
 
 
 def advance_positions(pos: torch.Tensor, stream=None) -> None:

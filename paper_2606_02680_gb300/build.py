@@ -11,7 +11,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libpbb.so")
 OBJ_DIR = os.path.join(PKG, "_build")
-SOURCES = ("pbb_api.cu", "pbb_decode.cu", "pbb_noalloc.cu")
+SOURCES = ("pbb_api.cu", "pbb_decode.cu", "pbb_forward.cu", "pbb_noalloc.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -23,7 +23,8 @@ def _nvcc() -> str:
 
 def _inputs():
     files = [os.path.join(CSRC, s) for s in SOURCES]
-    files += [os.path.join(CSRC, "pbb_internal.h"), os.path.join(INCLUDE, "pbb.h")]
+    files += [os.path.join(CSRC, h) for h in sorted(os.listdir(CSRC)) if h.endswith((".h", ".cuh"))]
+    files += [os.path.join(INCLUDE, "pbb.h")]
     return files
 
 

@@ -377,6 +377,57 @@ int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, voi
                        dtype, stream);
 }
 
+int pbb_forward(const void* q, const void* k, const void* v, void* out, float* lse, int batch, int Hq,
+                int Hkv, int n, int d, int B, pbb_dtype out_dtype, cudaStream_t stream)
+{
+    int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
+    if (rc != PBB_OK) return rc;
+    rc = check_group(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    if (n < 0 || elem_size(out_dtype) == 0) return PBB_ERR_INVALID_ARG;
+    if (batch == 0 || n == 0) return PBB_OK;
+    // TMA row coordinates are 32-bit: every (sequence, head, position) row must fit
+    if (static_cast<long long>(batch) * Hq * n >= (1LL << 31)) return PBB_ERR_UNSUPPORTED;
+    if (!q || !k || !v || !out) return PBB_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16) ||
+        (lse != nullptr && !aligned(lse, 4)))
+        return PBB_ERR_INVALID_ARG;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    pbb::ForwardArgs a{};
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.out = out;
+    a.lse = lse;
+    a.batch = batch;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.n = n;
+    a.d = d;
+    a.B = B;
+    a.out_f32 = out_dtype == PBB_F32 ? 1 : 0;
+    a.timeout_ns = g_timeout_ns.load();
+    return pbb::launch_forward(a, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
+}
+
+int pbb_ring_from_sequence(const void* k, const void* v, int n, void* k_ring, void* v_ring, int batch,
+                           int Hkv, int d, int B, pbb_dtype dtype, cudaStream_t stream)
+{
+    int rc = check_shape(batch, Hkv, d, B, dtype);
+    if (rc != PBB_OK) return rc;
+    if (n < 0) return PBB_ERR_INVALID_ARG;
+    if (batch == 0) return PBB_OK;
+    if (!k_ring || !v_ring || (n > 0 && (!k || !v))) return PBB_ERR_INVALID_ARG;
+    if (!aligned(k_ring, 16) || !aligned(v_ring, 16) || (n > 0 && (!aligned(k, 16) || !aligned(v, 16))))
+        return PBB_ERR_INVALID_ARG;
+    return pbb::launch_seq_ring(k, v, k_ring, v_ring, batch, Hkv, n, B, d * elem_size(dtype), stream) ==
+                   cudaSuccess
+               ? PBB_OK
+               : PBB_ERR_CUDA;
+}
+
 int pbb_advance_positions(int32_t* pos, int batch, cudaStream_t stream)
 {
     if (batch < 0) return PBB_ERR_INVALID_ARG;
@@ -390,8 +441,10 @@ int pbb_get_device_status(cudaStream_t stream)
     int dev = 0;
     int rc = current_device(&dev);
     if (rc != PBB_OK) return rc;
-    int status = 0;
+    int status = 0, fwd_status = 0;
     if (pbb::read_and_clear_status(&status, stream) != cudaSuccess) return PBB_ERR_CUDA;
+    if (pbb::read_and_clear_forward_status(&fwd_status) != cudaSuccess) return PBB_ERR_CUDA;
+    if (status == pbb::kDevOk && fwd_status != pbb::kDevOk) return PBB_ERR_DEVICE_TIMEOUT;  // forward kernels only time out
     if (status == pbb::kDevOk) return PBB_OK;
     {
         // An aborted step can leave split counters behind: zero them.

@@ -55,6 +55,9 @@
 #include <cudaTypedefs.h>
 #include <stdint.h>
 
+#include <mutex>
+
+#include "pbb_device.cuh"
 #include "pbb_internal.h"
 
 namespace pbb {
@@ -97,144 +100,6 @@ struct __align__(16) TileMeta {
     int b, kvh, chunk, nk;  // item and ring keys in this tile
     int nch, r, flags, pad; // chunks of the support, phase, kFirst/kLast/kCurrent/kEnd
 };
-
-// ---------------------------------------------------------------- PTX ----
-
-__device__ __forceinline__ uint32_t smem_addr(const void* p)
-{
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count)
-                 : "memory");
-}
-
-__device__ __forceinline__ void fence_mbar_init()
-{
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async()
-{
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
-                 "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_addr(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ bool mbar_try(uint64_t* bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_addr(bar)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-__device__ __forceinline__ unsigned long long global_ns()
-{
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-    return t;
-}
-
-// Wait for phase `parity` of `bar` to complete, giving up after `limit_ns`.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
-                                          unsigned long long limit_ns)
-{
-    if (mbar_test(bar, parity)) return true;
-    if (limit_ns == 0) return false;
-    const unsigned long long t0 = global_ns();
-    while (!mbar_try(bar, parity)) {
-        if (global_ns() - t0 > limit_ns) return false;
-    }
-    return true;
-}
-
-// 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
-            "r"(smem_addr(dst)),
-        "l"(src), "r"(bytes), "r"(smem_addr(bar))
-        : "memory");
-}
-
-// 2-D tiled TMA load of one box at (x = column, y = row) of a tensor map, completion on `bar`.
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, int x, int y, uint64_t* bar)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::
-            "r"(smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(smem_addr(bar))
-        : "memory");
-}
-
-__device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(addr));
-}
-
-__device__ __forceinline__ void ldmatrix_x4_trans(uint32_t (&r)[4], uint32_t addr)
-{
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-                 : "r"(addr));
-}
-
-// Transpose of an 8x8 b16 matrix held in the m8n8 fragment layout.
-__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t x)
-{
-    uint32_t y;
-    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
-    return y;
-}
-
-// d += a (16x16, row) * b (16x8, col), bf16 inputs, fp32 accumulation.
-__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1)
-{
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-        "{%0, %1, %2, %3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
-// Two floats -> bf16x2 (round to nearest even): lo in the low half, hi in the high half.
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
-{
-    const __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<const uint32_t*>(&v);
-}
-
-__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
 
 // ---------------------------------------------------------- elements ----
 
@@ -364,19 +229,6 @@ __device__ __forceinline__ void support_keys(int t, int B, int window, int& r, i
         n = bridge ? h + r : r;
         base = bridge ? h : 0;
     }
-}
-
-// 2^x with the SFU instruction (flushes subnormal results to zero; 2^-inf = 0).
-__device__ __forceinline__ float fast_exp2(float x)
-{
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
 // Barrier of the consumer warps through a shared-memory counter, bounded by
@@ -968,9 +820,6 @@ struct TcCfg {
     static_assert(BOX_BYTES % 1024 == 0, "swizzle atoms");
 };
 
-// Byte offset of 16-byte chunk `c` (0..7) of row `r` in a box written with the 128-byte swizzle.
-__device__ __forceinline__ uint32_t swz(int r, int c) { return static_cast<uint32_t>(r * 128 + ((c ^ (r & 7)) << 4)); }
-
 template <int D>
 __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
     decode_kernel_tc(const DecodeArgs a, const __grid_constant__ CUtensorMap kmap,
@@ -1436,16 +1285,18 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
 
 // Map a ring [rows][d] bf16 as a 2-D tensor read in boxes of 64 columns x box_rows
 // rows with the 128-byte swizzle. Caches the last maps built (rings rarely move).
-bool ring_tensor_map(CUtensorMap* map, void* ring, unsigned long long rows, int d, int box_rows)
+bool ring_tensor_map(CUtensorMap* map, const void* ring, unsigned long long rows, int d, int box_rows)
 {
     struct Entry {
-        void* ring;
+        const void* ring;
         unsigned long long rows;
         int d, box_rows;
         CUtensorMap map;
     };
+    static std::mutex mu;
     static Entry cache[8];
     static int next = 0;
+    std::lock_guard<std::mutex> lock(mu);
     for (auto& e : cache)
         if (e.ring == ring && e.rows == rows && e.d == d && e.box_rows == box_rows) {
             *map = e.map;
@@ -1458,7 +1309,7 @@ bool ring_tensor_map(CUtensorMap* map, void* ring, unsigned long long rows, int 
     const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(box_rows)};
     const cuuint32_t estr[2] = {1, 1};
     CUtensorMap m;
-    if (enc(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ring, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+    if (enc(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ring), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) !=
         CUDA_SUCCESS)
         return false;
@@ -1616,6 +1467,11 @@ cudaError_t launch_advance(int32_t* pos, int batch, cudaStream_t stream)
     const int blocks = (batch + 255) / 256 < 64 ? (batch + 255) / 256 : 64;
     advance_kernel<<<blocks, 256, 0, stream>>>(pos, batch);
     return cudaGetLastError();
+}
+
+bool rows_tensor_map(CUtensorMap* map, const void* base, unsigned long long rows, int d, int box_rows)
+{
+    return ring_tensor_map(map, base, rows, d, box_rows);
 }
 
 cudaError_t read_and_clear_status(int* status, cudaStream_t stream)

@@ -2,6 +2,7 @@
 // (pbb_decode.cu). Not installed; the public interface is include/pbb.h.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime_api.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -61,5 +62,27 @@ cudaError_t launch_advance(int32_t* pos, int batch, cudaStream_t stream);
 
 // Read (and clear) the device status word of the current device.
 cudaError_t read_and_clear_status(int* status, cudaStream_t stream);
+
+// 2-D bf16 tensor map over `rows` rows of d elements read in boxes of 64
+// columns x box_rows rows with the 128-byte swizzle (cached; false if the
+// driver's encoder is unavailable or refuses).
+bool rows_tensor_map(CUtensorMap* map, const void* base, unsigned long long rows, int d, int box_rows);
+
+// Whole-sequence forward (pbb_forward.cu).
+struct ForwardArgs {
+    const void* q;   // [batch][Hq][n][d] bf16
+    const void* k;   // [batch][Hkv][n][d] bf16
+    const void* v;   // [batch][Hkv][n][d] bf16
+    void* out;       // [batch][Hq][n][d] bf16 or fp32 (out_f32)
+    float* lse;      // [batch][Hq][n] or null
+    int batch, Hq, Hkv, n, d, B;
+    int out_f32;
+    unsigned long long timeout_ns;
+};
+cudaError_t launch_forward(const ForwardArgs& a, cudaStream_t stream);
+cudaError_t launch_seq_ring(const void* k, const void* v, void* k_ring, void* v_ring, int batch, int Hkv,
+                            int n, int B, int row_bytes, cudaStream_t stream);
+// Status word of the forward kernels (read and cleared; the caller synchronises first).
+cudaError_t read_and_clear_forward_status(int* status);
 
 }  // namespace pbb

@@ -1,4 +1,4 @@
-"""Seeded synthetic workloads for the PBB decode step.
+"""Seeded synthetic workloads for the PBB decode step and the whole-sequence forward.
 
 This module only draws numbers: it holds none of the method's arithmetic (no
 support, no slot mapping, no attention). Both the CUDA path's tests and the
@@ -23,7 +23,7 @@ from typing import Optional, Tuple
 import torch
 
 __all__ = ["Workload", "WORKLOADS", "sweep_workload", "start_positions", "history_window",
-           "step_inputs", "torch_dtype"]
+           "step_inputs", "torch_dtype", "SequenceWorkload", "FORWARD_WORKLOADS", "sequence_inputs"]
 
 
 @dataclass(frozen=True)
@@ -140,3 +140,44 @@ def step_inputs_stacked(w: Workload, steps: int, device="cpu", first: int = 0):
     """Stacked inputs of `steps` consecutive decode steps: ([steps, ...] x 3)."""
     qs, ks, vs = zip(*(step_inputs(w, first + i, device) for i in range(steps)))
     return torch.stack(qs), torch.stack(ks), torch.stack(vs)
+
+
+@dataclass(frozen=True)
+class SequenceWorkload:
+    """Whole sequences for the forward pass: q [batch, Hq, n, d], k/v [batch, Hkv, n, d], bf16."""
+    name: str
+    batch: int
+    Hq: int
+    Hkv: int
+    d: int
+    B: int
+    n: int
+    outlier_frac: float = 0.0
+    outlier_scale: float = 1.0
+    seed: int = 0
+    dtype: str = "bf16"
+
+    @property
+    def group(self) -> int:
+        return self.Hq // self.Hkv
+
+    def with_(self, **kw) -> "SequenceWorkload":
+        return replace(self, **kw)
+
+
+FORWARD_WORKLOADS = {
+    # the paper's local-layer geometry (head dim 64, block 128) at 8K context, group 4
+    "fwd_b16_n8192_B128": SequenceWorkload("fwd_b16_n8192_B128", batch=16, Hq=8, Hkv=2, d=64, B=128,
+                                           n=8192, seed=40),
+    # the decode benchmark's heads (Hq 32, Hkv 8, d 128) with 4096-token blocks at 32K context
+    "fwd_b2_n32768_B4096": SequenceWorkload("fwd_b2_n32768_B4096", batch=2, Hq=32, Hkv=8, d=128, B=4096,
+                                            n=32768, seed=41),
+}
+
+
+def sequence_inputs(w: SequenceWorkload, device="cpu") -> Tuple[torch.Tensor, torch.Tensor, torch.Tensor]:
+    """(q [batch, Hq, n, d], k [batch, Hkv, n, d], v [batch, Hkv, n, d]) of a sequence workload."""
+    q = _normal((w.batch, w.Hq, w.n, w.d), w, device, 20)
+    k = _normal((w.batch, w.Hkv, w.n, w.d), w, device, 21, outliers=True)
+    v = _normal((w.batch, w.Hkv, w.n, w.d), w, device, 22, outliers=True)
+    return q, k, v
