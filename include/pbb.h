@@ -165,9 +165,10 @@ int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, voi
  *                            NULL to skip
  * Device pointers owned by the caller; q, k, v, out 16-byte aligned. Same
  * group and head-size rules as the decode step; batch*Hq*n < 2^31. Runs on the
- * tensor cores (mma.sync, bf16 operands, fp32 accumulation; the softmax weights
- * are rounded to bf16 before P.V). Asynchronous on `stream`; a bounded wait that
- * runs out is reported by pbb_get_device_status as PBB_ERR_DEVICE_TIMEOUT.
+ * fifth-generation tensor cores (tcgen05, bf16 operands, fp32 accumulation in
+ * tensor memory; the softmax weights are rounded to bf16 before P.V), one
+ * persistent CTA per SM. Asynchronous on `stream`; a bounded wait that runs out
+ * is reported by pbb_get_device_status as PBB_ERR_DEVICE_TIMEOUT.
  */
 int pbb_forward(const void* q, const void* k, const void* v, void* out, float* lse, int batch, int Hq,
                 int Hkv, int n, int d, int B, pbb_dtype out_dtype, cudaStream_t stream);

@@ -1,4 +1,5 @@
-// PBB attention over whole sequences (the forward pass / prefill) for sm_103a.
+// PBB attention over whole sequences (the forward pass / prefill) for sm_103a,
+// on the fifth-generation tensor cores (tcgen05, accumulators in TMEM).
 //
 // Every position t of a sequence attends to the interval [a(t), t],
 // a(t) = max(0, h(floor(t/h) - 1)) (Eq. pbb_relay, the interval form of
@@ -7,27 +8,42 @@
 // also gets its natural-log partition lse = ln sum exp(z) (Eq. lse), which a
 // backward pass reuses.
 //
-// Work. A CTA takes QT consecutive positions t0 .. t0+QT-1 of all G query
-// heads of one KV head: M = G*QT = 64 query rows, stacked head-major, so every
-// K/V tile it streams serves all G heads (native GQA, K/V read once per CTA).
-// Its keys are [a(t0), t_last]; a(t) only grows with t, so that range covers
-// every row, and rows whose support starts later or ends earlier are masked in
-// the tiles that cross their bounds (no dense mask exists anywhere).
+// Work items. An item is QT consecutive positions t0 .. t0+QT-1 of all G query
+// heads of one KV head: M = G*QT = 128 query rows, stacked head-major, so every
+// K/V tile serves all G heads (native GQA). Its keys are [a(t0), t_last] (a(t)
+// only grows with t, so the range covers every row), streamed in tiles of 128
+// keys; rows whose support starts later or ends earlier are masked in the tiles
+// that cross their bounds. No dense mask exists anywhere. Persistent CTAs, one
+// per SM, take items round-robin; query tiles of a head are adjacent items, so
+// CTAs running together share K/V tiles in L2.
 //
-// Data movement. One producer lane issues TMA tensor copies (128-byte swizzle,
-// boxes of 64 columns): first the Q rows of the CTA, then the K/V tiles of 64
-// keys into a STAGES-deep ring of full/empty mbarriers.
-//
-// Math. Four consumer warps own 16 query rows each and run FlashAttention-style
-// tiles on mma.sync m16n8k16 (bf16 operands, fp32 accumulation): S = Q K^T from
-// ldmatrix fragments of the swizzled tiles, an online softmax in the base-2
-// domain (log2(e)/sqrt(d) folded into one scale; the output is rescaled only
-// when a row's running maximum grows), P rounded to bf16 as the A operand of
-// O += P V with V fragments from ldmatrix.trans. The epilogue divides by the
-// row sums and writes O (bf16 or fp32) and lse.
+// Roles (192 threads):
+//   warp 4, one lane   TMA producer: Q of an item (one 2-D tensor copy per head
+//                      and 64-column box; one or two Q buffers), then K and V tiles
+//                      into a 3- or 4-stage ring (128-byte swizzle), all on
+//                      full/empty mbarriers;
+//   warp 5, one lane   MMA issuer: S_j = Q K_j^T (M 128, N 128, both operands
+//                      K-major in shared memory) into one of two TMEM buffers, then
+//                      O += P_j V_j with P read from tensor memory and V MN-major in
+//                      shared memory, into the item's TMEM output buffer (two,
+//                      alternating between items); each group is completed through
+//                      tcgen05.commit;
+//   warps 0-3          softmax: thread r owns query row r (TMEM lane r). It reads
+//                      its row of S with tcgen05.ld, masks, keeps a running maximum
+//                      (base-2 domain, 1/sqrt(d) folded into one FFMA) that moves
+//                      only when it grows by more than 2^8 (then it rescales its O
+//                      row in TMEM), writes exp2(z - m) as bf16 pairs over the first
+//                      half of its S row (P aliases S, as the MMA reads it from TMEM),
+//                      and at the item's end divides its O row by the row sum and
+//                      writes O and lse.
+// S_{j+1} is computed while the softmax of tile j runs. MMAs of the one issuing
+// thread execute in order, so S_{j+2} overwrites a buffer only after P.V of tile
+// j has read its P.
 //
 // Every wait is bounded by the global timer; a wait that runs out records a
-// timeout in this file's status word, the CTA drains its copies and returns.
+// timeout in this file's status word and every role stops. Before the CTA exits,
+// the MMA issuer waits (bounded) for its MMAs, the producer for its copies, and
+// the TMEM columns are released.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -42,28 +58,33 @@ __device__ int g_fwd_status;  // first fault recorded by a forward kernel, kDevO
 
 namespace {
 
-constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken GPU can exceed
-constexpr int kFwdConsumers = 4;                         // warps that compute, 16 query rows each
-constexpr int kFwdThreads = (kFwdConsumers + 1) * 32;    // plus one producer warp
+constexpr int kFwdThreads = 192;                         // 4 softmax warps, producer, MMA issuer
+constexpr int kProducerWarp = 4;
+constexpr int kMmaWarp = 5;
+constexpr int kTmemCols = 512;
 
 template <int D, int G>
 struct FwdCfg {
-    static constexpr int M = 16 * kFwdConsumers;        // query rows of a CTA (G heads x QT positions)
-    static constexpr int QT = M / G;                    // positions of a CTA
-    static constexpr int NK = 64;                       // keys per K/V tile
+    static constexpr int M = 128;                       // query rows of an item (G heads x QT positions)
+    static constexpr int QT = M / G;                    // positions of an item
+    static constexpr int NK = 128;                      // keys per K/V tile
     static constexpr int BOXES = D / 64;                // 64-column boxes of a row
-    static constexpr int KBOX = NK * 128;               // bytes of one K (or V) box
     static constexpr int QBOX = M * 128;                // bytes of one Q box
-    static constexpr int STAGE = 2 * BOXES * KBOX;      // K boxes then V boxes
-    static constexpr int STAGES = D == 128 ? 2 : 3;
-    static constexpr int Q_OFF = STAGES * STAGE;
-    static constexpr int SMEM = Q_OFF + BOXES * QBOX + 1024;  // + alignment slack
-    static constexpr int KSTEPS = D / 16;               // k-steps of S = Q K^T
-    static constexpr int NT_S = NK / 8;                 // 8-key n-tiles of S
-    static constexpr int NT_O = D / 8;                  // 8-dim n-tiles of O
+    static constexpr int KBOX = NK * 128;               // bytes of one K (or V) box
+    static constexpr int QBUF = D == 64 ? 2 : 1;        // Q buffers (the next item's Q loads early)
+    static constexpr int STAGES = D == 64 ? 4 : 3;      // K/V tiles in flight
+    static constexpr int Q_OFF = 0;
+    static constexpr int Q_BYTES = BOXES * QBOX;
+    static constexpr int KV_OFF = Q_OFF + QBUF * Q_BYTES;
+    static constexpr int KV_STAGE = 2 * BOXES * KBOX;   // K boxes then V boxes
+    static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;  // + alignment slack
+    // TMEM columns: S buffers at 0 and NK, O buffers at 2 NK and 2 NK + D
+    static constexpr int T_S = 0;
+    static constexpr int T_O = 2 * NK;
+    static_assert(T_O + 2 * D <= kTmemCols, "TMEM budget");
     static_assert(QT % 8 == 0, "a head's Q rows must start on a swizzle atom (8 rows)");
-    static_assert(KBOX % 1024 == 0 && QBOX % 1024 == 0, "boxes keep 1024-byte alignment");
+    static_assert(SMEM <= 227 * 1024, "shared memory budget");
 };
 
 // Start of the PBB support of position t: a(t) = max(0, h (floor(t/h) - 1)).
@@ -73,271 +94,359 @@ __device__ __forceinline__ int support_start(int t, int h)
     return m > 0 ? h * (m - 1) : 0;
 }
 
+// A bounded wait whose outcome is the same in every lane of the warp (the
+// softmax warps run warp-collective tcgen05 loads after it).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)
+{
+    return __all_sync(0xffffffffu, mbar_wait(bar, parity, limit));
+}
+
+// One work item: (sequence, KV head) pair, first position, keys and tiles.
+struct Item {
+    int pair, t0, tl, lo, a_max, ntiles;
+};
+
+template <int QT, int NK>
+__device__ __forceinline__ Item make_item(int idx, int n, int B)
+{
+    const int nq = (n + QT - 1) / QT;
+    Item it;
+    it.pair = idx / nq;
+    it.t0 = (idx - it.pair * nq) * QT;
+    it.tl = min(it.t0 + QT, n) - 1;  // last valid position
+    const int h = B >> 1;
+    it.lo = support_start(it.t0, h);  // first key any row needs
+    it.a_max = support_start(it.tl, h);
+    it.ntiles = (it.tl - it.lo + NK) / NK;
+    return it;
+}
+
 template <int D, int G>
-__global__ void __launch_bounds__(kFwdThreads, 2)
+__global__ void __launch_bounds__(kFwdThreads, 1)
 forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                const __grid_constant__ CUtensorMap vmap, const ForwardArgs a)
 {
     using C = FwdCfg<D, G>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ unsigned char dsmem_raw[];
-    __shared__ __align__(8) uint64_t full_bar[STAGES];
-    __shared__ __align__(8) uint64_t empty_bar[STAGES];
-    __shared__ __align__(8) uint64_t q_bar;
+    constexpr int QBUF = C::QBUF;
+    __shared__ __align__(8) uint64_t q_full[QBUF], q_empty[QBUF], done_bar;
+    __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
+    __shared__ __align__(8) uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];
+    __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
         (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    // item -> (sequence, KV head, query tile); query tiles of a head are adjacent,
-    // so CTAs running together share K/V tiles in L2
-    const int nq = (a.n + C::QT - 1) / C::QT;
-    const int qtile = static_cast<int>(blockIdx.x % static_cast<unsigned>(nq));
-    const int pair = static_cast<int>(blockIdx.x / static_cast<unsigned>(nq));
-    const int b = pair / a.Hkv, kvh = pair - b * a.Hkv;
-    const int h = a.B >> 1;
-    const int t0 = qtile * C::QT;
-    const int tl = min(t0 + C::QT, a.n) - 1;   // last valid position of the CTA
-    const int lo = support_start(t0, h);       // first key any row needs
-    const int ntiles = (tl - lo + C::NK) / C::NK;
-    const int a_max = support_start(tl, h);    // latest support start among the rows
+    const int n_items = a.batch * a.Hkv * ((a.n + C::QT - 1) / C::QT);
 
     if (tid == 0) {
 #pragma unroll
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full_bar[s], 1);
-            mbar_init(&empty_bar[s], kFwdConsumers);
+        for (int q = 0; q < QBUF; ++q) {
+            mbar_init(&q_full[q], 1);
+            mbar_init(&q_empty[q], 1);
         }
-        mbar_init(&q_bar, 1);
+        mbar_init(&done_bar, 1);
+#pragma unroll
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 1);
+        }
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&s_full[b], 1);
+            mbar_init(&p_full[b], 128);
+            mbar_init(&pv_done[b], 1);
+            mbar_init(&o_free[b], 128);
+        }
         fence_mbar_init();
         abort_s = 0;
     }
+    if (warp == 0) tmem_alloc<kTmemCols>(&tmem_base_s);
+    tmem_fence_before();
     __syncthreads();
+    tmem_fence_after();
+    const uint32_t tmem = tmem_base_s;
+    const unsigned long long limit = a.timeout_ns;
 
-    int issued = 0;  // K/V tiles issued (producer lane only)
-    if (warp == kFwdConsumers) {
-        // ================= producer: one lane =================
+    if (warp == kProducerWarp) {
+        // ================= TMA producer =================
         if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&kmap)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
-            mbar_expect_tx(&q_bar, static_cast<uint32_t>(C::BOXES * C::QBOX));
-            const int qrow0 = (b * a.Hq + kvh * G) * a.n + t0;
-#pragma unroll
-            for (int gi = 0; gi < G; ++gi)
-#pragma unroll
-                for (int bx = 0; bx < C::BOXES; ++bx)
-                    tma_load_2d(dsmem + C::Q_OFF + bx * C::QBOX + gi * C::QT * 128, &qmap, bx * 64,
-                                qrow0 + gi * a.n, &q_bar);
-            const int krow0 = pair * a.n + lo;
-            for (int it = 0; it < ntiles; ++it) {
-                const int s = it % STAGES;
-                if (it >= STAGES &&
-                    !mbar_wait(&empty_bar[s], static_cast<uint32_t>((it / STAGES - 1) & 1), a.timeout_ns)) {
-                    abort_s = 1;
-                    atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+            uint32_t gt = 0, ic = 0, q_issued = 0;  // tiles, items and Q loads issued
+            bool ok = true;
+            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
+                const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+                const uint32_t qb = ic % QBUF;
+                if (ic >= QBUF && !mbar_wait(&q_empty[qb], ((ic / QBUF) - 1) & 1u, limit)) {
+                    ok = false;
                     break;
                 }
-                if (abort_s) break;
-                unsigned char* st = dsmem + s * C::STAGE;
-                mbar_expect_tx(&full_bar[s], static_cast<uint32_t>(C::STAGE));
+                mbar_expect_tx(&q_full[qb], static_cast<uint32_t>(C::Q_BYTES));
+                const int qrow0 = (b * a.Hq + kvh * G) * a.n + it.t0;
+                unsigned char* qdst = dsmem + C::Q_OFF + qb * C::Q_BYTES;
 #pragma unroll
-                for (int bx = 0; bx < C::BOXES; ++bx) {
-                    tma_load_2d(st + bx * C::KBOX, &kmap, bx * 64, krow0 + it * C::NK, &full_bar[s]);
-                    tma_load_2d(st + (C::BOXES + bx) * C::KBOX, &vmap, bx * 64, krow0 + it * C::NK, &full_bar[s]);
+                for (int gi = 0; gi < G; ++gi)
+#pragma unroll
+                    for (int bx = 0; bx < C::BOXES; ++bx)
+                        tma_load_2d(qdst + bx * C::QBOX + gi * C::QT * 128, &qmap, bx * 64, qrow0 + gi * a.n,
+                                    &q_full[qb]);
+                ++q_issued;
+                const int krow0 = it.pair * a.n + it.lo;
+                for (int j = 0; j < it.ntiles; ++j, ++gt) {
+                    const int s = gt % STAGES;
+                    if (gt >= STAGES && !mbar_wait(&kv_empty[s], ((gt / STAGES) - 1) & 1u, limit)) {
+                        ok = false;
+                        break;
+                    }
+                    if (abort_s) {
+                        ok = false;
+                        break;
+                    }
+                    unsigned char* st = dsmem + C::KV_OFF + s * C::KV_STAGE;
+                    mbar_expect_tx(&kv_full[s], static_cast<uint32_t>(C::KV_STAGE));
+#pragma unroll
+                    for (int bx = 0; bx < C::BOXES; ++bx) {
+                        tma_load_2d(st + bx * C::KBOX, &kmap, bx * 64, krow0 + j * C::NK, &kv_full[s]);
+                        tma_load_2d(st + (C::BOXES + bx) * C::KBOX, &vmap, bx * 64, krow0 + j * C::NK, &kv_full[s]);
+                    }
                 }
-                ++issued;
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+            }
+            // drain: the last copies into each stage and into Q land before shared memory goes away
+            for (uint32_t q = 0; q < QBUF && q < q_issued; ++q) {
+                const uint32_t j = q + QBUF * ((q_issued - 1 - q) / QBUF);
+                mbar_wait(&q_full[q], (j / QBUF) & 1u, kGuardNs);
+            }
+            for (uint32_t s = 0; s < STAGES && s < gt; ++s) {
+                const uint32_t j = s + STAGES * ((gt - 1 - s) / STAGES);
+                mbar_wait(&kv_full[s], (j / STAGES) & 1u, kGuardNs);
+            }
+        }
+    } else if (warp == kMmaWarp) {
+        // ================= MMA issuer =================
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, C::NK, 0);
+            constexpr uint32_t idesc_o = umma_idesc_bf16(C::M, D, 1);
+            const uint32_t kv_base = smem_addr(dsmem + C::KV_OFF);
+            uint32_t gt = 0, ic = 0, q_base = 0;
+            bool ok = true, issued_any = false;
+            // S_g = Q K_g^T into S buffer g % 2
+            auto issue_s = [&](uint32_t g) {
+                const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk & 3) * 32;  // 16 columns = 32 bytes into the 128-byte row
+                    const uint64_t ad = umma_desc_sw128(q_base + (kk >> 2) * C::QBOX + off, 16, 1024);
+                    const uint64_t bd = umma_desc_sw128(kb + (kk >> 2) * C::KBOX + off, 16, 1024);
+                    umma_bf16(tmem + C::T_S + (g & 1u) * C::NK, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&s_full[g & 1u]);
+            };
+            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
+                const uint32_t ob = ic & 1u;
+                const uint32_t qb = ic % QBUF;
+                q_base = smem_addr(dsmem + C::Q_OFF + qb * C::Q_BYTES);
+                if (!mbar_wait(&q_full[qb], (ic / QBUF) & 1u, limit) ||
+                    !mbar_wait(&kv_full[gt % STAGES], (gt / STAGES) & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                issue_s(gt);
+                issued_any = true;
+                if (it.ntiles == 1) umma_commit(&q_empty[qb]);
+                for (int j = 0; j < it.ntiles; ++j) {
+                    const uint32_t g = gt + j;
+                    if (j + 1 < it.ntiles) {
+                        if (!mbar_wait(&kv_full[(g + 1) % STAGES], ((g + 1) / STAGES) & 1u, limit)) {
+                            ok = false;
+                            break;
+                        }
+                        tmem_fence_after();
+                        issue_s(g + 1);
+                        if (j + 2 == it.ntiles) umma_commit(&q_empty[qb]);  // the item's last read of Q
+                    }
+                    if (!mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit) ||
+                        (j == 0 && ic >= 2 && !mbar_wait(&o_free[ob], ((ic >> 1) - 1) & 1u, limit))) {
+                        ok = false;
+                        break;
+                    }
+                    tmem_fence_after();
+                    // O (+)= P_g V_g: P from TMEM (bf16 pairs over S buffer g % 2), V MN-major
+                    const uint32_t pt = tmem + C::T_S + (g & 1u) * C::NK;
+                    const uint32_t vb = kv_base + (g % STAGES) * C::KV_STAGE + C::BOXES * C::KBOX;
+#pragma unroll
+                    for (int kk = 0; kk < C::NK / 16; ++kk) {
+                        const uint64_t bd = umma_desc_sw128(vb + kk * 2048, C::KBOX, 1024);
+                        umma_bf16_tmem_a(tmem + C::T_O + ob * D, pt + 8 * kk, bd, idesc_o, (j > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    umma_commit(&pv_done[g & 1u]);
+                    umma_commit(&kv_empty[g % STAGES]);
+                }
+                gt += it.ntiles;
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+            }
+            if (issued_any) {  // every MMA complete before TMEM is released
+                umma_commit(&done_bar);
+                mbar_wait(&done_bar, 0u, kGuardNs);
             }
         }
     } else {
-        // ================= consumers: 16 query rows per warp =================
-        const int g = lane >> 2, tig = lane & 3;  // fragment row group and thread in group
-        const int lm = lane >> 3;                 // which 8x8 matrix this lane addresses
+        // ================= softmax: thread r owns query row r =================
+        const int r = tid;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
         const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
-        // the warp's two rows per thread: r0 = 16 warp + g, r1 = r0 + 8 (CTA rows are head-major)
-        const int r0 = 16 * warp + g, r1 = r0 + 8;
-        const int tp0 = t0 + r0 % C::QT, tp1 = t0 + r1 % C::QT;    // their positions
-        const int as0 = support_start(tp0, h), as1 = support_start(tp1, h);
-
-        bool ok = mbar_wait(&q_bar, 0u, a.timeout_ns);
-        uint32_t qa[C::KSTEPS][4];  // Q A-fragments of the warp's 16 rows
-        if (ok) {
-            const uint32_t qbase = smem_addr(dsmem + C::Q_OFF);
-            const int row = 16 * warp + 8 * (lm & 1) + (lane & 7);
-#pragma unroll
-            for (int kk = 0; kk < C::KSTEPS; ++kk) {
-                const int ch = 2 * kk + (lm >> 1);
-                ldmatrix_x4(qa[kk], qbase + (ch >> 3) * C::QBOX + swz(row, ch & 7));
-            }
-        }
-        float o[C::NT_O][4];
-#pragma unroll
-        for (int nt = 0; nt < C::NT_O; ++nt)
-#pragma unroll
-            for (int x = 0; x < 4; ++x) o[nt][x] = 0.f;
-        float m0 = -INFINITY, m1 = -INFINITY;  // running maxima of rows r0, r1 (base-2 domain)
-        float l0 = 0.f, l1 = 0.f;              // this thread's share of their running sums
-
-        for (int it = 0; ok && it < ntiles; ++it) {
-            const int s = it % STAGES;
-            if (!mbar_wait(&full_bar[s], static_cast<uint32_t>((it / STAGES) & 1), a.timeout_ns)) {
-                ok = false;
-                break;
-            }
-            if (abort_s) {
-                ok = false;
-                break;
-            }
-            const uint32_t kbase = smem_addr(dsmem + s * C::STAGE);
-            const uint32_t vbase = kbase + C::BOXES * C::KBOX;
-            const int key0 = lo + it * C::NK;
-
-            // ---- S = Q K^T for 16 rows x 64 keys
-            float sc[C::NT_S][4];
-#pragma unroll
-            for (int nt = 0; nt < C::NT_S; ++nt)
-#pragma unroll
-                for (int x = 0; x < 4; ++x) sc[nt][x] = 0.f;
-#pragma unroll
-            for (int j = 0; j < C::NK / 16; ++j) {
-                const int krow = 16 * j + 8 * (lm >> 1) + (lane & 7);
-#pragma unroll
-                for (int kk = 0; kk < C::KSTEPS; ++kk) {
-                    const int ch = 2 * kk + (lm & 1);
-                    uint32_t kb[4];
-                    ldmatrix_x4(kb, kbase + (ch >> 3) * C::KBOX + swz(krow, ch & 7));
-                    mma_bf16_16816(sc[2 * j], qa[kk], kb[0], kb[1]);
-                    mma_bf16_16816(sc[2 * j + 1], qa[kk], kb[2], kb[3]);
+        const int h = a.B >> 1;
+        const int gi = r / C::QT, rp = r - gi * C::QT;
+        uint32_t gt = 0, ic = 0;
+        bool ok = true;
+        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
+            const uint32_t ob = ic & 1u;
+            const int t = it.t0 + rp;               // this row's position
+            const int as = support_start(t, h);     // and its support start
+            float m_used = -INFINITY, l = 0.f;
+            for (int j = 0; j < it.ntiles; ++j) {
+                const uint32_t g = gt + j;
+                if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(0xffffffffu, abort_s != 0)) {
+                    ok = false;
+                    break;
                 }
-            }
-            // ---- scale, mask where the tile crosses a row's bounds [a(t), t]
-            const bool edge = (key0 + C::NK - 1 > t0) || (key0 < a_max);
+                tmem_fence_after();
+                const uint32_t s_col = lane_base + C::T_S + (g & 1u) * C::NK;
+                float z[C::NK];  // raw scores q.k of this row
 #pragma unroll
-            for (int nt = 0; nt < C::NT_S; ++nt) {
+                for (int c = 0; c < C::NK / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(s_col + 32 * c, v);
 #pragma unroll
-                for (int x = 0; x < 4; ++x) {
-                    float z = sc[nt][x] * qscale;
-                    if (edge) {
-                        const int key = key0 + 8 * nt + 2 * tig + (x & 1);
-                        const bool vis = (x < 2) ? (key >= as0 && key <= tp0) : (key >= as1 && key <= tp1);
-                        z = vis ? z : -INFINITY;
+                    for (int x = 0; x < 32; ++x) z[32 * c + x] = __uint_as_float(v[x]);
+                }
+                tmem_wait_ld();
+                const int key0 = it.lo + j * C::NK;
+                if ((key0 + C::NK - 1 > it.t0) || (key0 < it.a_max)) {  // tile crosses some row's bounds
+#pragma unroll
+                    for (int c = 0; c < C::NK; ++c) {
+                        const int key = key0 + c;
+                        z[c] = (key >= as && key <= t) ? z[c] : -INFINITY;
                     }
-                    sc[nt][x] = z;
+                }
+                float mx = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < C::NK; ++c) mx = fmaxf(mx, z[c]);
+                mx *= qscale;  // the scale is positive: the maximum of the scaled scores
+                // the reference maximum moves only when the row maximum exceeds it by 2^8:
+                // weights stay below 2^8, and O and l are rescaled together, so o = O / l is exact
+                const bool grow = mx > m_used + 8.f;
+                const float m_new = grow ? mx : m_used;
+                if (__any_sync(0xffffffffu, grow)) {
+                    const float f = grow ? (m_used == -INFINITY ? 0.f : fast_exp2(m_used - m_new)) : 1.f;
+                    l *= f;
+                    if (j > 0) {  // O holds tiles 0 .. j-1 once P.V of tile j-1 is complete
+                        const uint32_t gp = g - 1;
+                        if (!warp_wait(&pv_done[gp & 1u], (gp >> 1) & 1u, limit)) {
+                            ok = false;
+                            break;
+                        }
+                        tmem_fence_after();
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint32_t v[32];
+                            const uint32_t ta = lane_base + C::T_O + ob * D + 32 * c;
+                            tmem_ld32(ta, v);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int x = 0; x < 32; ++x) v[x] = __float_as_uint(__uint_as_float(v[x]) * f);
+                            tmem_st32(ta, v);
+                        }
+                        tmem_wait_st();
+                    }
+                    m_used = m_new;
+                }
+                const float nbase = m_used == -INFINITY ? 0.f : -m_used;
+                // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row
+#pragma unroll
+                for (int c = 0; c < C::NK / 64; ++c) {
+                    uint32_t pk[32];
+#pragma unroll
+                    for (int x = 0; x < 32; ++x) {
+                        const float e0 = fast_exp2(fmaf(z[64 * c + 2 * x], qscale, nbase));
+                        const float e1 = fast_exp2(fmaf(z[64 * c + 2 * x + 1], qscale, nbase));
+                        l += e0 + e1;
+                        pk[x] = pack_bf16x2(e0, e1);
+                    }
+                    tmem_st32(s_col + 32 * c, pk);
+                }
+                tmem_wait_st();
+                tmem_fence_before();   // P is in TMEM and this row of S has been read
+                mbar_arrive(&p_full[g & 1u]);
+            }
+            if (!ok) break;
+            // ---- epilogue: O row / l, lse
+            const uint32_t gl = gt + it.ntiles - 1;
+            if (!warp_wait(&pv_done[gl & 1u], (gl >> 1) & 1u, limit)) {
+                ok = false;
+                break;
+            }
+            tmem_fence_after();
+            const bool valid = t < a.n;
+            const float inv = l > 0.f ? 1.f / l : 0.f;
+            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+            const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + t;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(lane_base + C::T_O + ob * D + 32 * c, v);
+                tmem_wait_ld();
+                if (valid) {
+                    if (a.out_f32) {
+                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 32 * c);
+#pragma unroll
+                        for (int x = 0; x < 8; ++x)
+                            dst[x] = make_float4(__uint_as_float(v[4 * x]) * inv, __uint_as_float(v[4 * x + 1]) * inv,
+                                                 __uint_as_float(v[4 * x + 2]) * inv, __uint_as_float(v[4 * x + 3]) * inv);
+                    } else {
+                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 32 * c);
+#pragma unroll
+                        for (int x = 0; x < 4; ++x) {
+                            uint4 pk;
+                            pk.x = pack_bf16x2(__uint_as_float(v[8 * x]) * inv, __uint_as_float(v[8 * x + 1]) * inv);
+                            pk.y = pack_bf16x2(__uint_as_float(v[8 * x + 2]) * inv, __uint_as_float(v[8 * x + 3]) * inv);
+                            pk.z = pack_bf16x2(__uint_as_float(v[8 * x + 4]) * inv, __uint_as_float(v[8 * x + 5]) * inv);
+                            pk.w = pack_bf16x2(__uint_as_float(v[8 * x + 6]) * inv, __uint_as_float(v[8 * x + 7]) * inv);
+                            dst[x] = pk;
+                        }
+                    }
                 }
             }
-            // ---- online softmax (base 2)
-            float mx0 = -INFINITY, mx1 = -INFINITY;
-#pragma unroll
-            for (int nt = 0; nt < C::NT_S; ++nt) {
-                mx0 = fmaxf(mx0, fmaxf(sc[nt][0], sc[nt][1]));
-                mx1 = fmaxf(mx1, fmaxf(sc[nt][2], sc[nt][3]));
+            tmem_fence_before();
+            mbar_arrive(&o_free[ob]);  // the next item on this O buffer may overwrite it
+            if (valid && a.lse != nullptr) {
+                // ln sum exp(z) = (m + log2 l) ln 2, m the base-2 reference maximum
+                a.lse[row] = (m_used + log2f(l)) * 0.6931471805599453f;
             }
-            mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, 1));
-            mx0 = fmaxf(mx0, __shfl_xor_sync(kFull, mx0, 2));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, 1));
-            mx1 = fmaxf(mx1, __shfl_xor_sync(kFull, mx1, 2));
-            const float mn0 = fmaxf(m0, mx0), mn1 = fmaxf(m1, mx1);
-            if (__any_sync(kFull, (mn0 > m0) || (mn1 > m1))) {
-                // a row with no visible key yet keeps m = -inf; its factor is 1 (o and l are 0)
-                const float al0 = (mn0 == -INFINITY) ? 1.f : fast_exp2(m0 - mn0);
-                const float al1 = (mn1 == -INFINITY) ? 1.f : fast_exp2(m1 - mn1);
-                l0 *= al0;
-                l1 *= al1;
-#pragma unroll
-                for (int nt = 0; nt < C::NT_O; ++nt) {
-                    o[nt][0] *= al0;
-                    o[nt][1] *= al0;
-                    o[nt][2] *= al1;
-                    o[nt][3] *= al1;
-                }
-            }
-            m0 = mn0;
-            m1 = mn1;
-            const float b0 = (mn0 == -INFINITY) ? 0.f : mn0;
-            const float b1 = (mn1 == -INFINITY) ? 0.f : mn1;
-            uint32_t pa[C::NK / 16][4];  // P as bf16 A-fragments, one per 16-key k-step
-#pragma unroll
-            for (int kk = 0; kk < C::NK / 16; ++kk) {
-                float p[2][4];
-#pragma unroll
-                for (int hlf = 0; hlf < 2; ++hlf) {
-                    const int nt = 2 * kk + hlf;
-                    p[hlf][0] = fast_exp2(sc[nt][0] - b0);
-                    p[hlf][1] = fast_exp2(sc[nt][1] - b0);
-                    p[hlf][2] = fast_exp2(sc[nt][2] - b1);
-                    p[hlf][3] = fast_exp2(sc[nt][3] - b1);
-                    l0 += p[hlf][0] + p[hlf][1];
-                    l1 += p[hlf][2] + p[hlf][3];
-                }
-                pa[kk][0] = pack_bf16x2(p[0][0], p[0][1]);
-                pa[kk][1] = pack_bf16x2(p[0][2], p[0][3]);
-                pa[kk][2] = pack_bf16x2(p[1][0], p[1][1]);
-                pa[kk][3] = pack_bf16x2(p[1][2], p[1][3]);
-            }
-            // ---- O += P V
-#pragma unroll
-            for (int kk = 0; kk < C::NK / 16; ++kk) {
-                const int vrow = 16 * kk + 8 * (lm & 1) + (lane & 7);
-#pragma unroll
-                for (int j = 0; j < D / 16; ++j) {
-                    const int ch = 2 * j + (lm >> 1);
-                    uint32_t vb[4];
-                    ldmatrix_x4_trans(vb, vbase + (ch >> 3) * C::KBOX + swz(vrow, ch & 7));
-                    mma_bf16_16816(o[2 * j], pa[kk], vb[0], vb[1]);
-                    mma_bf16_16816(o[2 * j + 1], pa[kk], vb[2], vb[3]);
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty_bar[s]);
+            gt += it.ntiles;
         }
         if (!ok) {
             abort_s = 1;
             atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
-        } else {
-            // ---- epilogue: row sums over the quad, normalise, write O and lse
-            l0 += __shfl_xor_sync(kFull, l0, 1);
-            l0 += __shfl_xor_sync(kFull, l0, 2);
-            l1 += __shfl_xor_sync(kFull, l1, 1);
-            l1 += __shfl_xor_sync(kFull, l1, 2);
-            const float inv0 = l0 > 0.f ? 1.f / l0 : 0.f;
-            const float inv1 = l1 > 0.f ? 1.f / l1 : 0.f;
-            const int gi0 = r0 / C::QT, gi1 = r1 / C::QT;
-            const size_t row0 = static_cast<size_t>(b * a.Hq + kvh * G + gi0) * a.n + tp0;
-            const size_t row1 = static_cast<size_t>(b * a.Hq + kvh * G + gi1) * a.n + tp1;
-            const bool w0 = tp0 < a.n, w1 = tp1 < a.n;
-            if (a.out_f32) {
-                float* out = static_cast<float*>(a.out);
-#pragma unroll
-                for (int nt = 0; nt < C::NT_O; ++nt) {
-                    const int dim = 8 * nt + 2 * tig;
-                    if (w0) *reinterpret_cast<float2*>(out + row0 * D + dim) = make_float2(o[nt][0] * inv0, o[nt][1] * inv0);
-                    if (w1) *reinterpret_cast<float2*>(out + row1 * D + dim) = make_float2(o[nt][2] * inv1, o[nt][3] * inv1);
-                }
-            } else {
-                uint32_t* out = static_cast<uint32_t*>(a.out);  // bf16 pairs
-#pragma unroll
-                for (int nt = 0; nt < C::NT_O; ++nt) {
-                    const int dim = 8 * nt + 2 * tig;
-                    if (w0) out[(row0 * D + dim) >> 1] = pack_bf16x2(o[nt][0] * inv0, o[nt][1] * inv0);
-                    if (w1) out[(row1 * D + dim) >> 1] = pack_bf16x2(o[nt][2] * inv1, o[nt][3] * inv1);
-                }
-            }
-            if (a.lse != nullptr && tig == 0) {
-                // ln sum exp(z) = (m2 + log2 l) ln 2, m2 the base-2 running maximum
-                constexpr float kLn2 = 0.6931471805599453f;
-                if (w0) a.lse[row0] = (m0 + log2f(l0)) * kLn2;
-                if (w1) a.lse[row1] = (m1 + log2f(l1)) * kLn2;
-            }
         }
     }
+    tmem_fence_before();
     __syncthreads();
-    if (abort_s && warp == kFwdConsumers && lane == 0) {
-        // drain: wait (bounded) for the copies this CTA issued before its shared memory goes away
-        mbar_wait(&q_bar, 0u, kGuardNs);
-        for (int s = 0; s < STAGES && s < issued; ++s) {
-            const int j = s + STAGES * ((issued - 1 - s) / STAGES);
-            mbar_wait(&full_bar[s], static_cast<uint32_t>((j / STAGES) & 1), kGuardNs);
-        }
-    }
+    tmem_fence_after();
+    if (warp == 0) tmem_dealloc<kTmemCols>(tmem);
 }
 
 // Sequence -> ring: slot j of each (sequence, KV head) ring gets the position
@@ -389,11 +498,15 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
     if (!rows_tensor_map(&qmap, a.q, qrows, D, C::QT) || !rows_tensor_map(&kmap, a.k, krows, D, C::NK) ||
         !rows_tensor_map(&vmap, a.v, krows, D, C::NK))
         return cudaErrorInvalidValue;
-    const long long nq = (a.n + C::QT - 1) / C::QT;
-    const long long grid = static_cast<long long>(a.batch) * a.Hkv * nq;
-    if (grid < 1) return cudaSuccess;
-    if (grid > 0x7fffffffLL) return cudaErrorInvalidValue;
-    forward_kernel<D, G><<<static_cast<unsigned>(grid), kFwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, a);
+    const long long items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::QT - 1) / C::QT);
+    if (items < 1) return cudaSuccess;
+    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    // one persistent CTA per SM (its shared memory and 512 TMEM columns admit no second)
+    const int grid = static_cast<int>(items < sms ? items : sms);
+    forward_kernel<D, G><<<grid, kFwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, a);
     return cudaGetLastError();
 }
 
