@@ -19,6 +19,7 @@ arrays. What each function computes is stated in the C file and below:
                        sliding-window attention (Sec. 2.3), the comparison pattern.
 * ``forward``          PBB attention for every position of whole sequences (the
                        forward pass / prefill), with the log-partition of Eq. (lse).
+* ``backward``         its gradients with respect to q, k and v.
 """
 from __future__ import annotations
 
@@ -85,6 +86,8 @@ def _load():
         lib.pbb_oracle_attend_window.restype = I
         lib.pbb_oracle_forward_rows.argtypes = [P, P, P, I, I, I, L, I, L, P, L, P, P, I]
         lib.pbb_oracle_forward_rows.restype = I
+        lib.pbb_oracle_backward.argtypes = [P, P, P, P, I, I, I, L, I, L, P, P, P, I]
+        lib.pbb_oracle_backward.restype = I
         lib.pbb_oracle_max_threads.argtypes = []
         lib.pbb_oracle_max_threads.restype = I
         _lib = lib
@@ -213,6 +216,26 @@ def forward(q, k, v, b: int, rows=None, n_threads: int = 0):
     if full:
         return out.reshape(batch, Hq, n, d), lse.reshape(batch, Hq, n)
     return out, lse
+
+
+def backward(q, k, v, dout, b: int, n_threads: int = 0):
+    """Gradients (dq, dk, dv) of the whole-sequence PBB attention for the upstream gradient
+    dout [batch, Hq, n, d] (chain rule through Eq. attention over A_PBB(t)); fp64."""
+    q = _f64(q)
+    kk = _f64(k)
+    vv = _f64(v)
+    do = _f64(dout)
+    batch, Hq, n, d = q.shape
+    _, Hkv, n2, d2 = kk.shape
+    assert n2 == n and d2 == d and vv.shape == kk.shape and do.shape == q.shape
+    dq = np.zeros_like(q)
+    dk = np.zeros_like(kk)
+    dv = np.zeros_like(vv)
+    rc = _load().pbb_oracle_backward(_ptr(q), _ptr(kk), _ptr(vv), _ptr(do), batch, Hq, Hkv, n, d, b,
+                                     _ptr(dq), _ptr(dk), _ptr(dv), n_threads)
+    if rc != ORACLE_OK:
+        raise OracleError(f"pbb_oracle_backward returned {rc}")
+    return dq, dk, dv
 
 
 class RingSim:

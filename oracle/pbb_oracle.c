@@ -21,7 +21,8 @@
  *   - sliding-window attention over {t-w+1, ..., t} (Sec. 2.3), the pattern
  *     the paper compares PBB with, for the window-ring decode control;
  *   - PBB attention for every position of whole sequences (the forward pass /
- *     prefill of Sec. 3) with its log-partition ln sum exp(z) (Eq. lse).
+ *     prefill of Sec. 3) with its log-partition ln sum exp(z) (Eq. lse), and
+ *     its gradients with respect to q, k and v (the backward pass).
  *
  * The brute-force evaluation visits every s in [0, t] and tests the support
  * predicate in its block/bridge form; it never uses the interval form, so the
@@ -220,6 +221,100 @@ int pbb_oracle_forward_rows(const double* q, const double* k, const double* v, i
         free(z);
         free(vr);
         free(kr);
+    }
+    return ORACLE_OK;
+}
+
+/*
+ * Gradients of the whole-sequence PBB attention: the backward pass of the
+ * paper's fused training kernel (Sec. 3; Appendix "exact union and numerical
+ * checks", bridge gradients into the previous block's K/V included). Given the
+ * upstream gradient dO of every output row, the chain rule through Eq.
+ * (attention) over A_PBB(t), written out per query row t and head j:
+ *   z_ts  = q_t . k_s / sqrt(d),  P_ts = exp(z_ts) / sum_{u in A(t)} exp(z_tu)
+ *   dP_ts = dO_t . v_s
+ *   dz_ts = P_ts (dP_ts - sum_{u in A(t)} P_tu dP_tu)
+ *   dq_t += dz_ts k_s / sqrt(d)    dk_s += dz_ts q_t / sqrt(d)    dv_s += P_ts dO_t
+ * for every s in A(t). K/V gradients collect every query head of the group
+ * (GQA) and every position whose support holds s.
+ *
+ *   q, dout     [batch][Hq][n][d]       dq   [batch][Hq][n][d]
+ *   k, v        [batch][Hkv][n][d]      dk, dv [batch][Hkv][n][d]
+ */
+int pbb_oracle_backward(const double* q, const double* k, const double* v, const double* dout, int batch,
+                        int Hq, int Hkv, long n, int d, long b, double* dq, double* dk, double* dv,
+                        int n_threads)
+{
+    if (batch < 0 || Hq <= 0 || Hkv <= 0 || d <= 0 || n <= 0 || b < 2 || (b % 2) || (Hq % Hkv))
+        return ORACLE_ERR_ARG;
+    const int group = Hq / Hkv;
+    const double scale = 1.0 / sqrt((double)d);
+    memset(dq, 0, sizeof(double) * (size_t)batch * Hq * n * d);
+    memset(dk, 0, sizeof(double) * (size_t)batch * Hkv * n * d);
+    memset(dv, 0, sizeof(double) * (size_t)batch * Hkv * n * d);
+#ifdef _OPENMP
+    if (n_threads > 0) omp_set_num_threads(n_threads);
+#else
+    (void)n_threads;
+#endif
+    /* one (sequence, KV head) pair per task: its dk, dv rows are written by no other task */
+#pragma omp parallel for schedule(dynamic, 1)
+    for (long pr = 0; pr < (long)batch * Hkv; ++pr) {
+        const long bi = pr / Hkv, kv = pr % Hkv;
+        long* src = (long*)malloc(sizeof(long) * (size_t)(b + 1));
+        double* P = (double*)malloc(sizeof(double) * (size_t)(b + 1));
+        double* dP = (double*)malloc(sizeof(double) * (size_t)(b + 1));
+        const double* kh = k + (size_t)pr * n * d;
+        const double* vh = v + (size_t)pr * n * d;
+        double* dkh = dk + (size_t)pr * n * d;
+        double* dvh = dv + (size_t)pr * n * d;
+        for (int jg = 0; jg < group; ++jg) {
+            const long j = kv * group + jg;
+            const size_t qh = ((size_t)bi * Hq + (size_t)j) * (size_t)n;
+            for (long t = 0; t < n; ++t) {
+                const double* qt = q + (qh + (size_t)t) * d;
+                const double* dot_ = dout + (qh + (size_t)t) * d;
+                double* dqt = dq + (qh + (size_t)t) * d;
+                long m = 0;
+                for (long s = 0; s <= t; ++s)
+                    if (pbb_oracle_in_support(t, s, b) && m < b + 1) src[m++] = s;
+                /* P over the support: two passes as in softmax_attend */
+                double zmax = -INFINITY;
+                for (long i = 0; i < m; ++i) {
+                    double z = 0.0;
+                    for (int c = 0; c < d; ++c) z += qt[c] * kh[src[i] * d + c];
+                    P[i] = z * scale;
+                    if (P[i] > zmax) zmax = P[i];
+                }
+                double den = 0.0;
+                for (long i = 0; i < m; ++i) {
+                    P[i] = exp(P[i] - zmax);
+                    den += P[i];
+                }
+                double sum_pdp = 0.0;
+                for (long i = 0; i < m; ++i) {
+                    P[i] /= den;
+                    double x = 0.0;
+                    for (int c = 0; c < d; ++c) x += dot_[c] * vh[src[i] * d + c];
+                    dP[i] = x;
+                    sum_pdp += P[i] * x;
+                }
+                for (long i = 0; i < m; ++i) {
+                    const double dz = P[i] * (dP[i] - sum_pdp);
+                    const double* ks = kh + src[i] * d;
+                    double* dks = dkh + src[i] * d;
+                    double* dvs = dvh + src[i] * d;
+                    for (int c = 0; c < d; ++c) {
+                        dqt[c] += dz * ks[c] * scale;
+                        dks[c] += dz * qt[c] * scale;
+                        dvs[c] += P[i] * dot_[c];
+                    }
+                }
+            }
+        }
+        free(dP);
+        free(P);
+        free(src);
     }
     return ORACLE_OK;
 }

@@ -519,3 +519,63 @@ def test_forward_rows_subset(oracle_mod):
     o2, l2 = oracle_mod.forward(q, k, v, 8, rows=rows)
     for i, (bi, j, t) in enumerate(rows):
         assert np.array_equal(o2[i], out[bi, j, t]) and l2[i] == lse[bi, j, t]
+
+
+# ----------------------------------------------------------------- backward --
+
+
+def _loss_and_grads(oracle_mod, q, k, v, w_out, b):
+    out, _ = oracle_mod.forward(q, k, v, b)
+    return float((out * w_out).sum()), oracle_mod.backward(q, k, v, w_out, b)
+
+
+@pytest.mark.parametrize("b,G", [(4, 1), (4, 2), (6, 3), (8, 2)])
+def test_backward_matches_finite_differences(oracle_mod, b, G):
+    """Central differences of L = sum(dO * O) through the forward oracle (pinned above)
+    against the analytic gradients, for every element of q, k and v."""
+    rng = np.random.default_rng(40 + b + G)
+    Hkv, n, d = 2, 13, 3
+    q = rng.standard_normal((1, Hkv * G, n, d))
+    k = rng.standard_normal((1, Hkv, n, d))
+    v = rng.standard_normal((1, Hkv, n, d))
+    w = rng.standard_normal((1, Hkv * G, n, d))
+    _, (dq, dk, dv) = _loss_and_grads(oracle_mod, q, k, v, w, b)
+    eps = 1e-6
+    for x, g in ((q, dq), (k, dk), (v, dv)):
+        num = np.zeros_like(x)
+        for idx in np.ndindex(x.shape):
+            old = x[idx]
+            x[idx] = old + eps
+            lp, _ = _loss_and_grads(oracle_mod, q, k, v, w, b)
+            x[idx] = old - eps
+            lm, _ = _loss_and_grads(oracle_mod, q, k, v, w, b)
+            x[idx] = old
+            num[idx] = (lp - lm) / (2 * eps)
+        assert np.allclose(g, num, rtol=1e-6, atol=1e-7)
+
+
+def test_backward_key_gradients_sum_to_zero(oracle_mod):
+    """A common shift c of every key adds q_t.c/sqrt(d) to all of a row's logits, which the
+    softmax ignores: sum_s dk_s = 0 for each (sequence, KV head)."""
+    rng = np.random.default_rng(41)
+    q = rng.standard_normal((2, 4, 50, 8))
+    k = rng.standard_normal((2, 2, 50, 8))
+    v = rng.standard_normal((2, 2, 50, 8))
+    w = rng.standard_normal((2, 4, 50, 8))
+    _, dk, _ = oracle_mod.backward(q, k, v, w, 16)
+    assert np.abs(dk.sum(axis=2)).max() < 1e-11
+
+
+def test_backward_zero_query_closed_form(oracle_mod):
+    """q = 0: P_ts = 1/|A(t)| on [a(t), t], so dv_s = sum over t with s in [a(t), t] of dO_t/|A(t)|."""
+    rng = np.random.default_rng(42)
+    b, n, d = 8, 40, 3
+    k = rng.standard_normal((1, 1, n, d))
+    v = rng.standard_normal((1, 1, n, d))
+    w = rng.standard_normal((1, 1, n, d))
+    _, _, dv = oracle_mod.backward(np.zeros((1, 1, n, d)), k, v, w, b)
+    ref = np.zeros((n, d))
+    for t in range(n):
+        a = interval_start(t, b)
+        ref[a:t + 1] += w[0, 0, t] / (t + 1 - a)
+    assert np.allclose(dv[0, 0], ref, atol=1e-13)
