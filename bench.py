@@ -19,7 +19,8 @@ on a bounded sample per step. --sweep prints one line per throughput-sweep point
 kernel family) instead, --pattern both prints the PBB line and then the
 control's; the control lines carry their own metric name. --forward times the
 whole-sequence forward (prefill) workloads, one line each, with a roofline
-against HBM or the tensor cores, whichever bounds the workload.
+against HBM or the tensor cores, whichever bounds the workload; --backward
+times the gradients (dq, dk, dv) on the same workloads.
 """
 from __future__ import annotations
 
@@ -41,6 +42,7 @@ if ROOT not in sys.path:
 METRIC = "PBB decode-core tokens*heads/s"
 METRIC_SWA = "SWA-B decode-core tokens*heads/s (control: window = B over the same ring)"
 METRIC_FWD = "PBB forward tokens*heads/s"
+METRIC_BWD = "PBB backward tokens*heads/s"
 UNIT = "tokens*heads/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
@@ -68,7 +70,9 @@ def parse_args():
                     help="attention pattern: PBB (default), the sliding-window control with window B, or both")
     ap.add_argument("--forward", action="store_true",
                     help="time the whole-sequence forward (prefill) workloads instead of the decode step")
-    ap.add_argument("--fwd-workload", default="", help="one forward workload (default: all)")
+    ap.add_argument("--backward", action="store_true",
+                    help="time the whole-sequence backward (dq, dk, dv) on the forward workloads")
+    ap.add_argument("--fwd-workload", default="", help="one forward/backward workload (default: all)")
     ap.add_argument("--graph", choices=["auto", "on", "off"], default="auto",
                     help="replay the timed steps as one CUDA graph (auto: when a step is under 100 us, "
                          "where host launch overhead would otherwise dominate)")
@@ -415,6 +419,22 @@ def forward_flops_bytes(w):
     return flops, bytes_
 
 
+def backward_flops_bytes(w):
+    """Algorithmic FLOPs of the backward: five products per (row, key) pair of a support
+    (S, dP = dO.V, dV, dK, dQ), 10 d |A(t)| per query head and position; bytes: bf16 q, k,
+    v, O, dO and fp32 lse read, fp32 dq, dk, dv written, the fp32 D row written and read."""
+    import numpy as np
+
+    from paper_2606_02680_gb300 import bytemodel
+
+    sizes = bytemodel.support_size(np.arange(w.n), w.B)
+    flops = 10 * w.d * w.batch * w.Hq * int(sizes.sum())
+    rows_q, rows_k = w.batch * w.Hq * w.n, w.batch * w.Hkv * w.n
+    bytes_ = (2 * w.d * (3 * rows_q + 2 * rows_k) + 4 * rows_q        # q, O, dO, k, v, lse
+              + 4 * w.d * (rows_q + 2 * rows_k) + 8 * rows_q)         # dq, dk, dv, D
+    return flops, bytes_
+
+
 def tensor_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -502,6 +522,117 @@ def time_forward_e2e(w, dev, steps, state):
             "api": "paper_2606_02680_gb300.forward (pinned host q/k/v in, out/lse back, one stream)"}
 
 
+def time_backward(w, dev, steps, warmup, dist=None):
+    """Eager backward calls (three kernels each) with CUDA events around each; inputs resident."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import inputs
+
+    q, k, v = inputs.sequence_inputs(w, device=dev)
+    g = torch.Generator(device=dev)
+    g.manual_seed(w.seed + 1000)
+    do = torch.randn((w.batch, w.Hq, w.n, w.d), generator=g, device=dev).to(torch.bfloat16)
+    out, lse = pbb.forward(q, k, v, w.B)
+    stream = torch.cuda.current_stream()
+    for _ in range(warmup):
+        pbb.backward(q, k, v, out, do, lse, w.B)
+    torch.cuda.synchronize()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    uuid = None
+    try:
+        uuid = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:  # noqa: BLE001
+        pass
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(uuid) as clocks:
+        start.record(stream)
+        for i in range(steps):
+            ev[2 * i].record(stream)
+            pbb.backward(q, k, v, out, do, lse, w.B)
+            ev[2 * i + 1].record(stream)
+        end.record(stream)
+        torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    if pbb.get_device_status() != pbb.PBB_OK:
+        raise RuntimeError("device status after the timed backward loop")
+    kern = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
+    return {"total_ms": start.elapsed_time(end), "kernel_ms_mean": sum(kern) / steps,
+            "kernel_ms_median": statistics.median(kern), "clocks": clocks.summary(),
+            "state": (q, k, v, out, do, lse)}
+
+
+def time_backward_e2e(w, dev, steps, state):
+    """The backward through the public API with host-resident tensors: q, k, v, O, dO, lse
+    copied in from pinned host memory and dq, dk, dv copied back, every step, one stream."""
+    import torch
+
+    import paper_2606_02680_gb300 as pbb
+
+    dev_t = state
+    host = [x.cpu().pin_memory() for x in dev_t]
+    stream = torch.cuda.current_stream()
+    outs = None
+
+    def step():
+        nonlocal outs
+        for d_, h_ in zip(dev_t, host):
+            d_.copy_(h_, non_blocking=True)
+        q, k, v, out, do, lse = dev_t
+        dq, dk, dv = pbb.backward(q, k, v, out, do, lse, w.B)
+        if outs is None:
+            outs = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in (dq, dk, dv)]
+        for h_, d_ in zip(outs, (dq, dk, dv)):
+            h_.copy_(d_, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record(stream)
+    for _ in range(steps):
+        step()
+    end.record(stream)
+    end.synchronize()
+    ms = start.elapsed_time(end)
+    return {"value": w.batch * w.Hq * w.n * steps / (ms / 1e3), "unit": UNIT,
+            "h2d_bytes_per_step": sum(x.numel() * x.element_size() for x in host),
+            "d2h_bytes_per_step": sum(x.numel() * x.element_size() for x in outs),
+            "ms_per_step": ms / steps,
+            "api": "paper_2606_02680_gb300.backward (pinned host q/k/v/O/dO/lse in, dq/dk/dv back, one stream)"}
+
+
+def oracle_backward_sample(w, seconds: float):
+    """The fp64 oracle backward on a prefix of one (sequence, KV head) slice of the workload,
+    grown until about `seconds` of CPU time; rows = positions x query heads of the prefix."""
+    import torch
+
+    import oracle
+    from paper_2606_02680_gb300 import inputs
+
+    oracle.build()
+    n = min(w.n, 2 * w.B)
+    done, elapsed = 0, 0.0
+    while True:
+        sub = w.with_(batch=1, Hq=w.group, Hkv=1, n=n)
+        q, k, v = inputs.sequence_inputs(sub)
+        do = torch.randn(q.shape, generator=torch.Generator().manual_seed(1)).to(torch.bfloat16)
+        t_start = time.perf_counter()
+        oracle.backward(q, k, v, do, w.B)
+        elapsed += time.perf_counter() - t_start
+        done += sub.Hq * n
+        if elapsed >= seconds:
+            break
+    return {"value": done / elapsed, "unit": UNIT, "cores": oracle.max_threads(), "kind": "oracle",
+            "seconds": elapsed,
+            "sample": f"{done} (position, query head) rows of {w.name}: repeated backward passes over the "
+                      f"first {n} positions of one sequence and KV head (fp64 chain rule, one thread per "
+                      f"(sequence, KV head), so a single slice runs on one core)"}
+
+
 def oracle_forward_sample(w, seconds: float, rows_per_call: int = 64):
     """The fp64 oracle forward on sampled rows of the workload (one sequence, one KV head)."""
     import numpy as np
@@ -537,13 +668,14 @@ def run_forward(args, dist, rank, world, dev):
     names = [args.fwd_workload] if args.fwd_workload else list(inputs.FORWARD_WORKLOADS)
     hbm, hbm_kind = hbm_peak()
     tpk, tpk_kind = tensor_peak()
+    bwd = args.backward
     for name in names:
         w = inputs.FORWARD_WORKLOADS[name]
         w = w.with_(batch=shard_batch(w.batch, rank, world))
-        res = time_forward(w, dev, args.steps, args.warmup, dist)
+        res = (time_backward if bwd else time_forward)(w, dev, args.steps, args.warmup, dist)
         total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
         units = sum_over_ranks(dist, w.batch * w.Hq * w.n * args.steps)
-        flops, bytes_ = forward_flops_bytes(w)
+        flops, bytes_ = (backward_flops_bytes if bwd else forward_flops_bytes)(w)
         kern_s = res["kernel_ms_mean"] / 1e3
         t_hbm, t_tc = bytes_ / (hbm * 1e9), flops / (tpk * 1e12)
         if t_tc >= t_hbm:
@@ -553,29 +685,34 @@ def run_forward(args, dist, rank, world, dev):
             roof = {"bound": "hbm", "achieved": bytes_ / kern_s / 1e9, "peak": hbm, "unit": "GB/s",
                     "peak_kind": hbm_kind}
         roof["frac"] = roof["achieved"] / roof["peak"]
-        roof.update({"traffic": None, "kernel": "forward_kernel<%d,%d>" % (w.d, w.group),
+        roof.update({"traffic": None,
+                     "kernel": ("bwd_kv_kernel<%d,%d> + bwd_q_kernel<%d,%d> + delta_kernel<%d> (one call)"
+                                % (w.d, w.group, w.d, w.group, w.d)) if bwd else
+                               "forward_kernel<%d,%d>" % (w.d, w.group),
                      "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,
                      "hbm_gbs": bytes_ / kern_s / 1e9, "tflops": flops / kern_s / 1e12,
                      "kernel_ms_mean": res["kernel_ms_mean"], "kernel_ms_median": res["kernel_ms_median"]})
         line = {
-            "metric": METRIC_FWD, "value": units / total_s, "unit": UNIT, "n_gpus": world,
+            "metric": METRIC_BWD if bwd else METRIC_FWD, "value": units / total_s, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
             "data": "synthetic (seeded N(0,1) q/k/v)",
-            "config": {"workload": f"{w.name}: batch {w.batch}, Hq {w.Hq}, Hkv {w.Hkv}, d {w.d}, B {w.B}, n {w.n}, bf16 out + fp32 lse",
+            "config": {"workload": f"{w.name}: batch {w.batch}, Hq {w.Hq}, Hkv {w.Hkv}, d {w.d}, B {w.B}, n {w.n}, "
+                                   + ("bf16 q/k/v/O/dO + fp32 lse in, fp32 dq/dk/dv out" if bwd else "bf16 out + fp32 lse"),
                        "batch_per_gpu": w.batch, "Hq": w.Hq, "Hkv": w.Hkv, "head_dim": w.d, "block": w.B,
                        "n": w.n, "l2": "inputs larger than L2: q/k/v/out %.2f GB" % (bytes_ / 1e9),
                        "parallelism": f"dp{world} (independent sequences, no collective)"},
             "roofline": roof, "clocks": res["clocks"],
-            "timing": "eager launches; CUDA events around every forward launch",
-            "gpu_launches": args.steps,
+            "timing": "eager calls; CUDA events around every " + ("backward call (3 launches)" if bwd else
+                                                                      "forward launch"),
+            "gpu_launches": (3 if bwd else 1) * args.steps,
         }
         if not args.no_e2e:
-            line["e2e"] = time_forward_e2e(w, dev, min(args.steps, 10), res["state"])
+            line["e2e"] = (time_backward_e2e if bwd else time_forward_e2e)(w, dev, min(args.steps, 10), res["state"])
         res.pop("state")
         torch.cuda.empty_cache()
         if rank == 0 and world == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = oracle_forward_sample(w, args.cpu_seconds)
+            line["cpu_baseline"] = (oracle_backward_sample if bwd else oracle_forward_sample)(w, args.cpu_seconds)
         if rank == 0:
             print(json.dumps(line), flush=True)
 
@@ -644,7 +781,7 @@ def run_ours(args):
     torch.cuda.set_device(dev)
     pbb.set_chunk_keys(args.chunk)
 
-    if args.forward:
+    if args.forward or args.backward:
         run_forward(args, dist, rank, world, dev)
         if dist is not None:
             dist.barrier()

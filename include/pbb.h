@@ -174,6 +174,27 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
                 int Hkv, int n, int d, int B, pbb_dtype out_dtype, cudaStream_t stream);
 
 /*
+ * Gradients of pbb_forward (the backward pass of the paper's fused training
+ * kernel, Sec. 3: bridge gradients flow into the previous half-block's K and V).
+ * With P_ts = exp(q_t.k_s/sqrt(d) - lse_t) on A(t) and D_t = dO_t . o_t:
+ *   dq_t = sum_s P_ts (dO_t.v_s - D_t) k_s / sqrt(d)
+ *   dk_s = sum over t (and the group's query heads) of P_ts (dO_t.v_s - D_t) q_t / sqrt(d)
+ *   dv_s = sum over t (and the group's query heads) of P_ts dO_t
+ *   q, out, dout [batch][Hq][n][d] bf16   out and lse from pbb_forward of q, k, v
+ *   k, v        [batch][Hkv][n][d] bf16   lse [batch][Hq][n] fp32
+ *   delta       [batch][Hq][n] fp32      scratch (receives D)
+ *   dq          [batch][Hq][n][d] fp32   dk, dv [batch][Hkv][n][d] fp32 (overwritten)
+ * Same shape rules as pbb_forward; 16-byte aligned tensors (lse, delta 4-byte).
+ * Runs on the tensor cores (mma.sync, bf16 operands with P and dS rounded to
+ * bf16, fp32 accumulation); no floating-point atomics, so results are bitwise
+ * deterministic. Asynchronous on `stream`; a bounded wait that runs out is
+ * reported by pbb_get_device_status as PBB_ERR_DEVICE_TIMEOUT.
+ */
+int pbb_backward(const void* q, const void* k, const void* v, const void* out, const void* dout, const float* lse,
+                 float* delta, float* dq, float* dk, float* dv, int batch, int Hq, int Hkv, int n, int d, int B,
+                 cudaStream_t stream);
+
+/*
  * Load the decode rings of sequences whose first n positions went through
  * pbb_forward (the cache-populating prefill, Appendix F.1): slot j of each ring
  * receives the position s in [n-B, n-1] with s = j (mod B), zeros where s < 0.

@@ -14,6 +14,7 @@ Names follow the C ABI:
 * ``swa_decode_step``                          the sliding-window control over the same rings
 * ``forward``, ``ring_from_sequence``          whole-sequence PBB attention (prefill / training
                                                forward) and the rings it leaves for decoding
+* ``backward``                                 its gradients dq, dk, dv
 * ``decode_step_host``, ``HostPipeline``       the same with host-resident inputs/outputs
                                                (one at a time / overlapped across steps)
 * ``advance_positions``, ``get_device_status``, ``reserve_workspace``,
@@ -31,7 +32,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step", "forward", "ring_from_sequence",
+    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step", "forward", "backward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -62,6 +63,7 @@ EXPORTS = {
     "pbb_swa_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_forward": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_ring_from_sequence": (_I, [_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P]),
+    "pbb_backward": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
     "pbb_get_device_status": (_I, [_P]),
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),
@@ -365,6 +367,31 @@ def forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, B: int, out: torc
                              _dev(lse, "lse", torch.float32) if lse is not None else None,
                              batch, Hq, Hkv, n, d, B, _dt(out.dtype), _stream(stream)), "pbb_forward")
     return out, lse
+
+
+def backward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tensor, dout: torch.Tensor,
+             lse: torch.Tensor, B: int, stream=None):
+    """Gradients (dq, dk, dv), fp32, of pbb_forward (pbb_backward). out and lse are the
+    forward's outputs for q, k, v; dout is the upstream gradient (bf16, shaped like out)."""
+    batch, Hq, n, d = q.shape
+    Hkv = k.shape[1]
+    for name, t, shape in (("k", k, (batch, Hkv, n, d)), ("v", v, (batch, Hkv, n, d)),
+                           ("out", out, (batch, Hq, n, d)), ("dout", dout, (batch, Hq, n, d)),
+                           ("lse", lse, (batch, Hq, n))):
+        if tuple(t.shape) != shape:
+            raise ValueError(f"{name} must have shape {shape}")
+    dev = q.device
+    delta = torch.empty((batch, Hq, n), dtype=torch.float32, device=dev)
+    dq = torch.empty((batch, Hq, n, d), dtype=torch.float32, device=dev)
+    dk = torch.empty((batch, Hkv, n, d), dtype=torch.float32, device=dev)
+    dv = torch.empty((batch, Hkv, n, d), dtype=torch.float32, device=dev)
+    bf = torch.bfloat16
+    _check(lib().pbb_backward(_dev(q, "q", bf), _dev(k, "k", bf), _dev(v, "v", bf), _dev(out, "out", bf),
+                              _dev(dout, "dout", bf), _dev(lse, "lse", torch.float32),
+                              _dev(delta, "delta", torch.float32), _dev(dq, "dq", torch.float32),
+                              _dev(dk, "dk", torch.float32), _dev(dv, "dv", torch.float32), batch, Hq, Hkv, n, d,
+                              B, _stream(stream)), "pbb_backward")
+    return dq, dk, dv
 
 
 def ring_from_sequence(k: torch.Tensor, v: torch.Tensor, k_ring: torch.Tensor, v_ring: torch.Tensor,

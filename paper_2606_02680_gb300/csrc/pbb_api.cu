@@ -412,6 +412,45 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
     return pbb::launch_forward(a, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
 
+int pbb_backward(const void* q, const void* k, const void* v, const void* out, const void* dout, const float* lse,
+                 float* delta, float* dq, float* dk, float* dv, int batch, int Hq, int Hkv, int n, int d, int B,
+                 cudaStream_t stream)
+{
+    int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
+    if (rc != PBB_OK) return rc;
+    rc = check_group(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    if (n < 0) return PBB_ERR_INVALID_ARG;
+    if (batch == 0 || n == 0) return PBB_OK;
+    if (static_cast<long long>(batch) * Hq * n >= (1LL << 31)) return PBB_ERR_UNSUPPORTED;
+    if (!q || !k || !v || !out || !dout || !lse || !delta || !dq || !dk || !dv) return PBB_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16) || !aligned(dout, 16) ||
+        !aligned(lse, 4) || !aligned(delta, 4) || !aligned(dq, 16) || !aligned(dk, 16) || !aligned(dv, 16))
+        return PBB_ERR_INVALID_ARG;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    pbb::BackwardArgs a{};
+    a.q = q;
+    a.k = k;
+    a.v = v;
+    a.out = out;
+    a.dout = dout;
+    a.lse = lse;
+    a.delta = delta;
+    a.dq = dq;
+    a.dk = dk;
+    a.dv = dv;
+    a.batch = batch;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.n = n;
+    a.d = d;
+    a.B = B;
+    a.timeout_ns = g_timeout_ns.load();
+    return pbb::launch_backward(a, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
+}
+
 int pbb_ring_from_sequence(const void* k, const void* v, int n, void* k_ring, void* v_ring, int batch,
                            int Hkv, int d, int B, pbb_dtype dtype, cudaStream_t stream)
 {
@@ -441,10 +480,12 @@ int pbb_get_device_status(cudaStream_t stream)
     int dev = 0;
     int rc = current_device(&dev);
     if (rc != PBB_OK) return rc;
-    int status = 0, fwd_status = 0;
+    int status = 0, fwd_status = 0, bwd_status = 0;
     if (pbb::read_and_clear_status(&status, stream) != cudaSuccess) return PBB_ERR_CUDA;
     if (pbb::read_and_clear_forward_status(&fwd_status) != cudaSuccess) return PBB_ERR_CUDA;
-    if (status == pbb::kDevOk && fwd_status != pbb::kDevOk) return PBB_ERR_DEVICE_TIMEOUT;  // forward kernels only time out
+    if (pbb::read_and_clear_backward_status(&bwd_status) != cudaSuccess) return PBB_ERR_CUDA;
+    if (status == pbb::kDevOk && (fwd_status != pbb::kDevOk || bwd_status != pbb::kDevOk))
+        return PBB_ERR_DEVICE_TIMEOUT;  // forward and backward kernels only time out
     if (status == pbb::kDevOk) return PBB_OK;
     {
         // An aborted step can leave split counters behind: zero them.

@@ -1294,7 +1294,7 @@ bool ring_tensor_map(CUtensorMap* map, const void* ring, unsigned long long rows
         CUtensorMap map;
     };
     static std::mutex mu;
-    static Entry cache[8];
+    static Entry cache[16];
     static int next = 0;
     std::lock_guard<std::mutex> lock(mu);
     for (auto& e : cache)
@@ -1314,7 +1314,7 @@ bool ring_tensor_map(CUtensorMap* map, const void* ring, unsigned long long rows
         CUDA_SUCCESS)
         return false;
     cache[next] = Entry{ring, rows, d, box_rows, m};
-    next = (next + 1) % 8;
+    next = (next + 1) % 16;
     *map = m;
     return true;
 }

@@ -85,4 +85,22 @@ cudaError_t launch_seq_ring(const void* k, const void* v, void* k_ring, void* v_
 // Status word of the forward kernels (read and cleared; the caller synchronises first).
 cudaError_t read_and_clear_forward_status(int* status);
 
+// Whole-sequence backward (pbb_backward.cu).
+struct BackwardArgs {
+    const void* q;      // [batch][Hq][n][d] bf16
+    const void* k;      // [batch][Hkv][n][d] bf16
+    const void* v;      // [batch][Hkv][n][d] bf16
+    const void* out;    // [batch][Hq][n][d] bf16, the forward's output
+    const void* dout;   // [batch][Hq][n][d] bf16, upstream gradient
+    const float* lse;   // [batch][Hq][n], the forward's log-partition
+    float* delta;       // [batch][Hq][n] scratch: dO . O per row
+    float* dq;          // [batch][Hq][n][d]
+    float* dk;          // [batch][Hkv][n][d]
+    float* dv;          // [batch][Hkv][n][d]
+    int batch, Hq, Hkv, n, d, B;
+    unsigned long long timeout_ns;
+};
+cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream);
+cudaError_t read_and_clear_backward_status(int* status);
+
 }  // namespace pbb
