@@ -68,6 +68,10 @@ def parse_args():
     ap.add_argument("--chunk", type=int, default=0, help="keys per CTA (0 = library plan)")
     ap.add_argument("--pattern", choices=["pbb", "swa", "both"], default="pbb",
                     help="attention pattern: PBB (default), the sliding-window control with window B, or both")
+    ap.add_argument("--layers", type=int, default=1,
+                    help="local layers per decode step (shared positions; their own rings and inputs)")
+    ap.add_argument("--layer-launches", choices=["one", "each"], default="one",
+                    help="with --layers > 1: one multi-layer launch per step, or one decode launch per layer")
     ap.add_argument("--forward", action="store_true",
                     help="time the whole-sequence forward (prefill) workloads instead of the decode step")
     ap.add_argument("--backward", action="store_true",
@@ -196,7 +200,10 @@ def describe(w):
             f"t0 ~ U[{w.t0_lo}, {w.t0_hi})")
 
 
-def setup_device_workload(w, dev, pool: int):
+def setup_device_workload(w, dev, pool: int, layers: int = 1):
+    """Rings prefilled at each sequence's start position and a pool of step inputs. With
+    layers > 1 every tensor holds layers x batch sequences (layer-major) that share the batch's
+    positions; pos stays [batch]."""
     import torch
 
     import paper_2606_02680_gb300 as pbb
@@ -205,27 +212,41 @@ def setup_device_workload(w, dev, pool: int):
     t0 = inputs.start_positions(w)
     pos = t0.to(torch.int32).to(dev)
     dt = inputs.torch_dtype(w)
-    k_ring = torch.empty((w.batch, w.Hkv, w.B, w.d), dtype=dt, device=dev)
+    wl = w.with_(batch=layers * w.batch)
+    t_all = t0.repeat(layers)
+    k_ring = torch.empty((wl.batch, w.Hkv, w.B, w.d), dtype=dt, device=dev)
     v_ring = torch.empty_like(k_ring)
-    hk, hv = inputs.history_window(w, t0, device=dev)
-    pbb.ring_prefill(hk, hv, pos, k_ring, v_ring)
+    hk, hv = inputs.history_window(wl, t_all, device=dev)
+    pbb.ring_prefill(hk, hv, t_all.to(torch.int32).to(dev), k_ring, v_ring)
     torch.cuda.synchronize()
     del hk, hv
     torch.cuda.empty_cache()
-    steps_in = [inputs.step_inputs(w, i, device=dev) for i in range(pool)]
+    steps_in = [inputs.step_inputs(wl, i, device=dev) for i in range(pool)]
     return t0, pos, k_ring, v_ring, steps_in
 
 
-def stepper(window):
-    """The decode call of a pattern: PBB (window None) or the sliding window."""
+def stepper(window, layers=1, launches="one"):
+    """The decode call of a step: PBB (window None) or the sliding window; with layers > 1 the
+    tensors hold layers x batch sequences and the step is one multi-layer launch or one launch
+    per layer."""
     import paper_2606_02680_gb300 as pbb
 
+    if layers > 1:
+        def multi(q, k, v, kr, vr, pos, out):
+            L = layers
+            sh = lambda x: x.view(L, x.shape[0] // L, *x.shape[1:])  # noqa: E731
+            if launches == "one":
+                pbb.decode_step_layers(sh(q), sh(k), sh(v), sh(kr), sh(vr), pos, sh(out))
+            else:
+                for l in range(L):
+                    pbb.decode_step(sh(q)[l], sh(k)[l], sh(v)[l], sh(kr)[l], sh(vr)[l], pos, sh(out)[l])
+        return multi
     if window is None:
         return pbb.decode_step
     return lambda q, k, v, kr, vr, pos, out: pbb.swa_decode_step(q, k, v, kr, vr, pos, out, window=window)
 
 
-def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None):
+def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None, layers=1, launches="one"):
     """Device-timed loop; returns dict of timings.
 
     Eager mode records a CUDA event pair around every decode launch inside the
@@ -239,10 +260,10 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None):
     from paper_2606_02680_gb300 import bytemodel
 
     pool = 8
-    decode = stepper(window)
-    t0, pos, k_ring, v_ring, steps_in = setup_device_workload(w, dev, pool)
-    out = torch.empty((w.batch, w.Hq, w.d), dtype=torch.float32, device=dev)
-    pbb.reserve_workspace(w.batch, w.Hq, w.Hkv, w.d, w.B)
+    decode = stepper(window, layers, launches)
+    t0, pos, k_ring, v_ring, steps_in = setup_device_workload(w, dev, pool, layers)
+    out = torch.empty((layers * w.batch, w.Hq, w.d), dtype=torch.float32, device=dev)
+    pbb.reserve_workspace(layers * w.batch, w.Hq, w.Hkv, w.d, w.B)
     stream = torch.cuda.current_stream()
     for i in range(warmup):
         q, k, v = steps_in[i % pool]
@@ -315,7 +336,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None):
             pbb.advance_positions(pos)
         torch.cuda.synchronize()
     kern_ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
-    launch_bytes = [bytemodel.step_bytes(t_np + first + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes, window)
+    launch_bytes = [layers * bytemodel.step_bytes(t_np + first + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes, window)
                     for i in range(steps)]
     res = {
         "total_ms": total_ms,
@@ -803,9 +824,10 @@ def run_ours(args):
     patterns = {"pbb": ["pbb"], "swa": ["swa"], "both": ["pbb", "swa"]}[args.pattern]
     for w, pattern in [(w, p) for w in points for p in patterns]:
         window = w.B if pattern == "swa" else None
-        res = time_device(w, dev, args.steps, args.warmup, dist, args.graph, window)
+        res = time_device(w, dev, args.steps, args.warmup, dist, args.graph, window, args.layers,
+                          args.layer_launches)
         total_s = max_over_ranks(dist, res["total_ms"] / 1e3)
-        units = sum_over_ranks(dist, w.batch * w.Hq * args.steps)
+        units = sum_over_ranks(dist, args.layers * w.batch * w.Hq * args.steps)
         value = units / total_s
         achieved = res["launch_bytes_mean"] / (res["kernel_ms_mean"] / 1e3) / 1e9
         key = w.name if window is None else f"{w.name}_swa"
@@ -841,13 +863,19 @@ def run_ours(args):
             "timing": res["timing"],
             "gpu_launches": 2 * args.steps,
         }
-        if not args.no_e2e and not args.sweep:
+        if not args.no_e2e and not args.sweep and args.layers == 1:
             line["e2e"] = time_e2e(w, dev, args.steps, res["state"], window)
         res.pop("state")
         torch.cuda.empty_cache()
         if window is not None:
             line["config"]["window"] = window
-        if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep and window is None:
+        if args.layers > 1:
+            line["config"]["layers"] = args.layers
+            line["config"]["layer_launches"] = ("one multi-layer launch per step" if args.layer_launches == "one"
+                                                else "one decode launch per layer")
+            line["gpu_launches"] = (2 if args.layer_launches == "one" else args.layers + 1) * args.steps
+        if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep and window is None and \
+                args.layers == 1:
             line["cpu_baseline"] = oracle_sample(w, args.cpu_seconds)
         if rank == 0:
             print(json.dumps(line), flush=True)

@@ -131,6 +131,25 @@ int pbb_decode_step_f32(const float* q, const float* k_new, const float* v_new, 
                         int Hkv, int d, int B, cudaStream_t stream);
 
 /*
+ * One decode step of `layers` PBB local-attention layers in a single launch
+ * (the paper's hybrid runs 15 local layers per token; one launch amortises the
+ * launch latency that dominates small batches). Every tensor gains a leading
+ * layer index, [layers][batch]...: q [layers][batch][Hq][d], k_new/v_new
+ * [layers][batch][Hkv][d], rings [layers][batch][Hkv][B][d], out
+ * [layers][batch][Hq][d]; pos [batch] is shared by all layers (they decode the
+ * same token). Layer l of sequence b computes exactly what pbb_decode_step would
+ * for that layer's tensors; the work of all layers forms one persistent grid.
+ * layers * batch <= 65535; other rules as pbb_decode_step (bf16) and
+ * pbb_decode_step_f32 (PBB_F32). The caller synchronises layer inputs: use this
+ * where every layer's q/k/v of the token are known before the step (batched
+ * evaluation of layers, or benchmarking), and per-layer calls inside a captured
+ * graph otherwise.
+ */
+int pbb_decode_step_layers(const void* q, const void* k_new, const void* v_new, void* k_ring, void* v_ring,
+                           const int32_t* pos, float* out, int layers, int batch, int Hq, int Hkv, int d, int B,
+                           pbb_dtype dtype, cudaStream_t stream);
+
+/*
  * Sliding-window attention decode step over the same rings: the control the
  * paper compares PBB with (Sec. 2.3; Sec. 3 notes that SWA with w = B can also
  * live in a B-slot ring). Identical to pbb_decode_step / pbb_decode_step_f32

@@ -11,6 +11,7 @@ Names follow the C ABI:
 * ``ring_bytes``, ``ring_alloc`` / ``Rings``   the B-slot K/V rings (Appendix F.1)
 * ``ring_prefill``                             load a ring from a history window
 * ``decode_step``                              append + attention over A(t) (Sec. 3)
+* ``decode_step_layers``                       one step of L layers in one launch
 * ``swa_decode_step``                          the sliding-window control over the same rings
 * ``forward``, ``ring_from_sequence``          whole-sequence PBB attention (prefill / training
                                                forward) and the rings it leaves for decoding
@@ -32,7 +33,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "swa_decode_step", "forward", "backward", "ring_from_sequence",
+    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -61,6 +62,7 @@ EXPORTS = {
     "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_swa_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
+    "pbb_decode_step_layers": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_forward": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_ring_from_sequence": (_I, [_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_backward": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
@@ -234,6 +236,33 @@ def decode_step(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_rin
               _dev(k_ring, "k_ring", dtype), _dev(v_ring, "v_ring", dtype),
               _dev(pos, "pos", torch.int32), _dev(out, "out", torch.float32), batch, Hq, Hkv, d, B,
               _stream(stream)), "pbb_decode_step")
+    return out
+
+
+def decode_step_layers(q: torch.Tensor, k_new: torch.Tensor, v_new: torch.Tensor, k_ring: torch.Tensor,
+                       v_ring: torch.Tensor, pos: torch.Tensor, out: torch.Tensor | None = None,
+                       stream=None) -> torch.Tensor:
+    """One decode step of L layers in one launch (pbb_decode_step_layers): q [L, batch, Hq, d],
+    k_new/v_new [L, batch, Hkv, d], rings [L, batch, Hkv, B, d], pos [batch] shared by the layers,
+    out [L, batch, Hq, d] fp32."""
+    L, batch, Hq, d = q.shape
+    _, _, Hkv, B, d2 = k_ring.shape
+    dtype = q.dtype
+    if d2 != d or tuple(k_ring.shape[:2]) != (L, batch) or tuple(v_ring.shape) != tuple(k_ring.shape):
+        raise ValueError("rings must be [L, batch, Hkv, B, d]")
+    if tuple(k_new.shape) != (L, batch, Hkv, d) or tuple(v_new.shape) != (L, batch, Hkv, d):
+        raise ValueError("k_new/v_new must be [L, batch, Hkv, d]")
+    if pos.numel() != batch:
+        raise ValueError("pos must have batch entries")
+    if out is None:
+        out = torch.empty((L, batch, Hq, d), dtype=torch.float32, device=q.device)
+    elif tuple(out.shape) != (L, batch, Hq, d):
+        raise ValueError("out must be [L, batch, Hq, d]")
+    _check(lib().pbb_decode_step_layers(_dev(q, "q", dtype), _dev(k_new, "k_new", dtype),
+                                        _dev(v_new, "v_new", dtype), _dev(k_ring, "k_ring", dtype),
+                                        _dev(v_ring, "v_ring", dtype), _dev(pos, "pos", torch.int32),
+                                        _dev(out, "out", torch.float32), L, batch, Hq, Hkv, d, B, _dt(dtype),
+                                        _stream(stream)), "pbb_decode_step_layers")
     return out
 
 

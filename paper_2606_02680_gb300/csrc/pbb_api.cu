@@ -203,7 +203,7 @@ int grow_workspace(int dev, size_t pairs, size_t pbytes, cudaStream_t stream, bo
 
 int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_ring, void* v_ring,
                 const int32_t* pos, float* out, int batch, int Hq, int Hkv, int d, int B,
-                int window, pbb_dtype dt, cudaStream_t stream)
+                int window, pbb_dtype dt, cudaStream_t stream, int pos_batch = 0)
 {
     int rc = check_shape(batch, Hkv, d, B, dt);
     if (rc != PBB_OK) return rc;
@@ -235,6 +235,7 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     a.d = d;
     a.B = B;
     a.window = window;
+    a.pos_batch = pos_batch > 0 ? pos_batch : batch;
     const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, group, window);
     a.whole = sp.whole;
     a.chunk = sp.chunk;
@@ -366,6 +367,16 @@ int pbb_decode_step_f32(const float* q, const float* k_new, const float* v_new, 
 {
     return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, batch, Hq, Hkv, d, B, 0, PBB_F32,
                        stream);
+}
+
+int pbb_decode_step_layers(const void* q, const void* k_new, const void* v_new, void* k_ring, void* v_ring,
+                           const int32_t* pos, float* out, int layers, int batch, int Hq, int Hkv, int d, int B,
+                           pbb_dtype dtype, cudaStream_t stream)
+{
+    if (layers < 1 || batch < 0) return PBB_ERR_INVALID_ARG;
+    if (static_cast<long long>(layers) * batch > 65535) return PBB_ERR_UNSUPPORTED;
+    return decode_impl(q, k_new, v_new, k_ring, v_ring, pos, out, layers * batch, Hq, Hkv, d, B, 0, dtype,
+                       stream, batch);
 }
 
 int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,

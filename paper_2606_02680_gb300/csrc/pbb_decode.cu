@@ -459,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     chunk = j % a.nchunk;
                 }
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
-                const int t = __ldg(a.pos + b);
+                const int t = __ldg(a.pos + (b < a.pos_batch ? b : b % a.pos_batch));  // layers share positions
                 if (t < 0) {
                     if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
                     continue;
@@ -875,7 +875,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     chunk = j % a.nchunk;
                 }
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
-                const int t = __ldg(a.pos + b);
+                const int t = __ldg(a.pos + (b < a.pos_batch ? b : b % a.pos_batch));  // layers share positions
                 if (t < 0) {
                     if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
                     continue;

@@ -25,6 +25,8 @@ struct DecodeArgs {
     int* counters;       // [batch][Hkv]                 finished chunks per (sequence, KV head)
     int* ctl;            // [2] work-queue head and finished CTAs; zero between launches
     int batch, Hq, Hkv, d, B;
+    int pos_batch;       // sequences with their own position: sequence b reads pos[b % pos_batch]
+                         // (layers of a multi-layer step are consecutive batches sharing positions)
     int window;          // 0: the PBB support [a(t), t]; w in [1, B]: the sliding window {t-w+1, ..., t}
     int whole;           // supports [0, whole) are one work item each
     int chunk;           // ring keys per work item of the later supports (a multiple of the tile)

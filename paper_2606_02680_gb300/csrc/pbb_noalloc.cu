@@ -93,6 +93,7 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
+    a.pos_batch = batch;
     const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, 2, group, 0);  // the same plan as pbb_decode_step
     if (sp.chunk <= 0) return PBB_ERR_CUDA;
     a.whole = sp.whole;
