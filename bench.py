@@ -709,7 +709,7 @@ def run_forward(args, dist, rank, world, dev):
         roof.update({"traffic": None,
                      "kernel": ("bwd_kv_kernel<%d,%d> + bwd_q_kernel<%d,%d> + delta_kernel<%d> (one call)"
                                 % (w.d, w.group, w.d, w.group, w.d)) if bwd else
-                               "forward_kernel<%d,%d>" % (w.d, w.group),
+                               "forward_kernel<%d,%d,%d>" % (w.d, w.group, 128 if w.B >= 512 else 64),
                      "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,
                      "hbm_gbs": bytes_ / kern_s / 1e9, "tflops": flops / kern_s / 1e12,
                      "kernel_ms_mean": res["kernel_ms_mean"], "kernel_ms_median": res["kernel_ms_median"]})

@@ -11,23 +11,24 @@
 // Work items. An item is QT consecutive positions t0 .. t0+QT-1 of all G query
 // heads of one KV head: M = G*QT = 128 query rows, stacked head-major, so every
 // K/V tile serves all G heads (native GQA). Its keys are [a(t0), t_last] (a(t)
-// only grows with t, so the range covers every row), streamed in tiles of 128
+// only grows with t, so the range covers every row), streamed in tiles of 64
 // keys; rows whose support starts later or ends earlier are masked in the tiles
-// that cross their bounds. No dense mask exists anywhere. Persistent CTAs, one
-// per SM, take items round-robin; query tiles of a head are adjacent items, so
-// CTAs running together share K/V tiles in L2.
+// that cross their bounds. No dense mask exists anywhere. Persistent CTAs (one
+// per SM with 128-key tiles for long supports, two per SM with 64-key tiles for
+// short ones; see FwdCfg) take items round-robin; query tiles of a head are
+// adjacent items, so CTAs running together share K/V tiles in L2.
 //
 // Roles (192 threads):
 //   warp 4, one lane   TMA producer: Q of an item (one 2-D tensor copy per head
 //                      and 64-column box; one or two Q buffers), then K and V tiles
-//                      into a 3- or 4-stage ring (128-byte swizzle), all on
+//                      into a 2- to 4-stage ring (128-byte swizzle), all on
 //                      full/empty mbarriers;
-//   warp 5, one lane   MMA issuer: S_j = Q K_j^T (M 128, N 128, both operands
+//   warp 5, one lane   MMA issuer: S_j = Q K_j^T (M 128, N = tile keys, both operands
 //                      K-major in shared memory) into one of two TMEM buffers, then
 //                      O += P_j V_j with P read from tensor memory and V MN-major in
-//                      shared memory, into the item's TMEM output buffer (two,
-//                      alternating between items); each group is completed through
-//                      tcgen05.commit;
+//                      shared memory, into the item's TMEM output buffer (two
+//                      alternating between items, one for narrow tiles at d = 128);
+//                      each group is completed through tcgen05.commit;
 //   warps 0-3          softmax: thread r owns query row r (TMEM lane r). It reads
 //                      its row of S with tcgen05.ld, masks, keeps a running maximum
 //                      (base-2 domain, 1/sqrt(d) folded into one FFMA) that moves
@@ -62,29 +63,38 @@ constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken G
 constexpr int kFwdThreads = 192;                         // 4 softmax warps, producer, MMA issuer
 constexpr int kProducerWarp = 4;
 constexpr int kMmaWarp = 5;
-constexpr int kTmemCols = 512;
 
-template <int D, int G>
+// Two shapes of the same kernel, chosen by the block size (see launch_fwd):
+//   wide   (NK = 128): one CTA per SM with all 512 TMEM columns and up to 225 KB of shared
+//          memory, for long supports (many tiles per item keep the tensor cores busy);
+//   narrow (NK = 64):  two CTAs per SM, each with 256 TMEM columns and under 114 KB, for
+//          short supports, where an item is one or two tiles and the other CTA's work
+//          hides each item's latencies.
+template <int D, int G, int NK_>
 struct FwdCfg {
+    static constexpr int NK = NK_;                      // keys per K/V tile
+    static constexpr bool WIDE = NK == 128;
+    static constexpr int CTAS = WIDE ? 1 : 2;           // CTAs per SM
+    static constexpr int TMEM_COLS = WIDE ? 512 : 256;
     static constexpr int M = 128;                       // query rows of an item (G heads x QT positions)
     static constexpr int QT = M / G;                    // positions of an item
-    static constexpr int NK = 128;                      // keys per K/V tile
     static constexpr int BOXES = D / 64;                // 64-column boxes of a row
     static constexpr int QBOX = M * 128;                // bytes of one Q box
     static constexpr int KBOX = NK * 128;               // bytes of one K (or V) box
     static constexpr int QBUF = D == 64 ? 2 : 1;        // Q buffers (the next item's Q loads early)
-    static constexpr int STAGES = D == 64 ? 4 : 3;      // K/V tiles in flight
+    static constexpr int STAGES = D == 64 ? 4 : (WIDE ? 3 : 2);  // K/V tiles in flight
+    static constexpr int OBUF = (WIDE || D == 64) ? 2 : 1;       // TMEM output buffers (alternate between items)
     static constexpr int Q_OFF = 0;
     static constexpr int Q_BYTES = BOXES * QBOX;
     static constexpr int KV_OFF = Q_OFF + QBUF * Q_BYTES;
     static constexpr int KV_STAGE = 2 * BOXES * KBOX;   // K boxes then V boxes
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;  // + alignment slack
-    // TMEM columns: S buffers at 0 and NK, O buffers at 2 NK and 2 NK + D
+    // TMEM columns: S buffers at 0 and NK, O buffers from 2 NK
     static constexpr int T_S = 0;
     static constexpr int T_O = 2 * NK;
-    static_assert(T_O + 2 * D <= kTmemCols, "TMEM budget");
+    static_assert(T_O + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(QT % 8 == 0, "a head's Q rows must start on a swizzle atom (8 rows)");
-    static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(CTAS * SMEM <= 227 * 1024, "shared memory budget");
 };
 
 // Start of the PBB support of position t: a(t) = max(0, h (floor(t/h) - 1)).
@@ -121,12 +131,12 @@ __device__ __forceinline__ Item make_item(int idx, int n, int B)
     return it;
 }
 
-template <int D, int G>
-__global__ void __launch_bounds__(kFwdThreads, 1)
+template <int D, int G, int NK>
+__global__ void __launch_bounds__(kFwdThreads, FwdCfg<D, G, NK>::CTAS)
 forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                const __grid_constant__ CUtensorMap vmap, const ForwardArgs a)
 {
-    using C = FwdCfg<D, G>;
+    using C = FwdCfg<D, G, NK>;
     constexpr int STAGES = C::STAGES;
     extern __shared__ unsigned char dsmem_raw[];
     constexpr int QBUF = C::QBUF;
@@ -162,7 +172,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         fence_mbar_init();
         abort_s = 0;
     }
-    if (warp == 0) tmem_alloc<kTmemCols>(&tmem_base_s);
+    if (warp == 0) tmem_alloc<C::TMEM_COLS>(&tmem_base_s);
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
@@ -251,7 +261,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             };
             for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
-                const uint32_t ob = ic & 1u;
+                const uint32_t ob = ic % C::OBUF;
                 const uint32_t qb = ic % QBUF;
                 q_base = smem_addr(dsmem + C::Q_OFF + qb * C::Q_BYTES);
                 if (!mbar_wait(&q_full[qb], (ic / QBUF) & 1u, limit) ||
@@ -275,7 +285,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         if (j + 2 == it.ntiles) umma_commit(&q_empty[qb]);  // the item's last read of Q
                     }
                     if (!mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit) ||
-                        (j == 0 && ic >= 2 && !mbar_wait(&o_free[ob], ((ic >> 1) - 1) & 1u, limit))) {
+                        (j == 0 && ic >= C::OBUF && !mbar_wait(&o_free[ob], ((ic / C::OBUF) - 1) & 1u, limit))) {
                         ok = false;
                         break;
                     }
@@ -313,7 +323,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         bool ok = true;
         for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
             const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
-            const uint32_t ob = ic & 1u;
+            const uint32_t ob = ic % C::OBUF;
             const int t = it.t0 + rp;               // this row's position
             const int as = support_start(t, h);     // and its support start
             float m_used = -INFINITY, l = 0.f;
@@ -446,7 +456,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
-    if (warp == 0) tmem_dealloc<kTmemCols>(tmem);
+    if (warp == 0) tmem_dealloc<C::TMEM_COLS>(tmem);
 }
 
 // Sequence -> ring: slot j of each (sequence, KV head) ring gets the position
@@ -479,16 +489,16 @@ __global__ void seq_ring_kernel(const unsigned char* __restrict__ k, const unsig
     }
 }
 
-template <int D, int G>
+template <int D, int G, int NK>
 cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
 {
-    using C = FwdCfg<D, G>;
+    using C = FwdCfg<D, G, NK>;
     static bool attr_set[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 64 && !attr_set[dev]) {
-        err = cudaFuncSetAttribute(forward_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        err = cudaFuncSetAttribute(forward_kernel<D, G, NK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
@@ -504,20 +514,35 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
     int sms = 0;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
-    // one persistent CTA per SM (its shared memory and 512 TMEM columns admit no second)
-    const int grid = static_cast<int>(items < sms ? items : sms);
-    forward_kernel<D, G><<<grid, kFwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, a);
+    // persistent CTAs: C::CTAS per SM, never more than TMEM holds
+    int per_sm = 0;
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, forward_kernel<D, G, NK>, kFwdThreads, C::SMEM);
+    if (err != cudaSuccess) return err;
+    if (per_sm < 1) per_sm = 1;
+    if (per_sm > C::CTAS) per_sm = C::CTAS;
+    const long long slots = static_cast<long long>(sms) * per_sm;
+    const int grid = static_cast<int>(items < slots ? items : slots);
+    forward_kernel<D, G, NK><<<grid, kFwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, a);
     return cudaGetLastError();
+}
+
+// Wide tiles for long supports: from B = 512 an item spans several 128-key tiles
+// (measured on GB300: 1,125 vs 537 TFLOP/s at B = 4096), narrow tiles and two CTAs per
+// SM below (2,169 vs 1,646 GB/s at B = 128, where an item is one tile).
+template <int D, int G>
+cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream)
+{
+    return a.B >= 512 ? launch_fwd<D, G, 128>(a, stream) : launch_fwd<D, G, 64>(a, stream);
 }
 
 template <int D>
 cudaError_t launch_fwd_d(const ForwardArgs& a, cudaStream_t stream)
 {
     switch (a.Hq / a.Hkv) {
-        case 1: return launch_fwd<D, 1>(a, stream);
-        case 2: return launch_fwd<D, 2>(a, stream);
-        case 4: return launch_fwd<D, 4>(a, stream);
-        case 8: return launch_fwd<D, 8>(a, stream);
+        case 1: return launch_fwd_shape<D, 1>(a, stream);
+        case 2: return launch_fwd_shape<D, 2>(a, stream);
+        case 4: return launch_fwd_shape<D, 4>(a, stream);
+        case 8: return launch_fwd_shape<D, 8>(a, stream);
         default: return cudaErrorInvalidValue;
     }
 }
