@@ -707,7 +707,7 @@ def run_forward(args, dist, rank, world, dev):
                     "peak_kind": hbm_kind}
         roof["frac"] = roof["achieved"] / roof["peak"]
         roof.update({"traffic": None,
-                     "kernel": ("bwd_kv_kernel<%d,%d> + bwd_q_kernel<%d,%d> + delta_kernel<%d> (one call)"
+                     "kernel": ("bwd_kv_tc_kernel<%d,%d> + bwd_q_tc_kernel<%d,%d> + delta_kernel<%d> (one call)"
                                 % (w.d, w.group, w.d, w.group, w.d)) if bwd else
                                "forward_kernel<%d,%d,%d>" % (w.d, w.group, 128 if w.B >= 512 else 64),
                      "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,

@@ -8,21 +8,21 @@
 // P is recomputed from the forward's log-partition: P_ts = exp(z_ts - lse_t).
 //
 // Three kernels, none with floating-point atomics (results are deterministic):
-//   delta_kernel   D for every row (dO . O);
-//   bwd_kv_kernel  one CTA per (sequence, KV head, tile of 64 keys): it streams
-//                  the query tiles whose supports hold any of its keys (positions
-//                  s0 .. h(floor(s_last/h) + 2) - 1: the key's own half-block and
-//                  the next one, bridge rows included) with all G heads of the group
-//                  stacked as 64 rows, and accumulates dK and dV for its keys in
-//                  registers (each warp owns 16 keys);
-//   bwd_q_kernel   one CTA per (sequence, KV head, 64 query rows): it streams the
-//                  key tiles of [a(t0), t_last] and accumulates dQ (each warp owns
-//                  16 query rows).
-// Tiles arrive by TMA (128-byte swizzle) through a full/empty mbarrier ring fed by
-// one producer lane; the products are mma.sync m16n8k16 (bf16 operands, fp32
-// accumulation), with P and dS rounded to bf16 as operands. Every wait is bounded by
-// the global timer; a wait that runs out records a timeout and the CTA drains its
-// copies and returns.
+//   delta_kernel       D for every row (dO . O);
+//   bwd_kv_tc_kernel   items of 128 keys of one (sequence, KV head): it streams the
+//                      query tiles (64 rows: the G heads of the group stacked) whose
+//                      supports hold any of its keys (positions s0 .. h(floor(s_last/h)+2)-1,
+//                      the keys' own half-block and the next one, bridge rows included)
+//                      and accumulates dK and dV in tensor memory;
+//   bwd_q_tc_kernel    items of 128 query rows: it streams the key tiles of [a(t0), t_last]
+//                      and accumulates dQ in tensor memory.
+// Both are persistent (one CTA per SM) on the fifth-generation tensor cores: a TMA
+// producer warp (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion
+// through tcgen05.commit on mbarriers) and four elementwise warps whose thread r
+// owns TMEM lane r; P, dS and their transposes are rounded to bf16 and written back
+// over the scores in tensor memory as the A operands of the next products. Every
+// wait is bounded by the global timer; a wait that runs out records a timeout, every
+// role stops, the MMAs and copies in flight are drained and TMEM is released.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -39,27 +39,10 @@ namespace {
 
 constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kGuardNs = 2000000000ull;
-constexpr int kBwdConsumers = 4;
-constexpr int kBwdThreads = (kBwdConsumers + 1) * 32;
 constexpr float kLog2e = 1.4426950408889634f;
-
-template <int D, int G>
-struct BwdCfg {
-    static constexpr int M = 64;              // query rows of a query tile (G heads x QT positions)
-    static constexpr int QT = M / G;
-    static constexpr int KT = 64;             // keys of a key tile (16 per warp)
-    static constexpr int BOXES = D / 64;
-    static constexpr int BOX = 64 * 128;      // one 64-row x 64-column bf16 box
-    static constexpr int TILE = BOXES * BOX;  // one 64-row tile of d columns
-    static constexpr int STAGES = 2;
-    static constexpr int STAGE = 2 * TILE;    // (Q, dO) or (K, V)
-    static constexpr int FIX_OFF = 0;         // the CTA's fixed pair of tiles
-    static constexpr int RING_OFF = 2 * TILE;
-    static constexpr int SMEM = RING_OFF + STAGES * STAGE + 1024;
-    static constexpr int KSTEPS = D / 16;
-    static constexpr int RC = D == 128 ? 16 : 32;  // query rows per inner step of the dK/dV kernel
-    static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
-};
+constexpr int kTcThreads = 192;  // 4 elementwise warps, producer, MMA issuer
+constexpr int kTcProducer = 4;
+constexpr int kTcMma = 5;
 
 __device__ __forceinline__ int support_start(int t, int h)
 {
@@ -67,11 +50,11 @@ __device__ __forceinline__ int support_start(int t, int h)
     return m > 0 ? h * (m - 1) : 0;
 }
 
-// Byte offset of 16-byte chunk ch (0 .. D/8 - 1) of row r in a 64-row tile of BOXES boxes.
-template <int BOX>
-__device__ __forceinline__ uint32_t tile_off(int r, int ch)
+// A bounded wait whose outcome is the same in every lane of the warp (warp-collective
+// tcgen05 loads and stores follow it).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)
 {
-    return static_cast<uint32_t>((ch >> 3) * BOX) + swz(r, ch & 7);
+    return __all_sync(kFull, mbar_wait(bar, parity, limit));
 }
 
 // ---------------------------------------------------------------- delta ----
@@ -101,426 +84,649 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
     if (row < rows && part == 0) delta[row] = acc;
 }
 
-// ------------------------------------------------------------- dK, dV ----
-
+// ------------------------------------------------------------------ dQ ----
+// Items of 128 query rows (G heads x QT positions), key tiles of 64. TMEM: S and dP,
+// two buffers each (dS is written back over S as bf16 pairs, the A operand of
+// dQ += dS K), and two dQ accumulators alternating between items.
 template <int D, int G>
-__global__ void __launch_bounds__(kBwdThreads, 1)
-bwd_kv_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
-              const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
-              const BackwardArgs a)
+struct BqCfg {
+    static constexpr int M = 128, QT = M / G, NK = 64, BOXES = D / 64;
+    static constexpr int QBOX = M * 128, KBOX = NK * 128;
+    static constexpr int Q_OFF = 0, DO_OFF = BOXES * QBOX;
+    static constexpr int KV_OFF = 2 * BOXES * QBOX;
+    static constexpr int KV_STAGE = 2 * BOXES * KBOX;
+    static constexpr int STAGES = 4;
+    static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
+    static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = 4 * NK;
+    static_assert(T_DQ + 2 * D <= 512, "TMEM budget");
+    static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
+};
+
+struct QItem {
+    int pair, t0, tl, lo, a_max, ntiles;
+};
+
+template <int QT, int NK>
+__device__ __forceinline__ QItem make_qitem(int idx, int n, int B)
 {
-    using C = BwdCfg<D, G>;
-    constexpr int STAGES = C::STAGES;
-    extern __shared__ unsigned char dsmem_raw[];
-    __shared__ __align__(8) uint64_t fix_bar, full_bar[STAGES], empty_bar[STAGES];
-    __shared__ volatile int abort_s;
-    unsigned char* dsmem = reinterpret_cast<unsigned char*>(
-        (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-    const int nk = (a.n + C::KT - 1) / C::KT;
-    const int ktile = static_cast<int>(blockIdx.x % static_cast<unsigned>(nk));
-    const int pair = static_cast<int>(blockIdx.x / static_cast<unsigned>(nk));
-    const int b = pair / a.Hkv, kvh = pair - b * a.Hkv;
-    const int h = a.B >> 1;
-    const int s0 = ktile * C::KT;
-    const int s_last = min(s0 + C::KT, a.n) - 1;
-    const int t_end = min(a.n, h * (s_last / h + 2));  // queries past t_end - 1 never see these keys
-    const int tq0 = (s0 / C::QT) * C::QT;             // first query tile (key s is seen from t = s)
-    const int nqt = (t_end - tq0 + C::QT - 1) / C::QT;
-
-    if (tid == 0) {
-        mbar_init(&fix_bar, 1);
-#pragma unroll
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full_bar[s], 1);
-            mbar_init(&empty_bar[s], kBwdConsumers);
-        }
-        fence_mbar_init();
-        abort_s = 0;
-    }
-    __syncthreads();
-
-    int issued = 0;
-    if (warp == kBwdConsumers) {
-        if (lane == 0) {
-            mbar_expect_tx(&fix_bar, static_cast<uint32_t>(2 * C::TILE));
-            const int krow = pair * a.n + s0;
-#pragma unroll
-            for (int bx = 0; bx < C::BOXES; ++bx) {
-                tma_load_2d(dsmem + C::FIX_OFF + bx * C::BOX, &kmap, bx * 64, krow, &fix_bar);
-                tma_load_2d(dsmem + C::FIX_OFF + C::TILE + bx * C::BOX, &vmap, bx * 64, krow, &fix_bar);
-            }
-            for (int it = 0; it < nqt; ++it) {
-                const int s = it % STAGES;
-                if (it >= STAGES &&
-                    !mbar_wait(&empty_bar[s], static_cast<uint32_t>((it / STAGES - 1) & 1), a.timeout_ns)) {
-                    abort_s = 1;
-                    atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
-                    break;
-                }
-                if (abort_s) break;
-                unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
-                mbar_expect_tx(&full_bar[s], static_cast<uint32_t>(C::STAGE));
-                const int t0 = tq0 + it * C::QT;
-#pragma unroll
-                for (int gi = 0; gi < G; ++gi) {
-                    const int qrow = (b * a.Hq + kvh * G + gi) * a.n + t0;
-#pragma unroll
-                    for (int bx = 0; bx < C::BOXES; ++bx) {
-                        tma_load_2d(st + bx * C::BOX + gi * C::QT * 128, &qmap, bx * 64, qrow, &full_bar[s]);
-                        tma_load_2d(st + C::TILE + bx * C::BOX + gi * C::QT * 128, &dmap, bx * 64, qrow,
-                                    &full_bar[s]);
-                    }
-                }
-                ++issued;
-            }
-        }
-    } else {
-        const int g = lane >> 2, tig = lane & 3, lm = lane >> 3;
-        const float sc2 = kLog2e * rsqrtf(static_cast<float>(D));  // base-2 logits
-        const float sc = rsqrtf(static_cast<float>(D));
-        const int key_a = s0 + 16 * warp + g, key_b = key_a + 8;   // this thread's keys (S^T rows)
-        float dk[D / 8][4], dv[D / 8][4];
-#pragma unroll
-        for (int nt = 0; nt < D / 8; ++nt)
-#pragma unroll
-            for (int x = 0; x < 4; ++x) dk[nt][x] = dv[nt][x] = 0.f;
-        bool ok = mbar_wait(&fix_bar, 0u, a.timeout_ns);
-        const uint32_t kbase = smem_addr(dsmem + C::FIX_OFF), vbase = kbase + C::TILE;
-        for (int it = 0; ok && it < nqt; ++it) {
-            const int s = it % STAGES;
-            if (!mbar_wait(&full_bar[s], static_cast<uint32_t>((it / STAGES) & 1), a.timeout_ns) || abort_s) {
-                ok = false;
-                break;
-            }
-            const uint32_t qbase = smem_addr(dsmem + C::RING_OFF + s * C::STAGE), dbase = qbase + C::TILE;
-            const int t0 = tq0 + it * C::QT;
-            constexpr int RC = C::RC, NT = RC / 8, KQ = RC / 16;
-#pragma unroll 1
-            for (int rc = 0; rc < C::M / RC; ++rc) {  // RC query rows at a time
-                // per-row data of the columns (query rows) this thread's fragments touch
-                float l2[NT][2], dl[NT][2];
-                int tpos[NT][2], tstart[NT][2];
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                    for (int e = 0; e < 2; ++e) {
-                        const int R = RC * rc + 8 * nt + 2 * tig + e;
-                        const int gi = R / C::QT;
-                        const int t = t0 + (R - gi * C::QT);
-                        tpos[nt][e] = t;
-                        tstart[nt][e] = support_start(t, h);
-                        const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + (t < a.n ? t : 0);
-                        l2[nt][e] = (t < a.n) ? a.lse[row] * kLog2e : 0.f;
-                        dl[nt][e] = (t < a.n) ? a.delta[row] : 0.f;
-                    }
-                // S^T = K_w Q^T and dP^T = V_w dO^T (16 keys x RC rows)
-                float st[NT][4], dpt[NT][4];
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-                    for (int x = 0; x < 4; ++x) st[nt][x] = dpt[nt][x] = 0.f;
-#pragma unroll
-                for (int kk = 0; kk < C::KSTEPS; ++kk) {
-                    uint32_t ka[4], va[4];
-                    const int arow = 16 * warp + 8 * (lm & 1) + (lane & 7);
-                    const int ach = 2 * kk + (lm >> 1);
-                    ldmatrix_x4(ka, kbase + tile_off<C::BOX>(arow, ach));
-                    ldmatrix_x4(va, vbase + tile_off<C::BOX>(arow, ach));
-#pragma unroll
-                    for (int p = 0; p < KQ; ++p) {
-                        const int brow = RC * rc + 16 * p + 8 * (lm >> 1) + (lane & 7);
-                        const int bch = 2 * kk + (lm & 1);
-                        uint32_t qb[4], db[4];
-                        ldmatrix_x4(qb, qbase + tile_off<C::BOX>(brow, bch));
-                        ldmatrix_x4(db, dbase + tile_off<C::BOX>(brow, bch));
-                        mma_bf16_16816(st[2 * p], ka, qb[0], qb[1]);
-                        mma_bf16_16816(st[2 * p + 1], ka, qb[2], qb[3]);
-                        mma_bf16_16816(dpt[2 * p], va, db[0], db[1]);
-                        mma_bf16_16816(dpt[2 * p + 1], va, db[2], db[3]);
-                    }
-                }
-                // P^T and dS^T, masked to a(t) <= s <= t
-                uint32_t pa[KQ][4], sa[KQ][4];
-#pragma unroll
-                for (int nt = 0; nt < NT; ++nt) {
-                    float p4[4], d4[4];
-#pragma unroll
-                    for (int x = 0; x < 4; ++x) {
-                        const int key = (x < 2) ? key_a : key_b;
-                        const int e = x & 1;
-                        const int t = tpos[nt][e];
-                        const bool vis = key < a.n && t < a.n && key <= t && key >= tstart[nt][e];
-                        const float p = vis ? fast_exp2(fmaf(st[nt][x], sc2, -l2[nt][e])) : 0.f;
-                        p4[x] = p;
-                        d4[x] = p * (dpt[nt][x] - dl[nt][e]);
-                    }
-                    const int kq = nt >> 1, hf = nt & 1;
-                    pa[kq][2 * hf] = pack_bf16x2(p4[0], p4[1]);
-                    pa[kq][2 * hf + 1] = pack_bf16x2(p4[2], p4[3]);
-                    sa[kq][2 * hf] = pack_bf16x2(d4[0], d4[1]);
-                    sa[kq][2 * hf + 1] = pack_bf16x2(d4[2], d4[3]);
-                }
-                // dV_w += P^T dO and dK_w += dS^T Q over these RC rows
-#pragma unroll
-                for (int kq = 0; kq < KQ; ++kq) {
-                    const int vrow = RC * rc + 16 * kq + 8 * (lm & 1) + (lane & 7);
-#pragma unroll
-                    for (int j = 0; j < D / 16; ++j) {
-                        const int ch = 2 * j + (lm >> 1);
-                        uint32_t db[4], qb[4];
-                        ldmatrix_x4_trans(db, dbase + tile_off<C::BOX>(vrow, ch));
-                        ldmatrix_x4_trans(qb, qbase + tile_off<C::BOX>(vrow, ch));
-                        mma_bf16_16816(dv[2 * j], pa[kq], db[0], db[1]);
-                        mma_bf16_16816(dv[2 * j + 1], pa[kq], db[2], db[3]);
-                        mma_bf16_16816(dk[2 * j], sa[kq], qb[0], qb[1]);
-                        mma_bf16_16816(dk[2 * j + 1], sa[kq], qb[2], qb[3]);
-                    }
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty_bar[s]);
-        }
-        if (!ok) {
-            abort_s = 1;
-            atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
-        } else {
-            // rows key_a, key_b; columns 8 nt + 2 tig, +1
-            const size_t base = static_cast<size_t>(pair) * a.n;
-#pragma unroll
-            for (int nt = 0; nt < D / 8; ++nt) {
-                const int col = 8 * nt + 2 * tig;
-                if (key_a < a.n) {
-                    *reinterpret_cast<float2*>(a.dk + (base + key_a) * D + col) = make_float2(dk[nt][0] * sc, dk[nt][1] * sc);
-                    *reinterpret_cast<float2*>(a.dv + (base + key_a) * D + col) = make_float2(dv[nt][0], dv[nt][1]);
-                }
-                if (key_b < a.n) {
-                    *reinterpret_cast<float2*>(a.dk + (base + key_b) * D + col) = make_float2(dk[nt][2] * sc, dk[nt][3] * sc);
-                    *reinterpret_cast<float2*>(a.dv + (base + key_b) * D + col) = make_float2(dv[nt][2], dv[nt][3]);
-                }
-            }
-        }
-    }
-    __syncthreads();
-    if (abort_s && warp == kBwdConsumers && lane == 0) {
-        mbar_wait(&fix_bar, 0u, kGuardNs);
-        for (int s = 0; s < STAGES && s < issued; ++s) {
-            const int j = s + STAGES * ((issued - 1 - s) / STAGES);
-            mbar_wait(&full_bar[s], static_cast<uint32_t>((j / STAGES) & 1), kGuardNs);
-        }
-    }
+    const int nq = (n + QT - 1) / QT;
+    QItem it;
+    it.pair = idx / nq;
+    it.t0 = (idx - it.pair * nq) * QT;
+    it.tl = min(it.t0 + QT, n) - 1;
+    const int h = B >> 1;
+    it.lo = support_start(it.t0, h);
+    it.a_max = support_start(it.tl, h);
+    it.ntiles = (it.tl - it.lo + NK) / NK;
+    return it;
 }
 
-// ------------------------------------------------------------------ dQ ----
-
 template <int D, int G>
-__global__ void __launch_bounds__(kBwdThreads, 1)
-bwd_q_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
-             const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
-             const BackwardArgs a)
+__global__ void __launch_bounds__(kTcThreads, 1)
+bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
+                const BackwardArgs a)
 {
-    using C = BwdCfg<D, G>;
-    constexpr int STAGES = C::STAGES;
+    using C = BqCfg<D, G>;
+    constexpr int STAGES = C::STAGES, NK = C::NK;
     extern __shared__ unsigned char dsmem_raw[];
-    __shared__ __align__(8) uint64_t fix_bar, full_bar[STAGES], empty_bar[STAGES];
+    __shared__ __align__(8) uint64_t q_full, q_empty, done_bar;
+    __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
+    __shared__ __align__(8) uint64_t s_full[2], ds_full[2], item_done[2], o_free[2];
+    __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
         (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-
-    const int nq = (a.n + C::QT - 1) / C::QT;
-    const int qtile = static_cast<int>(blockIdx.x % static_cast<unsigned>(nq));
-    const int pair = static_cast<int>(blockIdx.x / static_cast<unsigned>(nq));
-    const int b = pair / a.Hkv, kvh = pair - b * a.Hkv;
-    const int h = a.B >> 1;
-    const int t0 = qtile * C::QT;
-    const int tl = min(t0 + C::QT, a.n) - 1;
-    const int lo = support_start(t0, h);
-    const int ntiles = (tl - lo + C::KT) / C::KT;
-    const int a_max = support_start(tl, h);
-
+    const int n_items = a.batch * a.Hkv * ((a.n + C::QT - 1) / C::QT);
     if (tid == 0) {
-        mbar_init(&fix_bar, 1);
+        mbar_init(&q_full, 1);
+        mbar_init(&q_empty, 1);
+        mbar_init(&done_bar, 1);
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&full_bar[s], 1);
-            mbar_init(&empty_bar[s], kBwdConsumers);
+            mbar_init(&kv_full[s], 1);
+            mbar_init(&kv_empty[s], 1);
+        }
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&s_full[b], 1);
+            mbar_init(&ds_full[b], 128);
+            mbar_init(&item_done[b], 1);
+            mbar_init(&o_free[b], 128);
         }
         fence_mbar_init();
         abort_s = 0;
     }
+    if (warp == 0) tmem_alloc<512>(&tmem_base_s);
+    tmem_fence_before();
     __syncthreads();
+    tmem_fence_after();
+    const uint32_t tmem = tmem_base_s;
+    const unsigned long long limit = a.timeout_ns;
 
-    int issued = 0;
-    if (warp == kBwdConsumers) {
+    if (warp == kTcProducer) {
         if (lane == 0) {
-            mbar_expect_tx(&fix_bar, static_cast<uint32_t>(2 * C::TILE));
-#pragma unroll
-            for (int gi = 0; gi < G; ++gi) {
-                const int qrow = (b * a.Hq + kvh * G + gi) * a.n + t0;
-#pragma unroll
-                for (int bx = 0; bx < C::BOXES; ++bx) {
-                    tma_load_2d(dsmem + C::FIX_OFF + bx * C::BOX + gi * C::QT * 128, &qmap, bx * 64, qrow, &fix_bar);
-                    tma_load_2d(dsmem + C::FIX_OFF + C::TILE + bx * C::BOX + gi * C::QT * 128, &dmap, bx * 64, qrow,
-                                &fix_bar);
-                }
-            }
-            const int krow0 = pair * a.n + lo;
-            for (int it = 0; it < ntiles; ++it) {
-                const int s = it % STAGES;
-                if (it >= STAGES &&
-                    !mbar_wait(&empty_bar[s], static_cast<uint32_t>((it / STAGES - 1) & 1), a.timeout_ns)) {
-                    abort_s = 1;
-                    atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
+            uint32_t gt = 0, ic = 0, q_issued = 0;
+            bool ok = true;
+            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
+                const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+                if (ic > 0 && !mbar_wait(&q_empty, (ic - 1) & 1u, limit)) {
+                    ok = false;
                     break;
                 }
-                if (abort_s) break;
-                unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
-                mbar_expect_tx(&full_bar[s], static_cast<uint32_t>(C::STAGE));
+                mbar_expect_tx(&q_full, static_cast<uint32_t>(2 * C::BOXES * C::QBOX));
 #pragma unroll
-                for (int bx = 0; bx < C::BOXES; ++bx) {
-                    tma_load_2d(st + bx * C::BOX, &kmap, bx * 64, krow0 + it * C::KT, &full_bar[s]);
-                    tma_load_2d(st + C::TILE + bx * C::BOX, &vmap, bx * 64, krow0 + it * C::KT, &full_bar[s]);
+                for (int gi = 0; gi < G; ++gi) {
+                    const int qrow = (b * a.Hq + kvh * G + gi) * a.n + it.t0;
+#pragma unroll
+                    for (int bx = 0; bx < C::BOXES; ++bx) {
+                        tma_load_2d(dsmem + C::Q_OFF + bx * C::QBOX + gi * C::QT * 128, &qmap, bx * 64, qrow, &q_full);
+                        tma_load_2d(dsmem + C::DO_OFF + bx * C::QBOX + gi * C::QT * 128, &dmap, bx * 64, qrow, &q_full);
+                    }
                 }
-                ++issued;
+                ++q_issued;
+                const int krow0 = it.pair * a.n + it.lo;
+                for (int j = 0; j < it.ntiles; ++j, ++gt) {
+                    const int s = gt % STAGES;
+                    if (gt >= STAGES && !mbar_wait(&kv_empty[s], ((gt / STAGES) - 1) & 1u, limit)) {
+                        ok = false;
+                        break;
+                    }
+                    if (abort_s) {
+                        ok = false;
+                        break;
+                    }
+                    unsigned char* st = dsmem + C::KV_OFF + s * C::KV_STAGE;
+                    mbar_expect_tx(&kv_full[s], static_cast<uint32_t>(C::KV_STAGE));
+#pragma unroll
+                    for (int bx = 0; bx < C::BOXES; ++bx) {
+                        tma_load_2d(st + bx * C::KBOX, &kmap, bx * 64, krow0 + j * NK, &kv_full[s]);
+                        tma_load_2d(st + (C::BOXES + bx) * C::KBOX, &vmap, bx * 64, krow0 + j * NK, &kv_full[s]);
+                    }
+                }
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
+            }
+            // drain: the last copies into Q/dO and into each stage land before shared memory goes away
+            if (q_issued > 0) mbar_wait(&q_full, (q_issued - 1) & 1u, kGuardNs);
+            for (uint32_t s = 0; s < STAGES && s < gt; ++s) {
+                const uint32_t j = s + STAGES * ((gt - 1 - s) / STAGES);
+                mbar_wait(&kv_full[s], (j / STAGES) & 1u, kGuardNs);
+            }
+        }
+    } else if (warp == kTcMma) {
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NK, 0);
+            constexpr uint32_t idesc_q = umma_idesc_bf16(C::M, D, 1);
+            const uint32_t q_base = smem_addr(dsmem + C::Q_OFF), do_base = smem_addr(dsmem + C::DO_OFF);
+            const uint32_t kv_base = smem_addr(dsmem + C::KV_OFF);
+            uint32_t gt = 0, ic = 0;
+            bool ok = true, issued_any = false;
+            auto issue_sdp = [&](uint32_t g) {  // S = Q K^T and dP = dO V^T into buffer g % 2
+                const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE, vb = kb + C::BOXES * C::KBOX;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * C::QBOX + (kk & 3) * 32;
+                    const uint32_t koff = (kk >> 2) * C::KBOX + (kk & 3) * 32;
+                    umma_bf16(tmem + C::T_S + (g & 1u) * NK, umma_desc_sw128(q_base + off, 16, 1024),
+                              umma_desc_sw128(kb + koff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
+                    umma_bf16(tmem + C::T_DP + (g & 1u) * NK, umma_desc_sw128(do_base + off, 16, 1024),
+                              umma_desc_sw128(vb + koff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&s_full[g & 1u]);
+            };
+            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
+                const uint32_t ob = ic & 1u;
+                if (!mbar_wait(&q_full, ic & 1u, limit) || !mbar_wait(&kv_full[gt % STAGES], (gt / STAGES) & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                issue_sdp(gt);
+                issued_any = true;
+                if (it.ntiles == 1) umma_commit(&q_empty);
+                for (int j = 0; j < it.ntiles; ++j) {
+                    const uint32_t g = gt + j;
+                    if (j + 1 < it.ntiles) {
+                        if (!mbar_wait(&kv_full[(g + 1) % STAGES], ((g + 1) / STAGES) & 1u, limit)) {
+                            ok = false;
+                            break;
+                        }
+                        tmem_fence_after();
+                        issue_sdp(g + 1);
+                        if (j + 2 == it.ntiles) umma_commit(&q_empty);  // the item's last read of Q and dO
+                    }
+                    if (!mbar_wait(&ds_full[g & 1u], (g >> 1) & 1u, limit) ||
+                        (j == 0 && ic >= 2 && !mbar_wait(&o_free[ob], ((ic >> 1) - 1) & 1u, limit))) {
+                        ok = false;
+                        break;
+                    }
+                    tmem_fence_after();
+                    // dQ (+)= dS K: dS from TMEM (over S buffer g % 2), K MN-major
+                    const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
+#pragma unroll
+                    for (int kk = 0; kk < NK / 16; ++kk)
+                        umma_bf16_tmem_a(tmem + C::T_DQ + ob * D, tmem + C::T_S + (g & 1u) * NK + 8 * kk,
+                                         umma_desc_sw128(kb + kk * 2048, C::KBOX, 1024), idesc_q,
+                                         (j > 0 || kk > 0) ? 1u : 0u);
+                    umma_commit(&kv_empty[g % STAGES]);
+                }
+                if (!ok) break;
+                umma_commit(&item_done[ob]);
+                gt += it.ntiles;
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
+            }
+            if (issued_any) {  // every MMA complete before TMEM is released
+                umma_commit(&done_bar);
+                mbar_wait(&done_bar, 0u, kGuardNs);
             }
         }
     } else {
-        const int g = lane >> 2, tig = lane & 3, lm = lane >> 3;
-        const float sc2 = kLog2e * rsqrtf(static_cast<float>(D));
-        const float sc = rsqrtf(static_cast<float>(D));
-        const int r0 = 16 * warp + g, r1 = r0 + 8;
-        const int gi0 = r0 / C::QT, gi1 = r1 / C::QT;
-        const int tp0 = t0 + r0 - gi0 * C::QT, tp1 = t0 + r1 - gi1 * C::QT;
-        const int as0 = support_start(tp0, h), as1 = support_start(tp1, h);
-        const size_t row0 = static_cast<size_t>(b * a.Hq + kvh * G + gi0) * a.n + tp0;
-        const size_t row1 = static_cast<size_t>(b * a.Hq + kvh * G + gi1) * a.n + tp1;
-        const bool w0 = tp0 < a.n, w1 = tp1 < a.n;
-        const float l20 = w0 ? a.lse[row0] * kLog2e : 0.f, l21 = w1 ? a.lse[row1] * kLog2e : 0.f;
-        const float dl0 = w0 ? a.delta[row0] : 0.f, dl1 = w1 ? a.delta[row1] : 0.f;
-        float dq[D / 8][4];
+        // elementwise: thread r owns query row r
+        const int r = tid;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+        const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
+        const int h = a.B >> 1;
+        const int gi = r / C::QT, rp = r - gi * C::QT;
+        uint32_t gt = 0, ic = 0;
+        bool ok = true;
+        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
+            const uint32_t ob = ic & 1u;
+            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+            const int t = it.t0 + rp, as = support_start(t, h);
+            const bool valid = t < a.n;
+            const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + (valid ? t : 0);
+            const float l2 = valid ? a.lse[row] * kLog2e : 0.f, dr = valid ? a.delta[row] : 0.f;
+            for (int j = 0; j < it.ntiles; ++j) {
+                const uint32_t g = gt + j;
+                if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                const int key0 = it.lo + j * NK;
+                const bool edge = (key0 + NK - 1 > it.t0) || (key0 < it.a_max);
+                // 32 columns at a time: their dS (16 bf16-pair columns) goes over columns already read
 #pragma unroll
-        for (int nt = 0; nt < D / 8; ++nt)
+                for (int c = 0; c < NK / 32; ++c) {
+                    uint32_t v1[32], v2[32];
+                    tmem_ld32(lane_base + C::T_S + (g & 1u) * NK + 32 * c, v1);
+                    tmem_ld32(lane_base + C::T_DP + (g & 1u) * NK + 32 * c, v2);
+                    tmem_wait_ld();
+                    uint32_t pk[16];
 #pragma unroll
-            for (int x = 0; x < 4; ++x) dq[nt][x] = 0.f;
-        bool ok = mbar_wait(&fix_bar, 0u, a.timeout_ns);
-        uint32_t qa[C::KSTEPS][4], da[C::KSTEPS][4];
-        if (ok) {
-            const uint32_t qbase = smem_addr(dsmem + C::FIX_OFF), dbase = qbase + C::TILE;
-            const int row = 16 * warp + 8 * (lm & 1) + (lane & 7);
+                    for (int x = 0; x < 16; ++x) {
+                        float e[2];
 #pragma unroll
-            for (int kk = 0; kk < C::KSTEPS; ++kk) {
-                const int ch = 2 * kk + (lm >> 1);
-                ldmatrix_x4(qa[kk], qbase + tile_off<C::BOX>(row, ch));
-                ldmatrix_x4(da[kk], dbase + tile_off<C::BOX>(row, ch));
+                        for (int y = 0; y < 2; ++y) {
+                            const int key = key0 + 32 * c + 2 * x + y;
+                            const bool vis = valid && (!edge || (key >= as && key <= t));
+                            const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -l2)) : 0.f;
+                            e[y] = p * (__uint_as_float(v2[2 * x + y]) - dr);
+                        }
+                        pk[x] = pack_bf16x2(e[0], e[1]);
+                    }
+                    tmem_st16(lane_base + C::T_S + (g & 1u) * NK + 16 * c, pk);
+                }
+                tmem_wait_st();
+                tmem_fence_before();
+                mbar_arrive(&ds_full[g & 1u]);
             }
-        }
-        for (int it = 0; ok && it < ntiles; ++it) {
-            const int s = it % STAGES;
-            if (!mbar_wait(&full_bar[s], static_cast<uint32_t>((it / STAGES) & 1), a.timeout_ns) || abort_s) {
+            if (!ok) break;
+            if (!warp_wait(&item_done[ob], (ic >> 1) & 1u, limit)) {
                 ok = false;
                 break;
             }
-            const uint32_t kbase = smem_addr(dsmem + C::RING_OFF + s * C::STAGE), vbase = kbase + C::TILE;
-            const int key0 = lo + it * C::KT;
-            // S = Q_w K^T and dP = dO_w V^T (16 rows x 64 keys)
-            float sf[8][4], dp[8][4];
+            tmem_fence_after();
 #pragma unroll
-            for (int nt = 0; nt < 8; ++nt)
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(lane_base + C::T_DQ + ob * D + 32 * c, v);
+                tmem_wait_ld();
+                if (valid) {
+                    float4* dst = reinterpret_cast<float4*>(a.dq + row * D + 32 * c);
 #pragma unroll
-                for (int x = 0; x < 4; ++x) sf[nt][x] = dp[nt][x] = 0.f;
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int krow = 16 * j + 8 * (lm >> 1) + (lane & 7);
-#pragma unroll
-                for (int kk = 0; kk < C::KSTEPS; ++kk) {
-                    const int ch = 2 * kk + (lm & 1);
-                    uint32_t kb[4], vb[4];
-                    ldmatrix_x4(kb, kbase + tile_off<C::BOX>(krow, ch));
-                    ldmatrix_x4(vb, vbase + tile_off<C::BOX>(krow, ch));
-                    mma_bf16_16816(sf[2 * j], qa[kk], kb[0], kb[1]);
-                    mma_bf16_16816(sf[2 * j + 1], qa[kk], kb[2], kb[3]);
-                    mma_bf16_16816(dp[2 * j], da[kk], vb[0], vb[1]);
-                    mma_bf16_16816(dp[2 * j + 1], da[kk], vb[2], vb[3]);
+                    for (int x = 0; x < 8; ++x)
+                        dst[x] = make_float4(__uint_as_float(v[4 * x]) * sc, __uint_as_float(v[4 * x + 1]) * sc,
+                                             __uint_as_float(v[4 * x + 2]) * sc, __uint_as_float(v[4 * x + 3]) * sc);
                 }
             }
-            const bool edge = (key0 + C::KT - 1 > t0) || (key0 < a_max);
-            uint32_t sa[4][4];  // dS as bf16 A-fragments, one per 16-key k-step
-#pragma unroll
-            for (int nt = 0; nt < 8; ++nt) {
-                float d4[4];
-#pragma unroll
-                for (int x = 0; x < 4; ++x) {
-                    const int key = key0 + 8 * nt + 2 * tig + (x & 1);
-                    const bool hi = x >= 2;
-                    bool vis = hi ? w1 : w0;
-                    if (edge) vis = vis && (hi ? (key >= as1 && key <= tp1) : (key >= as0 && key <= tp0));
-                    const float p = vis ? fast_exp2(fmaf(sf[nt][x], sc2, -(hi ? l21 : l20))) : 0.f;
-                    d4[x] = p * (dp[nt][x] - (hi ? dl1 : dl0));
-                }
-                const int kq = nt >> 1, hf = nt & 1;
-                sa[kq][2 * hf] = pack_bf16x2(d4[0], d4[1]);
-                sa[kq][2 * hf + 1] = pack_bf16x2(d4[2], d4[3]);
-            }
-            // dQ_w += dS K
-#pragma unroll
-            for (int kq = 0; kq < 4; ++kq) {
-                const int krow = 16 * kq + 8 * (lm & 1) + (lane & 7);
-#pragma unroll
-                for (int j = 0; j < D / 16; ++j) {
-                    const int ch = 2 * j + (lm >> 1);
-                    uint32_t kb[4];
-                    ldmatrix_x4_trans(kb, kbase + tile_off<C::BOX>(krow, ch));
-                    mma_bf16_16816(dq[2 * j], sa[kq], kb[0], kb[1]);
-                    mma_bf16_16816(dq[2 * j + 1], sa[kq], kb[2], kb[3]);
-                }
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty_bar[s]);
+            tmem_fence_before();
+            mbar_arrive(&o_free[ob]);
+            gt += it.ntiles;
         }
         if (!ok) {
             abort_s = 1;
             atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
-        } else {
+        }
+    }
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    if (warp == 0) tmem_dealloc<512>(tmem);
+}
+
+// ------------------------------------------------------------- dK, dV ----
+// Items of 128 keys, query tiles of 64 rows (G heads x QT positions). TMEM: S^T and
+// dP^T, two buffers each (P^T and dS^T are written back over them as bf16 pairs, the
+// A operands of dV += P^T dO and dK += dS^T Q), then dV and dK. Per query tile the
+// producer warp also stages, for each of its 64 columns, the base-2 log-partition, D,
+// the position and its support start.
+template <int D, int G>
+struct BkvCfg {
+    static constexpr int M = 128, NQ = 64, QT = NQ / G, BOXES = D / 64;
+    static constexpr int KBOX = M * 128, QBOX = NQ * 128;
+    static constexpr int K_OFF = 0, V_OFF = BOXES * KBOX;
+    static constexpr int RING_OFF = 2 * BOXES * KBOX;
+    static constexpr int META = NQ * 16;                          // float4 per column
+    static constexpr int STAGE = 2 * BOXES * QBOX + META;         // Q, dO, metadata
+    static constexpr int STAGES = 3;
+    static constexpr int SMEM = RING_OFF + STAGES * STAGE + 1024;
+    static constexpr int T_ST = 0, T_DPT = 2 * NQ, T_DV = 4 * NQ, T_DK = 4 * NQ + D;
+    static_assert(T_DK + D <= 512, "TMEM budget");
+    static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
+    static_assert(STAGE % 1024 == 0, "stage boxes stay 1024-aligned");
+};
+
+struct KItem {
+    int pair, s0, tq0, nqt;
+};
+
+template <int QT>
+__device__ __forceinline__ KItem make_kitem(int idx, int n, int B)
+{
+    const int nk = (n + 127) / 128;
+    KItem it;
+    it.pair = idx / nk;
+    it.s0 = (idx - it.pair * nk) * 128;
+    const int s_last = min(it.s0 + 128, n) - 1;
+    const int h = B >> 1;
+    const int t_end = min(n, h * (s_last / h + 2));  // queries past t_end - 1 never see these keys
+    it.tq0 = (it.s0 / QT) * QT;
+    it.nqt = (t_end - it.tq0 + QT - 1) / QT;
+    return it;
+}
+
+template <int D, int G>
+__global__ void __launch_bounds__(kTcThreads, 1)
+bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                 const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
+                 const BackwardArgs a)
+{
+    using C = BkvCfg<D, G>;
+    constexpr int STAGES = C::STAGES, NQ = C::NQ;
+    extern __shared__ unsigned char dsmem_raw[];
+    __shared__ __align__(8) uint64_t kv_full, kv_empty, done_bar, item_done, o_free;
+    __shared__ __align__(8) uint64_t qd_full[STAGES], qd_empty[STAGES];
+    __shared__ __align__(8) uint64_t s_full[2], p_full[2];
+    __shared__ uint32_t tmem_base_s;
+    __shared__ volatile int abort_s;
+    unsigned char* dsmem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int n_items = a.batch * a.Hkv * ((a.n + 127) / 128);
+    if (tid == 0) {
+        mbar_init(&kv_full, 1);
+        mbar_init(&kv_empty, 1);
+        mbar_init(&done_bar, 1);
+        mbar_init(&item_done, 1);
+        mbar_init(&o_free, 128);
 #pragma unroll
-            for (int nt = 0; nt < D / 8; ++nt) {
-                const int col = 8 * nt + 2 * tig;
-                if (w0) *reinterpret_cast<float2*>(a.dq + row0 * D + col) = make_float2(dq[nt][0] * sc, dq[nt][1] * sc);
-                if (w1) *reinterpret_cast<float2*>(a.dq + row1 * D + col) = make_float2(dq[nt][2] * sc, dq[nt][3] * sc);
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&qd_full[s], 1);
+            mbar_init(&qd_empty[s], 1);
+        }
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(&s_full[b], 1);
+            mbar_init(&p_full[b], 128);
+        }
+        fence_mbar_init();
+        abort_s = 0;
+    }
+    if (warp == 0) tmem_alloc<512>(&tmem_base_s);
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    const uint32_t tmem = tmem_base_s;
+    const unsigned long long limit = a.timeout_ns;
+    const int h = a.B >> 1;
+
+    if (warp == kTcProducer) {
+        // the whole warp: lane 0 issues the copies, every lane stages two columns' metadata
+        uint32_t gt = 0, ic = 0, kv_issued = 0;
+        bool ok = true;
+        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
+            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+            if (ic > 0 && !warp_wait(&kv_empty, (ic - 1) & 1u, limit)) {
+                ok = false;
+                break;
+            }
+            if (lane == 0) {
+                mbar_expect_tx(&kv_full, static_cast<uint32_t>(2 * C::BOXES * C::KBOX));
+#pragma unroll
+                for (int bx = 0; bx < C::BOXES; ++bx) {
+                    tma_load_2d(dsmem + C::K_OFF + bx * C::KBOX, &kmap, bx * 64, it.pair * a.n + it.s0, &kv_full);
+                    tma_load_2d(dsmem + C::V_OFF + bx * C::KBOX, &vmap, bx * 64, it.pair * a.n + it.s0, &kv_full);
+                }
+            }
+            ++kv_issued;
+            for (int i = 0; i < it.nqt; ++i, ++gt) {
+                const int s = gt % STAGES;
+                if (gt >= STAGES && !warp_wait(&qd_empty[s], ((gt / STAGES) - 1) & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
+                if (__any_sync(kFull, abort_s != 0)) {
+                    ok = false;
+                    break;
+                }
+                unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
+                const int t0 = it.tq0 + i * C::QT;
+                float4* meta = reinterpret_cast<float4*>(st + 2 * C::BOXES * C::QBOX);
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int c = lane + 32 * e;
+                    const int gi = c / C::QT, t = t0 + (c - gi * C::QT);
+                    const bool valid = t < a.n;
+                    const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + (valid ? t : 0);
+                    meta[c] = make_float4(valid ? a.lse[row] * kLog2e : 0.f, valid ? a.delta[row] : 0.f,
+                                          __int_as_float(valid ? t : -1), __int_as_float(support_start(t, h)));
+                }
+                __threadfence_block();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_expect_tx(&qd_full[s], static_cast<uint32_t>(2 * C::BOXES * C::QBOX));
+#pragma unroll
+                    for (int gi = 0; gi < G; ++gi) {
+                        const int qrow = (b * a.Hq + kvh * G + gi) * a.n + t0;
+#pragma unroll
+                        for (int bx = 0; bx < C::BOXES; ++bx) {
+                            tma_load_2d(st + bx * C::QBOX + gi * C::QT * 128, &qmap, bx * 64, qrow, &qd_full[s]);
+                            tma_load_2d(st + (C::BOXES + bx) * C::QBOX + gi * C::QT * 128, &dmap, bx * 64, qrow,
+                                        &qd_full[s]);
+                        }
+                    }
+                }
             }
         }
-    }
-    __syncthreads();
-    if (abort_s && warp == kBwdConsumers && lane == 0) {
-        mbar_wait(&fix_bar, 0u, kGuardNs);
-        for (int s = 0; s < STAGES && s < issued; ++s) {
-            const int j = s + STAGES * ((issued - 1 - s) / STAGES);
-            mbar_wait(&full_bar[s], static_cast<uint32_t>((j / STAGES) & 1), kGuardNs);
+        if (!ok && lane == 0) {
+            abort_s = 1;
+            atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
+        }
+        if (lane == 0) {  // drain the copies still in flight
+            if (kv_issued > 0) mbar_wait(&kv_full, (kv_issued - 1) & 1u, kGuardNs);
+            for (uint32_t s = 0; s < STAGES && s < gt; ++s) {
+                const uint32_t j = s + STAGES * ((gt - 1 - s) / STAGES);
+                mbar_wait(&qd_full[s], (j / STAGES) & 1u, kGuardNs);
+            }
+        }
+    } else if (warp == kTcMma) {
+        if (lane == 0) {
+            constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NQ, 0);
+            constexpr uint32_t idesc_o = umma_idesc_bf16(C::M, D, 1);
+            const uint32_t k_base = smem_addr(dsmem + C::K_OFF), v_base = smem_addr(dsmem + C::V_OFF);
+            const uint32_t ring = smem_addr(dsmem + C::RING_OFF);
+            uint32_t gt = 0, ic = 0;
+            bool ok = true, issued_any = false;
+            auto issue_sdp = [&](uint32_t g) {  // S^T = K Q^T and dP^T = V dO^T into buffer g % 2
+                if (!mbar_wait(&qd_full[g % STAGES], (g / STAGES) & 1u, limit)) return false;
+                tmem_fence_after();
+                const uint32_t qb = ring + (g % STAGES) * C::STAGE, db = qb + C::BOXES * C::QBOX;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t koff = (kk >> 2) * C::KBOX + (kk & 3) * 32;
+                    const uint32_t qoff = (kk >> 2) * C::QBOX + (kk & 3) * 32;
+                    umma_bf16(tmem + C::T_ST + (g & 1u) * NQ, umma_desc_sw128(k_base + koff, 16, 1024),
+                              umma_desc_sw128(qb + qoff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
+                    umma_bf16(tmem + C::T_DPT + (g & 1u) * NQ, umma_desc_sw128(v_base + koff, 16, 1024),
+                              umma_desc_sw128(db + qoff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&s_full[g & 1u]);
+                return true;
+            };
+            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
+                if (!mbar_wait(&kv_full, ic & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                if (!issue_sdp(gt)) {
+                    ok = false;
+                    break;
+                }
+                issued_any = true;
+                for (int i = 0; i < it.nqt; ++i) {
+                    const uint32_t g = gt + i;
+                    if (i + 1 < it.nqt && !issue_sdp(g + 1)) {
+                        ok = false;
+                        break;
+                    }
+                    if (!mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit) ||
+                        (i == 0 && ic >= 1 && !mbar_wait(&o_free, (ic - 1) & 1u, limit))) {
+                        ok = false;
+                        break;
+                    }
+                    tmem_fence_after();
+                    // dV (+)= P^T dO and dK (+)= dS^T Q: A from TMEM, B (dO, Q) MN-major
+                    const uint32_t qb = ring + (g % STAGES) * C::STAGE, db = qb + C::BOXES * C::QBOX;
+#pragma unroll
+                    for (int kk = 0; kk < NQ / 16; ++kk) {
+                        const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+                        umma_bf16_tmem_a(tmem + C::T_DV, tmem + C::T_ST + (g & 1u) * NQ + 8 * kk,
+                                         umma_desc_sw128(db + kk * 2048, C::QBOX, 1024), idesc_o, acc);
+                        umma_bf16_tmem_a(tmem + C::T_DK, tmem + C::T_DPT + (g & 1u) * NQ + 8 * kk,
+                                         umma_desc_sw128(qb + kk * 2048, C::QBOX, 1024), idesc_o, acc);
+                    }
+                    umma_commit(&qd_empty[g % STAGES]);
+                }
+                if (!ok) break;
+                umma_commit(&kv_empty);
+                umma_commit(&item_done);
+                gt += it.nqt;
+            }
+            if (!ok) {
+                abort_s = 1;
+                atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
+            }
+            if (issued_any) {  // every MMA complete before TMEM is released
+                umma_commit(&done_bar);
+                mbar_wait(&done_bar, 0u, kGuardNs);
+            }
+        }
+    } else {
+        // elementwise: thread r owns key row r
+        const int r = tid;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+        const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
+        uint32_t gt = 0, ic = 0;
+        bool ok = true;
+        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
+            const int key = it.s0 + r;
+            const bool kvalid = key < a.n;
+            for (int i = 0; i < it.nqt; ++i) {
+                const uint32_t g = gt + i;
+                if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
+                                                                     2 * C::BOXES * C::QBOX);
+                // 32 columns at a time: their P^T and dS^T (16 bf16-pair columns each) go over
+                // columns already read
+#pragma unroll
+                for (int c = 0; c < NQ / 32; ++c) {
+                    uint32_t v1[32], v2[32];
+                    tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + 32 * c, v1);
+                    tmem_ld32(lane_base + C::T_DPT + (g & 1u) * NQ + 32 * c, v2);
+                    tmem_wait_ld();
+                    uint32_t pk[16], dk[16];
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) {
+                        float pe[2], de[2];
+#pragma unroll
+                        for (int y = 0; y < 2; ++y) {
+                            const int cc = 32 * c + 2 * x + y;
+                            const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc
+                            const int t = __float_as_int(m.z), at = __float_as_int(m.w);
+                            const bool vis = kvalid && key <= t && key >= at;
+                            const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -m.x)) : 0.f;
+                            pe[y] = p;
+                            de[y] = p * (__uint_as_float(v2[2 * x + y]) - m.y);
+                        }
+                        pk[x] = pack_bf16x2(pe[0], pe[1]);
+                        dk[x] = pack_bf16x2(de[0], de[1]);
+                    }
+                    tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, pk);
+                    tmem_st16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, dk);
+                }
+                tmem_wait_st();
+                tmem_fence_before();
+                mbar_arrive(&p_full[g & 1u]);
+            }
+            if (!ok) break;
+            if (!warp_wait(&item_done, ic & 1u, limit)) {
+                ok = false;
+                break;
+            }
+            tmem_fence_after();
+            const size_t row = static_cast<size_t>(it.pair) * a.n + (kvalid ? key : 0);
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32], w[32];
+                tmem_ld32(lane_base + C::T_DV + 32 * c, v);
+                tmem_ld32(lane_base + C::T_DK + 32 * c, w);
+                tmem_wait_ld();
+                if (kvalid) {
+                    float4* dv = reinterpret_cast<float4*>(a.dv + row * D + 32 * c);
+                    float4* dk = reinterpret_cast<float4*>(a.dk + row * D + 32 * c);
+#pragma unroll
+                    for (int x = 0; x < 8; ++x) {
+                        dv[x] = make_float4(__uint_as_float(v[4 * x]), __uint_as_float(v[4 * x + 1]),
+                                            __uint_as_float(v[4 * x + 2]), __uint_as_float(v[4 * x + 3]));
+                        dk[x] = make_float4(__uint_as_float(w[4 * x]) * sc, __uint_as_float(w[4 * x + 1]) * sc,
+                                            __uint_as_float(w[4 * x + 2]) * sc, __uint_as_float(w[4 * x + 3]) * sc);
+                    }
+                }
+            }
+            tmem_fence_before();
+            mbar_arrive(&o_free);
+            gt += it.nqt;
+        }
+        if (!ok) {
+            abort_s = 1;
+            atomicCAS(&g_bwd_status, kDevOk, kDevTimeout);
         }
     }
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    if (warp == 0) tmem_dealloc<512>(tmem);
 }
 
 template <int D, int G>
 cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
 {
-    using C = BwdCfg<D, G>;
+    using CQ = BqCfg<D, G>;
+    using CK = BkvCfg<D, G>;
     static bool attr_set[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 64 && !attr_set[dev]) {
-        err = cudaFuncSetAttribute(bwd_kv_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        err = cudaFuncSetAttribute(bwd_kv_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, CK::SMEM);
         if (err != cudaSuccess) return err;
-        err = cudaFuncSetAttribute(bwd_q_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        err = cudaFuncSetAttribute(bwd_q_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, CQ::SMEM);
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
     const unsigned long long qrows = static_cast<unsigned long long>(a.batch) * a.Hq * a.n;
     const unsigned long long krows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.n;
-    CUtensorMap qmap, kmap, vmap, dmap;
-    if (!rows_tensor_map(&qmap, a.q, qrows, D, C::QT) || !rows_tensor_map(&dmap, a.dout, qrows, D, C::QT) ||
-        !rows_tensor_map(&kmap, a.k, krows, D, C::KT) || !rows_tensor_map(&vmap, a.v, krows, D, C::KT))
+    // dQ pass: Q/dO in items of 128 rows, K/V in tiles of 64; dK/dV pass: K/V in items of
+    // 128 keys, Q/dO in tiles of 64 rows
+    CUtensorMap q1, d1, k1, v1, q2, d2, k2, v2;
+    if (!rows_tensor_map(&q1, a.q, qrows, D, CQ::QT) || !rows_tensor_map(&d1, a.dout, qrows, D, CQ::QT) ||
+        !rows_tensor_map(&k1, a.k, krows, D, CQ::NK) || !rows_tensor_map(&v1, a.v, krows, D, CQ::NK) ||
+        !rows_tensor_map(&q2, a.q, qrows, D, CK::QT) || !rows_tensor_map(&d2, a.dout, qrows, D, CK::QT) ||
+        !rows_tensor_map(&k2, a.k, krows, D, CK::M) || !rows_tensor_map(&v2, a.v, krows, D, CK::M))
         return cudaErrorInvalidValue;
     {
         constexpr int TPR = D / 8;
@@ -533,13 +739,16 @@ cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
         err = cudaGetLastError();
         if (err != cudaSuccess) return err;
     }
-    const long long kv_ctas = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::KT - 1) / C::KT);
-    const long long q_ctas = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::QT - 1) / C::QT);
-    if (kv_ctas > 0x7fffffffLL || q_ctas > 0x7fffffffLL) return cudaErrorInvalidValue;
-    bwd_kv_kernel<D, G><<<static_cast<unsigned>(kv_ctas), kBwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, dmap, a);
+    // one persistent CTA per SM for each pass (512 TMEM columns each)
+    const long long kv_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + 127) / 128);
+    const long long q_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + CQ::QT - 1) / CQ::QT);
+    if (kv_items > 0x7fffffffLL || q_items > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const int kv_grid = static_cast<int>(kv_items < sms ? kv_items : sms);
+    const int q_grid = static_cast<int>(q_items < sms ? q_items : sms);
+    bwd_kv_tc_kernel<D, G><<<kv_grid, kTcThreads, CK::SMEM, stream>>>(q2, k2, v2, d2, a);
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    bwd_q_kernel<D, G><<<static_cast<unsigned>(q_ctas), kBwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, dmap, a);
+    bwd_q_tc_kernel<D, G><<<q_grid, kTcThreads, CQ::SMEM, stream>>>(q1, k1, v1, d1, a);
     return cudaGetLastError();
 }
 
