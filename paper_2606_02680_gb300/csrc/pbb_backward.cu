@@ -18,9 +18,11 @@
 //                      and accumulates dQ in tensor memory.
 // Both are persistent (one CTA per SM) on the fifth-generation tensor cores: a TMA
 // producer warp (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion
-// through tcgen05.commit on mbarriers) and four elementwise warps whose thread r
-// owns TMEM lane r; P, dS and their transposes are rounded to bf16 and written back
-// over the scores in tensor memory as the A operands of the next products. Every
+// through tcgen05.commit on mbarriers) and two elementwise warpgroups that take
+// alternate tiles (the scores of tile g sit in TMEM buffer g % 2), so two tiles'
+// exponentials run at once; thread r of a warpgroup owns TMEM lane r. P, dS and
+// their transposes are rounded to bf16 and written back over the scores in tensor
+// memory as the A operands of the next products. Every
 // wait is bounded by the global timer; a wait that runs out records a timeout, every
 // role stops, the MMAs and copies in flight are drained and TMEM is released.
 #include <cuda.h>
@@ -40,9 +42,9 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kGuardNs = 2000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kTcThreads = 192;  // 4 elementwise warps, producer, MMA issuer
-constexpr int kTcProducer = 4;
-constexpr int kTcMma = 5;
+constexpr int kTcThreads = 320;  // 8 elementwise warps (two warpgroups), producer, MMA issuer
+constexpr int kTcProducer = 8;
+constexpr int kTcMma = 9;
 
 __device__ __forceinline__ int support_start(int t, int h)
 {
@@ -55,6 +57,23 @@ __device__ __forceinline__ int support_start(int t, int h)
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)
 {
     return __all_sync(kFull, mbar_wait(bar, parity, limit));
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane, and 8 columns stored.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8])
+{
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
 }
 
 // ---------------------------------------------------------------- delta ----
@@ -152,9 +171,9 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&ds_full[b], 128);
+            mbar_init(&ds_full[b], 128);   // the warpgroup that owns buffer b
             mbar_init(&item_done[b], 1);
-            mbar_init(&o_free[b], 128);
+            mbar_init(&o_free[b], 256);    // both warpgroups read half of the dQ row
         }
         fence_mbar_init();
         abort_s = 0;
@@ -291,9 +310,10 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             }
         }
     } else {
-        // elementwise: thread r owns query row r
-        const int r = tid;
-        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+        // elementwise: two warpgroups; warpgroup wg takes the tiles g with g % 2 == wg (S/dP
+        // buffer wg), and thread r of either owns query row r (TMEM lane r)
+        const int wg = warp >> 2, r = tid & 127;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
         const int h = a.B >> 1;
         const int gi = r / C::QT, rp = r - gi * C::QT;
@@ -309,6 +329,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             const float l2 = valid ? a.lse[row] * kLog2e : 0.f, dr = valid ? a.delta[row] : 0.f;
             for (int j = 0; j < it.ntiles; ++j) {
                 const uint32_t g = gt + j;
+                if (static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -349,12 +370,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             }
             tmem_fence_after();
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
+            for (int c = 0; c < D / 64; ++c) {  // this warpgroup's half of the row
+                const int col = wg * (D / 2) + 32 * c;
                 uint32_t v[32];
-                tmem_ld32(lane_base + C::T_DQ + ob * D + 32 * c, v);
+                tmem_ld32(lane_base + C::T_DQ + ob * D + col, v);
                 tmem_wait_ld();
                 if (valid) {
-                    float4* dst = reinterpret_cast<float4*>(a.dq + row * D + 32 * c);
+                    float4* dst = reinterpret_cast<float4*>(a.dq + row * D + col);
 #pragma unroll
                     for (int x = 0; x < 8; ++x)
                         dst[x] = make_float4(__uint_as_float(v[4 * x]) * sc, __uint_as_float(v[4 * x + 1]) * sc,
@@ -441,7 +463,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         mbar_init(&kv_empty, 1);
         mbar_init(&done_bar, 1);
         mbar_init(&item_done, 1);
-        mbar_init(&o_free, 128);
+        mbar_init(&o_free, 256);  // warpgroup 0 reads dV, warpgroup 1 dK
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&qd_full[s], 1);
@@ -450,7 +472,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&p_full[b], 128);
+            mbar_init(&p_full[b], 128);  // the warpgroup that owns buffer b
         }
         fence_mbar_init();
         abort_s = 0;
@@ -485,6 +507,19 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             ++kv_issued;
             for (int i = 0; i < it.nqt; ++i, ++gt) {
                 const int s = gt % STAGES;
+                const int t0 = it.tq0 + i * C::QT;
+                // this tile's per-column data: the loads are issued before the wait for a free
+                // stage, so their latency overlaps it
+                float4 mv[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int c = lane + 32 * e;
+                    const int gi = c / C::QT, t = t0 + (c - gi * C::QT);
+                    const bool valid = t < a.n;
+                    const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + (valid ? t : 0);
+                    mv[e] = make_float4(valid ? __ldg(a.lse + row) : 0.f, valid ? __ldg(a.delta + row) : 0.f,
+                                        __int_as_float(valid ? t : -1), __int_as_float(support_start(t, h)));
+                }
                 if (gt >= STAGES && !warp_wait(&qd_empty[s], ((gt / STAGES) - 1) & 1u, limit)) {
                     ok = false;
                     break;
@@ -494,16 +529,11 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     break;
                 }
                 unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
-                const int t0 = it.tq0 + i * C::QT;
                 float4* meta = reinterpret_cast<float4*>(st + 2 * C::BOXES * C::QBOX);
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
-                    const int c = lane + 32 * e;
-                    const int gi = c / C::QT, t = t0 + (c - gi * C::QT);
-                    const bool valid = t < a.n;
-                    const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + (valid ? t : 0);
-                    meta[c] = make_float4(valid ? a.lse[row] * kLog2e : 0.f, valid ? a.delta[row] : 0.f,
-                                          __int_as_float(valid ? t : -1), __int_as_float(support_start(t, h)));
+                    mv[e].x *= kLog2e;
+                    meta[lane + 32 * e] = mv[e];
                 }
                 __threadfence_block();
                 __syncwarp();
@@ -608,9 +638,10 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             }
         }
     } else {
-        // elementwise: thread r owns key row r
-        const int r = tid;
-        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+        // elementwise: two warpgroups; warpgroup wg takes the query tiles g with g % 2 == wg
+        // (S^T/dP^T buffer wg), and thread r of either owns key row r (TMEM lane r)
+        const int wg = warp >> 2, r = tid & 127;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
         uint32_t gt = 0, ic = 0;
         bool ok = true;
@@ -620,6 +651,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             const bool kvalid = key < a.n;
             for (int i = 0; i < it.nqt; ++i) {
                 const uint32_t g = gt + i;
+                if (static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -627,21 +659,21 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 tmem_fence_after();
                 const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
                                                                      2 * C::BOXES * C::QBOX);
-                // 32 columns at a time: their P^T and dS^T (16 bf16-pair columns each) go over
+                // 16 columns at a time: their P^T and dS^T (8 bf16-pair columns each) go over
                 // columns already read
 #pragma unroll
-                for (int c = 0; c < NQ / 32; ++c) {
-                    uint32_t v1[32], v2[32];
-                    tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + 32 * c, v1);
-                    tmem_ld32(lane_base + C::T_DPT + (g & 1u) * NQ + 32 * c, v2);
+                for (int c = 0; c < NQ / 16; ++c) {
+                    uint32_t v1[16], v2[16];
+                    tmem_ld16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, v1);
+                    tmem_ld16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, v2);
                     tmem_wait_ld();
-                    uint32_t pk[16], dk[16];
+                    uint32_t pk[8], dk[8];
 #pragma unroll
-                    for (int x = 0; x < 16; ++x) {
+                    for (int x = 0; x < 8; ++x) {
                         float pe[2], de[2];
 #pragma unroll
                         for (int y = 0; y < 2; ++y) {
-                            const int cc = 32 * c + 2 * x + y;
+                            const int cc = 16 * c + 2 * x + y;
                             const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc
                             const int t = __float_as_int(m.z), at = __float_as_int(m.w);
                             const bool vis = kvalid && key <= t && key >= at;
@@ -652,8 +684,8 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                         pk[x] = pack_bf16x2(pe[0], pe[1]);
                         dk[x] = pack_bf16x2(de[0], de[1]);
                     }
-                    tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, pk);
-                    tmem_st16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, dk);
+                    tmem_st8(lane_base + C::T_ST + (g & 1u) * NQ + 8 * c, pk);
+                    tmem_st8(lane_base + C::T_DPT + (g & 1u) * NQ + 8 * c, dk);
                 }
                 tmem_wait_st();
                 tmem_fence_before();
@@ -666,22 +698,21 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             }
             tmem_fence_after();
             const size_t row = static_cast<size_t>(it.pair) * a.n + (kvalid ? key : 0);
+            // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled by 1/sqrt(d))
+            const float f = wg == 0 ? 1.f : sc;
+            float* dst_row = (wg == 0 ? a.dv : a.dk) + row * D;
+            const uint32_t src = lane_base + (wg == 0 ? C::T_DV : C::T_DK);
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32], w[32];
-                tmem_ld32(lane_base + C::T_DV + 32 * c, v);
-                tmem_ld32(lane_base + C::T_DK + 32 * c, w);
+                uint32_t v[32];
+                tmem_ld32(src + 32 * c, v);
                 tmem_wait_ld();
                 if (kvalid) {
-                    float4* dv = reinterpret_cast<float4*>(a.dv + row * D + 32 * c);
-                    float4* dk = reinterpret_cast<float4*>(a.dk + row * D + 32 * c);
+                    float4* dst = reinterpret_cast<float4*>(dst_row + 32 * c);
 #pragma unroll
-                    for (int x = 0; x < 8; ++x) {
-                        dv[x] = make_float4(__uint_as_float(v[4 * x]), __uint_as_float(v[4 * x + 1]),
-                                            __uint_as_float(v[4 * x + 2]), __uint_as_float(v[4 * x + 3]));
-                        dk[x] = make_float4(__uint_as_float(w[4 * x]) * sc, __uint_as_float(w[4 * x + 1]) * sc,
-                                            __uint_as_float(w[4 * x + 2]) * sc, __uint_as_float(w[4 * x + 3]) * sc);
-                    }
+                    for (int x = 0; x < 8; ++x)
+                        dst[x] = make_float4(__uint_as_float(v[4 * x]) * f, __uint_as_float(v[4 * x + 1]) * f,
+                                             __uint_as_float(v[4 * x + 2]) * f, __uint_as_float(v[4 * x + 3]) * f);
                 }
             }
             tmem_fence_before();
