@@ -60,41 +60,48 @@ __device__ int g_fwd_status;  // first fault recorded by a forward kernel, kDevO
 namespace {
 
 constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken GPU can exceed
-constexpr int kFwdThreads = 192;                         // 4 softmax warps, producer, MMA issuer
-constexpr int kProducerWarp = 4;
-constexpr int kMmaWarp = 5;
 
-// Two shapes of the same kernel, chosen by the block size (see launch_fwd):
-//   wide   (NK = 128): one CTA per SM with all 512 TMEM columns and up to 225 KB of shared
-//          memory, for long supports (many tiles per item keep the tensor cores busy);
-//   narrow (NK = 64):  two CTAs per SM, each with 256 TMEM columns and under 114 KB, for
-//          short supports, where an item is one or two tiles and the other CTA's work
-//          hides each item's latencies.
-template <int D, int G, int NK_>
+// Shapes of the same kernel (chosen by the block size, see launch_fwd_shape):
+//   NK    keys per K/V tile (128 or 64);
+//   WGS   softmax warpgroups (1, or 2 taking alternate tiles with an output buffer each);
+//   CTAS  CTAs per SM: 1 owns all 512 TMEM columns, 2 share them (256 each) so one CTA's
+//         latencies overlap the other's work.
+// Long supports (many tiles per item) use one CTA per SM; short ones, where an item is one
+// or two tiles, two CTAs per SM with 64-key tiles.
+template <int D, int G, int NK_, int WGS_, int CTAS_>
 struct FwdCfg {
-    static constexpr int NK = NK_;                      // keys per K/V tile
-    static constexpr bool WIDE = NK == 128;
-    static constexpr int CTAS = WIDE ? 1 : 2;           // CTAs per SM
-    static constexpr int TMEM_COLS = WIDE ? 512 : 256;
+    static constexpr int NK = NK_;
+    static constexpr int WGS = WGS_;
+    static constexpr int CTAS = CTAS_;
+    static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
     static constexpr int M = 128;                       // query rows of an item (G heads x QT positions)
     static constexpr int QT = M / G;                    // positions of an item
     static constexpr int BOXES = D / 64;                // 64-column boxes of a row
     static constexpr int QBOX = M * 128;                // bytes of one Q box
     static constexpr int KBOX = NK * 128;               // bytes of one K (or V) box
     static constexpr int QBUF = D == 64 ? 2 : 1;        // Q buffers (the next item's Q loads early)
-    static constexpr int STAGES = D == 64 ? 4 : (WIDE ? 3 : 2);  // K/V tiles in flight
-    static constexpr int OBUF = (WIDE || D == 64) ? 2 : 1;       // TMEM output buffers (alternate between items)
+    static constexpr int KV_STAGE = 2 * BOXES * KBOX;   // K boxes then V boxes
     static constexpr int Q_OFF = 0;
     static constexpr int Q_BYTES = BOXES * QBOX;
     static constexpr int KV_OFF = Q_OFF + QBUF * Q_BYTES;
-    static constexpr int KV_STAGE = 2 * BOXES * KBOX;   // K boxes then V boxes
+    // the kernel's static shared memory (barriers; with two warpgroups the (m, l) exchange)
+    static constexpr int STATIC_SMEM = WGS == 2 ? 4608 : 512;
+    // K/V tiles in flight: as many as the shared memory of this shape holds, at most 4
+    static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - STATIC_SMEM - 1024 - KV_OFF) / KV_STAGE;
+    static constexpr int STAGES = STAGE_ROOM < 4 ? STAGE_ROOM : 4;
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;  // + alignment slack
-    // TMEM columns: S buffers at 0 and NK, O buffers from 2 NK
+    // TMEM columns: S buffers at 0 and NK, output buffers from 2 NK: one per warpgroup with
+    // two warpgroups, else two alternating between items where they fit
     static constexpr int T_S = 0;
     static constexpr int T_O = 2 * NK;
+    static constexpr int OBUF = WGS == 2 ? 2 : (T_O + 2 * D <= TMEM_COLS ? 2 : 1);
+    static constexpr int THREADS = 128 * WGS + 64;      // softmax warps, producer warp, MMA warp
+    static constexpr int PRODUCER_WARP = 4 * WGS;
+    static constexpr int MMA_WARP = 4 * WGS + 1;
+    static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_O + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(QT % 8 == 0, "a head's Q rows must start on a swizzle atom (8 rows)");
-    static_assert(CTAS * SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(CTAS * (SMEM + STATIC_SMEM) <= 227 * 1024, "shared memory budget");
 };
 
 // Start of the PBB support of position t: a(t) = max(0, h (floor(t/h) - 1)).
@@ -131,18 +138,21 @@ __device__ __forceinline__ Item make_item(int idx, int n, int B)
     return it;
 }
 
-template <int D, int G, int NK>
-__global__ void __launch_bounds__(kFwdThreads, FwdCfg<D, G, NK>::CTAS)
+template <int D, int G, int NK, int WGS_, int CTAS_>
+__global__ void __launch_bounds__(FwdCfg<D, G, NK, WGS_, CTAS_>::THREADS, CTAS_)
 forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                const __grid_constant__ CUtensorMap vmap, const ForwardArgs a)
 {
-    using C = FwdCfg<D, G, NK>;
+    using C = FwdCfg<D, G, NK, WGS_, CTAS_>;
     constexpr int STAGES = C::STAGES;
+    constexpr int WGS = C::WGS;
     extern __shared__ unsigned char dsmem_raw[];
     constexpr int QBUF = C::QBUF;
-    __shared__ __align__(8) uint64_t q_full[QBUF], q_empty[QBUF], done_bar;
+    __shared__ __align__(8) uint64_t q_full[QBUF], q_empty[QBUF], done_bar, merge_bar;
     __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
     __shared__ __align__(8) uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];
+    // per item parity, (m, l) of each warpgroup's rows (used with two warpgroups only)
+    __shared__ float2 ml_s[WGS == 2 ? 2 : 1][WGS][WGS == 2 ? 128 : 1];
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
@@ -157,6 +167,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             mbar_init(&q_empty[q], 1);
         }
         mbar_init(&done_bar, 1);
+        mbar_init(&merge_bar, 128 * WGS);
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&kv_full[s], 1);
@@ -165,9 +176,9 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&p_full[b], 128);
+            mbar_init(&p_full[b], 128);         // the warpgroup that owns S buffer b
             mbar_init(&pv_done[b], 1);
-            mbar_init(&o_free[b], 128);
+            mbar_init(&o_free[b], 128 * WGS);   // every softmax thread, after reading the output
         }
         fence_mbar_init();
         abort_s = 0;
@@ -179,7 +190,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
     const uint32_t tmem = tmem_base_s;
     const unsigned long long limit = a.timeout_ns;
 
-    if (warp == kProducerWarp) {
+    if (warp == C::PRODUCER_WARP) {
         // ================= TMA producer =================
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
@@ -239,7 +250,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 mbar_wait(&kv_full[s], (j / STAGES) & 1u, kGuardNs);
             }
         }
-    } else if (warp == kMmaWarp) {
+    } else if (warp == C::MMA_WARP) {
         // ================= MMA issuer =================
         if (lane == 0) {
             constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, C::NK, 0);
@@ -284,19 +295,28 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         issue_s(g + 1);
                         if (j + 2 == it.ntiles) umma_commit(&q_empty[qb]);  // the item's last read of Q
                     }
-                    if (!mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit) ||
-                        (j == 0 && ic >= C::OBUF && !mbar_wait(&o_free[ob], ((ic / C::OBUF) - 1) & 1u, limit))) {
+                    // before the item's first P.V: the output buffers are free once every softmax thread
+                    // has read the previous item's (both warpgroups' accumulators, or buffer ob)
+                    bool free_ok = true;
+                    if (j == 0) {
+                        if (WGS == 2 && ic >= 1) free_ok = mbar_wait(&o_free[0], (ic - 1) & 1u, limit);
+                        if (WGS == 1 && ic >= C::OBUF) free_ok = mbar_wait(&o_free[ob], ((ic / C::OBUF) - 1) & 1u, limit);
+                    }
+                    if (!free_ok || !mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit)) {
                         ok = false;
                         break;
                     }
                     tmem_fence_after();
-                    // O (+)= P_g V_g: P from TMEM (bf16 pairs over S buffer g % 2), V MN-major
+                    // O (+)= P_g V_g: P from TMEM (bf16 pairs over S buffer g % 2), V MN-major. With two
+                    // warpgroups, tile g accumulates into warpgroup (g % 2)'s buffer, starting at its first tile.
                     const uint32_t pt = tmem + C::T_S + (g & 1u) * C::NK;
                     const uint32_t vb = kv_base + (g % STAGES) * C::KV_STAGE + C::BOXES * C::KBOX;
+                    const uint32_t o_dst = tmem + C::T_O + (WGS == 2 ? (g & 1u) : ob) * D;
+                    const bool first = WGS == 2 ? j < 2 : j == 0;
 #pragma unroll
                     for (int kk = 0; kk < C::NK / 16; ++kk) {
                         const uint64_t bd = umma_desc_sw128(vb + kk * 2048, C::KBOX, 1024);
-                        umma_bf16_tmem_a(tmem + C::T_O + ob * D, pt + 8 * kk, bd, idesc_o, (j > 0 || kk > 0) ? 1u : 0u);
+                        umma_bf16_tmem_a(o_dst, pt + 8 * kk, bd, idesc_o, (!first || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(&pv_done[g & 1u]);
                     umma_commit(&kv_empty[g % STAGES]);
@@ -313,9 +333,11 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             }
         }
     } else {
-        // ================= softmax: thread r owns query row r =================
-        const int r = tid;
-        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * warp) << 16);
+        // ================= softmax =================
+        // Warpgroup wg takes the tiles g with g % WGS == wg; thread r owns query row r
+        // (TMEM lane r) and keeps its own running maximum and sum for those tiles.
+        const int wg = warp >> 2, r = tid & 127;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
         const int h = a.B >> 1;
         const int gi = r / C::QT, rp = r - gi * C::QT;
@@ -324,18 +346,23 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
             const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
             const uint32_t ob = ic % C::OBUF;
+            const uint32_t o_col = C::T_O + (WGS == 2 ? static_cast<uint32_t>(wg) : ob) * D;
             const int t = it.t0 + rp;               // this row's position
             const int as = support_start(t, h);     // and its support start
             float m_used = -INFINITY, l = 0.f;
+            int last = -1;                          // this warpgroup's last tile of the item
             for (int j = 0; j < it.ntiles; ++j) {
                 const uint32_t g = gt + j;
+                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
+                const bool has_prev = last >= 0;    // an earlier tile of this warpgroup holds O
+                last = j;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(0xffffffffu, abort_s != 0)) {
                     ok = false;
                     break;
                 }
                 tmem_fence_after();
                 const uint32_t s_col = lane_base + C::T_S + (g & 1u) * C::NK;
-                float z[C::NK];  // raw scores q.k of this row
+                float z[C::NK];  // raw scores q.k of this row: every load issued, one wait
 #pragma unroll
                 for (int c = 0; c < C::NK / 32; ++c) {
                     uint32_t v[32];
@@ -363,8 +390,8 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 if (__any_sync(0xffffffffu, grow)) {
                     const float f = grow ? (m_used == -INFINITY ? 0.f : fast_exp2(m_used - m_new)) : 1.f;
                     l *= f;
-                    if (j > 0) {  // O holds tiles 0 .. j-1 once P.V of tile j-1 is complete
-                        const uint32_t gp = g - 1;
+                    if (has_prev) {  // O holds this warpgroup's earlier tiles once P.V of the previous one is complete
+                        const uint32_t gp = g - WGS;
                         if (!warp_wait(&pv_done[gp & 1u], (gp >> 1) & 1u, limit)) {
                             ok = false;
                             break;
@@ -373,7 +400,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
 #pragma unroll
                         for (int c = 0; c < D / 32; ++c) {
                             uint32_t v[32];
-                            const uint32_t ta = lane_base + C::T_O + ob * D + 32 * c;
+                            const uint32_t ta = lane_base + o_col + 32 * c;
                             tmem_ld32(ta, v);
                             tmem_wait_ld();
 #pragma unroll
@@ -403,48 +430,75 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 mbar_arrive(&p_full[g & 1u]);
             }
             if (!ok) break;
-            // ---- epilogue: O row / l, lse
-            const uint32_t gl = gt + it.ntiles - 1;
-            if (!warp_wait(&pv_done[gl & 1u], (gl >> 1) & 1u, limit)) {
-                ok = false;
-                break;
+            // ---- epilogue: this warpgroup's last P.V, then o = O / l and lse
+            if (last >= 0) {
+                const uint32_t gl = gt + last;
+                if (!warp_wait(&pv_done[gl & 1u], (gl >> 1) & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
             }
-            tmem_fence_after();
             const bool valid = t < a.n;
-            const float inv = l > 0.f ? 1.f / l : 0.f;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
             const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + t;
-#pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(lane_base + C::T_O + ob * D + 32 * c, v);
+            float m_tot = m_used, l_tot = l, f0 = 1.f, f1 = 0.f, w0 = 1.f, w1 = 0.f;
+            int c0 = 0, c1 = D / 32;  // columns of the output this thread writes (32 at a time)
+            if (WGS == 2) {
+                // fuse the two warpgroups' partial results (Eq. lse): each writes half of the columns
+                ml_s[ic & 1u][wg][r] = make_float2(m_used, l);
+                mbar_arrive(&merge_bar);
+                if (!warp_wait(&merge_bar, ic & 1u, limit)) {
+                    ok = false;
+                    break;
+                }
+                const float2 p0 = ml_s[ic & 1u][0][r], p1 = ml_s[ic & 1u][1][r];
+                m_tot = fmaxf(p0.x, p1.x);
+                f0 = p0.y > 0.f ? fast_exp2(p0.x - m_tot) : 0.f;
+                f1 = p1.y > 0.f ? fast_exp2(p1.x - m_tot) : 0.f;
+                l_tot = f0 * p0.y + f1 * p1.y;
+                w0 = p0.y > 0.f ? 1.f : 0.f;  // a warpgroup without tiles left its buffer stale: never read it
+                w1 = p1.y > 0.f ? 1.f : 0.f;
+                c0 = wg * (D / 64);
+                c1 = c0 + D / 64;
+            }
+            tmem_fence_after();
+            const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
+            for (int c = c0; c < c1; ++c) {
+                uint32_t v[32], u[32];
+                tmem_ld32(lane_base + (WGS == 2 ? C::T_O : o_col) + 32 * c, v);
+                if (WGS == 2) tmem_ld32(lane_base + C::T_O + D + 32 * c, u);
                 tmem_wait_ld();
+                float o[32];
+#pragma unroll
+                for (int x = 0; x < 32; ++x) {
+                    const float a0 = w0 > 0.f ? __uint_as_float(v[x]) * f0 : 0.f;
+                    const float a1 = (WGS == 2 && w1 > 0.f) ? __uint_as_float(u[x]) * f1 : 0.f;
+                    o[x] = (a0 + a1) * inv;
+                }
                 if (valid) {
                     if (a.out_f32) {
                         float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 32 * c);
 #pragma unroll
-                        for (int x = 0; x < 8; ++x)
-                            dst[x] = make_float4(__uint_as_float(v[4 * x]) * inv, __uint_as_float(v[4 * x + 1]) * inv,
-                                                 __uint_as_float(v[4 * x + 2]) * inv, __uint_as_float(v[4 * x + 3]) * inv);
+                        for (int x = 0; x < 8; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
                     } else {
                         uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 32 * c);
 #pragma unroll
                         for (int x = 0; x < 4; ++x) {
                             uint4 pk;
-                            pk.x = pack_bf16x2(__uint_as_float(v[8 * x]) * inv, __uint_as_float(v[8 * x + 1]) * inv);
-                            pk.y = pack_bf16x2(__uint_as_float(v[8 * x + 2]) * inv, __uint_as_float(v[8 * x + 3]) * inv);
-                            pk.z = pack_bf16x2(__uint_as_float(v[8 * x + 4]) * inv, __uint_as_float(v[8 * x + 5]) * inv);
-                            pk.w = pack_bf16x2(__uint_as_float(v[8 * x + 6]) * inv, __uint_as_float(v[8 * x + 7]) * inv);
+                            pk.x = pack_bf16x2(o[8 * x], o[8 * x + 1]);
+                            pk.y = pack_bf16x2(o[8 * x + 2], o[8 * x + 3]);
+                            pk.z = pack_bf16x2(o[8 * x + 4], o[8 * x + 5]);
+                            pk.w = pack_bf16x2(o[8 * x + 6], o[8 * x + 7]);
                             dst[x] = pk;
                         }
                     }
                 }
             }
             tmem_fence_before();
-            mbar_arrive(&o_free[ob]);  // the next item on this O buffer may overwrite it
-            if (valid && a.lse != nullptr) {
+            mbar_arrive(&o_free[WGS == 2 ? 0u : ob]);  // the next item may overwrite the output buffer
+            if (valid && a.lse != nullptr && wg == 0) {
                 // ln sum exp(z) = (m + log2 l) ln 2, m the base-2 reference maximum
-                a.lse[row] = (m_used + log2f(l)) * 0.6931471805599453f;
+                a.lse[row] = (m_tot + log2f(l_tot)) * 0.6931471805599453f;
             }
             gt += it.ntiles;
         }
@@ -489,16 +543,17 @@ __global__ void seq_ring_kernel(const unsigned char* __restrict__ k, const unsig
     }
 }
 
-template <int D, int G, int NK>
+template <int D, int G, int NK, int WGS, int CTAS>
 cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
 {
-    using C = FwdCfg<D, G, NK>;
+    using C = FwdCfg<D, G, NK, WGS, CTAS>;
+    auto kernel = forward_kernel<D, G, NK, WGS, CTAS>;
     static bool attr_set[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 64 && !attr_set[dev]) {
-        err = cudaFuncSetAttribute(forward_kernel<D, G, NK>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
@@ -516,23 +571,33 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     // persistent CTAs: C::CTAS per SM, never more than TMEM holds
     int per_sm = 0;
-    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, forward_kernel<D, G, NK>, kFwdThreads, C::SMEM);
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, C::THREADS, C::SMEM);
     if (err != cudaSuccess) return err;
     if (per_sm < 1) per_sm = 1;
     if (per_sm > C::CTAS) per_sm = C::CTAS;
     const long long slots = static_cast<long long>(sms) * per_sm;
     const int grid = static_cast<int>(items < slots ? items : slots);
-    forward_kernel<D, G, NK><<<grid, kFwdThreads, C::SMEM, stream>>>(qmap, kmap, vmap, a);
+    kernel<<<grid, C::THREADS, C::SMEM, stream>>>(qmap, kmap, vmap, a);
     return cudaGetLastError();
 }
 
-// Wide tiles for long supports: from B = 512 an item spans several 128-key tiles
-// (measured on GB300: 1,125 vs 537 TFLOP/s at B = 4096), narrow tiles and two CTAs per
-// SM below (2,169 vs 1,646 GB/s at B = 128, where an item is one tile).
+// The shape for long supports (B >= 512: an item spans several tiles) is a build-time choice:
+// 0 = 128-key tiles, one softmax warpgroup; 1 = 64-key tiles, two softmax warpgroups.
+#ifndef PBB_FWD_LONG_SHAPE
+#define PBB_FWD_LONG_SHAPE 0
+#endif
+
+// Short supports: 64-key tiles, two CTAs per SM (measured on GB300 at B = 128: 2,169 GB/s,
+// against 1,646 GB/s for the long-support shape, where an item is one tile).
 template <int D, int G>
 cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream)
 {
-    return a.B >= 512 ? launch_fwd<D, G, 128>(a, stream) : launch_fwd<D, G, 64>(a, stream);
+    if (a.B < 512) return launch_fwd<D, G, 64, 1, 2>(a, stream);
+#if PBB_FWD_LONG_SHAPE == 1
+    return launch_fwd<D, G, 64, 2, 1>(a, stream);
+#else
+    return launch_fwd<D, G, 128, 1, 1>(a, stream);
+#endif
 }
 
 template <int D>
