@@ -59,6 +59,7 @@ def parse_args():
     ap.add_argument("--block", type=int, default=4096)
     ap.add_argument("--hq", type=int, default=0, help="query heads of the throughput point (default 32)")
     ap.add_argument("--hkv", type=int, default=0, help="KV heads of the throughput point (default 8)")
+    ap.add_argument("--head-dim", type=int, default=0, help="head size of the throughput point (default 128)")
     ap.add_argument("--sweep", action="store_true", help="one line per throughput-sweep point")
     ap.add_argument("--workload", default="", help="a named workload of paper_2606_02680_gb300.inputs "
                     "(default: the throughput point given by --batch/--block)")
@@ -816,9 +817,9 @@ def run_ours(args):
                   for b in inputs.SWEEP_BATCHES for B in inputs.SWEEP_BLOCKS]
     else:
         w0 = inputs.sweep_workload(shard_batch(args.batch, rank, world), args.block)
-        if args.hq or args.hkv:
-            hq, hkv = args.hq or w0.Hq, args.hkv or w0.Hkv
-            w0 = w0.with_(Hq=hq, Hkv=hkv, name=f"{w0.name}_Hq{hq}_Hkv{hkv}")
+        if args.hq or args.hkv or args.head_dim:
+            hq, hkv, hd = args.hq or w0.Hq, args.hkv or w0.Hkv, args.head_dim or w0.d
+            w0 = w0.with_(Hq=hq, Hkv=hkv, d=hd, name=f"{w0.name}_Hq{hq}_Hkv{hkv}" + (f"_d{hd}" if hd != w0.d else ""))
         points = [w0]
     peak, peak_kind = hbm_peak()
     patterns = {"pbb": ["pbb"], "swa": ["swa"], "both": ["pbb", "swa"]}[args.pattern]

@@ -36,7 +36,10 @@
  *     layout above or come from pbb_ring_alloc.
  *   - Calls are asynchronous on `stream` (0 = the legacy default stream) and
  *     never synchronise. Sizes: batch >= 0, Hq % Hkv == 0 with
- *     Hq/Hkv in {1, 2, 4, 8}, d in {64, 128}, B even and 2 <= B <= 2^20.
+ *     Hq/Hkv in {1, 2, 4, 6, 8}, d in {64, 128}, B even and 2 <= B <= 2^20.
+ *     A group of 6 (12 query heads on 2 KV heads, the paper's models of Sec. 5)
+ *     runs on the group-8 CUDA-core kernel with two zero query rows that are
+ *     computed and never written.
  *   - Return value: PBB_OK or a negative PBB_ERR_* code; nothing is launched
  *     when argument checking fails. Faults the device finds (a negative
  *     position, a wait that ran out) are kept in a device-side status word
@@ -183,7 +186,9 @@ int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, voi
  *                            log-partition of Eq. (lse) a backward pass reuses;
  *                            NULL to skip
  * Device pointers owned by the caller; q, k, v, out 16-byte aligned. Same
- * group and head-size rules as the decode step; batch*Hq*n < 2^31. Runs on the
+ * head-size rules as the decode step; Hq/Hkv in {1, 2, 4, 8} (a tile stacks
+ * Hq/Hkv heads x 128/(Hq/Hkv) positions as 128 rows, so 6 returns
+ * PBB_ERR_UNSUPPORTED); batch*Hq*n < 2^31. Runs on the
  * fifth-generation tensor cores (tcgen05, bf16 operands, fp32 accumulation in
  * tensor memory; the softmax weights are rounded to bf16 before P.V), one
  * persistent CTA per SM. Asynchronous on `stream`; a bounded wait that runs out
@@ -204,9 +209,11 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
  *   delta       [batch][Hq][n] fp32      scratch (receives D)
  *   dq          [batch][Hq][n][d] fp32   dk, dv [batch][Hkv][n][d] fp32 (overwritten)
  * Same shape rules as pbb_forward; 16-byte aligned tensors (lse, delta 4-byte).
- * Runs on the tensor cores (mma.sync, bf16 operands with P and dS rounded to
- * bf16, fp32 accumulation); no floating-point atomics, so results are bitwise
- * deterministic. Asynchronous on `stream`; a bounded wait that runs out is
+ * Runs on the fifth-generation tensor cores (tcgen05: S, dP and the gradients
+ * accumulate in fp32 in tensor memory; bf16 operands, with P and dS rounded to
+ * bf16): one pass over key tiles for dK and dV, one over query tiles for dQ,
+ * each persistent with one CTA per SM. No floating-point atomics, so results
+ * are bitwise deterministic. Asynchronous on `stream`; a bounded wait that runs out is
  * reported by pbb_get_device_status as PBB_ERR_DEVICE_TIMEOUT.
  */
 int pbb_backward(const void* q, const void* k, const void* v, const void* out, const void* dout, const float* lse,

@@ -48,14 +48,36 @@ int check_shape(int batch, int Hkv, int d, int B, pbb_dtype dt)
     return PBB_OK;
 }
 
+// Decode steps: groups 1, 2, 4, 6 and 8 (6, the paper's models with 12 query heads on 2 KV
+// heads, runs on the group-8 kernel with two padded heads).
 int check_group(int Hq, int Hkv)
 {
     if (Hq <= 0 || Hkv <= 0) return PBB_ERR_INVALID_ARG;
     if (Hq % Hkv != 0) return PBB_ERR_UNSUPPORTED;
     const int g = Hq / Hkv;
-    if (g != 1 && g != 2 && g != 4 && g != 8) return PBB_ERR_UNSUPPORTED;
+    if (g != 1 && g != 2 && g != 4 && g != 6 && g != 8) return PBB_ERR_UNSUPPORTED;
     return PBB_OK;
 }
+
+// The whole-sequence kernels stack G heads x 128/G positions as 128 rows: G must divide 128.
+int check_group_sequence(int Hq, int Hkv)
+{
+    const int rc = check_group(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    return (Hq / Hkv) == 6 ? PBB_ERR_UNSUPPORTED : PBB_OK;
+}
+
+// The group G a decode kernel runs, which lays out the split partials: the tensor-core kernel
+// always runs 8 query columns, the CUDA-core kernel runs a group of 6 as 8. plan_split takes
+// the real group.
+int kernel_group(const pbb::DecodeArgs& a, int elem)
+{
+    if (pbb::use_tensor_cores(a, elem)) return 8;
+    return a.gq == 6 ? 8 : a.gq;
+}
+
+// An upper bound of kernel_group for every step of this group.
+int max_kernel_group(int group) { return (group == 6 || pbb::tc_group(group)) ? 8 : group; }
 
 int current_device(int* dev)
 {
@@ -137,7 +159,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
         // (measured: +29 % at B 4096 and +6 % at B 2048, but -12 to -15 % at B <= 1024 and
         // -19 % for the tensor-core kernel, whose two consumer warps combine slowly).
         const bool long_supports = max_keys >= 2047 && pbb::tile_keys(elem, d, group) == tile &&
-                                   !(window == 0 && elem == 2 && group == 8 && B % 64 == 0);
+                                   !(window == 0 && elem == 2 && pbb::tc_group(group) && B % 64 == 0);
         if (R == 0 || 2 * R > G || !long_supports) {  // no split
             sp.whole = static_cast<int>(pairs);
             sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
@@ -219,7 +241,6 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     rc = current_device(&dev);
     if (rc != PBB_OK) return rc;
     const int elem = elem_size(dt);
-    const int group = Hq / Hkv;
 
     pbb::DecodeArgs a{};
     a.q = q;
@@ -234,9 +255,10 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
+    a.gq = Hq / Hkv;
     a.window = window;
     a.pos_batch = pos_batch > 0 ? pos_batch : batch;
-    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, group, window);
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, Hq / Hkv, window);
     a.whole = sp.whole;
     a.chunk = sp.chunk;
     a.nchunk = sp.nchunk;
@@ -246,6 +268,7 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     const size_t items = static_cast<size_t>(sp.whole) + (pairs - static_cast<size_t>(sp.whole)) * sp.nchunk;
     if (items > static_cast<size_t>(INT_MAX)) return PBB_ERR_UNSUPPORTED;
     a.total_items = static_cast<int>(items);
+    const int group = kernel_group(a, elem);
     {
         const size_t pbytes = static_cast<size_t>(sp.whole) < pairs ? parts_bytes(batch, Hkv, d, group, sp) : 0;
         std::lock_guard<std::mutex> lock(g_mutex);
@@ -337,13 +360,13 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
     rc = current_device(&dev);
     if (rc != PBB_OK) return rc;
     const int elem = elem_size(dtype);
-    const int group = Hq / Hkv;
+    const int group = max_kernel_group(Hq / Hkv);
     // Every batch up to max_batch (the plan's split depends on the batch), for
     // PBB steps and for window steps with window = B.
     size_t need = 0;
     for (int bsz = 1; bsz <= max_batch; ++bsz) {
         for (int window : {0, B}) {
-            const pbb::SplitPlan sp = pbb::plan_split(bsz, Hkv, d, B, elem, group, window);
+            const pbb::SplitPlan sp = pbb::plan_split(bsz, Hkv, d, B, elem, Hq / Hkv, window);
             if (static_cast<size_t>(sp.whole) >= static_cast<size_t>(bsz) * Hkv) continue;
             const size_t w = parts_bytes(bsz, Hkv, d, group, sp);
             if (w > need) need = w;
@@ -393,7 +416,7 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
 {
     int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
     if (rc != PBB_OK) return rc;
-    rc = check_group(Hq, Hkv);
+    rc = check_group_sequence(Hq, Hkv);
     if (rc != PBB_OK) return rc;
     if (n < 0 || elem_size(out_dtype) == 0) return PBB_ERR_INVALID_ARG;
     if (batch == 0 || n == 0) return PBB_OK;
@@ -429,7 +452,7 @@ int pbb_backward(const void* q, const void* k, const void* v, const void* out, c
 {
     int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
     if (rc != PBB_OK) return rc;
-    rc = check_group(Hq, Hkv);
+    rc = check_group_sequence(Hq, Hkv);
     if (rc != PBB_OK) return rc;
     if (n < 0) return PBB_ERR_INVALID_ARG;
     if (batch == 0 || n == 0) return PBB_OK;
@@ -541,6 +564,7 @@ int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
     if (rc != PBB_OK) return rc;
     pbb::DecodeArgs a{};
     a.batch = batch;
+    a.gq = Hq / Hkv;
     a.Hq = Hq;
     a.Hkv = Hkv;
     a.d = d;

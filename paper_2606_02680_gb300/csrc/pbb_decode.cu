@@ -333,7 +333,7 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
                 O = fmaf(merge_o[(w * G) * D + e], sc, O);
             }
             if (mt.nch == 1) {
-                a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D + e] = O / L;
+                if (j < a.gq) a.out[(static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * a.gq) * D + e] = O / L;
             } else {
                 a.part_o[part * G * D + e] = O;
                 if ((e % D) == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
@@ -350,7 +350,7 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
             __threadfence();
             const float* po = a.part_o + (head - a.whole) * a.nchunk * G * D;
             const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + (head - a.whole) * a.nchunk * G;
-            float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * G) * D;
+            float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * a.gq) * D;
             if (mt.nch <= NC * D) {
                 // weight of every (chunk, head) in shared memory: e^(m_c - M) / L, with M and
                 // L reduced across the chunks by one warp per head
@@ -375,7 +375,7 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
                 }
                 ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
                 if (ok) {
-                    for (int e = ctid; e < G * D; e += NC * 32) {
+                    for (int e = ctid; e < a.gq * D; e += NC * 32) {  // the real query heads
                         const int j = e / D;
                         float O = 0.f;
 #pragma unroll 8
@@ -384,7 +384,7 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
                     }
                 }
             } else {
-                for (int e = ctid; e < G * D; e += NC * 32) {
+                for (int e = ctid; e < a.gq * D; e += NC * 32) {  // the real query heads
                     const int j = e / D;
                     float M = -INFINITY;
                     for (int c = 0; c < mt.nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
@@ -436,6 +436,13 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
         sbar_gen = 0;
         abort_s = 0;
         issued_s = 0;
+    }
+    if (a.gq < G) {
+        // a group of gq < G heads runs as G: the query rows gq .. G-1 of every stage are never
+        // loaded and stay zero, so the padded heads compute finite values that are never written
+        for (int s = 0; s < kStages; ++s)
+            for (int x = threadIdx.x; x < (G - a.gq) * C::ROW / 16; x += blockDim.x)
+                reinterpret_cast<uint4*>(dsmem + s * C::STAGE + C::Q_OFF + a.gq * C::ROW)[x] = make_uint4(0u, 0u, 0u, 0u);
     }
     __syncthreads();
 
@@ -504,7 +511,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     mt.pad = 0;
                     meta_s[s] = mt;
                     unsigned char* st = dsmem + s * C::STAGE;
-                    const uint32_t bytes = static_cast<uint32_t>(2 * nk * C::ROW + (first ? G * C::ROW : 0) +
+                    const uint32_t bytes = static_cast<uint32_t>(2 * nk * C::ROW + (first ? a.gq * C::ROW : 0) +
                                                                  (current ? 2 * C::ROW : 0));
                     fence_proxy_async();
                     mbar_expect_tx(&full_bar[s], bytes);  // arrives (release): the descriptor is visible
@@ -522,8 +529,8 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     }
                     if (first) {
                         const unsigned char* qg = static_cast<const unsigned char*>(a.q) +
-                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * C::ROW;
-                        bulk_g2s(st + C::Q_OFF, qg, G * C::ROW, &full_bar[s]);
+                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * a.gq) * C::ROW;
+                        bulk_g2s(st + C::Q_OFF, qg, a.gq * C::ROW, &full_bar[s]);
                     }
                     if (current) {
                         bulk_g2s(st + C::KN_OFF, static_cast<const unsigned char*>(a.k_new) + head * C::ROW,
@@ -853,6 +860,13 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
         abort_s = 0;
         issued_s = 0;
     }
+    if (a.gq < G) {
+        // a group of gq < 8 heads fills the score tile's columns gq .. 7 with zero query rows,
+        // never loaded: those heads compute finite values that are never written
+        for (int s = 0; s < kTcStages; ++s)
+            for (int x = threadIdx.x; x < (G - a.gq) * C::ROW / 16; x += blockDim.x)
+                reinterpret_cast<uint4*>(dsmem + s * C::STAGE + C::Q_OFF + a.gq * C::ROW)[x] = make_uint4(0u, 0u, 0u, 0u);
+    }
     __syncthreads();
 
     if (warp == kTcConsumers) {
@@ -922,7 +936,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     meta_s[s] = mt;
                     unsigned char* st = dsmem + s * C::STAGE;
                     const uint32_t bytes = static_cast<uint32_t>((nk > 0 ? 2 * C::BOXES * C::BOX_BYTES : 0) +
-                                                                 (first ? G * C::ROW : 0) + (current ? 2 * C::ROW : 0));
+                                                                 (first ? a.gq * C::ROW : 0) + (current ? 2 * C::ROW : 0));
                     fence_proxy_async();
                     mbar_expect_tx(&full_bar[s], bytes);
                     if (nk > 0) {
@@ -939,8 +953,8 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     }
                     if (first) {
                         const unsigned char* qg = static_cast<const unsigned char*>(a.q) +
-                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * G) * C::ROW;
-                        bulk_g2s(st + C::Q_OFF, qg, G * C::ROW, &full_bar[s]);
+                                                  (static_cast<size_t>(b) * a.Hq + static_cast<size_t>(kvh) * a.gq) * C::ROW;
+                        bulk_g2s(st + C::Q_OFF, qg, a.gq * C::ROW, &full_bar[s]);
                     }
                     if (current) {
                         bulk_g2s(st + C::KN_OFF, static_cast<const unsigned char*>(a.k_new) + static_cast<size_t>(head) * C::ROW,
@@ -1337,14 +1351,14 @@ int occupancy_tc()
     return n;
 }
 
-// Whether a step takes the tensor-core path: bf16, GQA group 8, block a multiple
+// Whether a step takes the tensor-core path: bf16, GQA group 8 (or 4 or 6, padded), block a multiple
 // of two tiles (no tile straddles the ring end), chunks whole tiles, row
 // coordinates within int32.
 bool tc_eligible(const DecodeArgs& a, int elem_bytes)
 {
     // PBB only: its tiles start at multiples of the tile in slot order (slots 0 and
     // h), which whole TMA boxes need; a window's run starts at any slot.
-    if (a.window != 0 || elem_bytes != 2 || a.Hq != 8 * a.Hkv || (a.d != 64 && a.d != 128)) return false;
+    if (a.window != 0 || elem_bytes != 2 || !tc_group(a.gq) || (a.d != 64 && a.d != 128)) return false;
     constexpr int tk = 16 * kTcConsumers;
     if (a.B % (2 * tk) != 0 || a.chunk % tk != 0) return false;
     const unsigned long long rows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.B;
@@ -1378,6 +1392,7 @@ cudaError_t launch_g(const DecodeArgs& a, cudaStream_t stream)
         case 1: return launch_t<ELEM, D, 1>(a, stream);
         case 2: return launch_t<ELEM, D, 2>(a, stream);
         case 4: return launch_t<ELEM, D, 4>(a, stream);
+        case 6:  // six query heads per KV head run on the group-8 kernel with two padded heads
         case 8: return launch_t<ELEM, D, 8>(a, stream);
         default: return cudaErrorInvalidValue;
     }
@@ -1390,6 +1405,7 @@ int occupancy_g(int group)
         case 1: return occupancy_t<ELEM, D, 1>();
         case 2: return occupancy_t<ELEM, D, 2>();
         case 4: return occupancy_t<ELEM, D, 4>();
+        case 6:
         case 8: return occupancy_t<ELEM, D, 8>();
         default: return 0;
     }
@@ -1402,6 +1418,7 @@ int tile_g(int group)
         case 1: return Cfg<ELEM, D, 1>::TK;
         case 2: return Cfg<ELEM, D, 2>::TK;
         case 4: return Cfg<ELEM, D, 4>::TK;
+        case 6:
         case 8: return Cfg<ELEM, D, 8>::TK;
         default: return 0;
     }
@@ -1420,7 +1437,7 @@ int tile_keys(int elem_bytes, int d, int group)
 
 int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window)
 {
-    if (window == 0 && elem_bytes == 2 && group == 8 && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
+    if (window == 0 && elem_bytes == 2 && tc_group(group) && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
         tensor_map_encoder() != nullptr)
         return d == 64 ? occupancy_tc<64>() : occupancy_tc<128>();
     if (elem_bytes == 2 && d == 64) return occupancy_g<2, 64>(group);

@@ -25,6 +25,7 @@ struct DecodeArgs {
     int* counters;       // [batch][Hkv]                 finished chunks per (sequence, KV head)
     int* ctl;            // [2] work-queue head and finished CTAs; zero between launches
     int batch, Hq, Hkv, d, B;
+    int gq;              // query heads per KV head (Hq / Hkv); the kernel's group G is gq, or 8 for gq = 6
     int pos_batch;       // sequences with their own position: sequence b reads pos[b % pos_batch]
                          // (layers of a multi-layer step are consecutive batches sharing positions)
     int window;          // 0: the PBB support [a(t), t]; w in [1, B]: the sliding window {t-w+1, ..., t}
@@ -37,6 +38,17 @@ struct DecodeArgs {
 
 // Keys per shared-memory tile of a kernel instance (rows of K and of V).
 int tile_keys(int elem_bytes, int d, int group);
+
+// GQA groups the tensor-core decode kernel serves: its score tile has 8 query columns, and a
+// group of 4 or 6 fills the rest with zero query rows (PBB_TC_MIN_GROUP = 8 keeps those groups
+// on the CUDA-core kernel).
+#ifndef PBB_TC_MIN_GROUP
+#define PBB_TC_MIN_GROUP 4
+#endif
+inline bool tc_group(int group)
+{
+    return group == 8 || (group >= PBB_TC_MIN_GROUP && (group == 4 || group == 6));
+}
 
 // Resident CTAs per SM of the decode kernel a step of this shape runs (0 if unsupported).
 int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window);

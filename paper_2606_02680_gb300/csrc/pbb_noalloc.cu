@@ -69,8 +69,8 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     if ((B % 2) != 0 || B > (1 << 20) || (d != 64 && d != 128) || batch > 65535 || Hkv > 65535)
         return PBB_ERR_UNSUPPORTED;
     if (Hq % Hkv != 0) return PBB_ERR_UNSUPPORTED;
-    const int group = Hq / Hkv;
-    if (group != 1 && group != 2 && group != 4 && group != 8) return PBB_ERR_UNSUPPORTED;
+    const int gq = Hq / Hkv;
+    if (gq != 1 && gq != 2 && gq != 4 && gq != 6 && gq != 8) return PBB_ERR_UNSUPPORTED;
     if (batch == 0) return PBB_OK;
     if (!q || !k_new || !v_new || !k_ring || !v_ring || !pos || !out) return PBB_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k_new, 16) || !aligned(v_new, 16) || !aligned(k_ring, 16) ||
@@ -93,8 +93,9 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     a.Hkv = Hkv;
     a.d = d;
     a.B = B;
+    a.gq = gq;
     a.pos_batch = batch;
-    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, 2, group, 0);  // the same plan as pbb_decode_step
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, 2, gq, 0);  // the same plan as pbb_decode_step
     if (sp.chunk <= 0) return PBB_ERR_CUDA;
     a.whole = sp.whole;
     a.chunk = sp.chunk;
@@ -102,6 +103,9 @@ extern "C" int pbb_decode_step_noalloc(const void* q, const void* k_new, const v
     if (a.nchunk > 65535) return PBB_ERR_UNSUPPORTED;
     a.timeout_ns = 1000000000ull;
 
+    // the partials' head layout is the launched kernel's group: 8 on the tensor cores, and 8
+    // for six heads on the CUDA cores
+    const int group = (pbb::use_tensor_cores(a, 2) || gq == 6) ? 8 : gq;
     const size_t pairs = static_cast<size_t>(batch) * Hkv;
     const size_t parts = (pairs - static_cast<size_t>(sp.whole)) * a.nchunk * group;
     const size_t o_bytes = round_up(parts * d * sizeof(float), 256);

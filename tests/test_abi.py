@@ -115,6 +115,20 @@ def test_product_path_does_not_use_the_oracle():
                 assert "pbb_oracle" not in text, f
 
 
+def test_group6_decode_only(pbb):
+    """GQA group 6 (12 query heads on 2 KV heads) is a decode shape; the whole-sequence
+    forward and backward, whose tiles stack the group's heads into 128 rows, refuse it
+    before looking at any pointer. Batch 0 makes the decode calls no-ops."""
+    lib = pbb.lib()
+    assert lib.pbb_decode_step(None, None, None, None, None, None, None, 0, 12, 2, 64, 128, None) == 0
+    assert lib.pbb_swa_decode_step(None, None, None, None, None, None, None, 0, 12, 2, 64, 128,
+                                   128, 0, None) == 0
+    assert lib.pbb_forward(None, None, None, None, None, 1, 12, 2, 128, 64, 128, 0, None) == -2
+    assert lib.pbb_backward(None, None, None, None, None, None, None, None, None, None, 1, 12, 2,
+                            128, 64, 128, None) == -2
+    assert lib.pbb_decode_step(None, None, None, None, None, None, None, 0, 24, 2, 64, 128, None) == -2
+
+
 def test_window_checked_before_launch(pbb):
     """pbb_swa_decode_step: a window outside [1, B] is refused before anything
     else; batch 0 with a valid window is a no-op (no device work)."""

@@ -91,6 +91,13 @@ def test_group8_tensor_core_layers():
     run_layers(w, 2, 30)
 
 
+def test_group6_layers():
+    """Two local layers of the paper's model shape (12 query heads on 2 KV heads, d 64)."""
+    w = inputs.Workload("layers_g6", batch=3, Hq=12, Hkv=2, d=64, B=128, dtype="bf16", steps=0,
+                        t0_lo=0, t0_hi=2000, seed=304)
+    run_layers(w, 2, 30)
+
+
 def test_fp32_layers():
     w = inputs.Workload("layers_f32", batch=2, Hq=8, Hkv=2, d=64, B=128, dtype="f32", steps=0,
                         t0_lo=0, t0_hi=600, seed=303)

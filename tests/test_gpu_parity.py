@@ -64,7 +64,7 @@ def test_fp32_one_layer_split(chunk_keys):
     run_and_check(w, chunk_keys, chunk=32, ring_every=100)
 
 
-@pytest.mark.parametrize("group", [1, 2, 4, 8])
+@pytest.mark.parametrize("group", [1, 2, 4, 6, 8])
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("chunk", [0, 32])
 def test_bf16_groups_and_dims(chunk_keys, group, d, chunk):
@@ -79,13 +79,27 @@ def test_bf16_groups_and_dims(chunk_keys, group, d, chunk):
 
 
 @pytest.mark.parametrize("group,d,dtype", [(4, 128, "bf16"), (8, 128, "bf16"), (4, 64, "f32"),
-                                           (2, 128, "f32")])
+                                           (2, 128, "f32"), (6, 64, "bf16"), (6, 128, "f32")])
 def test_ragged_prefilled(chunk_keys, group, d, dtype):
     """Ragged start positions with rings loaded by pbb_ring_prefill; every step checked."""
     w = inputs.Workload("ragged", batch=5, Hq=2 * group, Hkv=2, d=d, B=256, dtype=dtype,
                         steps=300, t0_lo=0, t0_hi=5000, seed=7 + group)
     run_and_check(w, chunk_keys, chunk=0)
     run_and_check(w, chunk_keys, chunk=64)
+
+
+def test_paper_model_shape_group6(chunk_keys):
+    """The paper's models (Sec. 5): 12 query heads on 2 KV heads, head size 64, block 128.
+    GQA group 6 runs on the tensor-core kernel with two zero query rows that are never
+    written: batch 1 from t = 0 across 5 block boundaries, every step, then ragged
+    prefilled positions with every support split into 32-key chunks. (The CUDA-core kernel
+    runs group 6 for fp32, windows and blocks that are not a multiple of 64.)"""
+    w = inputs.Workload("paper_g6", batch=1, Hq=12, Hkv=2, d=64, B=128, dtype="bf16",
+                        steps=5 * 128 + 3, t0_lo=0, t0_hi=1, seed=612)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
+    run_and_check(w, chunk_keys, ring_every=128)
+    w = w.with_(name="paper_g6_ragged", batch=5, steps=200, t0_hi=50000, seed=613)
+    run_and_check(w, chunk_keys, chunk=32)
 
 
 def test_prefill_is_bit_exact(chunk_keys):
@@ -297,11 +311,28 @@ def test_bf16_group8_tensor_core_path(chunk_keys, B, d, chunk):
     run_and_check(w, chunk_keys, chunk=chunk)
 
 
+@pytest.mark.parametrize("group", [4, 6])
+@pytest.mark.parametrize("B", [64, 256])
 @pytest.mark.parametrize("d", [64, 128])
-def test_bf16_group8_tensor_core_ragged_outliers(chunk_keys, d):
+@pytest.mark.parametrize("chunk", [0, 64])
+def test_bf16_padded_group_tensor_core_path(chunk_keys, group, B, d, chunk):
+    """GQA groups 4 and 6 on the tensor-core kernel: the score tile's 8 query columns hold the
+    group's heads and zero rows for the rest, whose outputs are never written. Every step of
+    3 blocks from t = 0, batch 3, against the oracle; the output rows of neighbouring KV
+    groups must come out untouched by the padded heads."""
+    w = inputs.Workload(f"tcpad_g{group}_B{B}_d{d}", batch=3, Hq=2 * group, Hkv=2, d=d, B=B,
+                        dtype="bf16", steps=3 * B + 3, t0_lo=0, t0_hi=1, seed=400 + group + B + d)
+    chunk_keys(chunk)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
+    run_and_check(w, chunk_keys, chunk=chunk)
+
+
+@pytest.mark.parametrize("group", [4, 6, 8])
+@pytest.mark.parametrize("d", [64, 128])
+def test_bf16_tensor_core_ragged_outliers(chunk_keys, group, d):
     """Tensor-core path with ragged prefilled rings and x20 outliers (large logits)."""
-    w = inputs.Workload("tc_outlier", batch=6, Hq=8, Hkv=1, d=d, B=512, dtype="bf16", steps=80,
-                        t0_lo=0, t0_hi=20000, outlier_frac=0.01, outlier_scale=20.0, seed=77 + d)
+    w = inputs.Workload("tc_outlier", batch=6, Hq=group, Hkv=1, d=d, B=512, dtype="bf16", steps=80,
+                        t0_lo=0, t0_hi=20000, outlier_frac=0.01, outlier_scale=20.0, seed=77 + d + group)
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
     run_and_check(w, chunk_keys, chunk=0)
     run_and_check(w, chunk_keys, chunk=128)

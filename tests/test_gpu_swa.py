@@ -51,7 +51,7 @@ def run_and_check(w, window, check_every=1, ring_every=None):
     assert pbb.get_device_status() == pbb.PBB_OK
 
 
-@pytest.mark.parametrize("group", [1, 2, 4, 8])
+@pytest.mark.parametrize("group", [1, 2, 4, 6, 8])
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("chunk", [0, 32])
 def test_window_B_groups_and_dims(chunk_keys, group, d, chunk):

@@ -40,14 +40,17 @@ def _state(pbb, w, t0, wk, wv, dev):
     return pos, kr, vr
 
 
-def test_noalloc_matches_decode_step_on_two_calls(lib):
+@pytest.mark.parametrize("Hq,Hkv,d", [(16, 4, 128), (12, 2, 64), (8, 4, 128)])
+def test_noalloc_matches_decode_step_on_two_calls(lib, Hq, Hkv, d):
     pbb = lib
     from paper_2606_02680_gb300 import inputs
 
     dev = torch.device("cuda", 0)
-    # small batch: the plan splits every support across many CTAs, so the scratch is used
-    w = inputs.Workload("noalloc", batch=4, Hq=16, Hkv=4, d=128, B=2048, dtype="bf16", steps=2,
-                        t0_lo=2048, t0_hi=100000, seed=77)
+    # small batch: the plan splits every support across many CTAs, so the scratch is used;
+    # (12, 2, 64) is the paper's model shape, GQA group 6; groups 4 and 6 run on the tensor
+    # cores, group 2 on the CUDA cores
+    w = inputs.Workload("noalloc", batch=4, Hq=Hq, Hkv=Hkv, d=d, B=2048, dtype="bf16", steps=2,
+                        t0_lo=2048, t0_hi=100000, seed=77 + Hq)
     assert pbb.plan_chunk_keys(w.batch, w.Hq, w.Hkv, w.d, w.B) < w.B - 1
     t0 = inputs.start_positions(w)
     wk, wv = inputs.history_window(w, t0, device=dev)
