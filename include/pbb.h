@@ -263,11 +263,24 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
 /*
  * Which kernel a decode step of this shape runs on the current device:
  * PBB_KERNEL_CUDA_CORES (packed fp32 FMAs; every shape) or PBB_KERNEL_TENSOR_CORES
- * (bf16 with Hq/Hkv = 8, where the scores of a 16-key block against the 8 query
- * heads form a dense mma tile; needs B a multiple of 64). Negative on error.
+ * (bf16 PBB steps with Hq/Hkv = 8, where the scores of a 16-key block against the
+ * 8 query heads form a dense mma tile, or Hq/Hkv = 4 or 6 with the tile's other
+ * columns zero; needs B a multiple of 64). Groups 4 and 6 take the tensor cores
+ * only when batch*Hkv fills the resident CTAs. Negative on error.
  */
-enum { PBB_KERNEL_CUDA_CORES = 0, PBB_KERNEL_TENSOR_CORES = 1 };
+enum { PBB_KERNEL_AUTO = -1, PBB_KERNEL_CUDA_CORES = 0, PBB_KERNEL_TENSOR_CORES = 1 };
 int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
+ * Kernel choice for the decode steps that follow (process-wide, like
+ * pbb_set_chunk_keys): PBB_KERNEL_AUTO (the default) lets the library choose;
+ * PBB_KERNEL_CUDA_CORES runs every step on the CUDA-core kernel;
+ * PBB_KERNEL_TENSOR_CORES runs every step the tensor-core kernel supports (bf16
+ * PBB steps, Hq/Hkv in {4, 6, 8}, B a multiple of 64) on it whatever the batch,
+ * the rest on the CUDA cores. Returns the previous choice, or
+ * PBB_ERR_INVALID_ARG (and no change) for any other value.
+ */
+int pbb_set_kernel(int kernel);
 
 /*
  * No counterpart in the paper: a library-usage variant for callers that cannot

@@ -33,7 +33,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
+    "lib", "lib_path", "set_kernel", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -70,6 +70,7 @@ EXPORTS = {
     "pbb_get_device_status": (_I, [_P]),
     "pbb_set_wait_timeout_ns": (_I, [_ULL]),
     "pbb_set_chunk_keys": (_I, [_I]),
+    "pbb_set_kernel": (_I, [_I]),
     "pbb_plan_chunk_keys": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_plan_kernel": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_error_string": (ctypes.c_char_p, [_I]),
@@ -469,8 +470,23 @@ def plan_chunk_keys(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.b
     return int(lib().pbb_plan_chunk_keys(batch, Hq, Hkv, d, B, _dt(dtype)))
 
 
+PBB_KERNEL_AUTO = -1
 PBB_KERNEL_CUDA_CORES = 0
 PBB_KERNEL_TENSOR_CORES = 1
+_KERNEL_NAMES = {"auto": PBB_KERNEL_AUTO, "cuda_cores": PBB_KERNEL_CUDA_CORES,
+                 "tensor_cores": PBB_KERNEL_TENSOR_CORES}
+
+
+def set_kernel(kernel: str) -> str:
+    """Kernel choice for later decode steps: 'auto' (default), 'cuda_cores', or
+    'tensor_cores' (every step the tensor-core kernel supports, whatever the batch).
+    Returns the previous choice."""
+    if kernel not in _KERNEL_NAMES:
+        raise ValueError(f"kernel must be one of {sorted(_KERNEL_NAMES)}")
+    prev = int(lib().pbb_set_kernel(_KERNEL_NAMES[kernel]))
+    if prev < PBB_KERNEL_AUTO:
+        raise PbbError(prev, "pbb_set_kernel")
+    return {v: k for k, v in _KERNEL_NAMES.items()}[prev]
 
 
 def plan_kernel(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> str:

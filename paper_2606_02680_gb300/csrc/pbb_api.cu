@@ -117,6 +117,11 @@ int min_split_keys(int d, int elem, int tile)
 
 }  // namespace
 
+// Whether the tensor-core kernel also splits a partly filled last round of long supports.
+#ifndef PBB_TC_SPLIT_LAST_ROUND
+#define PBB_TC_SPLIT_LAST_ROUND 0
+#endif
+
 namespace pbb {
 
 SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int window)
@@ -150,7 +155,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
         sp.nchunk = (max_keys + chunk - 1) / chunk;
         return sp;
     }
-    int per_sm = pbb::decode_ctas_per_sm(elem, d, group, B, window);
+    int per_sm = pbb::decode_ctas_per_sm(batch, Hkv, elem, d, group, B, window);
     if (per_sm <= 0) per_sm = 1;
     const long long G = static_cast<long long>(sm_count(dev)) * per_sm;
     if (pairs >= G) {
@@ -159,7 +164,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
         // (measured: +29 % at B 4096 and +6 % at B 2048, but -12 to -15 % at B <= 1024 and
         // -19 % for the tensor-core kernel, whose two consumer warps combine slowly).
         const bool long_supports = max_keys >= 2047 && pbb::tile_keys(elem, d, group) == tile &&
-                                   !(window == 0 && elem == 2 && pbb::tc_group(group) && B % 64 == 0);
+                                   (PBB_TC_SPLIT_LAST_ROUND || !pbb::tensor_core_shape(batch, Hkv, d, B, elem, group, window));
         if (R == 0 || 2 * R > G || !long_supports) {  // no split
             sp.whole = static_cast<int>(pairs);
             sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
@@ -543,6 +548,13 @@ int pbb_set_chunk_keys(int keys)
 {
     if (keys < 0) return PBB_ERR_INVALID_ARG;
     return g_chunk_override.exchange(keys);
+}
+
+int pbb_set_kernel(int kernel)
+{
+    if (kernel != PBB_KERNEL_AUTO && kernel != PBB_KERNEL_CUDA_CORES && kernel != PBB_KERNEL_TENSOR_CORES)
+        return PBB_ERR_INVALID_ARG;
+    return pbb::set_kernel_choice(kernel);
 }
 
 int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)

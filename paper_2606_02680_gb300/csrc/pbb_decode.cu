@@ -55,8 +55,10 @@
 #include <cudaTypedefs.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <mutex>
 
+#include "pbb.h"
 #include "pbb_device.cuh"
 #include "pbb_internal.h"
 
@@ -1351,18 +1353,53 @@ int occupancy_tc()
     return n;
 }
 
-// Whether a step takes the tensor-core path: bf16, GQA group 8 (or 4 or 6, padded), block a multiple
-// of two tiles (no tile straddles the ring end), chunks whole tiles, row
-// coordinates within int32.
+int device_sms()
+{
+    static int cache[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    if (dev < 64 && cache[dev] > 0) return cache[dev];
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    if (dev < 64) cache[dev] = n;
+    return n;
+}
+
+// Padded groups (4 and 6 heads in the 8-column score tile) take the tensor cores only when the
+// supports at least fill the resident CTAs. With fewer supports every support is split, and
+// there the CUDA-core kernel, whose four consumer warps merge and combine the split partials
+// faster, wins (measured on GB300: 7-34 % at batch 1 to 32, Hq 32, Hkv 8).
+#ifndef PBB_TC_PAD_MIN_FILL
+#define PBB_TC_PAD_MIN_FILL 1
+#endif
+
+// Whether a step of this shape runs the tensor-core kernel, before the chunk check: a bf16 PBB
+// step (its tiles start at multiples of the tile in slot order, slots 0 and h, as whole TMA
+// boxes need; a window's run starts at any slot), GQA group 8 (or 4 or 6, padded), d 64 or
+// 128, block a multiple of two tiles (no tile straddles the ring end), row coordinates within
+// int32.
+std::atomic<int> g_kernel_choice{PBB_KERNEL_AUTO};
+
+bool tc_shape(int batch, int Hkv, int d, int B, int elem_bytes, int group, int window)
+{
+    const int choice = g_kernel_choice.load();
+    if (choice == PBB_KERNEL_CUDA_CORES) return false;
+    if (window != 0 || elem_bytes != 2 || !tc_group(group) || (d != 64 && d != 128)) return false;
+    if (B % (32 * kTcConsumers) != 0 || tensor_map_encoder() == nullptr) return false;
+    const unsigned long long rows = static_cast<unsigned long long>(batch) * Hkv * B;
+    if (rows >= (1ull << 31)) return false;
+    if (PBB_TC_PAD_MIN_FILL && group != 8 && choice == PBB_KERNEL_AUTO) {
+        const long long ctas = static_cast<long long>(device_sms()) * (d == 64 ? occupancy_tc<64>() : occupancy_tc<128>());
+        if (static_cast<long long>(batch) * Hkv < ctas) return false;
+    }
+    return true;
+}
+
+// The tensor-core path also needs chunks of whole tiles.
 bool tc_eligible(const DecodeArgs& a, int elem_bytes)
 {
-    // PBB only: its tiles start at multiples of the tile in slot order (slots 0 and
-    // h), which whole TMA boxes need; a window's run starts at any slot.
-    if (a.window != 0 || elem_bytes != 2 || !tc_group(a.gq) || (a.d != 64 && a.d != 128)) return false;
     constexpr int tk = 16 * kTcConsumers;
-    if (a.B % (2 * tk) != 0 || a.chunk % tk != 0) return false;
-    const unsigned long long rows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.B;
-    return rows < (1ull << 31) && tensor_map_encoder() != nullptr;
+    return tc_shape(a.batch, a.Hkv, a.d, a.B, elem_bytes, a.gq, a.window) && a.chunk % tk == 0;
 }
 
 template <int D>
@@ -1435,11 +1472,16 @@ int tile_keys(int elem_bytes, int d, int group)
     return 0;
 }
 
-int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window)
+int set_kernel_choice(int kernel) { return g_kernel_choice.exchange(kernel); }
+
+bool tensor_core_shape(int batch, int Hkv, int d, int B, int elem_bytes, int group, int window)
 {
-    if (window == 0 && elem_bytes == 2 && tc_group(group) && (d == 64 || d == 128) && B % (32 * kTcConsumers) == 0 &&
-        tensor_map_encoder() != nullptr)
-        return d == 64 ? occupancy_tc<64>() : occupancy_tc<128>();
+    return tc_shape(batch, Hkv, d, B, elem_bytes, group, window);
+}
+
+int decode_ctas_per_sm(int batch, int Hkv, int elem_bytes, int d, int group, int B, int window)
+{
+    if (tc_shape(batch, Hkv, d, B, elem_bytes, group, window)) return d == 64 ? occupancy_tc<64>() : occupancy_tc<128>();
     if (elem_bytes == 2 && d == 64) return occupancy_g<2, 64>(group);
     if (elem_bytes == 2 && d == 128) return occupancy_g<2, 128>(group);
     if (elem_bytes == 4 && d == 64) return occupancy_g<4, 64>(group);

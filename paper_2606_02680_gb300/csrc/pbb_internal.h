@@ -50,8 +50,16 @@ inline bool tc_group(int group)
     return group == 8 || (group >= PBB_TC_MIN_GROUP && (group == 4 || group == 6));
 }
 
+// The kernel choice of pbb_set_kernel (PBB_KERNEL_AUTO, _CUDA_CORES or _TENSOR_CORES); returns
+// the previous one.
+int set_kernel_choice(int kernel);
+
+// Whether a decode step of this shape runs the tensor-core kernel (given chunks of whole
+// tiles, which plan_split makes for it).
+bool tensor_core_shape(int batch, int Hkv, int d, int B, int elem_bytes, int group, int window);
+
 // Resident CTAs per SM of the decode kernel a step of this shape runs (0 if unsupported).
-int decode_ctas_per_sm(int elem_bytes, int d, int group, int B, int window);
+int decode_ctas_per_sm(int batch, int Hkv, int elem_bytes, int d, int group, int B, int window);
 
 // The split plan of a step (see plan_split in pbb_api.cu): supports [0, whole)
 // run whole, every later one in nchunk chunks of `chunk` ring keys. window as

@@ -129,6 +129,20 @@ def test_group6_decode_only(pbb):
     assert lib.pbb_decode_step(None, None, None, None, None, None, None, 0, 24, 2, 64, 128, None) == -2
 
 
+def test_kernel_choice_roundtrip(pbb):
+    """pbb_set_kernel needs no device: it records the choice for later steps."""
+    lib = pbb.lib()
+    assert lib.pbb_set_kernel(5) == -1 and lib.pbb_set_kernel(-2) == -1
+    prev = pbb.set_kernel("cuda_cores")
+    try:
+        assert pbb.set_kernel("tensor_cores") == "cuda_cores"
+        assert pbb.set_kernel("auto") == "tensor_cores"
+        with pytest.raises(ValueError):
+            pbb.set_kernel("mma")
+    finally:
+        pbb.set_kernel(prev)
+
+
 def test_window_checked_before_launch(pbb):
     """pbb_swa_decode_step: a window outside [1, B] is refused before anything
     else; batch 0 with a valid window is a no-op (no device work)."""

@@ -37,6 +37,14 @@ def chunk_keys():
     pbb.set_chunk_keys(prev)
 
 
+@pytest.fixture
+def kernel():
+    """pbb.set_kernel for the test, restored afterwards."""
+    prev = pbb.set_kernel("auto")
+    yield pbb.set_kernel
+    pbb.set_kernel(prev)
+
+
 def run_and_check(w, chunk_keys, chunk=0, check_every=1, ring_every=None):
     chunk_keys(chunk)
     run = SequentialRun(w)
@@ -88,15 +96,18 @@ def test_ragged_prefilled(chunk_keys, group, d, dtype):
     run_and_check(w, chunk_keys, chunk=64)
 
 
-def test_paper_model_shape_group6(chunk_keys):
+@pytest.mark.parametrize("which", ["cuda_cores", "tensor_cores"])
+def test_paper_model_shape_group6(chunk_keys, kernel, which):
     """The paper's models (Sec. 5): 12 query heads on 2 KV heads, head size 64, block 128.
-    GQA group 6 runs on the tensor-core kernel with two zero query rows that are never
-    written: batch 1 from t = 0 across 5 block boundaries, every step, then ragged
-    prefilled positions with every support split into 32-key chunks. (The CUDA-core kernel
-    runs group 6 for fp32, windows and blocks that are not a multiple of 64.)"""
+    GQA group 6 runs on either kernel's 8 query columns with two zero query rows that are
+    never written (at batch 1 the library picks the CUDA cores): batch 1 from t = 0 across
+    5 block boundaries, every step, then ragged prefilled positions with every support
+    split into 32-key chunks."""
     w = inputs.Workload("paper_g6", batch=1, Hq=12, Hkv=2, d=64, B=128, dtype="bf16",
                         steps=5 * 128 + 3, t0_lo=0, t0_hi=1, seed=612)
-    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "cuda_cores"
+    kernel(which)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == which
     run_and_check(w, chunk_keys, ring_every=128)
     w = w.with_(name="paper_g6_ragged", batch=5, steps=200, t0_hi=50000, seed=613)
     run_and_check(w, chunk_keys, chunk=32)
@@ -315,7 +326,7 @@ def test_bf16_group8_tensor_core_path(chunk_keys, B, d, chunk):
 @pytest.mark.parametrize("B", [64, 256])
 @pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("chunk", [0, 64])
-def test_bf16_padded_group_tensor_core_path(chunk_keys, group, B, d, chunk):
+def test_bf16_padded_group_tensor_core_path(chunk_keys, kernel, group, B, d, chunk):
     """GQA groups 4 and 6 on the tensor-core kernel: the score tile's 8 query columns hold the
     group's heads and zero rows for the rest, whose outputs are never written. Every step of
     3 blocks from t = 0, batch 3, against the oracle; the output rows of neighbouring KV
@@ -323,19 +334,46 @@ def test_bf16_padded_group_tensor_core_path(chunk_keys, group, B, d, chunk):
     w = inputs.Workload(f"tcpad_g{group}_B{B}_d{d}", batch=3, Hq=2 * group, Hkv=2, d=d, B=B,
                         dtype="bf16", steps=3 * B + 3, t0_lo=0, t0_hi=1, seed=400 + group + B + d)
     chunk_keys(chunk)
+    kernel("tensor_cores")  # batch 3 alone would stay on the CUDA cores
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
     run_and_check(w, chunk_keys, chunk=chunk)
 
 
 @pytest.mark.parametrize("group", [4, 6, 8])
 @pytest.mark.parametrize("d", [64, 128])
-def test_bf16_tensor_core_ragged_outliers(chunk_keys, group, d):
+def test_bf16_tensor_core_ragged_outliers(chunk_keys, kernel, group, d):
     """Tensor-core path with ragged prefilled rings and x20 outliers (large logits)."""
+    kernel("tensor_cores")
     w = inputs.Workload("tc_outlier", batch=6, Hq=group, Hkv=1, d=d, B=512, dtype="bf16", steps=80,
                         t0_lo=0, t0_hi=20000, outlier_frac=0.01, outlier_scale=20.0, seed=77 + d + group)
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
     run_and_check(w, chunk_keys, chunk=0)
     run_and_check(w, chunk_keys, chunk=128)
+
+
+def test_kernel_choice(kernel):
+    """The library's choice: group 8 always on the tensor cores; groups 4 and 6 there once
+    the supports fill the resident CTAs (3 per SM), else on the CUDA cores; fp32, windows,
+    groups 1 and 2 and blocks that are not a multiple of 64 on the CUDA cores. pbb_set_kernel
+    overrides it within what each kernel supports."""
+    import torch as _t
+    assert pbb.plan_kernel(1, 16, 2, 128, 4096) == "tensor_cores"
+    assert pbb.plan_kernel(512, 32, 8, 128, 4096) == "tensor_cores"
+    assert pbb.plan_kernel(8, 32, 8, 128, 4096) == "cuda_cores"
+    assert pbb.plan_kernel(32, 16, 4, 128, 1024) == "cuda_cores"
+    assert pbb.plan_kernel(512, 12, 2, 64, 128) == "tensor_cores"  # the paper's heads, 1,024 supports
+    assert pbb.plan_kernel(1, 12, 2, 64, 128) == "cuda_cores"
+    assert pbb.plan_kernel(512, 16, 2, 128, 96) == "cuda_cores"
+    assert pbb.plan_kernel(512, 32, 8, 128, 4096, _t.float32) == "cuda_cores"
+    assert pbb.plan_kernel(512, 16, 8, 128, 4096) == "cuda_cores"  # group 2
+    assert kernel("cuda_cores") == "auto"
+    assert pbb.plan_kernel(512, 32, 8, 128, 4096) == "cuda_cores"
+    assert pbb.plan_kernel(1, 16, 2, 128, 4096) == "cuda_cores"
+    assert kernel("tensor_cores") == "cuda_cores"
+    assert pbb.plan_kernel(1, 32, 8, 128, 4096) == "tensor_cores"
+    assert pbb.plan_kernel(1, 16, 8, 128, 4096) == "cuda_cores"  # group 2: no tensor-core kernel
+    with pytest.raises(ValueError):
+        kernel("fastest")
 
 
 def test_host_pipeline_matches_device_steps():
