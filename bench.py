@@ -685,6 +685,7 @@ def oracle_forward_sample(w, seconds: float, rows_per_call: int = 64):
 def run_forward(args, dist, rank, world, dev):
     import torch
 
+    import paper_2606_02680_gb300 as pbb
     from paper_2606_02680_gb300 import inputs
 
     names = [args.fwd_workload] if args.fwd_workload else list(inputs.FORWARD_WORKLOADS)
@@ -710,7 +711,8 @@ def run_forward(args, dist, rank, world, dev):
         roof.update({"traffic": None,
                      "kernel": ("bwd_kv_tc_kernel<%d,%d> + bwd_q_tc_kernel<%d,%d> + delta_kernel<%d> (one call)"
                                 % (w.d, w.group, w.d, w.group, w.d)) if bwd else
-                               "forward_kernel<%d,%d,%d>" % (w.d, w.group, 128 if w.B >= 512 else 64),
+                               "forward_kernel<%d,%d,%d keys,%d CTAs/SM>" % ((w.d, w.group) + pbb.plan_forward(
+                                   w.batch, w.Hq, w.Hkv, w.n, w.d, w.B)),
                      "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,
                      "hbm_gbs": bytes_ / kern_s / 1e9, "tflops": flops / kern_s / 1e12,
                      "kernel_ms_mean": res["kernel_ms_mean"], "kernel_ms_median": res["kernel_ms_median"]})

@@ -198,6 +198,15 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
                 int Hkv, int n, int d, int B, pbb_dtype out_dtype, cudaStream_t stream);
 
 /*
+ * The launch shape pbb_forward would use for these sizes on the current device
+ * (nothing is launched): *keys_per_tile, the keys of one K/V tile (128 for
+ * B >= 512; 32 at d = 64 and 64 at d = 128 below), and *ctas_per_sm, the
+ * persistent CTAs sharing an SM's tensor memory (0 when there is no work).
+ * Same shape rules as pbb_forward; PBB_ERR_INVALID_ARG for null outputs.
+ */
+int pbb_plan_forward(int batch, int Hq, int Hkv, int n, int d, int B, int* keys_per_tile, int* ctas_per_sm);
+
+/*
  * Gradients of pbb_forward (the backward pass of the paper's fused training
  * kernel, Sec. 3: bridge gradients flow into the previous half-block's K and V).
  * With P_ts = exp(q_t.k_s/sqrt(d) - lse_t) on A(t) and D_t = dO_t . o_t:

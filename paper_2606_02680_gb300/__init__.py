@@ -33,7 +33,7 @@ __all__ = [
     "PBB_OK", "PBB_ERR_INVALID_ARG", "PBB_ERR_UNSUPPORTED", "PBB_ERR_CUDA",
     "PBB_ERR_DEVICE_TIMEOUT", "PBB_ERR_WORKSPACE", "PBB_ERR_DEVICE_POSITION",
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
-    "lib", "lib_path", "set_kernel", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
+    "lib", "lib_path", "set_kernel", "plan_forward", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
     "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
 ]
@@ -64,6 +64,7 @@ EXPORTS = {
     "pbb_swa_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_layers": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_forward": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
+    "pbb_plan_forward": (_I, [_I, _I, _I, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I)]),
     "pbb_ring_from_sequence": (_I, [_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_backward": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
@@ -475,6 +476,14 @@ PBB_KERNEL_CUDA_CORES = 0
 PBB_KERNEL_TENSOR_CORES = 1
 _KERNEL_NAMES = {"auto": PBB_KERNEL_AUTO, "cuda_cores": PBB_KERNEL_CUDA_CORES,
                  "tensor_cores": PBB_KERNEL_TENSOR_CORES}
+
+
+def plan_forward(batch: int, Hq: int, Hkv: int, n: int, d: int, B: int) -> tuple:
+    """(keys per K/V tile, persistent CTAs per SM) of pbb_forward for these sizes."""
+    nk, ctas = _I(0), _I(0)
+    _check(int(lib().pbb_plan_forward(batch, Hq, Hkv, n, d, B, ctypes.byref(nk), ctypes.byref(ctas))),
+           "pbb_plan_forward")
+    return nk.value, ctas.value
 
 
 def set_kernel(kernel: str) -> str:

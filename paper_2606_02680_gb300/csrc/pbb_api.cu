@@ -451,6 +451,31 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
     return pbb::launch_forward(a, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
 
+int pbb_plan_forward(int batch, int Hq, int Hkv, int n, int d, int B, int* keys_per_tile, int* ctas_per_sm)
+{
+    if (!keys_per_tile || !ctas_per_sm) return PBB_ERR_INVALID_ARG;
+    int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
+    if (rc != PBB_OK) return rc;
+    rc = check_group_sequence(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    if (n < 0) return PBB_ERR_INVALID_ARG;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    pbb::ForwardArgs a{};
+    a.batch = batch;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.n = n;
+    a.d = d;
+    a.B = B;
+    pbb::ForwardPlan plan{};
+    if (pbb::plan_forward(a, &plan) != cudaSuccess) return PBB_ERR_CUDA;
+    *keys_per_tile = plan.keys_per_tile;
+    *ctas_per_sm = plan.ctas_per_sm;
+    return PBB_OK;
+}
+
 int pbb_backward(const void* q, const void* k, const void* v, const void* out, const void* dout, const float* lse,
                  float* delta, float* dq, float* dk, float* dv, int batch, int Hq, int Hkv, int n, int d, int B,
                  cudaStream_t stream)

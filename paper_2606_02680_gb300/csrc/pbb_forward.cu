@@ -50,6 +50,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <algorithm>
+
 #include "pbb_device.cuh"
 #include "pbb_internal.h"
 
@@ -62,10 +64,10 @@ namespace {
 constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken GPU can exceed
 
 // Shapes of the same kernel (chosen by the block size, see launch_fwd_shape):
-//   NK    keys per K/V tile (128 or 64);
+//   NK    keys per K/V tile (128, 64 or 32);
 //   WGS   softmax warpgroups (1, or 2 taking alternate tiles with an output buffer each);
-//   CTAS  CTAs per SM: 1 owns all 512 TMEM columns, 2 share them (256 each) so one CTA's
-//         latencies overlap the other's work.
+//   CTAS  CTAs per SM: 1 owns all 512 TMEM columns, 2 to 4 share them (256 or 128 each) so
+//         one CTA's latencies overlap the others' work.
 // Long supports (many tiles per item) use one CTA per SM; short ones, where an item is one
 // or two tiles, two CTAs per SM with 64-key tiles.
 template <int D, int G, int NK_, int WGS_, int CTAS_>
@@ -73,13 +75,13 @@ struct FwdCfg {
     static constexpr int NK = NK_;
     static constexpr int WGS = WGS_;
     static constexpr int CTAS = CTAS_;
-    static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
+    static constexpr int TMEM_COLS = CTAS == 1 ? 512 : (CTAS == 2 ? 256 : 128);  // a power of 2
     static constexpr int M = 128;                       // query rows of an item (G heads x QT positions)
     static constexpr int QT = M / G;                    // positions of an item
     static constexpr int BOXES = D / 64;                // 64-column boxes of a row
     static constexpr int QBOX = M * 128;                // bytes of one Q box
     static constexpr int KBOX = NK * 128;               // bytes of one K (or V) box
-    static constexpr int QBUF = D == 64 ? 2 : 1;        // Q buffers (the next item's Q loads early)
+    static constexpr int QBUF = (D == 64 && CTAS <= 2) ? 2 : 1;  // Q buffers (the next item's Q loads early)
     static constexpr int KV_STAGE = 2 * BOXES * KBOX;   // K boxes then V boxes
     static constexpr int Q_OFF = 0;
     static constexpr int Q_BYTES = BOXES * QBOX;
@@ -99,6 +101,7 @@ struct FwdCfg {
     static constexpr int PRODUCER_WARP = 4 * WGS;
     static constexpr int MMA_WARP = 4 * WGS + 1;
     static_assert(STAGES >= 2, "shared memory budget");
+    static_assert(NK == 32 || NK % 64 == 0, "P is packed 32 or 64 scores at a time");
     static_assert(T_O + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(QT % 8 == 0, "a head's Q rows must start on a swizzle atom (8 rows)");
     static_assert(CTAS * (SMEM + STATIC_SMEM) <= 227 * 1024, "shared memory budget");
@@ -116,6 +119,17 @@ __device__ __forceinline__ int support_start(int t, int h)
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)
 {
     return __all_sync(0xffffffffu, mbar_wait(bar, parity, limit));
+}
+
+// 16-column TMEM load (the shapes with three or four CTAs per SM work in 16-column chunks to
+// stay within their registers).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
 }
 
 // One work item: (sequence, KV head) pair, first position, keys and tiles.
@@ -397,15 +411,28 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                             break;
                         }
                         tmem_fence_after();
+                        if constexpr (C::CTAS >= 3) {
 #pragma unroll
-                        for (int c = 0; c < D / 32; ++c) {
-                            uint32_t v[32];
-                            const uint32_t ta = lane_base + o_col + 32 * c;
-                            tmem_ld32(ta, v);
-                            tmem_wait_ld();
+                            for (int c = 0; c < D / 16; ++c) {
+                                uint32_t v[16];
+                                const uint32_t ta = lane_base + o_col + 16 * c;
+                                tmem_ld16(ta, v);
+                                tmem_wait_ld();
 #pragma unroll
-                            for (int x = 0; x < 32; ++x) v[x] = __float_as_uint(__uint_as_float(v[x]) * f);
-                            tmem_st32(ta, v);
+                                for (int x = 0; x < 16; ++x) v[x] = __float_as_uint(__uint_as_float(v[x]) * f);
+                                tmem_st16(ta, v);
+                            }
+                        } else {
+#pragma unroll
+                            for (int c = 0; c < D / 32; ++c) {
+                                uint32_t v[32];
+                                const uint32_t ta = lane_base + o_col + 32 * c;
+                                tmem_ld32(ta, v);
+                                tmem_wait_ld();
+#pragma unroll
+                                for (int x = 0; x < 32; ++x) v[x] = __float_as_uint(__uint_as_float(v[x]) * f);
+                                tmem_st32(ta, v);
+                            }
                         }
                         tmem_wait_st();
                     }
@@ -413,17 +440,29 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 }
                 const float nbase = m_used == -INFINITY ? 0.f : -m_used;
                 // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row
+                if constexpr (C::NK == 32) {
+                    uint32_t pk[16];
 #pragma unroll
-                for (int c = 0; c < C::NK / 64; ++c) {
-                    uint32_t pk[32];
-#pragma unroll
-                    for (int x = 0; x < 32; ++x) {
-                        const float e0 = fast_exp2(fmaf(z[64 * c + 2 * x], qscale, nbase));
-                        const float e1 = fast_exp2(fmaf(z[64 * c + 2 * x + 1], qscale, nbase));
+                    for (int x = 0; x < 16; ++x) {
+                        const float e0 = fast_exp2(fmaf(z[2 * x], qscale, nbase));
+                        const float e1 = fast_exp2(fmaf(z[2 * x + 1], qscale, nbase));
                         l += e0 + e1;
                         pk[x] = pack_bf16x2(e0, e1);
                     }
-                    tmem_st32(s_col + 32 * c, pk);
+                    tmem_st16(s_col, pk);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < C::NK / 64; ++c) {
+                        uint32_t pk[32];
+#pragma unroll
+                        for (int x = 0; x < 32; ++x) {
+                            const float e0 = fast_exp2(fmaf(z[64 * c + 2 * x], qscale, nbase));
+                            const float e1 = fast_exp2(fmaf(z[64 * c + 2 * x + 1], qscale, nbase));
+                            l += e0 + e1;
+                            pk[x] = pack_bf16x2(e0, e1);
+                        }
+                        tmem_st32(s_col + 32 * c, pk);
+                    }
                 }
                 tmem_wait_st();
                 tmem_fence_before();   // P is in TMEM and this row of S has been read
@@ -463,6 +502,37 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             }
             tmem_fence_after();
             const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
+            if constexpr (C::CTAS >= 3 && WGS == 1) {
+                // one output buffer, 16 columns at a time
+#pragma unroll
+                for (int c = 0; c < D / 16; ++c) {
+                    uint32_t v[16];
+                    tmem_ld16(lane_base + o_col + 16 * c, v);
+                    tmem_wait_ld();
+                    float o[16];
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) o[x] = __uint_as_float(v[x]) * inv;
+                    if (valid) {
+                        if (a.out_f32) {
+                            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 16 * c);
+#pragma unroll
+                            for (int x = 0; x < 4; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+                        } else {
+                            uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 16 * c);
+#pragma unroll
+                            for (int x = 0; x < 2; ++x) {
+                                uint4 pk;
+                                pk.x = pack_bf16x2(o[8 * x], o[8 * x + 1]);
+                                pk.y = pack_bf16x2(o[8 * x + 2], o[8 * x + 3]);
+                                pk.z = pack_bf16x2(o[8 * x + 4], o[8 * x + 5]);
+                                pk.w = pack_bf16x2(o[8 * x + 6], o[8 * x + 7]);
+                                dst[x] = pk;
+                            }
+                        }
+                    }
+                }
+                c1 = c0;  // done: skip the 32-column loop below
+            }
             for (int c = c0; c < c1; ++c) {
                 uint32_t v[32], u[32];
                 tmem_ld32(lane_base + (WGS == 2 ? C::T_O : o_col) + 32 * c, v);
@@ -543,8 +613,33 @@ __global__ void seq_ring_kernel(const unsigned char* __restrict__ k, const unsig
     }
 }
 
+// Resident CTAs per SM from the resources the SM checks (registers, shared memory, threads),
+// at most `want`. The runtime's occupancy calculator answers 1 for these tcgen05 kernels even
+// where two fit, and two did run together on GB300 (measured: the B = 128 forward 2,155 ->
+// 2,958 GB/s with two per SM); TMEM is shared by construction (TMEM_COLS x CTAS <= 512).
+template <typename K>
+int resident_ctas(K kernel, int threads, int dyn_smem, int want, int dev)
+{
+    cudaFuncAttributes fa{};
+    int smem_sm = 0, regs_sm = 0, reserved = 0, threads_sm = 0;
+    if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess ||
+        cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess)
+        return 1;
+    const int warps = (threads + 31) / 32;
+    const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;  // allocated per warp in 256-register units
+    const long long smem_cta = static_cast<long long>(dyn_smem) + fa.sharedSizeBytes + reserved;
+    int n = want;
+    n = std::min<long long>(n, smem_sm / smem_cta);
+    n = std::min(n, regs_sm / (regs_warp * warps));
+    n = std::min(n, threads_sm / threads);
+    return n < 1 ? 1 : n;
+}
+
 template <int D, int G, int NK, int WGS, int CTAS>
-cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
+cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
     using C = FwdCfg<D, G, NK, WGS, CTAS>;
     auto kernel = forward_kernel<D, G, NK, WGS, CTAS>;
@@ -557,26 +652,34 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
         if (err != cudaSuccess) return err;
         attr_set[dev] = true;
     }
+    const long long items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::QT - 1) / C::QT);
+    if (items < 1) {
+        if (plan != nullptr) *plan = ForwardPlan{NK, 0, 0};
+        return cudaSuccess;
+    }
+    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    // persistent CTAs: C::CTAS per SM where they fit, never more than TMEM holds
+    static int per_sm_cache[64] = {};
+    int per_sm = dev < 64 ? per_sm_cache[dev] : 0;
+    if (per_sm == 0) {
+        per_sm = resident_ctas(kernel, C::THREADS, C::SMEM, C::CTAS, dev);
+        if (dev < 64) per_sm_cache[dev] = per_sm;
+    }
+    const long long slots = static_cast<long long>(sms) * per_sm;
+    const int grid = static_cast<int>(items < slots ? items : slots);
+    if (plan != nullptr) {
+        *plan = ForwardPlan{NK, per_sm, grid};
+        return cudaSuccess;
+    }
     CUtensorMap qmap, kmap, vmap;
     const unsigned long long qrows = static_cast<unsigned long long>(a.batch) * a.Hq * a.n;
     const unsigned long long krows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.n;
     if (!rows_tensor_map(&qmap, a.q, qrows, D, C::QT) || !rows_tensor_map(&kmap, a.k, krows, D, C::NK) ||
         !rows_tensor_map(&vmap, a.v, krows, D, C::NK))
         return cudaErrorInvalidValue;
-    const long long items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::QT - 1) / C::QT);
-    if (items < 1) return cudaSuccess;
-    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;
-    int sms = 0;
-    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (err != cudaSuccess) return err;
-    // persistent CTAs: C::CTAS per SM, never more than TMEM holds
-    int per_sm = 0;
-    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, C::THREADS, C::SMEM);
-    if (err != cudaSuccess) return err;
-    if (per_sm < 1) per_sm = 1;
-    if (per_sm > C::CTAS) per_sm = C::CTAS;
-    const long long slots = static_cast<long long>(sms) * per_sm;
-    const int grid = static_cast<int>(items < slots ? items : slots);
     kernel<<<grid, C::THREADS, C::SMEM, stream>>>(qmap, kmap, vmap, a);
     return cudaGetLastError();
 }
@@ -587,39 +690,51 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream)
 #define PBB_FWD_LONG_SHAPE 0
 #endif
 
-// Short supports: 64-key tiles, two CTAs per SM (measured on GB300 at B = 128: 2,169 GB/s,
-// against 1,646 GB/s for the long-support shape, where an item is one tile).
+// Short supports (B < 512, an item is one to three tiles): 64-key tiles and two CTAs per SM, or
+// at d = 64 (build option PBB_FWD_SHORT_SHAPE) 32-key tiles with three (1) or four (2) CTAs.
+#ifndef PBB_FWD_SHORT_SHAPE
+#define PBB_FWD_SHORT_SHAPE 1
+#endif
+
 template <int D, int G>
-cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream)
+cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
-    if (a.B < 512) return launch_fwd<D, G, 64, 1, 2>(a, stream);
+    if (a.B < 512) {
+        if constexpr (D == 64 && PBB_FWD_SHORT_SHAPE == 1) return launch_fwd<D, G, 32, 1, 3>(a, stream, plan);
+        if constexpr (D == 64 && PBB_FWD_SHORT_SHAPE == 2) return launch_fwd<D, G, 32, 1, 4>(a, stream, plan);
+        return launch_fwd<D, G, 64, 1, 2>(a, stream, plan);
+    }
 #if PBB_FWD_LONG_SHAPE == 1
-    return launch_fwd<D, G, 64, 2, 1>(a, stream);
+    return launch_fwd<D, G, 64, 2, 1>(a, stream, plan);
 #else
-    return launch_fwd<D, G, 128, 1, 1>(a, stream);
+    return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
 #endif
 }
 
 template <int D>
-cudaError_t launch_fwd_d(const ForwardArgs& a, cudaStream_t stream)
+cudaError_t launch_fwd_d(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
     switch (a.Hq / a.Hkv) {
-        case 1: return launch_fwd_shape<D, 1>(a, stream);
-        case 2: return launch_fwd_shape<D, 2>(a, stream);
-        case 4: return launch_fwd_shape<D, 4>(a, stream);
-        case 8: return launch_fwd_shape<D, 8>(a, stream);
+        case 1: return launch_fwd_shape<D, 1>(a, stream, plan);
+        case 2: return launch_fwd_shape<D, 2>(a, stream, plan);
+        case 4: return launch_fwd_shape<D, 4>(a, stream, plan);
+        case 8: return launch_fwd_shape<D, 8>(a, stream, plan);
         default: return cudaErrorInvalidValue;
     }
 }
 
-}  // namespace
-
-cudaError_t launch_forward(const ForwardArgs& a, cudaStream_t stream)
+cudaError_t forward_dispatch(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
-    if (a.d == 64) return launch_fwd_d<64>(a, stream);
-    if (a.d == 128) return launch_fwd_d<128>(a, stream);
+    if (a.d == 64) return launch_fwd_d<64>(a, stream, plan);
+    if (a.d == 128) return launch_fwd_d<128>(a, stream, plan);
     return cudaErrorInvalidValue;
 }
+
+}  // namespace
+
+cudaError_t launch_forward(const ForwardArgs& a, cudaStream_t stream) { return forward_dispatch(a, stream, nullptr); }
+
+cudaError_t plan_forward(const ForwardArgs& a, ForwardPlan* plan) { return forward_dispatch(a, nullptr, plan); }
 
 cudaError_t launch_seq_ring(const void* k, const void* v, void* k_ring, void* v_ring, int batch, int Hkv,
                             int n, int B, int row_bytes, cudaStream_t stream)

@@ -102,6 +102,12 @@ struct ForwardArgs {
     unsigned long long timeout_ns;
 };
 cudaError_t launch_forward(const ForwardArgs& a, cudaStream_t stream);
+// The shape launch_forward runs for these arguments (nothing is launched): keys per K/V tile,
+// persistent CTAs per SM and the grid.
+struct ForwardPlan {
+    int keys_per_tile, ctas_per_sm, grid;
+};
+cudaError_t plan_forward(const ForwardArgs& a, ForwardPlan* plan);
 cudaError_t launch_seq_ring(const void* k, const void* v, void* k_ring, void* v_ring, int batch, int Hkv,
                             int n, int B, int row_bytes, cudaStream_t stream);
 // Status word of the forward kernels (read and cleared; the caller synchronises first).

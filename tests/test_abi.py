@@ -129,6 +129,16 @@ def test_group6_decode_only(pbb):
     assert lib.pbb_decode_step(None, None, None, None, None, None, None, 0, 24, 2, 64, 128, None) == -2
 
 
+def test_forward_plan_checks_before_the_device(pbb):
+    import ctypes
+
+    lib = pbb.lib()
+    x = ctypes.c_int(0)
+    assert lib.pbb_plan_forward(1, 8, 2, 64, 64, 128, None, ctypes.byref(x)) == -1
+    assert lib.pbb_plan_forward(1, 12, 2, 64, 64, 128, ctypes.byref(x), ctypes.byref(x)) == -2  # group 6
+    assert lib.pbb_plan_forward(1, 8, 2, 64, 96, 128, ctypes.byref(x), ctypes.byref(x)) == -2   # d 96
+
+
 def test_kernel_choice_roundtrip(pbb):
     """pbb_set_kernel needs no device: it records the choice for later steps."""
     lib = pbb.lib()

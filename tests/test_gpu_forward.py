@@ -185,3 +185,15 @@ def test_ring_from_sequence_then_decode(n, B):
         assert err <= 1e-2, (t, err)
         sim.append(ks, vs, np.full(w.batch, t))
     assert np.array_equal(ring_bytes_np(kr), sim.k) and np.array_equal(ring_bytes_np(vr), sim.v)
+
+
+def test_launch_shapes():
+    """Long supports (B >= 512) run 128-key tiles with one CTA per SM (all 512 TMEM columns);
+    short ones run 32-key tiles with three CTAs per SM at d = 64 (128 columns each) and
+    64-key tiles with two at d = 128 (256 each): more CTAs overlap the per-item latencies
+    of one- to four-tile items."""
+    assert pbb.plan_forward(2, 32, 8, 32768, 128, 4096) == (128, 1)
+    assert pbb.plan_forward(16, 8, 2, 8192, 64, 128) == (32, 3)
+    assert pbb.plan_forward(16, 8, 2, 8192, 128, 128) == (64, 2)
+    assert pbb.plan_forward(1, 8, 2, 0, 64, 128)[1] == 0  # no work
+
