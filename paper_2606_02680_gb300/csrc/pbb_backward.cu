@@ -42,9 +42,6 @@ namespace {
 constexpr unsigned kFull = 0xffffffffu;
 constexpr unsigned long long kGuardNs = 2000000000ull;
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr int kTcThreads = 320;  // 8 elementwise warps (two warpgroups), producer, MMA issuer
-constexpr int kTcProducer = 8;
-constexpr int kTcMma = 9;
 
 __device__ __forceinline__ int support_start(int t, int h)
 {
@@ -104,22 +101,31 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
 }
 
 // ------------------------------------------------------------------ dQ ----
-// Items of 128 query rows (G heads x QT positions), key tiles of 64. TMEM: S and dP,
+// Items of 128 query rows (G heads x QT positions), key tiles of NK. TMEM: S and dP,
 // two buffers each (dS is written back over S as bf16 pairs, the A operand of
-// dQ += dS K), and two dQ accumulators alternating between items.
-template <int D, int G>
+// dQ += dS K), and one or two dQ accumulators alternating between items.
+// Shapes: NK keys per tile (64 or 32), WGS elementwise warpgroups (2 taking alternate
+// tiles, or 1), CTAS CTAs per SM sharing its 512 TMEM columns (1, or 2 with 256 each).
+template <int D, int G, int NK_, int WGS_, int CTAS_>
 struct BqCfg {
-    static constexpr int M = 128, QT = M / G, NK = 64, BOXES = D / 64;
+    static constexpr int NK = NK_, WGS = WGS_, CTAS = CTAS_;
+    static constexpr int M = 128, QT = M / G, BOXES = D / 64;
+    static constexpr int THREADS = 128 * WGS + 64, PRODUCER = 4 * WGS, MMA = 4 * WGS + 1;
+    static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
     static constexpr int QBOX = M * 128, KBOX = NK * 128;
     static constexpr int Q_OFF = 0, DO_OFF = BOXES * QBOX;
     static constexpr int KV_OFF = 2 * BOXES * QBOX;
     static constexpr int KV_STAGE = 2 * BOXES * KBOX;
-    static constexpr int STAGES = 4;
+    static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - KV_OFF) / KV_STAGE;
+    static constexpr int STAGES = STAGE_ROOM < 4 ? STAGE_ROOM : 4;
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
     static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = 4 * NK;
-    static_assert(T_DQ + 2 * D <= 512, "TMEM budget");
-    static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static constexpr int OBUF = T_DQ + 2 * D <= TMEM_COLS ? 2 : 1;
+    static_assert(STAGES >= 2, "shared memory budget");
+    static_assert(T_DQ + OBUF * D <= TMEM_COLS, "TMEM budget");
+    static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
     static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
+    static_assert(NK % 32 == 0 && D % (32 * WGS) == 0, "32-column chunks");
 };
 
 struct QItem {
@@ -141,14 +147,14 @@ __device__ __forceinline__ QItem make_qitem(int idx, int n, int B)
     return it;
 }
 
-template <int D, int G>
-__global__ void __launch_bounds__(kTcThreads, 1)
+template <int D, int G, int NK_, int WGS_, int CTAS_>
+__global__ void __launch_bounds__(BqCfg<D, G, NK_, WGS_, CTAS_>::THREADS, CTAS_)
 bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                 const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
                 const BackwardArgs a)
 {
-    using C = BqCfg<D, G>;
-    constexpr int STAGES = C::STAGES, NK = C::NK;
+    using C = BqCfg<D, G, NK_, WGS_, CTAS_>;
+    constexpr int STAGES = C::STAGES, NK = C::NK, WGS = C::WGS, OBUF = C::OBUF;
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t q_full, q_empty, done_bar;
     __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
@@ -171,21 +177,21 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&ds_full[b], 128);   // the warpgroup that owns buffer b
+            mbar_init(&ds_full[b], 128);        // the warpgroup that owns buffer b
             mbar_init(&item_done[b], 1);
-            mbar_init(&o_free[b], 256);    // both warpgroups read half of the dQ row
+            mbar_init(&o_free[b], 128 * WGS);   // every warpgroup reads its share of the dQ row
         }
         fence_mbar_init();
         abort_s = 0;
     }
-    if (warp == 0) tmem_alloc<512>(&tmem_base_s);
+    if (warp == 0) tmem_alloc<C::TMEM_COLS>(&tmem_base_s);
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
     const uint32_t tmem = tmem_base_s;
     const unsigned long long limit = a.timeout_ns;
 
-    if (warp == kTcProducer) {
+    if (warp == C::PRODUCER) {
         if (lane == 0) {
             uint32_t gt = 0, ic = 0, q_issued = 0;
             bool ok = true;
@@ -238,7 +244,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 mbar_wait(&kv_full[s], (j / STAGES) & 1u, kGuardNs);
             }
         }
-    } else if (warp == kTcMma) {
+    } else if (warp == C::MMA) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NK, 0);
             constexpr uint32_t idesc_q = umma_idesc_bf16(C::M, D, 1);
@@ -261,7 +267,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             };
             for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
-                const uint32_t ob = ic & 1u;
+                const uint32_t ob = ic % OBUF;
                 if (!mbar_wait(&q_full, ic & 1u, limit) || !mbar_wait(&kv_full[gt % STAGES], (gt / STAGES) & 1u, limit)) {
                     ok = false;
                     break;
@@ -282,7 +288,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                         if (j + 2 == it.ntiles) umma_commit(&q_empty);  // the item's last read of Q and dO
                     }
                     if (!mbar_wait(&ds_full[g & 1u], (g >> 1) & 1u, limit) ||
-                        (j == 0 && ic >= 2 && !mbar_wait(&o_free[ob], ((ic >> 1) - 1) & 1u, limit))) {
+                        (j == 0 && ic >= OBUF && !mbar_wait(&o_free[ob], ((ic / OBUF) - 1) & 1u, limit))) {
                         ok = false;
                         break;
                     }
@@ -310,8 +316,8 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             }
         }
     } else {
-        // elementwise: two warpgroups; warpgroup wg takes the tiles g with g % 2 == wg (S/dP
-        // buffer wg), and thread r of either owns query row r (TMEM lane r)
+        // elementwise: with two warpgroups, warpgroup wg takes the tiles g with g % 2 == wg (S/dP
+        // buffer wg); one warpgroup takes them all. Thread r owns query row r (TMEM lane r)
         const int wg = warp >> 2, r = tid & 127;
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
@@ -321,7 +327,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         bool ok = true;
         for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
             const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
-            const uint32_t ob = ic & 1u;
+            const uint32_t ob = ic % OBUF;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
             const int t = it.t0 + rp, as = support_start(t, h);
             const bool valid = t < a.n;
@@ -329,7 +335,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             const float l2 = valid ? a.lse[row] * kLog2e : 0.f, dr = valid ? a.delta[row] : 0.f;
             for (int j = 0; j < it.ntiles; ++j) {
                 const uint32_t g = gt + j;
-                if (static_cast<int>(g & 1u) != wg) continue;
+                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -364,14 +370,14 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 mbar_arrive(&ds_full[g & 1u]);
             }
             if (!ok) break;
-            if (!warp_wait(&item_done[ob], (ic >> 1) & 1u, limit)) {
+            if (!warp_wait(&item_done[ob], (ic / OBUF) & 1u, limit)) {
                 ok = false;
                 break;
             }
             tmem_fence_after();
 #pragma unroll
-            for (int c = 0; c < D / 64; ++c) {  // this warpgroup's half of the row
-                const int col = wg * (D / 2) + 32 * c;
+            for (int c = 0; c < D / (32 * WGS); ++c) {  // this warpgroup's share of the row
+                const int col = wg * (D / WGS) + 32 * c;
                 uint32_t v[32];
                 tmem_ld32(lane_base + C::T_DQ + ob * D + col, v);
                 tmem_wait_ld();
@@ -395,7 +401,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
-    if (warp == 0) tmem_dealloc<512>(tmem);
+    if (warp == 0) tmem_dealloc<C::TMEM_COLS>(tmem);
 }
 
 // ------------------------------------------------------------- dK, dV ----
@@ -404,21 +410,29 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 // A operands of dV += P^T dO and dK += dS^T Q), then dV and dK. Per query tile the
 // producer warp also stages, for each of its 64 columns, the base-2 log-partition, D,
 // the position and its support start.
-template <int D, int G>
+// Shapes as for the dQ pass: NQ query rows per tile (64 or 32), WGS elementwise warpgroups,
+// CTAS CTAs per SM.
+template <int D, int G, int NQ_, int WGS_, int CTAS_>
 struct BkvCfg {
-    static constexpr int M = 128, NQ = 64, QT = NQ / G, BOXES = D / 64;
+    static constexpr int NQ = NQ_, WGS = WGS_, CTAS = CTAS_;
+    static constexpr int M = 128, QT = NQ / G, BOXES = D / 64;
+    static constexpr int THREADS = 128 * WGS + 64, PRODUCER = 4 * WGS, MMA = 4 * WGS + 1;
+    static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
     static constexpr int KBOX = M * 128, QBOX = NQ * 128;
     static constexpr int K_OFF = 0, V_OFF = BOXES * KBOX;
     static constexpr int RING_OFF = 2 * BOXES * KBOX;
     static constexpr int META = NQ * 16;                          // float4 per column
-    static constexpr int STAGE = 2 * BOXES * QBOX + META;         // Q, dO, metadata
-    static constexpr int STAGES = 3;
+    static constexpr int STAGE = (2 * BOXES * QBOX + META + 1023) / 1024 * 1024;  // Q, dO, metadata
+    static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - RING_OFF) / STAGE;
+    static constexpr int STAGE_MAX = CTAS == 1 ? 3 : 4;
+    static constexpr int STAGES = STAGE_ROOM < STAGE_MAX ? STAGE_ROOM : STAGE_MAX;
     static constexpr int SMEM = RING_OFF + STAGES * STAGE + 1024;
     static constexpr int T_ST = 0, T_DPT = 2 * NQ, T_DV = 4 * NQ, T_DK = 4 * NQ + D;
-    static_assert(T_DK + D <= 512, "TMEM budget");
-    static_assert(SMEM <= 227 * 1024, "shared memory budget");
+    static_assert(STAGES >= 2, "shared memory budget");
+    static_assert(T_DK + D <= TMEM_COLS, "TMEM budget");
+    static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
     static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
-    static_assert(STAGE % 1024 == 0, "stage boxes stay 1024-aligned");
+    static_assert(NQ % 32 == 0, "the producer warp stages NQ / 32 columns per lane");
 };
 
 struct KItem {
@@ -440,14 +454,15 @@ __device__ __forceinline__ KItem make_kitem(int idx, int n, int B)
     return it;
 }
 
-template <int D, int G>
-__global__ void __launch_bounds__(kTcThreads, 1)
+template <int D, int G, int NQ_, int WGS_, int CTAS_>
+__global__ void __launch_bounds__(BkvCfg<D, G, NQ_, WGS_, CTAS_>::THREADS, CTAS_)
 bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                  const __grid_constant__ CUtensorMap vmap, const __grid_constant__ CUtensorMap dmap,
                  const BackwardArgs a)
 {
-    using C = BkvCfg<D, G>;
-    constexpr int STAGES = C::STAGES, NQ = C::NQ;
+    using C = BkvCfg<D, G, NQ_, WGS_, CTAS_>;
+    constexpr int STAGES = C::STAGES, NQ = C::NQ, WGS = C::WGS;
+    constexpr int MV = NQ / 32;  // columns of metadata each producer lane stages per tile
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t kv_full, kv_empty, done_bar, item_done, o_free;
     __shared__ __align__(8) uint64_t qd_full[STAGES], qd_empty[STAGES];
@@ -463,7 +478,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         mbar_init(&kv_empty, 1);
         mbar_init(&done_bar, 1);
         mbar_init(&item_done, 1);
-        mbar_init(&o_free, 256);  // warpgroup 0 reads dV, warpgroup 1 dK
+        mbar_init(&o_free, 128 * WGS);  // with two warpgroups, 0 reads dV and 1 dK
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&qd_full[s], 1);
@@ -477,7 +492,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         fence_mbar_init();
         abort_s = 0;
     }
-    if (warp == 0) tmem_alloc<512>(&tmem_base_s);
+    if (warp == 0) tmem_alloc<C::TMEM_COLS>(&tmem_base_s);
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
@@ -485,7 +500,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
     const unsigned long long limit = a.timeout_ns;
     const int h = a.B >> 1;
 
-    if (warp == kTcProducer) {
+    if (warp == C::PRODUCER) {
         // the whole warp: lane 0 issues the copies, every lane stages two columns' metadata
         uint32_t gt = 0, ic = 0, kv_issued = 0;
         bool ok = true;
@@ -510,9 +525,9 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 const int t0 = it.tq0 + i * C::QT;
                 // this tile's per-column data: the loads are issued before the wait for a free
                 // stage, so their latency overlaps it
-                float4 mv[2];
+                float4 mv[MV];
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
+                for (int e = 0; e < MV; ++e) {
                     const int c = lane + 32 * e;
                     const int gi = c / C::QT, t = t0 + (c - gi * C::QT);
                     const bool valid = t < a.n;
@@ -531,7 +546,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
                 float4* meta = reinterpret_cast<float4*>(st + 2 * C::BOXES * C::QBOX);
 #pragma unroll
-                for (int e = 0; e < 2; ++e) {
+                for (int e = 0; e < MV; ++e) {
                     mv[e].x *= kLog2e;
                     meta[lane + 32 * e] = mv[e];
                 }
@@ -563,7 +578,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 mbar_wait(&qd_full[s], (j / STAGES) & 1u, kGuardNs);
             }
         }
-    } else if (warp == kTcMma) {
+    } else if (warp == C::MMA) {
         if (lane == 0) {
             constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NQ, 0);
             constexpr uint32_t idesc_o = umma_idesc_bf16(C::M, D, 1);
@@ -638,8 +653,8 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             }
         }
     } else {
-        // elementwise: two warpgroups; warpgroup wg takes the query tiles g with g % 2 == wg
-        // (S^T/dP^T buffer wg), and thread r of either owns key row r (TMEM lane r)
+        // elementwise: with two warpgroups, warpgroup wg takes the query tiles g with g % 2 == wg
+        // (S^T/dP^T buffer wg); one warpgroup takes them all. Thread r owns key row r (TMEM lane r)
         const int wg = warp >> 2, r = tid & 127;
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
@@ -651,7 +666,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             const bool kvalid = key < a.n;
             for (int i = 0; i < it.nqt; ++i) {
                 const uint32_t g = gt + i;
-                if (static_cast<int>(g & 1u) != wg) continue;
+                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -698,21 +713,25 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             }
             tmem_fence_after();
             const size_t row = static_cast<size_t>(it.pair) * a.n + (kvalid ? key : 0);
-            // warpgroup 0 writes dV, warpgroup 1 writes dK (scaled by 1/sqrt(d))
-            const float f = wg == 0 ? 1.f : sc;
-            float* dst_row = (wg == 0 ? a.dv : a.dk) + row * D;
-            const uint32_t src = lane_base + (wg == 0 ? C::T_DV : C::T_DK);
+            // dV, then dK scaled by 1/sqrt(d): with two warpgroups, 0 writes dV and 1 writes dK
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t v[32];
-                tmem_ld32(src + 32 * c, v);
-                tmem_wait_ld();
-                if (kvalid) {
-                    float4* dst = reinterpret_cast<float4*>(dst_row + 32 * c);
+            for (int o = 0; o < 2; ++o) {
+                if (WGS == 2 && o != wg) continue;
+                const float f = o == 0 ? 1.f : sc;
+                float* dst_row = (o == 0 ? a.dv : a.dk) + row * D;
+                const uint32_t src = lane_base + (o == 0 ? C::T_DV : C::T_DK);
 #pragma unroll
-                    for (int x = 0; x < 8; ++x)
-                        dst[x] = make_float4(__uint_as_float(v[4 * x]) * f, __uint_as_float(v[4 * x + 1]) * f,
-                                             __uint_as_float(v[4 * x + 2]) * f, __uint_as_float(v[4 * x + 3]) * f);
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(src + 32 * c, v);
+                    tmem_wait_ld();
+                    if (kvalid) {
+                        float4* dst = reinterpret_cast<float4*>(dst_row + 32 * c);
+#pragma unroll
+                        for (int x = 0; x < 8; ++x)
+                            dst[x] = make_float4(__uint_as_float(v[4 * x]) * f, __uint_as_float(v[4 * x + 1]) * f,
+                                                 __uint_as_float(v[4 * x + 2]) * f, __uint_as_float(v[4 * x + 3]) * f);
+                    }
                 }
             }
             tmem_fence_before();
@@ -727,23 +746,29 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
     tmem_fence_before();
     __syncthreads();
     tmem_fence_after();
-    if (warp == 0) tmem_dealloc<512>(tmem);
+    if (warp == 0) tmem_dealloc<C::TMEM_COLS>(tmem);
 }
 
-template <int D, int G>
-cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
+// One backward call: delta, the dK/dV pass (shape CK) and the dQ pass (shape CQ), each pass a
+// persistent grid of CTAS CTAs per SM where they fit.
+template <int D, typename CQ, typename CK>
+cudaError_t launch_bwd_shape(const BackwardArgs& a, cudaStream_t stream)
 {
-    using CQ = BqCfg<D, G>;
-    using CK = BkvCfg<D, G>;
+    constexpr int G = CQ::M / CQ::QT;
+    auto kv_kernel = bwd_kv_tc_kernel<D, G, CK::NQ, CK::WGS, CK::CTAS>;
+    auto q_kernel = bwd_q_tc_kernel<D, G, CQ::NK, CQ::WGS, CQ::CTAS>;
     static bool attr_set[64] = {};
+    static int kv_per_sm[64] = {}, q_per_sm[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
     if (dev < 64 && !attr_set[dev]) {
-        err = cudaFuncSetAttribute(bwd_kv_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, CK::SMEM);
+        err = cudaFuncSetAttribute(kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CK::SMEM);
         if (err != cudaSuccess) return err;
-        err = cudaFuncSetAttribute(bwd_q_tc_kernel<D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, CQ::SMEM);
+        err = cudaFuncSetAttribute(q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CQ::SMEM);
         if (err != cudaSuccess) return err;
+        kv_per_sm[dev] = resident_ctas(kv_kernel, CK::THREADS, CK::SMEM, CK::CTAS, dev);
+        q_per_sm[dev] = resident_ctas(q_kernel, CQ::THREADS, CQ::SMEM, CQ::CTAS, dev);
         attr_set[dev] = true;
     }
     int sms = 0;
@@ -751,8 +776,8 @@ cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
     if (err != cudaSuccess) return err;
     const unsigned long long qrows = static_cast<unsigned long long>(a.batch) * a.Hq * a.n;
     const unsigned long long krows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.n;
-    // dQ pass: Q/dO in items of 128 rows, K/V in tiles of 64; dK/dV pass: K/V in items of
-    // 128 keys, Q/dO in tiles of 64 rows
+    // dQ pass: Q/dO in items of 128 rows, K/V in tiles of NK; dK/dV pass: K/V in items of
+    // 128 keys, Q/dO in tiles of NQ rows
     CUtensorMap q1, d1, k1, v1, q2, d2, k2, v2;
     if (!rows_tensor_map(&q1, a.q, qrows, D, CQ::QT) || !rows_tensor_map(&d1, a.dout, qrows, D, CQ::QT) ||
         !rows_tensor_map(&k1, a.k, krows, D, CQ::NK) || !rows_tensor_map(&v1, a.v, krows, D, CQ::NK) ||
@@ -770,17 +795,37 @@ cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
         err = cudaGetLastError();
         if (err != cudaSuccess) return err;
     }
-    // one persistent CTA per SM for each pass (512 TMEM columns each)
     const long long kv_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + 127) / 128);
     const long long q_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + CQ::QT - 1) / CQ::QT);
     if (kv_items > 0x7fffffffLL || q_items > 0x7fffffffLL) return cudaErrorInvalidValue;
-    const int kv_grid = static_cast<int>(kv_items < sms ? kv_items : sms);
-    const int q_grid = static_cast<int>(q_items < sms ? q_items : sms);
-    bwd_kv_tc_kernel<D, G><<<kv_grid, kTcThreads, CK::SMEM, stream>>>(q2, k2, v2, d2, a);
+    const long long kv_slots = static_cast<long long>(sms) * (dev < 64 ? kv_per_sm[dev] : 1);
+    const long long q_slots = static_cast<long long>(sms) * (dev < 64 ? q_per_sm[dev] : 1);
+    const int kv_grid = static_cast<int>(kv_items < kv_slots ? kv_items : kv_slots);
+    const int q_grid = static_cast<int>(q_items < q_slots ? q_items : q_slots);
+    kv_kernel<<<kv_grid, CK::THREADS, CK::SMEM, stream>>>(q2, k2, v2, d2, a);
     err = cudaGetLastError();
     if (err != cudaSuccess) return err;
-    bwd_q_tc_kernel<D, G><<<q_grid, kTcThreads, CQ::SMEM, stream>>>(q1, k1, v1, d1, a);
+    q_kernel<<<q_grid, CQ::THREADS, CQ::SMEM, stream>>>(q1, k1, v1, d1, a);
     return cudaGetLastError();
+}
+
+// Shapes: long supports (B >= 512), and d = 128 or GQA group 8, run both passes with 64-row
+// tiles, two elementwise warpgroups and one CTA per SM (512 TMEM columns). Short supports at
+// d = 64 and G <= 4 run 32-row tiles, one elementwise warpgroup and two CTAs per SM (256
+// columns each), so one CTA's per-item latencies overlap the other's work. Build option
+// PBB_BWD_SHORT_SHAPE = 0 keeps every call on the long shape.
+#ifndef PBB_BWD_SHORT_SHAPE
+#define PBB_BWD_SHORT_SHAPE 1
+#endif
+
+template <int D, int G>
+cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
+{
+    if constexpr (D == 64 && G <= 4 && PBB_BWD_SHORT_SHAPE == 1) {
+        if (a.B < 512)
+            return launch_bwd_shape<D, BqCfg<D, G, 32, 1, 2>, BkvCfg<D, G, 32, 1, 2>>(a, stream);
+    }
+    return launch_bwd_shape<D, BqCfg<D, G, 64, 2, 1>, BkvCfg<D, G, 64, 2, 1>>(a, stream);
 }
 
 template <int D>

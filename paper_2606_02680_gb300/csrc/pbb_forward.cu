@@ -50,8 +50,6 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
-#include <algorithm>
-
 #include "pbb_device.cuh"
 #include "pbb_internal.h"
 
@@ -130,6 +128,14 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
           "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
         : "r"(taddr));
+}
+
+// max(a, b, c) in one instruction (three-input max.f32, sm_100 and later).
+__device__ __forceinline__ float fmax3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
 }
 
 // One work item: (sequence, KV head) pair, first position, keys and tiles.
@@ -386,16 +392,24 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 }
                 tmem_wait_ld();
                 const int key0 = it.lo + j * C::NK;
-                if ((key0 + C::NK - 1 > it.t0) || (key0 < it.a_max)) {  // tile crosses some row's bounds
+                if (key0 + C::NK - 1 > it.t0) {  // the diagonal: keys past some row's own position
+                    const int hi = t - key0;     // this row's last visible column
 #pragma unroll
-                    for (int c = 0; c < C::NK; ++c) {
-                        const int key = key0 + c;
-                        z[c] = (key >= as && key <= t) ? z[c] : -INFINITY;
-                    }
+                    for (int c = 0; c < C::NK; ++c) z[c] = c <= hi ? z[c] : -INFINITY;
                 }
-                float mx = -INFINITY;
+                if (key0 < it.a_max) {           // some row's support starts inside this tile
+                    const int lo = as - key0;    // this row's first visible column
 #pragma unroll
-                for (int c = 0; c < C::NK; ++c) mx = fmaxf(mx, z[c]);
+                    for (int c = 0; c < C::NK; ++c) z[c] = c >= lo ? z[c] : -INFINITY;
+                }
+                // row maximum: two independent chains of three-input maxima
+                float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < C::NK; c += 4) {
+                    mx0 = fmax3(mx0, z[c], z[c + 1]);
+                    mx1 = fmax3(mx1, z[c + 2], z[c + 3]);
+                }
+                float mx = fmaxf(mx0, mx1);
                 mx *= qscale;  // the scale is positive: the maximum of the scaled scores
                 // the reference maximum moves only when the row maximum exceeds it by 2^8:
                 // weights stay below 2^8, and O and l are rescaled together, so o = O / l is exact
@@ -439,15 +453,18 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                     m_used = m_new;
                 }
                 const float nbase = m_used == -INFINITY ? 0.f : -m_used;
-                // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row
+                // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row;
+                // the arguments and the row sum use packed two-lane FMA and add
+                const float2 sc2 = make_float2(qscale, qscale), nb2 = make_float2(nbase, nbase);
+                float2 lacc = make_float2(0.f, 0.f);
                 if constexpr (C::NK == 32) {
                     uint32_t pk[16];
 #pragma unroll
                     for (int x = 0; x < 16; ++x) {
-                        const float e0 = fast_exp2(fmaf(z[2 * x], qscale, nbase));
-                        const float e1 = fast_exp2(fmaf(z[2 * x + 1], qscale, nbase));
-                        l += e0 + e1;
-                        pk[x] = pack_bf16x2(e0, e1);
+                        const float2 arg = __ffma2_rn(make_float2(z[2 * x], z[2 * x + 1]), sc2, nb2);
+                        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                        lacc = __fadd2_rn(lacc, e);
+                        pk[x] = pack_bf16x2(e.x, e.y);
                     }
                     tmem_st16(s_col, pk);
                 } else {
@@ -456,14 +473,15 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         uint32_t pk[32];
 #pragma unroll
                         for (int x = 0; x < 32; ++x) {
-                            const float e0 = fast_exp2(fmaf(z[64 * c + 2 * x], qscale, nbase));
-                            const float e1 = fast_exp2(fmaf(z[64 * c + 2 * x + 1], qscale, nbase));
-                            l += e0 + e1;
-                            pk[x] = pack_bf16x2(e0, e1);
+                            const float2 arg = __ffma2_rn(make_float2(z[64 * c + 2 * x], z[64 * c + 2 * x + 1]), sc2, nb2);
+                            const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                            lacc = __fadd2_rn(lacc, e);
+                            pk[x] = pack_bf16x2(e.x, e.y);
                         }
                         tmem_st32(s_col + 32 * c, pk);
                     }
                 }
+                l += lacc.x + lacc.y;
                 tmem_wait_st();
                 tmem_fence_before();   // P is in TMEM and this row of S has been read
                 mbar_arrive(&p_full[g & 1u]);
@@ -611,31 +629,6 @@ __global__ void seq_ring_kernel(const unsigned char* __restrict__ k, const unsig
         *reinterpret_cast<uint4*>(k_ring + dst) = kv;
         *reinterpret_cast<uint4*>(v_ring + dst) = vv;
     }
-}
-
-// Resident CTAs per SM from the resources the SM checks (registers, shared memory, threads),
-// at most `want`. The runtime's occupancy calculator answers 1 for these tcgen05 kernels even
-// where two fit, and two did run together on GB300 (measured: the B = 128 forward 2,155 ->
-// 2,958 GB/s with two per SM); TMEM is shared by construction (TMEM_COLS x CTAS <= 512).
-template <typename K>
-int resident_ctas(K kernel, int threads, int dyn_smem, int want, int dev)
-{
-    cudaFuncAttributes fa{};
-    int smem_sm = 0, regs_sm = 0, reserved = 0, threads_sm = 0;
-    if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess ||
-        cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess)
-        return 1;
-    const int warps = (threads + 31) / 32;
-    const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;  // allocated per warp in 256-register units
-    const long long smem_cta = static_cast<long long>(dyn_smem) + fa.sharedSizeBytes + reserved;
-    int n = want;
-    n = std::min<long long>(n, smem_sm / smem_cta);
-    n = std::min(n, regs_sm / (regs_warp * warps));
-    n = std::min(n, threads_sm / threads);
-    return n < 1 ? 1 : n;
 }
 
 template <int D, int G, int NK, int WGS, int CTAS>

@@ -131,4 +131,29 @@ struct BackwardArgs {
 cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream);
 cudaError_t read_and_clear_backward_status(int* status);
 
+// Resident CTAs per SM of `kernel` from the resources the SM checks (registers, shared memory,
+// threads), at most `want`. The runtime's occupancy calculator answers 1 for the tcgen05
+// kernels even where two fit (and two did run together on GB300); the callers keep TMEM
+// shared by construction (columns per CTA x want <= 512).
+template <typename K>
+int resident_ctas(K kernel, int threads, int dyn_smem, int want, int dev)
+{
+    cudaFuncAttributes fa{};
+    int smem_sm = 0, regs_sm = 0, reserved = 0, threads_sm = 0;
+    if (cudaFuncGetAttributes(&fa, kernel) != cudaSuccess ||
+        cudaDeviceGetAttribute(&smem_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&regs_sm, cudaDevAttrMaxRegistersPerMultiprocessor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&threads_sm, cudaDevAttrMaxThreadsPerMultiProcessor, dev) != cudaSuccess)
+        return 1;
+    const int warps = (threads + 31) / 32;
+    const int regs_warp = (fa.numRegs * 32 + 255) / 256 * 256;  // allocated per warp in 256-register units
+    const long long smem_cta = static_cast<long long>(dyn_smem) + fa.sharedSizeBytes + reserved;
+    long long n = want;
+    if (smem_sm / smem_cta < n) n = smem_sm / smem_cta;
+    if (regs_warp > 0 && regs_sm / (regs_warp * warps) < n) n = regs_sm / (regs_warp * warps);
+    if (threads_sm / threads < n) n = threads_sm / threads;
+    return n < 1 ? 1 : static_cast<int>(n);
+}
+
 }  // namespace pbb
