@@ -78,6 +78,9 @@ def parse_args():
     ap.add_argument("--backward", action="store_true",
                     help="time the whole-sequence backward (dq, dk, dv) on the forward workloads")
     ap.add_argument("--fwd-workload", default="", help="one forward/backward workload (default: all)")
+    ap.add_argument("--kernel", choices=["auto", "cuda_cores", "tensor_cores"], default="auto",
+                    help="decode kernel choice (pbb_set_kernel); cuda_cores compares PBB and the window "
+                         "control on the same kernel")
     ap.add_argument("--graph", choices=["auto", "on", "off"], default="auto",
                     help="replay the timed steps as one CUDA graph (auto: when a step is under 100 us, "
                          "where host launch overhead would otherwise dominate)")
@@ -804,6 +807,7 @@ def run_ours(args):
     dev = torch.device("cuda", local if dist is not None else 0)
     torch.cuda.set_device(dev)
     pbb.set_chunk_keys(args.chunk)
+    pbb.set_kernel(args.kernel)
 
     if args.forward or args.backward:
         run_forward(args, dist, rank, world, dev)

@@ -104,6 +104,11 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
 // Items of 128 query rows (G heads x QT positions), key tiles of NK. TMEM: S and dP,
 // two buffers each (dS is written back over S as bf16 pairs, the A operand of
 // dQ += dS K), and one or two dQ accumulators alternating between items.
+// Columns of S and dP the elementwise threads load before each wait (32 or 64).
+#ifndef PBB_BWD_Q_QC
+#define PBB_BWD_Q_QC 64
+#endif
+
 // Shapes: NK keys per tile (64 or 32), WGS elementwise warpgroups (2 taking alternate
 // tiles, or 1), CTAS CTAs per SM sharing its 512 TMEM columns (1, or 2 with 256 each).
 template <int D, int G, int NK_, int WGS_, int CTAS_>
@@ -343,27 +348,39 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 tmem_fence_after();
                 const int key0 = it.lo + j * NK;
                 const bool edge = (key0 + NK - 1 > it.t0) || (key0 < it.a_max);
-                // 32 columns at a time: their dS (16 bf16-pair columns) goes over columns already read
+                // QC columns at a time (all their loads before one wait): their dS (QC/2
+                // bf16-pair columns) goes over columns already read
+                constexpr int QC = PBB_BWD_Q_QC < NK ? PBB_BWD_Q_QC : NK;
 #pragma unroll
-                for (int c = 0; c < NK / 32; ++c) {
-                    uint32_t v1[32], v2[32];
-                    tmem_ld32(lane_base + C::T_S + (g & 1u) * NK + 32 * c, v1);
-                    tmem_ld32(lane_base + C::T_DP + (g & 1u) * NK + 32 * c, v2);
+                for (int c = 0; c < NK / QC; ++c) {
+                    uint32_t v1[QC], v2[QC];
+#pragma unroll
+                    for (int h32 = 0; h32 < QC / 32; ++h32) {
+                        uint32_t* a1 = v1 + 32 * h32;
+                        uint32_t* a2 = v2 + 32 * h32;
+                        tmem_ld32(lane_base + C::T_S + (g & 1u) * NK + QC * c + 32 * h32,
+                                  *reinterpret_cast<uint32_t(*)[32]>(a1));
+                        tmem_ld32(lane_base + C::T_DP + (g & 1u) * NK + QC * c + 32 * h32,
+                                  *reinterpret_cast<uint32_t(*)[32]>(a2));
+                    }
                     tmem_wait_ld();
-                    uint32_t pk[16];
+                    uint32_t pk[QC / 2];
 #pragma unroll
-                    for (int x = 0; x < 16; ++x) {
+                    for (int x = 0; x < QC / 2; ++x) {
                         float e[2];
 #pragma unroll
                         for (int y = 0; y < 2; ++y) {
-                            const int key = key0 + 32 * c + 2 * x + y;
+                            const int key = key0 + QC * c + 2 * x + y;
                             const bool vis = valid && (!edge || (key >= as && key <= t));
                             const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -l2)) : 0.f;
                             e[y] = p * (__uint_as_float(v2[2 * x + y]) - dr);
                         }
                         pk[x] = pack_bf16x2(e[0], e[1]);
                     }
-                    tmem_st16(lane_base + C::T_S + (g & 1u) * NK + 16 * c, pk);
+#pragma unroll
+                    for (int h16 = 0; h16 < QC / 32; ++h16)
+                        tmem_st16(lane_base + C::T_S + (g & 1u) * NK + (QC / 2) * c + 16 * h16,
+                                  *reinterpret_cast<const uint32_t(*)[16]>(pk + 16 * h16));
                 }
                 tmem_wait_st();
                 tmem_fence_before();
@@ -412,6 +429,11 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 // the position and its support start.
 // Shapes as for the dQ pass: NQ query rows per tile (64 or 32), WGS elementwise warpgroups,
 // CTAS CTAs per SM.
+// Columns of S^T and dP^T the elementwise threads load before each wait (16 or 32): fewer waits
+// per tile against more registers.
+#ifndef PBB_BWD_KV_KC
+#define PBB_BWD_KV_KC 16
+#endif
 template <int D, int G, int NQ_, int WGS_, int CTAS_>
 struct BkvCfg {
     static constexpr int NQ = NQ_, WGS = WGS_, CTAS = CTAS_;
@@ -674,21 +696,27 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 tmem_fence_after();
                 const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
                                                                      2 * C::BOXES * C::QBOX);
-                // 16 columns at a time: their P^T and dS^T (8 bf16-pair columns each) go over
+                // KC columns at a time: their P^T and dS^T (KC/2 bf16-pair columns each) go over
                 // columns already read
+                constexpr int KC = PBB_BWD_KV_KC < NQ ? PBB_BWD_KV_KC : NQ;
 #pragma unroll
-                for (int c = 0; c < NQ / 16; ++c) {
-                    uint32_t v1[16], v2[16];
-                    tmem_ld16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, v1);
-                    tmem_ld16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, v2);
+                for (int c = 0; c < NQ / KC; ++c) {
+                    uint32_t v1[KC], v2[KC];
+                    if constexpr (KC == 32) {
+                        tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + KC * c, v1);
+                        tmem_ld32(lane_base + C::T_DPT + (g & 1u) * NQ + KC * c, v2);
+                    } else {
+                        tmem_ld16(lane_base + C::T_ST + (g & 1u) * NQ + KC * c, v1);
+                        tmem_ld16(lane_base + C::T_DPT + (g & 1u) * NQ + KC * c, v2);
+                    }
                     tmem_wait_ld();
-                    uint32_t pk[8], dk[8];
+                    uint32_t pk[KC / 2], dk[KC / 2];
 #pragma unroll
-                    for (int x = 0; x < 8; ++x) {
+                    for (int x = 0; x < KC / 2; ++x) {
                         float pe[2], de[2];
 #pragma unroll
                         for (int y = 0; y < 2; ++y) {
-                            const int cc = 16 * c + 2 * x + y;
+                            const int cc = KC * c + 2 * x + y;
                             const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc
                             const int t = __float_as_int(m.z), at = __float_as_int(m.w);
                             const bool vis = kvalid && key <= t && key >= at;
@@ -699,8 +727,13 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                         pk[x] = pack_bf16x2(pe[0], pe[1]);
                         dk[x] = pack_bf16x2(de[0], de[1]);
                     }
-                    tmem_st8(lane_base + C::T_ST + (g & 1u) * NQ + 8 * c, pk);
-                    tmem_st8(lane_base + C::T_DPT + (g & 1u) * NQ + 8 * c, dk);
+                    if constexpr (KC == 32) {
+                        tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, pk);
+                        tmem_st16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, dk);
+                    } else {
+                        tmem_st8(lane_base + C::T_ST + (g & 1u) * NQ + 8 * c, pk);
+                        tmem_st8(lane_base + C::T_DPT + (g & 1u) * NQ + 8 * c, dk);
+                    }
                 }
                 tmem_wait_st();
                 tmem_fence_before();

@@ -14,11 +14,12 @@
 // only grows with t, so the range covers every row), streamed in tiles of 64
 // keys; rows whose support starts later or ends earlier are masked in the tiles
 // that cross their bounds. No dense mask exists anywhere. Persistent CTAs (one
-// per SM with 128-key tiles for long supports, two per SM with 64-key tiles for
-// short ones; see FwdCfg) take items round-robin; query tiles of a head are
-// adjacent items, so CTAs running together share K/V tiles in L2.
+// per SM with 128-key tiles for long supports; for short ones three per SM with
+// 32-key tiles at d = 64, two with 64-key tiles at d = 128; see FwdCfg) take items
+// round-robin; query tiles of a head are adjacent items, so CTAs running together
+// share K/V tiles in L2.
 //
-// Roles (192 threads):
+// Roles (192 threads; 320 with two softmax warpgroups, whose warps come first):
 //   warp 4, one lane   TMA producer: Q of an item (one 2-D tensor copy per head
 //                      and 64-column box; one or two Q buffers), then K and V tiles
 //                      into a 2- to 4-stage ring (128-byte swizzle), all on
@@ -29,7 +30,9 @@
 //                      shared memory, into the item's TMEM output buffer (two
 //                      alternating between items, one for narrow tiles at d = 128);
 //                      each group is completed through tcgen05.commit;
-//   warps 0-3          softmax: thread r owns query row r (TMEM lane r). It reads
+//   warps 0-3          softmax: thread r owns query row r (TMEM lane r; with two
+//                      warpgroups each takes half of the row's columns and they
+//                      exchange partial maxima and sums). It reads
 //                      its row of S with tcgen05.ld, masks, keeps a running maximum
 //                      (base-2 domain, 1/sqrt(d) folded into one FFMA) that moves
 //                      only when it grows by more than 2^8 (then it rescales its O
@@ -63,7 +66,8 @@ constexpr unsigned long long kGuardNs = 2000000000ull;  // waits only a broken G
 
 // Shapes of the same kernel (chosen by the block size, see launch_fwd_shape):
 //   NK    keys per K/V tile (128, 64 or 32);
-//   WGS   softmax warpgroups (1, or 2 taking alternate tiles with an output buffer each);
+//   WGS   softmax warpgroups (1, or 2 sharing every tile: each takes half of the score
+//         columns and half of the output columns);
 //   CTAS  CTAs per SM: 1 owns all 512 TMEM columns, 2 to 4 share them (256 or 128 each) so
 //         one CTA's latencies overlap the others' work.
 // Long supports (many tiles per item) use one CTA per SM; short ones, where an item is one
@@ -84,17 +88,18 @@ struct FwdCfg {
     static constexpr int Q_OFF = 0;
     static constexpr int Q_BYTES = BOXES * QBOX;
     static constexpr int KV_OFF = Q_OFF + QBUF * Q_BYTES;
-    // the kernel's static shared memory (barriers; with two warpgroups the (m, l) exchange)
+    // the kernel's static shared memory (barriers; with two warpgroups the exchanges of the
+    // partial row maxima and sums, 2 x 2 x 128 floats each)
     static constexpr int STATIC_SMEM = WGS == 2 ? 4608 : 512;
     // K/V tiles in flight: as many as the shared memory of this shape holds, at most 4
     static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - STATIC_SMEM - 1024 - KV_OFF) / KV_STAGE;
     static constexpr int STAGES = STAGE_ROOM < 4 ? STAGE_ROOM : 4;
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;  // + alignment slack
-    // TMEM columns: S buffers at 0 and NK, output buffers from 2 NK: one per warpgroup with
-    // two warpgroups, else two alternating between items where they fit
+    // TMEM columns: S buffers at 0 and NK, output buffers from 2 NK: two alternating between
+    // items where they fit
     static constexpr int T_S = 0;
     static constexpr int T_O = 2 * NK;
-    static constexpr int OBUF = WGS == 2 ? 2 : (T_O + 2 * D <= TMEM_COLS ? 2 : 1);
+    static constexpr int OBUF = T_O + 2 * D <= TMEM_COLS ? 2 : 1;
     static constexpr int THREADS = 128 * WGS + 64;      // softmax warps, producer warp, MMA warp
     static constexpr int PRODUCER_WARP = 4 * WGS;
     static constexpr int MMA_WARP = 4 * WGS + 1;
@@ -168,11 +173,12 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
     constexpr int WGS = C::WGS;
     extern __shared__ unsigned char dsmem_raw[];
     constexpr int QBUF = C::QBUF;
-    __shared__ __align__(8) uint64_t q_full[QBUF], q_empty[QBUF], done_bar, merge_bar;
+    __shared__ __align__(8) uint64_t q_full[QBUF], q_empty[QBUF], done_bar, lsum_bar, xch_bar[2];
     __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
     __shared__ __align__(8) uint64_t s_full[2], p_full[2], pv_done[2], o_free[2];
-    // per item parity, (m, l) of each warpgroup's rows (used with two warpgroups only)
-    __shared__ float2 ml_s[WGS == 2 ? 2 : 1][WGS][WGS == 2 ? 128 : 1];
+    // with two warpgroups, by tile (item) parity: each warpgroup's partial row maxima (sums)
+    __shared__ float xch_s[WGS == 2 ? 2 : 1][WGS][WGS == 2 ? 128 : 1];
+    __shared__ float lsum_s[WGS == 2 ? 2 : 1][WGS][WGS == 2 ? 128 : 1];
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
@@ -187,7 +193,9 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             mbar_init(&q_empty[q], 1);
         }
         mbar_init(&done_bar, 1);
-        mbar_init(&merge_bar, 128 * WGS);
+        mbar_init(&lsum_bar, 128 * WGS);
+        mbar_init(&xch_bar[0], 128 * WGS);
+        mbar_init(&xch_bar[1], 128 * WGS);
 #pragma unroll
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&kv_full[s], 1);
@@ -196,7 +204,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&p_full[b], 128);         // the warpgroup that owns S buffer b
+            mbar_init(&p_full[b], 128 * WGS);   // every softmax thread, after writing its P
             mbar_init(&pv_done[b], 1);
             mbar_init(&o_free[b], 128 * WGS);   // every softmax thread, after reading the output
         }
@@ -315,24 +323,20 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         issue_s(g + 1);
                         if (j + 2 == it.ntiles) umma_commit(&q_empty[qb]);  // the item's last read of Q
                     }
-                    // before the item's first P.V: the output buffers are free once every softmax thread
-                    // has read the previous item's (both warpgroups' accumulators, or buffer ob)
+                    // before the item's first P.V: output buffer ob is free once every softmax thread
+                    // has read the item before that used it
                     bool free_ok = true;
-                    if (j == 0) {
-                        if (WGS == 2 && ic >= 1) free_ok = mbar_wait(&o_free[0], (ic - 1) & 1u, limit);
-                        if (WGS == 1 && ic >= C::OBUF) free_ok = mbar_wait(&o_free[ob], ((ic / C::OBUF) - 1) & 1u, limit);
-                    }
+                    if (j == 0 && ic >= C::OBUF) free_ok = mbar_wait(&o_free[ob], ((ic / C::OBUF) - 1) & 1u, limit);
                     if (!free_ok || !mbar_wait(&p_full[g & 1u], (g >> 1) & 1u, limit)) {
                         ok = false;
                         break;
                     }
                     tmem_fence_after();
-                    // O (+)= P_g V_g: P from TMEM (bf16 pairs over S buffer g % 2), V MN-major. With two
-                    // warpgroups, tile g accumulates into warpgroup (g % 2)'s buffer, starting at its first tile.
+                    // O (+)= P_g V_g: P from TMEM (bf16 pairs over S buffer g % 2), V MN-major
                     const uint32_t pt = tmem + C::T_S + (g & 1u) * C::NK;
                     const uint32_t vb = kv_base + (g % STAGES) * C::KV_STAGE + C::BOXES * C::KBOX;
-                    const uint32_t o_dst = tmem + C::T_O + (WGS == 2 ? (g & 1u) : ob) * D;
-                    const bool first = WGS == 2 ? j < 2 : j == 0;
+                    const uint32_t o_dst = tmem + C::T_O + ob * D;
+                    const bool first = j == 0;
 #pragma unroll
                     for (int kk = 0; kk < C::NK / 16; ++kk) {
                         const uint64_t bd = umma_desc_sw128(vb + kk * 2048, C::KBOX, 1024);
@@ -354,8 +358,13 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         }
     } else {
         // ================= softmax =================
-        // Warpgroup wg takes the tiles g with g % WGS == wg; thread r owns query row r
-        // (TMEM lane r) and keeps its own running maximum and sum for those tiles.
+        // Thread r of a warpgroup owns query row r (TMEM lane r). With two warpgroups both take
+        // every tile: warpgroup wg works on the score columns [wg NK/2, (wg+1) NK/2) and the
+        // output columns [wg d/2, (wg+1) d/2) of its rows. They exchange their partial row maxima
+        // through shared memory every tile, so both keep the same reference maximum, and their
+        // partial row sums at the item's end.
+        constexpr int HC = C::NK / WGS;  // score columns of this thread
+        constexpr int OC = D / WGS;      // output columns of this thread
         const int wg = warp >> 2, r = tid & 127;
         const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
@@ -366,51 +375,64 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
             const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
             const uint32_t ob = ic % C::OBUF;
-            const uint32_t o_col = C::T_O + (WGS == 2 ? static_cast<uint32_t>(wg) : ob) * D;
+            const uint32_t o_col = C::T_O + ob * D + wg * OC;  // this thread's output columns
             const int t = it.t0 + rp;               // this row's position
             const int as = support_start(t, h);     // and its support start
             float m_used = -INFINITY, l = 0.f;
-            int last = -1;                          // this warpgroup's last tile of the item
             for (int j = 0; j < it.ntiles; ++j) {
                 const uint32_t g = gt + j;
-                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
-                const bool has_prev = last >= 0;    // an earlier tile of this warpgroup holds O
-                last = j;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(0xffffffffu, abort_s != 0)) {
                     ok = false;
                     break;
                 }
                 tmem_fence_after();
-                const uint32_t s_col = lane_base + C::T_S + (g & 1u) * C::NK;
-                float z[C::NK];  // raw scores q.k of this row: every load issued, one wait
+                const uint32_t s_row = lane_base + C::T_S + (g & 1u) * C::NK;
+                float z[HC];  // raw scores q.k of this thread's columns: every load issued, one wait
+                if constexpr (HC >= 32) {
 #pragma unroll
-                for (int c = 0; c < C::NK / 32; ++c) {
-                    uint32_t v[32];
-                    tmem_ld32(s_col + 32 * c, v);
+                    for (int c = 0; c < HC / 32; ++c) {
+                        uint32_t v[32];
+                        tmem_ld32(s_row + wg * HC + 32 * c, v);
 #pragma unroll
-                    for (int x = 0; x < 32; ++x) z[32 * c + x] = __uint_as_float(v[x]);
+                        for (int x = 0; x < 32; ++x) z[32 * c + x] = __uint_as_float(v[x]);
+                    }
+                } else {
+                    uint32_t v[16];
+                    tmem_ld16(s_row + wg * HC, v);
+#pragma unroll
+                    for (int x = 0; x < 16; ++x) z[x] = __uint_as_float(v[x]);
                 }
                 tmem_wait_ld();
-                const int key0 = it.lo + j * C::NK;
-                if (key0 + C::NK - 1 > it.t0) {  // the diagonal: keys past some row's own position
-                    const int hi = t - key0;     // this row's last visible column
+                const int tile0 = it.lo + j * C::NK;   // first key of the tile
+                const int key0 = tile0 + wg * HC;      // first key of this thread's columns
+                if (tile0 + C::NK - 1 > it.t0) {       // the diagonal: keys past some row's own position
+                    const int hi = t - key0;           // this row's last visible column
 #pragma unroll
-                    for (int c = 0; c < C::NK; ++c) z[c] = c <= hi ? z[c] : -INFINITY;
+                    for (int c = 0; c < HC; ++c) z[c] = c <= hi ? z[c] : -INFINITY;
                 }
-                if (key0 < it.a_max) {           // some row's support starts inside this tile
-                    const int lo = as - key0;    // this row's first visible column
+                if (tile0 < it.a_max) {                // some row's support starts inside this tile
+                    const int lo = as - key0;          // this row's first visible column
 #pragma unroll
-                    for (int c = 0; c < C::NK; ++c) z[c] = c >= lo ? z[c] : -INFINITY;
+                    for (int c = 0; c < HC; ++c) z[c] = c >= lo ? z[c] : -INFINITY;
                 }
                 // row maximum: two independent chains of three-input maxima
                 float mx0 = -INFINITY, mx1 = -INFINITY;
 #pragma unroll
-                for (int c = 0; c < C::NK; c += 4) {
+                for (int c = 0; c < HC; c += 4) {
                     mx0 = fmax3(mx0, z[c], z[c + 1]);
                     mx1 = fmax3(mx1, z[c + 2], z[c + 3]);
                 }
-                float mx = fmaxf(mx0, mx1);
-                mx *= qscale;  // the scale is positive: the maximum of the scaled scores
+                float mx = fmaxf(mx0, mx1) * qscale;  // the scale is positive: the maximum of the scaled scores
+                if constexpr (WGS == 2) {
+                    // the other warpgroup's half of the row (both warps read both halves' maxima)
+                    xch_s[g & 1u][wg][r] = mx;
+                    mbar_arrive(&xch_bar[g & 1u]);
+                    if (!warp_wait(&xch_bar[g & 1u], (g >> 1) & 1u, limit)) {
+                        ok = false;
+                        break;
+                    }
+                    mx = fmaxf(mx, xch_s[g & 1u][wg ^ 1][r]);
+                }
                 // the reference maximum moves only when the row maximum exceeds it by 2^8:
                 // weights stay below 2^8, and O and l are rescaled together, so o = O / l is exact
                 const bool grow = mx > m_used + 8.f;
@@ -418,8 +440,8 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 if (__any_sync(0xffffffffu, grow)) {
                     const float f = grow ? (m_used == -INFINITY ? 0.f : fast_exp2(m_used - m_new)) : 1.f;
                     l *= f;
-                    if (has_prev) {  // O holds this warpgroup's earlier tiles once P.V of the previous one is complete
-                        const uint32_t gp = g - WGS;
+                    if (j > 0) {  // O holds the item's earlier tiles once P.V of the previous one is complete
+                        const uint32_t gp = g - 1;
                         if (!warp_wait(&pv_done[gp & 1u], (gp >> 1) & 1u, limit)) {
                             ok = false;
                             break;
@@ -427,7 +449,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         tmem_fence_after();
                         if constexpr (C::CTAS >= 3) {
 #pragma unroll
-                            for (int c = 0; c < D / 16; ++c) {
+                            for (int c = 0; c < OC / 16; ++c) {
                                 uint32_t v[16];
                                 const uint32_t ta = lane_base + o_col + 16 * c;
                                 tmem_ld16(ta, v);
@@ -438,7 +460,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                             }
                         } else {
 #pragma unroll
-                            for (int c = 0; c < D / 32; ++c) {
+                            for (int c = 0; c < OC / 32; ++c) {
                                 uint32_t v[32];
                                 const uint32_t ta = lane_base + o_col + 32 * c;
                                 tmem_ld32(ta, v);
@@ -453,11 +475,12 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                     m_used = m_new;
                 }
                 const float nbase = m_used == -INFINITY ? 0.f : -m_used;
-                // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row;
-                // the arguments and the row sum use packed two-lane FMA and add
+                // P = exp2(z * scale - m) as bf16 pairs over the first NK/2 columns of the S row (this
+                // thread's HC/2 of them, over columns read before the exchange); the arguments and the
+                // row sum use packed two-lane FMA and add
                 const float2 sc2 = make_float2(qscale, qscale), nb2 = make_float2(nbase, nbase);
                 float2 lacc = make_float2(0.f, 0.f);
-                if constexpr (C::NK == 32) {
+                if constexpr (HC == 32) {
                     uint32_t pk[16];
 #pragma unroll
                     for (int x = 0; x < 16; ++x) {
@@ -466,10 +489,10 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                         lacc = __fadd2_rn(lacc, e);
                         pk[x] = pack_bf16x2(e.x, e.y);
                     }
-                    tmem_st16(s_col, pk);
+                    tmem_st16(s_row + wg * 16, pk);
                 } else {
 #pragma unroll
-                    for (int c = 0; c < C::NK / 64; ++c) {
+                    for (int c = 0; c < HC / 64; ++c) {
                         uint32_t pk[32];
 #pragma unroll
                         for (int x = 0; x < 32; ++x) {
@@ -478,7 +501,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                             lacc = __fadd2_rn(lacc, e);
                             pk[x] = pack_bf16x2(e.x, e.y);
                         }
-                        tmem_st32(s_col + 32 * c, pk);
+                        tmem_st32(s_row + wg * (HC / 2) + 32 * c, pk);
                     }
                 }
                 l += lacc.x + lacc.y;
@@ -487,91 +510,49 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 mbar_arrive(&p_full[g & 1u]);
             }
             if (!ok) break;
-            // ---- epilogue: this warpgroup's last P.V, then o = O / l and lse
-            if (last >= 0) {
-                const uint32_t gl = gt + last;
+            // ---- epilogue: the item's last P.V, then o = O / l and lse
+            {
+                const uint32_t gl = gt + it.ntiles - 1;
                 if (!warp_wait(&pv_done[gl & 1u], (gl >> 1) & 1u, limit)) {
                     ok = false;
                     break;
                 }
             }
-            const bool valid = t < a.n;
-            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
-            const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + t;
-            float m_tot = m_used, l_tot = l, f0 = 1.f, f1 = 0.f, w0 = 1.f, w1 = 0.f;
-            int c0 = 0, c1 = D / 32;  // columns of the output this thread writes (32 at a time)
-            if (WGS == 2) {
-                // fuse the two warpgroups' partial results (Eq. lse): each writes half of the columns
-                ml_s[ic & 1u][wg][r] = make_float2(m_used, l);
-                mbar_arrive(&merge_bar);
-                if (!warp_wait(&merge_bar, ic & 1u, limit)) {
+            float l_tot = l;
+            if constexpr (WGS == 2) {  // the row sum is the two warpgroups' partial sums (same reference)
+                lsum_s[ic & 1u][wg][r] = l;
+                mbar_arrive(&lsum_bar);
+                if (!warp_wait(&lsum_bar, ic & 1u, limit)) {
                     ok = false;
                     break;
                 }
-                const float2 p0 = ml_s[ic & 1u][0][r], p1 = ml_s[ic & 1u][1][r];
-                m_tot = fmaxf(p0.x, p1.x);
-                f0 = p0.y > 0.f ? fast_exp2(p0.x - m_tot) : 0.f;
-                f1 = p1.y > 0.f ? fast_exp2(p1.x - m_tot) : 0.f;
-                l_tot = f0 * p0.y + f1 * p1.y;
-                w0 = p0.y > 0.f ? 1.f : 0.f;  // a warpgroup without tiles left its buffer stale: never read it
-                w1 = p1.y > 0.f ? 1.f : 0.f;
-                c0 = wg * (D / 64);
-                c1 = c0 + D / 64;
+                l_tot = lsum_s[ic & 1u][0][r] + lsum_s[ic & 1u][1][r];
             }
+            const bool valid = t < a.n;
+            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+            const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + t;
             tmem_fence_after();
             const float inv = l_tot > 0.f ? 1.f / l_tot : 0.f;
-            if constexpr (C::CTAS >= 3 && WGS == 1) {
-                // one output buffer, 16 columns at a time
+            constexpr int EC = C::CTAS >= 3 ? 16 : 32;  // output columns per TMEM load
 #pragma unroll
-                for (int c = 0; c < D / 16; ++c) {
-                    uint32_t v[16];
-                    tmem_ld16(lane_base + o_col + 16 * c, v);
-                    tmem_wait_ld();
-                    float o[16];
-#pragma unroll
-                    for (int x = 0; x < 16; ++x) o[x] = __uint_as_float(v[x]) * inv;
-                    if (valid) {
-                        if (a.out_f32) {
-                            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 16 * c);
-#pragma unroll
-                            for (int x = 0; x < 4; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
-                        } else {
-                            uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 16 * c);
-#pragma unroll
-                            for (int x = 0; x < 2; ++x) {
-                                uint4 pk;
-                                pk.x = pack_bf16x2(o[8 * x], o[8 * x + 1]);
-                                pk.y = pack_bf16x2(o[8 * x + 2], o[8 * x + 3]);
-                                pk.z = pack_bf16x2(o[8 * x + 4], o[8 * x + 5]);
-                                pk.w = pack_bf16x2(o[8 * x + 6], o[8 * x + 7]);
-                                dst[x] = pk;
-                            }
-                        }
-                    }
-                }
-                c1 = c0;  // done: skip the 32-column loop below
-            }
-            for (int c = c0; c < c1; ++c) {
-                uint32_t v[32], u[32];
-                tmem_ld32(lane_base + (WGS == 2 ? C::T_O : o_col) + 32 * c, v);
-                if (WGS == 2) tmem_ld32(lane_base + C::T_O + D + 32 * c, u);
+            for (int c = 0; c < OC / EC; ++c) {
+                uint32_t v[EC];
+                if constexpr (EC == 16) tmem_ld16(lane_base + o_col + EC * c, v);
+                else tmem_ld32(lane_base + o_col + EC * c, v);
                 tmem_wait_ld();
-                float o[32];
+                float o[EC];
 #pragma unroll
-                for (int x = 0; x < 32; ++x) {
-                    const float a0 = w0 > 0.f ? __uint_as_float(v[x]) * f0 : 0.f;
-                    const float a1 = (WGS == 2 && w1 > 0.f) ? __uint_as_float(u[x]) * f1 : 0.f;
-                    o[x] = (a0 + a1) * inv;
-                }
+                for (int x = 0; x < EC; ++x) o[x] = __uint_as_float(v[x]) * inv;
                 if (valid) {
+                    const size_t e0 = row * D + wg * OC + EC * c;  // first output element of the chunk
                     if (a.out_f32) {
-                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 32 * c);
+                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + e0);
 #pragma unroll
-                        for (int x = 0; x < 8; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
+                        for (int x = 0; x < EC / 4; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
                     } else {
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 32 * c);
+                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + e0);
 #pragma unroll
-                        for (int x = 0; x < 4; ++x) {
+                        for (int x = 0; x < EC / 8; ++x) {
                             uint4 pk;
                             pk.x = pack_bf16x2(o[8 * x], o[8 * x + 1]);
                             pk.y = pack_bf16x2(o[8 * x + 2], o[8 * x + 3]);
@@ -583,10 +564,10 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 }
             }
             tmem_fence_before();
-            mbar_arrive(&o_free[WGS == 2 ? 0u : ob]);  // the next item may overwrite the output buffer
+            mbar_arrive(&o_free[ob]);  // the next item may overwrite the output buffer
             if (valid && a.lse != nullptr && wg == 0) {
                 // ln sum exp(z) = (m + log2 l) ln 2, m the base-2 reference maximum
-                a.lse[row] = (m_tot + log2f(l_tot)) * 0.6931471805599453f;
+                a.lse[row] = (m_used + log2f(l_tot)) * 0.6931471805599453f;
             }
             gt += it.ntiles;
         }
@@ -678,7 +659,8 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* p
 }
 
 // The shape for long supports (B >= 512: an item spans several tiles) is a build-time choice:
-// 0 = 128-key tiles, one softmax warpgroup; 1 = 64-key tiles, two softmax warpgroups.
+// 0 = 128-key tiles, one softmax warpgroup; 1 = 128-key tiles, two softmax warpgroups sharing
+// every tile.
 #ifndef PBB_FWD_LONG_SHAPE
 #define PBB_FWD_LONG_SHAPE 0
 #endif
@@ -698,7 +680,7 @@ cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream, ForwardP
         return launch_fwd<D, G, 64, 1, 2>(a, stream, plan);
     }
 #if PBB_FWD_LONG_SHAPE == 1
-    return launch_fwd<D, G, 64, 2, 1>(a, stream, plan);
+    return launch_fwd<D, G, 128, 2, 1>(a, stream, plan);
 #else
     return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
 #endif
