@@ -582,6 +582,434 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
     if (warp == 0) tmem_dealloc<C::TMEM_COLS>(tmem);
 }
 
+// ------------------------------------------------------------ paired items ----
+// Long supports (B a multiple of 256, so every support starts on a 128-key tile boundary):
+// each CTA takes two consecutive query tiles (items A and B) of one (sequence, KV head), which
+// need the same keys except where B's support starts a half-block later, and streams their
+// union once. Warps 0-3 run the softmax of A, warps 4-7 that of B, each over its own S and
+// output in TMEM, so one warpgroup's softmax runs while the tensor pipe works on the other's
+// products, and the issuing thread queues four groups (S and P.V of both) per K/V tile. The
+// softmax warpgroups take 216 registers a thread (setmaxnreg) from the warpgroup of the producer,
+// MMA and spare warps.
+template <int D, int G>
+struct PairCfg {
+    static constexpr int NK = 128, M = 128, QT = M / G, BOXES = D / 64;
+    static constexpr int QBOX = M * 128, KBOX = NK * 128;
+    static constexpr int Q_BYTES = BOXES * QBOX;           // one item's Q
+    static constexpr int TILE = BOXES * KBOX;              // one K or V tile
+    static constexpr int Q_OFF = 0;                        // Q of A, then Q of B
+    static constexpr int K_OFF = 2 * Q_BYTES;
+    static constexpr int STATIC_SMEM = 1024;
+    static constexpr int BUDGET = 228 * 1024 - 1024 - STATIC_SMEM - 1024;
+    static constexpr int TILE_ROOM = (BUDGET - K_OFF) / TILE;
+    static constexpr int KSTAGES = (TILE_ROOM + 1) / 2 < 4 ? (TILE_ROOM + 1) / 2 : 4;
+    static constexpr int VSTAGES = TILE_ROOM - KSTAGES < 4 ? TILE_ROOM - KSTAGES : 4;
+    static constexpr int V_OFF = K_OFF + KSTAGES * TILE;
+    static constexpr int SMEM = V_OFF + VSTAGES * TILE + 1024;
+    static constexpr int T_S = 0, T_O = 2 * NK;            // S of A and B, then the outputs
+    // warps 0-7 softmax, 8 Q and K producer, 9 V producer, 10 MMA issuer, 11 spare; at launch
+    // 168 registers each (12 warps, three per SMSP). setmaxnreg is uniform per warpgroup and
+    // the register file is split between the SMSPs, so each SMSP's three warps (two softmax,
+    // one of warpgroup 2) must fit their launch share: 2 x 216 + 72 = 3 x 168, and over the
+    // CTA 256 x 216 + 128 x 72 = 384 x 168
+    static constexpr int THREADS = 384, W_QK = 8, W_V = 9, W_MMA = 10;
+    static constexpr int LAUNCH_REGS = 168;
+    static constexpr int SOFTMAX_REGS = 216, OTHER_REGS = 72;
+    static_assert(2 * SOFTMAX_REGS + OTHER_REGS <= 3 * LAUNCH_REGS, "register split per SMSP");
+    static_assert(256 * SOFTMAX_REGS + 128 * OTHER_REGS <= THREADS * LAUNCH_REGS, "register split");
+    static_assert(T_O + 2 * D <= 512, "TMEM budget");
+    static_assert(KSTAGES >= 2 && VSTAGES >= 2, "shared memory budget");
+    static_assert(SMEM + STATIC_SMEM + 1024 <= 228 * 1024, "shared memory budget");
+    static_assert(QT % 8 == 0, "a head's Q rows must start on a swizzle atom (8 rows)");
+};
+
+// Two items of one (sequence, KV head): A = query tile 2s, B = 2s + 1 (absent past the end).
+// Their keys are [loA, end], in tiles of NK from loA; A takes tiles [0, ntA), B [jB0, nt).
+struct PItem {
+    int pair, t0, tlA, tlB, loA, loB, amaxA, amaxB, nt, ntA, jB0;
+    bool hasB;
+};
+
+template <int QT, int NK>
+__device__ __forceinline__ PItem make_pitem(int sidx, int n, int B)
+{
+    const int nq = (n + QT - 1) / QT;
+    const int nsp = (nq + 1) / 2;
+    PItem it;
+    it.pair = sidx / nsp;
+    it.t0 = (sidx - it.pair * nsp) * 2 * QT;
+    it.tlA = min(it.t0 + QT, n) - 1;
+    it.hasB = it.t0 + QT < n;
+    it.tlB = it.hasB ? min(it.t0 + 2 * QT, n) - 1 : it.tlA;
+    const int h = B >> 1;
+    it.loA = support_start(it.t0, h);
+    it.amaxA = support_start(it.tlA, h);
+    it.loB = it.hasB ? support_start(it.t0 + QT, h) : it.loA;
+    it.amaxB = support_start(it.tlB, h);
+    it.nt = (it.tlB - it.loA + NK) / NK;
+    it.ntA = (it.tlA - it.loA + NK) / NK;
+    it.jB0 = (it.loB - it.loA) / NK;  // exact: supports start on multiples of h, h a multiple of NK
+    return it;
+}
+
+// setmaxnreg is a warpgroup instruction: the four warps of a warpgroup execute the same one.
+__device__ __forceinline__ void regs_inc_softmax() { asm volatile("setmaxnreg.inc.sync.aligned.u32 216;\n" ::: "memory"); }
+__device__ __forceinline__ void regs_dec_others() { asm volatile("setmaxnreg.dec.sync.aligned.u32 72;\n" ::: "memory"); }
+
+template <int D, int G>
+__global__ void __launch_bounds__(PairCfg<D, G>::THREADS, 1)
+forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                    const __grid_constant__ CUtensorMap vmap, const ForwardArgs a)
+{
+    using C = PairCfg<D, G>;
+    constexpr int NK = C::NK, KS = C::KSTAGES, VS = C::VSTAGES;
+    extern __shared__ unsigned char dsmem_raw[];
+    __shared__ __align__(8) uint64_t q_full[2], q_empty[2], done_bar;
+    __shared__ __align__(8) uint64_t k_full[KS], k_empty[KS], v_full[VS], v_empty[VS];
+    __shared__ __align__(8) uint64_t s_full[2], p_full[2], pv_last[2], o_free[2];  // per item (A, B)
+    __shared__ uint32_t tmem_base_s;
+    __shared__ volatile int abort_s;
+    unsigned char* dsmem = reinterpret_cast<unsigned char*>(
+        (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nq = (a.n + C::QT - 1) / C::QT;
+    const int n_sitems = a.batch * a.Hkv * ((nq + 1) / 2);
+
+    if (tid == 0) {
+#pragma unroll
+        for (int x = 0; x < 2; ++x) {
+            mbar_init(&q_full[x], 1);
+            mbar_init(&q_empty[x], 1);
+            mbar_init(&s_full[x], 1);
+            mbar_init(&p_full[x], 128);
+            mbar_init(&pv_last[x], 1);
+            mbar_init(&o_free[x], 128);
+        }
+        mbar_init(&done_bar, 1);
+#pragma unroll
+        for (int s = 0; s < KS; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+        }
+#pragma unroll
+        for (int s = 0; s < VS; ++s) {
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
+        }
+        fence_mbar_init();
+        abort_s = 0;
+    }
+    if (warp == 0) tmem_alloc<512>(&tmem_base_s);
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    const uint32_t tmem = tmem_base_s;
+    const unsigned long long limit = a.timeout_ns;
+    // warpgroup 2 (producers, MMA issuer, spare) gives registers to warpgroups 0 and 1 (softmax):
+    // each warpgroup's four warps run one setmaxnreg, at one place, ahead of its roles
+    if (warp >= 8) {
+        regs_dec_others();
+        if (warp == C::W_QK || warp == C::W_V) {
+            // ================= TMA producers: Q of both items and K tiles; V tiles =================
+            const bool qk = warp == C::W_QK;
+            if (lane == 0) {
+                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(qk ? &kmap : &vmap)) : "memory");
+                if (qk) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
+                uint32_t gt = 0, issued = 0, ic[2] = {0, 0}, q_issued[2] = {0, 0};
+                bool ok = true;
+                for (int sidx = blockIdx.x; ok && sidx < n_sitems; sidx += gridDim.x) {
+                    const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
+                    const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+                    if (qk) {
+                        for (int x = 0; x < (it.hasB ? 2 : 1); ++x) {
+                            if (ic[x] >= 1 && !mbar_wait(&q_empty[x], (ic[x] - 1) & 1u, limit)) {
+                                ok = false;
+                                break;
+                            }
+                            mbar_expect_tx(&q_full[x], static_cast<uint32_t>(C::Q_BYTES));
+                            const int qrow0 = (b * a.Hq + kvh * G) * a.n + it.t0 + x * C::QT;
+                            unsigned char* qdst = dsmem + C::Q_OFF + x * C::Q_BYTES;
+#pragma unroll
+                            for (int gi = 0; gi < G; ++gi)
+#pragma unroll
+                                for (int bx = 0; bx < C::BOXES; ++bx)
+                                    tma_load_2d(qdst + bx * C::QBOX + gi * C::QT * 128, &qmap, bx * 64,
+                                                qrow0 + gi * a.n, &q_full[x]);
+                            ++ic[x];
+                            q_issued[x] = ic[x];
+                        }
+                        if (!ok) break;
+                    }
+                    const int row0 = it.pair * a.n + it.loA;
+                    for (int j = 0; j < it.nt; ++j, ++gt) {
+                        if (abort_s) {
+                            ok = false;
+                            break;
+                        }
+                        const int ns = qk ? KS : VS;
+                        const int s = gt % ns;
+                        uint64_t* fullb = qk ? &k_full[s] : &v_full[s];
+                        uint64_t* emptyb = qk ? &k_empty[s] : &v_empty[s];
+                        if (gt >= static_cast<uint32_t>(ns) && !mbar_wait(emptyb, ((gt / ns) - 1) & 1u, limit)) {
+                            ok = false;
+                            break;
+                        }
+                        unsigned char* st = dsmem + (qk ? C::K_OFF : C::V_OFF) + s * C::TILE;
+                        mbar_expect_tx(fullb, static_cast<uint32_t>(C::TILE));
+#pragma unroll
+                        for (int bx = 0; bx < C::BOXES; ++bx)
+                            tma_load_2d(st + bx * C::KBOX, qk ? &kmap : &vmap, bx * 64, row0 + j * NK, fullb);
+                        issued = gt + 1;
+                    }
+                }
+                if (!ok) {
+                    abort_s = 1;
+                    atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+                }
+                // drain the copies still in flight before shared memory goes away
+                for (int x = 0; x < 2; ++x)
+                    if (q_issued[x] > 0) mbar_wait(&q_full[x], (q_issued[x] - 1) & 1u, kGuardNs);
+                const uint32_t ns = qk ? KS : VS;
+                for (uint32_t s = 0; s < ns && s < issued; ++s) {
+                    const uint32_t jj = s + ns * ((issued - 1 - s) / ns);
+                    mbar_wait(qk ? &k_full[s] : &v_full[s], (jj / ns) & 1u, kGuardNs);
+                }
+            }
+        } else if (warp == C::W_MMA) {
+            // ================= MMA issuer =================
+            if (lane == 0) {
+                constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NK, 0);
+                constexpr uint32_t idesc_o = umma_idesc_bf16(C::M, D, 1);
+                const uint32_t q_base = smem_addr(dsmem + C::Q_OFF);
+                const uint32_t k_base = smem_addr(dsmem + C::K_OFF), v_base = smem_addr(dsmem + C::V_OFF);
+                uint32_t gk = 0, gv = 0;                  // K and V tiles consumed
+                uint32_t ic[2] = {0, 0}, gp[2] = {0, 0};  // items and P tiles consumed, per item slot
+                bool ok = true, issued_any = false;
+                for (int sidx = blockIdx.x; ok && sidx < n_sitems; sidx += gridDim.x) {
+                    const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
+                    const int jb[2] = {0, it.hasB ? it.jB0 : it.nt};  // first and end tile of each item
+                    const int je[2] = {it.ntA, it.nt};
+                    for (int j = 0; ok && j <= it.nt; ++j) {
+                        bool need_k = false, need_v = false;
+#pragma unroll
+                        for (int x = 0; x < 2; ++x) {
+                            need_k |= j >= jb[x] && j < je[x];
+                            need_v |= j >= jb[x] + 1 && j - 1 < je[x];
+                        }
+                        if ((need_k && !mbar_wait(&k_full[gk % KS], (gk / KS) & 1u, limit)) ||
+                            (need_v && !mbar_wait(&v_full[gv % VS], (gv / VS) & 1u, limit))) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t kb = k_base + (gk % KS) * C::TILE, vb = v_base + (gv % VS) * C::TILE;
+#pragma unroll
+                        for (int x = 0; x < 2; ++x) {
+                            const bool pv = j >= jb[x] + 1 && j - 1 < je[x];  // P_x V of tile j - 1
+                            const bool sk = j >= jb[x] && j < je[x];          // S_x of tile j
+                            if (pv) {
+                                const bool first = j - 1 == jb[x];
+                                if ((first && ic[x] >= 1 && !mbar_wait(&o_free[x], (ic[x] - 1) & 1u, limit)) ||
+                                    !mbar_wait(&p_full[x], gp[x] & 1u, limit)) {
+                                    ok = false;
+                                    break;
+                                }
+                                tmem_fence_after();
+                                const uint32_t pt = tmem + C::T_S + x * NK, o_dst = tmem + C::T_O + x * D;
+#pragma unroll
+                                for (int kk = 0; kk < NK / 16; ++kk) {
+                                    const uint64_t bd = umma_desc_sw128(vb + kk * 2048, C::KBOX, 1024);
+                                    umma_bf16_tmem_a(o_dst, pt + 8 * kk, bd, idesc_o, (!first || kk > 0) ? 1u : 0u);
+                                }
+                                ++gp[x];
+                            }
+                            if (sk) {
+                                if (j == jb[x]) {
+                                    if (!mbar_wait(&q_full[x], ic[x] & 1u, limit)) {
+                                        ok = false;
+                                        break;
+                                    }
+                                    tmem_fence_after();
+                                }
+                                const uint32_t qb = q_base + x * C::Q_BYTES;
+#pragma unroll
+                                for (int kk = 0; kk < D / 16; ++kk) {
+                                    const uint32_t off = (kk & 3) * 32;
+                                    const uint64_t ad = umma_desc_sw128(qb + (kk >> 2) * C::QBOX + off, 16, 1024);
+                                    const uint64_t bd = umma_desc_sw128(kb + (kk >> 2) * C::KBOX + off, 16, 1024);
+                                    umma_bf16(tmem + C::T_S + x * NK, ad, bd, idesc_s, kk > 0 ? 1u : 0u);
+                                }
+                                umma_commit(&s_full[x]);      // S_x of tile j, and P_x V of tile j - 1
+                                if (j == je[x] - 1) umma_commit(&q_empty[x]);
+                            } else if (pv) {
+                                umma_commit(&pv_last[x]);     // the item's last P.V
+                                ++ic[x];
+                            }
+                            issued_any = true;
+                        }
+                        if (!ok) break;
+                        if (need_k) umma_commit(&k_empty[gk++ % KS]);
+                        if (need_v) umma_commit(&v_empty[gv++ % VS]);
+                    }
+                }
+                if (!ok) {
+                    abort_s = 1;
+                    atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+                }
+                if (issued_any) {  // every MMA complete before TMEM is released
+                    umma_commit(&done_bar);
+                    mbar_wait(&done_bar, 0u, kGuardNs);
+                }
+            }
+        }  // warp 11 has no role: its registers went to the softmax warpgroups
+    } else {
+        regs_inc_softmax();
+        // ================= softmax of item x (warps 4x .. 4x + 3) =================
+        const int x = warp >> 2, r = tid & 127;
+        const uint32_t lane_base = tmem + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+        const uint32_t s_row = lane_base + C::T_S + x * NK, o_row = lane_base + C::T_O + x * D;
+        const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
+        const int h = a.B >> 1;
+        const int gi = r / C::QT, rp = r - gi * C::QT;
+        uint32_t g = 0, ic = 0;  // this item slot's tiles and items so far
+        bool ok = true;
+        for (int sidx = blockIdx.x; ok && sidx < n_sitems; sidx += gridDim.x) {
+            const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
+            if (x == 1 && !it.hasB) continue;
+            const int t0 = it.t0 + x * C::QT, tl = x == 0 ? it.tlA : it.tlB;
+            const int amax = x == 0 ? it.amaxA : it.amaxB;
+            const int jb = x == 0 ? 0 : it.jB0, je = x == 0 ? it.ntA : it.nt;
+            const int t = t0 + rp;                  // this row's position
+            const int as = support_start(t, h);     // and its support start
+            float m_used = -INFINITY, l = 0.f;
+            for (int j = jb; j < je; ++j, ++g) {
+                if (!warp_wait(&s_full[x], g & 1u, limit) || __any_sync(0xffffffffu, abort_s != 0)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
+                float z[NK];  // raw scores q.k of this row: every load issued, one wait
+#pragma unroll
+                for (int c = 0; c < NK / 32; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(s_row + 32 * c, v);
+#pragma unroll
+                    for (int y = 0; y < 32; ++y) z[32 * c + y] = __uint_as_float(v[y]);
+                }
+                tmem_wait_ld();
+                const int key0 = it.loA + j * NK;
+                if (key0 + NK - 1 > t0) {  // the diagonal: keys past some row's own position
+                    const int hi = t - key0;
+#pragma unroll
+                    for (int c = 0; c < NK; ++c) z[c] = c <= hi ? z[c] : -INFINITY;
+                }
+                if (key0 < amax) {         // some row's support starts inside this tile
+                    const int lo = as - key0;
+#pragma unroll
+                    for (int c = 0; c < NK; ++c) z[c] = c >= lo ? z[c] : -INFINITY;
+                }
+                float mx0 = -INFINITY, mx1 = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < NK; c += 4) {
+                    mx0 = fmax3(mx0, z[c], z[c + 1]);
+                    mx1 = fmax3(mx1, z[c + 2], z[c + 3]);
+                }
+                const float mx = fmaxf(mx0, mx1) * qscale;
+                // the reference maximum moves only when the row maximum exceeds it by 2^8
+                // (see forward_kernel); s_full of this tile also covers P.V of the previous one,
+                // so O holds every earlier tile when it is rescaled
+                const bool grow = mx > m_used + 8.f;
+                const float m_new = grow ? mx : m_used;
+                if (__any_sync(0xffffffffu, grow)) {
+                    const float f = grow ? (m_used == -INFINITY ? 0.f : fast_exp2(m_used - m_new)) : 1.f;
+                    l *= f;
+                    if (j > jb) {
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint32_t v[32];
+                            tmem_ld32(o_row + 32 * c, v);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int y = 0; y < 32; ++y) v[y] = __float_as_uint(__uint_as_float(v[y]) * f);
+                            tmem_st32(o_row + 32 * c, v);
+                        }
+                        tmem_wait_st();
+                    }
+                    m_used = m_new;
+                }
+                const float nbase = m_used == -INFINITY ? 0.f : -m_used;
+                const float2 sc2 = make_float2(qscale, qscale), nb2 = make_float2(nbase, nbase);
+                float2 lacc = make_float2(0.f, 0.f);
+#pragma unroll
+                for (int c = 0; c < NK / 64; ++c) {
+                    uint32_t pk[32];
+#pragma unroll
+                    for (int y = 0; y < 32; ++y) {
+                        const float2 arg = __ffma2_rn(make_float2(z[64 * c + 2 * y], z[64 * c + 2 * y + 1]), sc2, nb2);
+                        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                        lacc = __fadd2_rn(lacc, e);
+                        pk[y] = pack_bf16x2(e.x, e.y);
+                    }
+                    tmem_st32(s_row + 32 * c, pk);
+                }
+                l += lacc.x + lacc.y;
+                tmem_wait_st();
+                tmem_fence_before();
+                mbar_arrive(&p_full[x]);
+            }
+            if (!ok) break;
+            // ---- epilogue: the item's last P.V, then o = O / l and lse
+            if (!warp_wait(&pv_last[x], ic & 1u, limit)) {
+                ok = false;
+                break;
+            }
+            tmem_fence_after();
+            const bool valid = t < a.n && t <= tl;
+            const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
+            const size_t row = static_cast<size_t>(b * a.Hq + kvh * G + gi) * a.n + t;
+            const float inv = l > 0.f ? 1.f / l : 0.f;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t v[32];
+                tmem_ld32(o_row + 32 * c, v);
+                tmem_wait_ld();
+                float o[32];
+#pragma unroll
+                for (int y = 0; y < 32; ++y) o[y] = __uint_as_float(v[y]) * inv;
+                if (valid) {
+                    if (a.out_f32) {
+                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 32 * c);
+#pragma unroll
+                        for (int y = 0; y < 8; ++y) dst[y] = make_float4(o[4 * y], o[4 * y + 1], o[4 * y + 2], o[4 * y + 3]);
+                    } else {
+                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 32 * c);
+#pragma unroll
+                        for (int y = 0; y < 4; ++y) {
+                            uint4 pk;
+                            pk.x = pack_bf16x2(o[8 * y], o[8 * y + 1]);
+                            pk.y = pack_bf16x2(o[8 * y + 2], o[8 * y + 3]);
+                            pk.z = pack_bf16x2(o[8 * y + 4], o[8 * y + 5]);
+                            pk.w = pack_bf16x2(o[8 * y + 6], o[8 * y + 7]);
+                            dst[y] = pk;
+                        }
+                    }
+                }
+            }
+            tmem_fence_before();
+            mbar_arrive(&o_free[x]);  // the next item of this slot may overwrite the output
+            if (valid && a.lse != nullptr) a.lse[row] = (m_used + log2f(l)) * 0.6931471805599453f;
+            ++ic;
+        }
+        if (!ok) {
+            abort_s = 1;
+            atomicCAS(&g_fwd_status, kDevOk, kDevTimeout);
+        }
+    }
+    tmem_fence_before();
+    __syncthreads();
+    tmem_fence_after();
+    if (warp == 0) tmem_dealloc<512>(tmem);
+}
+
 // Sequence -> ring: slot j of each (sequence, KV head) ring gets the position
 // s in [n-B, n-1] with s = j (mod B), zeros where s < 0 (Appendix F.1).
 __global__ void seq_ring_kernel(const unsigned char* __restrict__ k, const unsigned char* __restrict__ v,
@@ -671,6 +1099,58 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* p
 #define PBB_FWD_SHORT_SHAPE 1
 #endif
 
+// Long supports with B a multiple of 256 run the paired-item kernel (build option
+// PBB_FWD_PAIR = 0 keeps them on forward_kernel's one-item shape).
+#ifndef PBB_FWD_PAIR
+#define PBB_FWD_PAIR 1
+#endif
+
+template <int D, int G>
+cudaError_t launch_fwd_pair(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
+{
+    using C = PairCfg<D, G>;
+    auto kernel = forward_pair_kernel<D, G>;
+    static int state[64] = {};  // 0 unknown, 1 usable, -1 the register split does not hold
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    if (dev < 64 && state[dev] == 0) {
+        err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (err != cudaSuccess) return err;
+        // setmaxnreg moves registers within the block's launch allocation: the split is only
+        // valid if the kernel launches with LAUNCH_REGS per thread (else an increase would wait
+        // forever), so anything else falls back to the one-item kernel
+        cudaFuncAttributes fa{};
+        err = cudaFuncGetAttributes(&fa, kernel);
+        if (err != cudaSuccess) return err;
+        state[dev] = fa.numRegs == C::LAUNCH_REGS ? 1 : -1;
+    }
+    if (dev >= 64 || state[dev] != 1) return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
+    const long long nq = (a.n + C::QT - 1) / C::QT;
+    const long long sitems = static_cast<long long>(a.batch) * a.Hkv * ((nq + 1) / 2);
+    if (sitems < 1) {
+        if (plan != nullptr) *plan = ForwardPlan{C::NK, 0, 0};
+        return cudaSuccess;
+    }
+    if (sitems > 0x7fffffffLL) return cudaErrorInvalidValue;
+    int sms = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    const int grid = static_cast<int>(sitems < sms ? sitems : sms);
+    if (plan != nullptr) {
+        *plan = ForwardPlan{C::NK, 1, grid};
+        return cudaSuccess;
+    }
+    CUtensorMap qmap, kmap, vmap;
+    const unsigned long long qrows = static_cast<unsigned long long>(a.batch) * a.Hq * a.n;
+    const unsigned long long krows = static_cast<unsigned long long>(a.batch) * a.Hkv * a.n;
+    if (!rows_tensor_map(&qmap, a.q, qrows, D, C::QT) || !rows_tensor_map(&kmap, a.k, krows, D, C::NK) ||
+        !rows_tensor_map(&vmap, a.v, krows, D, C::NK))
+        return cudaErrorInvalidValue;
+    kernel<<<grid, C::THREADS, C::SMEM, stream>>>(qmap, kmap, vmap, a);
+    return cudaGetLastError();
+}
+
 // Blocks below this run the short-support shapes (measured at B = 4096, d = 128: the 64-key,
 // two-CTA shape reaches 963 TFLOP/s against 1,186 for the 128-key, one-CTA shape).
 #ifndef PBB_FWD_SHORT_MAX_B
@@ -688,6 +1168,7 @@ cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream, ForwardP
 #if PBB_FWD_LONG_SHAPE == 1
     return launch_fwd<D, G, 128, 2, 1>(a, stream, plan);
 #else
+    if (PBB_FWD_PAIR && (a.B / 2) % 128 == 0) return launch_fwd_pair<D, G>(a, stream, plan);
     return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
 #endif
 }

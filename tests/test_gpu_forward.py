@@ -83,6 +83,17 @@ def test_block_sizes(B):
     run_full(w)
 
 
+@pytest.mark.parametrize("group", [1, 2, 4, 8])
+@pytest.mark.parametrize("d", [64, 128])
+def test_long_blocks_groups_and_dims(group, d):
+    """Long supports (B = 512, the 128-key-tile shape) for every group and head size;
+    n = 777 gives an odd number of 128-row query tiles per (sequence, KV head) and a ragged
+    last tile."""
+    w = inputs.SequenceWorkload(f"fwd_long_g{group}_d{d}", batch=2, Hq=2 * group, Hkv=2, d=d, B=512,
+                                n=777, seed=90 + group + d)
+    run_full(w)
+
+
 @pytest.mark.parametrize("n", [1, 7, 8, 63, 64, 65])
 def test_short_sequences(n):
     w = inputs.SequenceWorkload(f"fwd_n{n}", batch=3, Hq=4, Hkv=1, d=64, B=32, n=n, seed=70 + n)
