@@ -108,9 +108,13 @@ int sm_count(int dev)
 // whole, while splitting only the last round's supports paid for long supports
 // (see below); a positive pbb_set_chunk_keys override splits every support
 // into chunks of that many keys.
+#ifndef PBB_MIN_CHUNK_KB
+#define PBB_MIN_CHUNK_KB 64
+#endif
+
 int min_split_keys(int d, int elem, int tile)
 {
-    constexpr int kMinChunkBytes = 64 * 1024;
+    constexpr int kMinChunkBytes = PBB_MIN_CHUNK_KB * 1024;
     const int k = kMinChunkBytes / (2 * d * elem);
     return k < tile ? tile : k;
 }

@@ -377,12 +377,21 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
                 }
                 ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
                 if (ok) {
-                    for (int e = ctid; e < a.gq * D; e += NC * 32) {  // the real query heads
+                    // four consecutive elements (one head: D is a multiple of 4) per thread, as
+                    // 16-byte loads of every chunk's partial (partials and out are 16-byte aligned)
+                    for (int e = 4 * ctid; e < a.gq * D; e += 4 * NC * 32) {  // the real query heads
                         const int j = e / D;
-                        float O = 0.f;
+                        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll 8
-                        for (int c = 0; c < mt.nch; ++c) O = fmaf(__ldcg(po + c * G * D + e), wgt[c * G + j], O);
-                        out_g[e] = O;
+                        for (int c = 0; c < mt.nch; ++c) {
+                            const float4 p = __ldcg(reinterpret_cast<const float4*>(po + c * G * D + e));
+                            const float w = wgt[c * G + j];
+                            O.x = fmaf(p.x, w, O.x);
+                            O.y = fmaf(p.y, w, O.y);
+                            O.z = fmaf(p.z, w, O.z);
+                            O.w = fmaf(p.w, w, O.w);
+                        }
+                        *reinterpret_cast<float4*>(out_g + e) = O;
                     }
                 }
             } else {
