@@ -109,6 +109,16 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
 #define PBB_BWD_Q_QC 64
 #endif
 
+// In the one-CTA shapes, tiles with no masked entry take a packed path (1) or the masked one
+// (0): PBB_BWD_Q_INNER for the dQ pass, PBB_BWD_KV_INNER for the dK/dV pass. The two-CTA
+// shapes always take the masked path (measured faster there).
+#ifndef PBB_BWD_Q_INNER
+#define PBB_BWD_Q_INNER 1
+#endif
+#ifndef PBB_BWD_KV_INNER
+#define PBB_BWD_KV_INNER 1
+#endif
+
 // Shapes: NK keys per tile (64 or 32), WGS elementwise warpgroups (2 taking alternate
 // tiles, or 1), CTAS CTAs per SM sharing its 512 TMEM columns (1, or 2 with 256 each).
 template <int D, int G, int NK_, int WGS_, int CTAS_>
@@ -126,6 +136,7 @@ struct BqCfg {
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
     static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = 4 * NK;
     static constexpr int OBUF = T_DQ + 2 * D <= TMEM_COLS ? 2 : 1;
+    static constexpr bool INNER = PBB_BWD_Q_INNER && CTAS == 1;
     static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_DQ + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
@@ -348,6 +359,8 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 tmem_fence_after();
                 const int key0 = it.lo + j * NK;
                 const bool edge = (key0 + NK - 1 > it.t0) || (key0 < it.a_max);
+                // every key of the tile in every valid row's support: the packed path
+                const bool inner = C::INNER && !edge && __all_sync(kFull, valid);
                 // QC columns at a time (all their loads before one wait): their dS (QC/2
                 // bf16-pair columns) goes over columns already read
                 constexpr int QC = PBB_BWD_Q_QC < NK ? PBB_BWD_Q_QC : NK;
@@ -365,17 +378,31 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     }
                     tmem_wait_ld();
                     uint32_t pk[QC / 2];
+                    if (inner) {
 #pragma unroll
-                    for (int x = 0; x < QC / 2; ++x) {
-                        float e[2];
-#pragma unroll
-                        for (int y = 0; y < 2; ++y) {
-                            const int key = key0 + QC * c + 2 * x + y;
-                            const bool vis = valid && (!edge || (key >= as && key <= t));
-                            const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -l2)) : 0.f;
-                            e[y] = p * (__uint_as_float(v2[2 * x + y]) - dr);
+                        for (int x = 0; x < QC / 2; ++x) {
+                            const float2 arg = __ffma2_rn(
+                                make_float2(__uint_as_float(v1[2 * x]), __uint_as_float(v1[2 * x + 1])),
+                                make_float2(sc2, sc2), make_float2(-l2, -l2));
+                            const float2 e = __fmul2_rn(
+                                make_float2(fast_exp2(arg.x), fast_exp2(arg.y)),
+                                __fadd2_rn(make_float2(__uint_as_float(v2[2 * x]), __uint_as_float(v2[2 * x + 1])),
+                                           make_float2(-dr, -dr)));
+                            pk[x] = pack_bf16x2(e.x, e.y);
                         }
-                        pk[x] = pack_bf16x2(e[0], e[1]);
+                    } else {
+#pragma unroll
+                        for (int x = 0; x < QC / 2; ++x) {
+                            float e[2];
+#pragma unroll
+                            for (int y = 0; y < 2; ++y) {
+                                const int key = key0 + QC * c + 2 * x + y;
+                                const bool vis = valid && (!edge || (key >= as && key <= t));
+                                const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -l2)) : 0.f;
+                                e[y] = p * (__uint_as_float(v2[2 * x + y]) - dr);
+                            }
+                            pk[x] = pack_bf16x2(e[0], e[1]);
+                        }
                     }
 #pragma unroll
                     for (int h16 = 0; h16 < QC / 32; ++h16)
@@ -443,7 +470,10 @@ struct BkvCfg {
     static constexpr int KBOX = M * 128, QBOX = NQ * 128;
     static constexpr int K_OFF = 0, V_OFF = BOXES * KBOX;
     static constexpr int RING_OFF = 2 * BOXES * KBOX;
-    static constexpr int META = NQ * 16;                          // float4 per column
+    // per column (lse2, D, t, a(t)) as a float4 (one load per entry on the masked path); with
+    // the packed path, (-lse2, -D) again as a float2 array (one load per column pair)
+    static constexpr bool INNER = PBB_BWD_KV_INNER && CTAS == 1;
+    static constexpr int META = NQ * (INNER ? 24 : 16);
     static constexpr int STAGE = (2 * BOXES * QBOX + META + 1023) / 1024 * 1024;  // Q, dO, metadata
     static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - RING_OFF) / STAGE;
     static constexpr int STAGE_MAX = CTAS == 1 ? 3 : 4;
@@ -571,6 +601,8 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 for (int e = 0; e < MV; ++e) {
                     mv[e].x *= kLog2e;
                     meta[lane + 32 * e] = mv[e];
+                    if constexpr (C::INNER)
+                        reinterpret_cast<float2*>(meta + NQ)[lane + 32 * e] = make_float2(-mv[e].x, -mv[e].y);
                 }
                 __threadfence_block();
                 __syncwarp();
@@ -696,6 +728,12 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 tmem_fence_after();
                 const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
                                                                      2 * C::BOXES * C::QBOX);
+                const float2* meta_ld = reinterpret_cast<const float2*>(meta + NQ);
+                // a tile whose every query sees every key of the warp's rows needs no mask: the
+                // packed path (bit-identical arithmetic, half the instructions)
+                const int tq0 = it.tq0 + i * C::QT, tql = tq0 + C::QT - 1;
+                const bool inner =
+                    C::INNER && __all_sync(kFull, kvalid && tql < a.n && key <= tq0 && key >= support_start(tql, h));
                 // KC columns at a time: their P^T and dS^T (KC/2 bf16-pair columns each) go over
                 // columns already read
                 constexpr int KC = PBB_BWD_KV_KC < NQ ? PBB_BWD_KV_KC : NQ;
@@ -711,21 +749,38 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     }
                     tmem_wait_ld();
                     uint32_t pk[KC / 2], dk[KC / 2];
+                    if (inner) {
 #pragma unroll
-                    for (int x = 0; x < KC / 2; ++x) {
-                        float pe[2], de[2];
-#pragma unroll
-                        for (int y = 0; y < 2; ++y) {
-                            const int cc = KC * c + 2 * x + y;
-                            const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc
-                            const int t = __float_as_int(m.z), at = __float_as_int(m.w);
-                            const bool vis = kvalid && key <= t && key >= at;
-                            const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -m.x)) : 0.f;
-                            pe[y] = p;
-                            de[y] = p * (__uint_as_float(v2[2 * x + y]) - m.y);
+                        for (int x = 0; x < KC / 2; ++x) {
+                            // (-lse2, -D) of columns cc and cc + 1
+                            const float4 m = *reinterpret_cast<const float4*>(meta_ld + KC * c + 2 * x);
+                            const float2 arg = __ffma2_rn(
+                                make_float2(__uint_as_float(v1[2 * x]), __uint_as_float(v1[2 * x + 1])),
+                                make_float2(sc2, sc2), make_float2(m.x, m.z));
+                            const float2 p = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                            const float2 ds = __fmul2_rn(
+                                p, __fadd2_rn(make_float2(__uint_as_float(v2[2 * x]), __uint_as_float(v2[2 * x + 1])),
+                                              make_float2(m.y, m.w)));
+                            pk[x] = pack_bf16x2(p.x, p.y);
+                            dk[x] = pack_bf16x2(ds.x, ds.y);
                         }
-                        pk[x] = pack_bf16x2(pe[0], pe[1]);
-                        dk[x] = pack_bf16x2(de[0], de[1]);
+                    } else {
+#pragma unroll
+                        for (int x = 0; x < KC / 2; ++x) {
+                            float pe[2], de[2];
+#pragma unroll
+                            for (int y = 0; y < 2; ++y) {
+                                const int cc = KC * c + 2 * x + y;
+                                const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc; t = -1 past n
+                                const int t = __float_as_int(m.z), at = __float_as_int(m.w);
+                                const bool vis = kvalid && key <= t && key >= at;
+                                const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -m.x)) : 0.f;
+                                pe[y] = p;
+                                de[y] = p * (__uint_as_float(v2[2 * x + y]) - m.y);
+                            }
+                            pk[x] = pack_bf16x2(pe[0], pe[1]);
+                            dk[x] = pack_bf16x2(de[0], de[1]);
+                        }
                     }
                     if constexpr (KC == 32) {
                         tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, pk);
