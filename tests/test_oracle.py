@@ -579,3 +579,24 @@ def test_backward_zero_query_closed_form(oracle_mod):
         a = interval_start(t, b)
         ref[a:t + 1] += w[0, 0, t] / (t + 1 - a)
     assert np.allclose(dv[0, 0], ref, atol=1e-13)
+
+
+def test_backward_bridge_gradients_reach_exactly_the_bridge_keys(oracle_mod):
+    """The paper's multi-block gradient check at B = 8 (h = 4): upstream gradient only on the
+    bridge queries 8..11 of block 1. By Eq. (pbb) they attend to the previous block's second
+    half (keys 4..7, the bridge) and to their own block up to themselves, so dk and dv are
+    nonzero on keys 4..11 (each of them, for generic inputs) and exactly zero on keys 0..3 and
+    12 onward; dq is zero outside rows 8..11."""
+    rng = np.random.default_rng(43)
+    b, n, d = 8, 24, 4
+    q = rng.standard_normal((1, 2, n, d))
+    k = rng.standard_normal((1, 1, n, d))
+    v = rng.standard_normal((1, 1, n, d))
+    w = np.zeros((1, 2, n, d))
+    w[:, :, 8:12] = rng.standard_normal((1, 2, 4, d))
+    dq, dk, dv = oracle_mod.backward(q, k, v, w, b)
+    for g in (dk, dv):
+        assert np.all(np.abs(g[0, 0, 4:12]).max(axis=-1) > 0)
+        assert np.abs(g[0, 0, :4]).max() == 0.0 and np.abs(g[0, 0, 12:]).max() == 0.0
+    assert np.abs(dq[0, :, :8]).max() == 0.0 and np.abs(dq[0, :, 12:]).max() == 0.0
+    assert np.all(np.abs(dq[0, :, 8:12]).max(axis=-1) > 0)
