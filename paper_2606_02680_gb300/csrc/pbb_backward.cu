@@ -845,20 +845,21 @@ cudaError_t launch_bwd_shape(const BackwardArgs& a, cudaStream_t stream)
     constexpr int G = CQ::M / CQ::QT;
     auto kv_kernel = bwd_kv_tc_kernel<D, G, CK::NQ, CK::WGS, CK::CTAS>;
     auto q_kernel = bwd_q_tc_kernel<D, G, CQ::NK, CQ::WGS, CQ::CTAS>;
-    static bool attr_set[64] = {};
-    static int kv_per_sm[64] = {}, q_per_sm[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    if (dev < 64 && !attr_set[dev]) {
+    // each pass's shared-memory opt-in and its resident CTAs per SM, once per device
+    static std::atomic<int> kv_cache[kMaxCachedDevices] = {}, q_cache[kMaxCachedDevices] = {};
+    const int kv_per_sm = cached_per_device(kv_cache, dev, [&] {
         err = cudaFuncSetAttribute(kv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CK::SMEM);
-        if (err != cudaSuccess) return err;
+        return err == cudaSuccess ? resident_ctas(kv_kernel, CK::THREADS, CK::SMEM, CK::CTAS, dev) : 0;
+    });
+    if (kv_per_sm < 1) return err;
+    const int q_per_sm = cached_per_device(q_cache, dev, [&] {
         err = cudaFuncSetAttribute(q_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, CQ::SMEM);
-        if (err != cudaSuccess) return err;
-        kv_per_sm[dev] = resident_ctas(kv_kernel, CK::THREADS, CK::SMEM, CK::CTAS, dev);
-        q_per_sm[dev] = resident_ctas(q_kernel, CQ::THREADS, CQ::SMEM, CQ::CTAS, dev);
-        attr_set[dev] = true;
-    }
+        return err == cudaSuccess ? resident_ctas(q_kernel, CQ::THREADS, CQ::SMEM, CQ::CTAS, dev) : 0;
+    });
+    if (q_per_sm < 1) return err;
     int sms = 0;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
@@ -886,8 +887,8 @@ cudaError_t launch_bwd_shape(const BackwardArgs& a, cudaStream_t stream)
     const long long kv_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + 127) / 128);
     const long long q_items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + CQ::QT - 1) / CQ::QT);
     if (kv_items > 0x7fffffffLL || q_items > 0x7fffffffLL) return cudaErrorInvalidValue;
-    const long long kv_slots = static_cast<long long>(sms) * (dev < 64 ? kv_per_sm[dev] : 1);
-    const long long q_slots = static_cast<long long>(sms) * (dev < 64 ? q_per_sm[dev] : 1);
+    const long long kv_slots = static_cast<long long>(sms) * kv_per_sm;
+    const long long q_slots = static_cast<long long>(sms) * q_per_sm;
     const int kv_grid = static_cast<int>(kv_items < kv_slots ? kv_items : kv_slots);
     const int q_grid = static_cast<int>(q_items < q_slots ? q_items : q_slots);
     kv_kernel<<<kv_grid, CK::THREADS, CK::SMEM, stream>>>(q2, k2, v2, d2, a);

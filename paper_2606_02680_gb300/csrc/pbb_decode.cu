@@ -1245,31 +1245,32 @@ __global__ void advance_kernel(int32_t* pos, int batch)
 template <int ELEM, int D, int G>
 cudaError_t ensure_smem_attr()
 {
-    static bool attr_set[64] = {};
+    static std::atomic<int> done[kMaxCachedDevices] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    if (dev < 64 && attr_set[dev]) return cudaSuccess;
-    err = cudaFuncSetAttribute(decode_kernel<ELEM, D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               Cfg<ELEM, D, G>::SMEM);
-    if (err == cudaSuccess && dev < 64) attr_set[dev] = true;
-    return err;
+    const int ok = cached_per_device(done, dev, [&] {
+        err = cudaFuncSetAttribute(decode_kernel<ELEM, D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   Cfg<ELEM, D, G>::SMEM);
+        return err == cudaSuccess ? 1 : 0;
+    });
+    return ok > 0 ? cudaSuccess : err;
 }
 
 template <int ELEM, int D, int G>
 int occupancy_t()
 {
-    static int cache[64] = {};
+    static std::atomic<int> cache[kMaxCachedDevices] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev < 64 && cache[dev] > 0) return cache[dev];
-    int n = 0;
-    if (ensure_smem_attr<ELEM, D, G>() != cudaSuccess) return 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<ELEM, D, G>, kThreads,
-                                                      Cfg<ELEM, D, G>::SMEM) != cudaSuccess)
-        return 0;
-    if (dev < 64) cache[dev] = n;
-    return n;
+    return cached_per_device(cache, dev, [] {
+        int n = 0;
+        if (ensure_smem_attr<ELEM, D, G>() != cudaSuccess) return 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel<ELEM, D, G>, kThreads,
+                                                          Cfg<ELEM, D, G>::SMEM) != cudaSuccess)
+            return 0;
+        return n;
+    });
 }
 
 template <int ELEM, int D, int G>
@@ -1294,17 +1295,16 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t stream)
 
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder()
 {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    static bool tried = false;
-    if (!tried) {
-        tried = true;
+    // looked up once: one thread initialises a function-local static while any others wait
+    static const PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
         void* p = nullptr;
         cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
                 cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }
+            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        return static_cast<PFN_cuTensorMapEncodeTiled_v12000>(nullptr);
+    }();
     return fn;
 }
 
@@ -1347,31 +1347,30 @@ bool ring_tensor_map(CUtensorMap* map, const void* ring, unsigned long long rows
 template <int D>
 int occupancy_tc()
 {
-    static int cache[64] = {};
+    static std::atomic<int> cache[kMaxCachedDevices] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev < 64 && cache[dev] > 0) return cache[dev];
-    if (cudaFuncSetAttribute(decode_kernel_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<D>::SMEM) !=
-        cudaSuccess)
-        return 0;
-    int n = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel_tc<D>, kTcThreads, TcCfg<D>::SMEM) !=
-        cudaSuccess)
-        return 0;
-    if (dev < 64) cache[dev] = n;
-    return n;
+    return cached_per_device(cache, dev, [] {
+        if (cudaFuncSetAttribute(decode_kernel_tc<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 TcCfg<D>::SMEM) != cudaSuccess)
+            return 0;
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, decode_kernel_tc<D>, kTcThreads, TcCfg<D>::SMEM) !=
+            cudaSuccess)
+            return 0;
+        return n;
+    });
 }
 
 int device_sms()
 {
-    static int cache[64] = {};
+    static std::atomic<int> cache[kMaxCachedDevices] = {};
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-    if (dev < 64 && cache[dev] > 0) return cache[dev];
-    int n = 0;
-    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    if (dev < 64) cache[dev] = n;
-    return n;
+    return cached_per_device(cache, dev, [dev] {
+        int n = 0;
+        return cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess ? n : 0;
+    });
 }
 
 // Padded groups (4 and 6 heads in the 8-column score tile) take the tensor cores only when the

@@ -1045,15 +1045,17 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* p
 {
     using C = FwdCfg<D, G, NK, WGS, CTAS>;
     auto kernel = forward_kernel<D, G, NK, WGS, CTAS>;
-    static bool attr_set[64] = {};
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    if (dev < 64 && !attr_set[dev]) {
+    // the shared-memory opt-in, then persistent CTAs: C::CTAS per SM where they fit, never more
+    // than TMEM holds
+    static std::atomic<int> per_sm_cache[kMaxCachedDevices] = {};
+    const int per_sm = cached_per_device(per_sm_cache, dev, [&] {
         err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (err != cudaSuccess) return err;
-        attr_set[dev] = true;
-    }
+        return err == cudaSuccess ? resident_ctas(kernel, C::THREADS, C::SMEM, C::CTAS, dev) : 0;
+    });
+    if (per_sm < 1) return err;
     const long long items = static_cast<long long>(a.batch) * a.Hkv * ((a.n + C::QT - 1) / C::QT);
     if (items < 1) {
         if (plan != nullptr) *plan = ForwardPlan{NK, 0, 0};
@@ -1063,13 +1065,6 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* p
     int sms = 0;
     err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err != cudaSuccess) return err;
-    // persistent CTAs: C::CTAS per SM where they fit, never more than TMEM holds
-    static int per_sm_cache[64] = {};
-    int per_sm = dev < 64 ? per_sm_cache[dev] : 0;
-    if (per_sm == 0) {
-        per_sm = resident_ctas(kernel, C::THREADS, C::SMEM, C::CTAS, dev);
-        if (dev < 64) per_sm_cache[dev] = per_sm;
-    }
     const long long slots = static_cast<long long>(sms) * per_sm;
     const int grid = static_cast<int>(items < slots ? items : slots);
     if (plan != nullptr) {
@@ -1110,22 +1105,24 @@ cudaError_t launch_fwd_pair(const ForwardArgs& a, cudaStream_t stream, ForwardPl
 {
     using C = PairCfg<D, G>;
     auto kernel = forward_pair_kernel<D, G>;
-    static int state[64] = {};  // 0 unknown, 1 usable, -1 the register split does not hold
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    if (dev < 64 && state[dev] == 0) {
+    // 1: usable; 2: the register split does not hold. setmaxnreg moves registers within the
+    // block's launch allocation, so the split is only valid if the kernel launches with
+    // LAUNCH_REGS per thread (else an increase would wait forever); anything else falls back to
+    // the one-item kernel
+    static std::atomic<int> state[kMaxCachedDevices] = {};
+    const int usable = cached_per_device(state, dev, [&] {
         err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (err != cudaSuccess) return err;
-        // setmaxnreg moves registers within the block's launch allocation: the split is only
-        // valid if the kernel launches with LAUNCH_REGS per thread (else an increase would wait
-        // forever), so anything else falls back to the one-item kernel
+        if (err != cudaSuccess) return 0;
         cudaFuncAttributes fa{};
         err = cudaFuncGetAttributes(&fa, kernel);
-        if (err != cudaSuccess) return err;
-        state[dev] = fa.numRegs == C::LAUNCH_REGS ? 1 : -1;
-    }
-    if (dev >= 64 || state[dev] != 1) return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
+        if (err != cudaSuccess) return 0;
+        return fa.numRegs == C::LAUNCH_REGS ? 1 : 2;
+    });
+    if (usable < 1) return err;
+    if (usable != 1) return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
     const long long nq = (a.n + C::QT - 1) / C::QT;
     const long long sitems = static_cast<long long>(a.batch) * a.Hkv * ((nq + 1) / 2);
     if (sitems < 1) {

@@ -7,6 +7,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include <atomic>
+
 namespace pbb {
 
 // Device status codes (the word read by pbb_get_device_status).
@@ -130,6 +132,27 @@ struct BackwardArgs {
 };
 cudaError_t launch_backward(const BackwardArgs& a, cudaStream_t stream);
 cudaError_t read_and_clear_backward_status(int* status);
+
+// Per-device values worked out once: a kernel's shared-memory opt-in with its resident CTAs, the
+// SM count. Slot `dev` of `cache` holds 0 until a call on that device stores the positive result
+// of `make`; a result of 0 or less (a failed query) is returned without being stored. Host
+// threads calling at once may each run `make`, which only issues idempotent queries and
+// settings; the release store publishes those with the value. Devices at or past
+// kMaxCachedDevices run `make` on every call.
+constexpr int kMaxCachedDevices = 64;
+
+template <typename F>
+int cached_per_device(std::atomic<int>* cache, int dev, F make)
+{
+    const bool slot = dev >= 0 && dev < kMaxCachedDevices;
+    if (slot) {
+        const int v = cache[dev].load(std::memory_order_acquire);
+        if (v > 0) return v;
+    }
+    const int v = make();
+    if (slot && v > 0) cache[dev].store(v, std::memory_order_release);
+    return v;
+}
 
 // Resident CTAs per SM of `kernel` from the resources the SM checks (registers, shared memory,
 // threads), at most `want`. The runtime's occupancy calculator answers 1 for the tcgen05
