@@ -110,6 +110,13 @@ int pbb_ring_prefill(const void* k_hist, const void* v_hist, const int32_t* pos,
  * per-split partial (max, sum, output) of Eq. (lse) and one counter per
  * (sequence, KV head); a decode step grows it on demand, which allocates, so
  * call this first when decode steps are to be captured in a CUDA graph.
+ *   - Every decode step on a device (pbb_decode_step, _f32, _layers and
+ *     pbb_swa_decode_step) uses this one workspace, including its work-queue
+ *     head: steps whose execution overlaps on the GPU (different streams, or
+ *     graphs replayed on different streams) race on it, and the caller must
+ *     order them. Issuing calls from several host threads is safe: the library
+ *     serialises its own bookkeeping, and a growth waits for the steps already
+ *     launched before it frees the old buffers.
  */
 int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
 

@@ -291,8 +291,10 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
             a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(g_ws[dev].parts) +
                                                  round_up(parts * d * sizeof(float), 256));
         }
+        // launched with the lock held: a call on another host thread that grows the workspace
+        // frees these buffers only after its cudaDeviceSynchronize, which waits for this launch
+        return pbb::launch_decode(a, elem, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
     }
-    return pbb::launch_decode(a, elem, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
 
 }  // namespace
