@@ -109,9 +109,9 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
 #define PBB_BWD_Q_QC 64
 #endif
 
-// In the one-CTA shapes, tiles with no masked entry take a packed path (1) or the masked one
-// (0): PBB_BWD_Q_INNER for the dQ pass, PBB_BWD_KV_INNER for the dK/dV pass. The two-CTA
-// shapes always take the masked path (measured faster there).
+// Tiles with no masked entry take a packed path (1) or the masked one (0): PBB_BWD_Q_INNER for
+// the dQ pass (every shape), PBB_BWD_KV_INNER for the dK/dV pass (one-CTA shapes; the two-CTA
+// shape keeps the masked path, measured faster there).
 #ifndef PBB_BWD_Q_INNER
 #define PBB_BWD_Q_INNER 1
 #endif
@@ -136,7 +136,7 @@ struct BqCfg {
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
     static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = 4 * NK;
     static constexpr int OBUF = T_DQ + 2 * D <= TMEM_COLS ? 2 : 1;
-    static constexpr bool INNER = PBB_BWD_Q_INNER && CTAS == 1;
+    static constexpr bool INNER = PBB_BWD_Q_INNER;
     static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_DQ + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
