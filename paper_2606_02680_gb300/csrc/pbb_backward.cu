@@ -16,15 +16,19 @@
 //                      and accumulates dK and dV in tensor memory;
 //   bwd_q_tc_kernel    items of 128 query rows: it streams the key tiles of [a(t0), t_last]
 //                      and accumulates dQ in tensor memory.
-// Both are persistent (one CTA per SM) on the fifth-generation tensor cores: a TMA
-// producer warp (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion
-// through tcgen05.commit on mbarriers) and two elementwise warpgroups that take
-// alternate tiles (the scores of tile g sit in TMEM buffer g % 2), so two tiles'
-// exponentials run at once; thread r of a warpgroup owns TMEM lane r. P, dS and
-// their transposes are rounded to bf16 and written back over the scores in tensor
-// memory as the A operands of the next products. Every
-// wait is bounded by the global timer; a wait that runs out records a timeout, every
-// role stops, the MMAs and copies in flight are drained and TMEM is released.
+// Both are persistent on the fifth-generation tensor cores: a TMA producer warp
+// (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion through
+// tcgen05.commit on mbarriers) and elementwise warpgroups; thread r of a warpgroup owns
+// TMEM lane r. The long shape runs one CTA per SM with two elementwise warpgroups that
+// take alternate tiles (the scores of tile g sit in TMEM buffer g % 2), so two tiles'
+// exponentials run at once; the short shape (short supports, d = 64) runs two CTAs per
+// SM with one warpgroup each, on half the TMEM. P, dS and their transposes are rounded
+// to bf16 and written back over the scores in tensor memory as the A operands of the
+// next products. Tiles with no masked entry take a packed path (two columns per
+// ffma2/fadd2/fmul2, rounded like the scalar operations, so the results are the same
+// bits). Every wait is bounded by the global timer; a wait that runs out records a
+// timeout, every role stops, the MMAs and copies in flight are drained and TMEM is
+// released.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
