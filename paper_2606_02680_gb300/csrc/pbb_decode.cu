@@ -18,7 +18,7 @@
 // it appends k_new/v_new to slot r (never a slot that is read) and folds the
 // token into its softmax. Chunks past the end of a short support are skipped.
 //
-// Persistent CTAs, one per SM. A producer lane takes items from a device-wide
+// Persistent CTAs, as many per SM as fit. A producer lane takes items from a device-wide
 // queue (an atomic counter) and streams them without a break: every item
 // becomes tiles of TK keys, and each tile lands in one stage of a 3-stage
 // shared-memory ring through 1-D bulk copies (cp.async.bulk, completion
@@ -790,9 +790,12 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
 // GQA group 8 makes the score product a dense tile: for a block of 16 keys,
 // S^T [16 keys x 8 heads] = K [16 x d] . Q^T [d x 8] is an mma.m16n8k16 chain
 // over d, and the output O^T [d x 8 heads] += V^T [d x 16 keys] . P^T
-// [16 keys x 8 heads] is one mma per 16 output dims. This kernel serves
-// bf16, G = 8 and block sizes that are multiples of twice the tile, so that no
-// tile straddles the end of a ring. It keeps the persistent producer /
+// [16 keys x 8 heads] is one mma per 16 output dims. This kernel serves bf16
+// PBB steps with G = 8, or G = 4 and 6 with their query columns padded to 8 by
+// zero rows (whose outputs are not written), and block sizes that are multiples
+// of twice the tile, so that no tile straddles the end of a ring. The step is
+// bound by HBM (each K/V byte feeds 2G flops), so the warp-level mma is enough to
+// keep up with the copies. It keeps the persistent producer /
 // consumer structure, work queue, merge and combine of decode_kernel; what
 // changes is how a consumer warp handles its 16 keys of a tile:
 //   - K and V tiles arrive by 2-D TMA copies with the 128-byte swizzle, one

@@ -44,6 +44,10 @@
 // thread execute in order, so S_{j+2} overwrites a buffer only after P.V of tile
 // j has read its P.
 //
+// Long supports with B a multiple of 256 run forward_pair_kernel instead (the
+// "paired items" section below): two adjacent query items of a head share every K/V
+// tile, each with its own softmax warpgroup, S buffer and O buffer in TMEM.
+//
 // Every wait is bounded by the global timer; a wait that runs out records a
 // timeout in this file's status word and every role stops. Before the CTA exits,
 // the MMA issuer waits (bounded) for its MMAs, the producer for its copies, and
