@@ -161,3 +161,46 @@ def test_window_checked_before_launch(pbb):
         rc = lib.pbb_swa_decode_step(None, None, None, None, None, None, None, 0, 8, 2, 128, 128,
                                      window, 0, None)
         assert rc == code, (window, rc)
+
+
+def test_whole_sequence_arguments_checked_before_the_device(pbb):
+    """pbb_forward, pbb_backward and pbb_ring_from_sequence refuse bad arguments (null or
+    misaligned pointers, negative lengths, row counts past 32-bit TMA coordinates) and treat
+    empty work as a no-op, all before any device call. Pointers are never dereferenced."""
+    lib = pbb.lib()
+    p = 0x1000
+    # pbb_forward(q, k, v, out, lse, batch, Hq, Hkv, n, d, B, out_dtype, stream)
+    fwd = lib.pbb_forward
+    assert fwd(None, None, None, None, None, 0, 8, 2, 128, 64, 128, 0, None) == 0       # batch 0
+    assert fwd(None, None, None, None, None, 1, 8, 2, 0, 64, 128, 0, None) == 0         # n 0
+    assert fwd(None, None, None, None, None, 1, 8, 2, -1, 64, 128, 0, None) == -1       # n < 0
+    assert fwd(p, p, p, p, None, 1, 8, 2, 128, 64, 128, 7, None) == -1                  # out dtype
+    assert fwd(None, p, p, p, None, 1, 8, 2, 128, 64, 128, 0, None) == -1               # null q
+    assert fwd(p, p, p, p + 8, None, 1, 8, 2, 128, 64, 128, 0, None) == -1              # out misaligned
+    assert fwd(p, p, p, p, p + 2, 1, 8, 2, 128, 64, 128, 1, None) == -1                 # lse misaligned
+    assert fwd(p, p, p, p, None, 1 << 12, 32, 8, 1 << 14, 128, 128, 0, None) == -2      # 2^31 rows
+    assert fwd(p, p, p, p, None, 1, 8, 2, 128, 64, 127, 0, None) == -2                  # B odd
+    # pbb_backward(q, k, v, out, dout, lse, delta, dq, dk, dv, batch, Hq, Hkv, n, d, B, stream)
+    bwd = lib.pbb_backward
+    nul = (None,) * 10
+    assert bwd(*nul, 0, 8, 2, 128, 64, 128, None) == 0                                  # batch 0
+    assert bwd(*nul, 1, 8, 2, 0, 64, 128, None) == 0                                    # n 0
+    assert bwd(*nul, 1, 8, 2, -3, 64, 128, None) == -1                                  # n < 0
+    ptrs = [p] * 10
+    for i in range(10):                                                                 # each null pointer
+        args = list(ptrs)
+        args[i] = None
+        assert bwd(*args, 1, 8, 2, 128, 64, 128, None) == -1, i
+    for i, off in ((0, 8), (5, 2), (6, 2), (7, 4)):                                     # q, lse, delta, dq
+        args = list(ptrs)
+        args[i] = p + off
+        assert bwd(*args, 1, 8, 2, 128, 64, 128, None) == -1, i
+    assert bwd(*ptrs, 1 << 12, 32, 8, 1 << 14, 128, 128, None) == -2                    # 2^31 rows
+    assert bwd(*ptrs, 1, 8, 2, 128, 80, 128, None) == -2                                # d 80
+    # pbb_ring_from_sequence(k, v, n, k_ring, v_ring, batch, Hkv, d, B, dtype, stream)
+    rfs = lib.pbb_ring_from_sequence
+    assert rfs(None, None, 5, None, None, 0, 2, 64, 128, 0, None) == 0                  # batch 0
+    assert rfs(None, None, -1, p, p, 1, 2, 64, 128, 0, None) == -1                      # n < 0
+    assert rfs(None, None, 5, p, p, 1, 2, 64, 128, 0, None) == -1                       # null history
+    assert rfs(p, p, 5, None, p, 1, 2, 64, 128, 0, None) == -1                          # null ring
+    assert rfs(p + 4, p, 5, p, p, 1, 2, 64, 128, 0, None) == -1                         # misaligned
