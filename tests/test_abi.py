@@ -204,3 +204,34 @@ def test_whole_sequence_arguments_checked_before_the_device(pbb):
     assert rfs(None, None, 5, p, p, 1, 2, 64, 128, 0, None) == -1                       # null history
     assert rfs(p, p, 5, None, p, 1, 2, 64, 128, 0, None) == -1                          # null ring
     assert rfs(p + 4, p, 5, p, p, 1, 2, 64, 128, 0, None) == -1                         # misaligned
+
+
+def test_binding_refuses_host_tensors(pbb):
+    """No CPU fallback: every compute call of the binding raises on host tensors before the
+    library runs anything."""
+    import torch
+
+    bf = torch.bfloat16
+    batch, Hq, Hkv, d, B, n = 1, 8, 2, 64, 128, 16
+    q = torch.zeros(batch, Hq, d, dtype=bf)
+    kn = torch.zeros(batch, Hkv, d, dtype=bf)
+    ring = torch.zeros(batch, Hkv, B, d, dtype=bf)
+    pos = torch.zeros(batch, dtype=torch.int32)
+    calls = [
+        lambda: pbb.decode_step(q, kn, kn, ring, ring.clone(), pos),
+        lambda: pbb.swa_decode_step(q, kn, kn, ring, ring.clone(), pos, window=B),
+        lambda: pbb.decode_step_layers(q[None], kn[None], kn[None], ring[None], ring[None].clone(), pos),
+        lambda: pbb.ring_prefill(ring, ring.clone(), pos, ring.clone(), ring.clone()),
+        lambda: pbb.advance_positions(pos),
+    ]
+    qs = torch.zeros(batch, Hq, n, d, dtype=bf)
+    ks = torch.zeros(batch, Hkv, n, d, dtype=bf)
+    lse = torch.zeros(batch, Hq, n, dtype=torch.float32)
+    calls += [
+        lambda: pbb.forward(qs, ks, ks.clone(), B),
+        lambda: pbb.backward(qs, ks, ks.clone(), qs.clone(), qs.clone(), lse, B),
+        lambda: pbb.ring_from_sequence(ks, ks.clone(), ring.clone(), ring.clone()),
+    ]
+    for i, call in enumerate(calls):
+        with pytest.raises(TypeError, match="CUDA tensor"):
+            call()
