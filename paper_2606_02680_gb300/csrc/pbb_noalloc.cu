@@ -4,10 +4,9 @@
 //
 // Who needs it: callers that must not, or cannot, allocate device memory
 // while they run decode steps. Examples are a serving runtime that hands all
-// of HBM to its own pool up front and forbids any other allocation, code
-// running inside a CUDA stream capture (allocation there breaks or
-// invalidates the capture), and latency-critical loops where cudaMalloc's
-// implicit device synchronisation is unacceptable. pbb_decode_step keeps its
+// of HBM to its own pool up front and forbids any other allocation, and
+// latency-critical loops where the device-wide synchronisation a cudaMalloc
+// can bring is unacceptable. pbb_decode_step keeps its
 // scratch in a workspace it grows with cudaMalloc on demand; this variant
 // never calls cudaMalloc, cudaFree or any allocating library routine.
 //

@@ -152,6 +152,7 @@ class DeviceRun:
         w, i = self.w, self.step_i
         q, k, v = inputs.step_inputs(w, i, device=self.dev)
         out = _decode(q, k, v, self.k_ring, self.v_ring, self.pos, self.window)
+        self.out = out  # every sequence's output of this step, on the device
         pbb.advance_positions(self.pos)
         idx = torch.as_tensor(self.sample, device=self.dev)
         ks, vs = k.index_select(0, idx).cpu(), v.index_select(0, idx).cpu()

@@ -104,3 +104,63 @@ def test_sweep_point(batch, B):
         check_close(out, run.oracle_out(), w.dtype, f"b{batch} B{B} step {i}")
     run.check_rings()
     assert pbb.get_device_status() == pbb.PBB_OK
+
+
+def _edge_start_positions(batch: int, B: int, seed: int) -> torch.Tensor:
+    """Start positions at chosen phases r = t mod B: the first sequences cycle through
+    r in {0, 1, h-2, h-1, h, h+1, B-2, B-1} (a two-step run then crosses the bridge/no-bridge
+    edge at h-1 -> h and the block boundary at B-1 -> 0), the rest are uniform; every block
+    index is at least 1, so the bridge exists (Eq. pbb)."""
+    h = B // 2
+    edges = [0, 1, h - 2, h - 1, h, h + 1, B - 2, B - 1]
+    g = torch.Generator().manual_seed(seed)
+    blk = torch.randint(1, (1 << 20) // B, (batch,), generator=g, dtype=torch.int64)
+    r = torch.randint(0, B, (batch,), generator=g, dtype=torch.int64)
+    n_edge = min(batch, 4 * len(edges))
+    r[:n_edge] = torch.tensor([edges[i % len(edges)] for i in range(n_edge)], dtype=torch.int64)
+    return blk * B + r
+
+
+def test_headline_every_sequence_at_edge_phases():
+    """The benchmark's timed shape (batch 512, Hq 32, Hkv 8, d 128, B 4096, bf16; the library's
+    plan, which runs group 4 padded to 8 on the tensor-core kernel) checked on EVERY sequence
+    on two consecutive steps, with 32 sequences placed on the phase edges of Eq. (pbb) at
+    B = 4096, and every sequence's rings byte for byte at the end against the oracle's ring
+    simulator."""
+    w = inputs.sweep_workload(512, 4096, steps=2)
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, torch.bfloat16) == "tensor_cores"
+    dev = torch.device("cuda", 0)
+    t0 = _edge_start_positions(w.batch, w.B, seed=23)
+    pos = t0.to(torch.int32).to(dev)
+    hk_d, hv_d = inputs.history_window(w, t0, device=dev)  # positions t0-B .. t0-1
+    k_ring = torch.empty((w.batch, w.Hkv, w.B, w.d), dtype=torch.bfloat16, device=dev)
+    v_ring = torch.empty_like(k_ring)
+    pbb.ring_prefill(hk_d, hv_d, pos, k_ring, v_ring)
+    new_k, new_v = [], []
+    chunk = 32
+    for i in range(w.steps):
+        q, k, v = inputs.step_inputs(w, i, device=dev)
+        out = pbb.decode_step(q, k, v, k_ring, v_ring, pos).cpu()
+        pbb.advance_positions(pos)
+        new_k.append(k.cpu())
+        new_v.append(v.cpu())
+        t = (t0 + i).numpy()
+        qc = q.cpu()
+        for lo in range(0, w.batch, chunk):
+            sl = slice(lo, lo + chunk)
+            # window of B+1 rows ending at the current token: positions t-B .. t
+            wk = torch.cat([hk_d[sl].cpu()] + [x[sl].unsqueeze(2) for x in new_k], dim=2)[:, :, i:]
+            wv = torch.cat([hv_d[sl].cpu()] + [x[sl].unsqueeze(2) for x in new_v], dim=2)[:, :, i:]
+            ref = oracle.attend(qc[sl], wk, wv, s0=t[sl] - w.B, t=t[sl], b=w.B)
+            check_close(out[sl], ref, w.dtype, f"step {i} sequences {lo}..{lo + chunk - 1}")
+    assert pbb.get_device_status() == pbb.PBB_OK
+    from pbb_testlib import ring_bytes_np
+
+    for lo in range(0, w.batch, chunk):
+        sl = slice(lo, lo + chunk)
+        sim = oracle.RingSim(chunk, w.Hkv, w.d, w.B, 2)
+        sim.replay(hk_d[sl].cpu(), hv_d[sl].cpu(), (t0[sl] - w.B).numpy())
+        for i in range(w.steps):
+            sim.append(new_k[i][sl], new_v[i][sl], (t0[sl] + i).numpy())
+        assert np.array_equal(ring_bytes_np(k_ring[sl]), sim.k), f"K rings {lo}..{lo + chunk - 1}"
+        assert np.array_equal(ring_bytes_np(v_ring[sl]), sim.v), f"V rings {lo}..{lo + chunk - 1}"

@@ -1,18 +1,22 @@
-"""pbb_decode_step_noalloc against pbb_decode_step, through the C ABI.
+"""pbb_decode_step_noalloc through the C ABI: against pbb_decode_step and the fp64 oracle.
 
-The no-allocation entry point serves callers that cannot allocate device
-memory while they decode (a runtime that owns all of HBM through its own pool,
-code inside a CUDA stream capture, loops that cannot afford cudaMalloc's
-implicit synchronisation). Its split scratch is a fixed array inside the
-library instead of the workspace pbb_decode_step grows with cudaMalloc. This
-file is collected last on purpose, so a run that stops at the first failure
-has already run every other test; it also passes when run alone.
+The no-allocation entry point is for callers that cannot allocate device memory
+while they decode: a serving runtime that hands all of HBM to its own pool and
+forbids any other allocation, or a loop that cannot afford the device-wide
+synchronisation a cudaMalloc can bring. Its split scratch is a fixed array
+inside the library instead of the workspace pbb_decode_step grows with
+cudaMalloc. This file is collected last on purpose, so a run that stops at the
+first failure has already run every other test; it also passes when run alone.
 """
 import ctypes
 
 import numpy as np
 import pytest
 import torch
+
+from pbb_testlib import check_close, ring_bytes_np
+
+import oracle
 
 pytestmark = pytest.mark.gpu
 
@@ -24,6 +28,7 @@ def lib():
     from paper_2606_02680_gb300 import build as nvbuild
 
     nvbuild.build()
+    oracle.build()
     import paper_2606_02680_gb300 as pbb
 
     torch.cuda.set_device(0)
@@ -42,7 +47,7 @@ def _state(pbb, w, t0, wk, wv, dev):
 
 @pytest.mark.parametrize("Hq,Hkv,d,kernel", [(16, 4, 128, "auto"), (12, 2, 64, "auto"), (8, 4, 128, "auto"),
                                               (16, 4, 128, "tensor_cores"), (12, 2, 64, "tensor_cores")])
-def test_noalloc_matches_decode_step_on_two_calls(lib, Hq, Hkv, d, kernel):
+def test_noalloc_matches_decode_step_and_oracle_on_two_calls(lib, Hq, Hkv, d, kernel):
     pbb = lib
     from paper_2606_02680_gb300 import inputs
 
@@ -65,6 +70,11 @@ def _noalloc_against_decode_step(pbb, inputs, Hq, Hkv, d):
     wk, wv = inputs.history_window(w, t0, device=dev)
     pos_a, kr_a, vr_a = _state(pbb, w, t0, wk, wv, dev)
     pos_b, kr_b, vr_b = _state(pbb, w, t0, wk, wv, dev)
+    # the oracle's side: host history (positions t0-B .. t0-1, then one row per step) and its
+    # ring simulator
+    hk, hv = [wk.cpu()], [wv.cpu()]
+    sim = oracle.RingSim(w.batch, w.Hkv, w.d, w.B, 2)
+    sim.replay(hk[0], hv[0], (t0 - w.B).numpy())
     stream = torch.cuda.current_stream()
     s = ctypes.c_void_p(stream.cuda_stream)
     L = pbb.lib()
@@ -83,29 +93,46 @@ def _noalloc_against_decode_step(pbb, inputs, Hq, Hkv, d):
         assert L.pbb_advance_positions(pos_a.data_ptr(), w.batch, s) == pbb.PBB_OK
         assert L.pbb_advance_positions(pos_b.data_ptr(), w.batch, s) == pbb.PBB_OK
         torch.cuda.synchronize()
-        a = out_a.cpu().double().numpy()
-        b = out_b.cpu().double().numpy()
-        assert np.all(np.isfinite(b))
-        err = np.abs(a - b)
-        assert err.max() <= 1e-2 and (err / np.maximum(np.abs(a), 1.0)).max() <= 1e-2, step
+        # same split plan and kernel, deterministic combine order: bitwise the same result
+        assert torch.equal(out_a, out_b), step
         assert torch.equal(kr_a.view(torch.int16), kr_b.view(torch.int16))
         assert torch.equal(vr_a.view(torch.int16), vr_b.view(torch.int16))
+        # and the fp64 oracle over the history window ending at the current token
+        hk.append(k.cpu().unsqueeze(2))
+        hv.append(v.cpu().unsqueeze(2))
+        t = (t0 + step).numpy()
+        sim.append(k.cpu(), v.cpu(), t)
+        win_k = torch.cat(hk, dim=2)[:, :, step:w.B + step + 1]
+        win_v = torch.cat(hv, dim=2)[:, :, step:w.B + step + 1]
+        ref = oracle.attend(q.cpu(), win_k, win_v, s0=t - w.B, t=t, b=w.B)
+        check_close(out_b.cpu(), ref, "bf16", f"no-alloc step {step}")
+        assert np.array_equal(ring_bytes_np(kr_b), sim.k), "K ring differs from the oracle's"
+        assert np.array_equal(ring_bytes_np(vr_b), sim.v), "V ring differs from the oracle's"
     assert L.pbb_get_device_status(s) == pbb.PBB_OK
 
 
 def test_noalloc_rejects_steps_beyond_its_scratch(lib):
+    """A step whose split partials exceed the fixed array is refused before any launch. The
+    buffers are sized for the step all the same, so that a kernel launched by mistake would
+    stay inside them instead of touching memory it does not own."""
     pbb = lib
     dev = torch.device("cuda", 0)
     batch, Hq, Hkv, d, B = 64, 32, 8, 128, 4096
     prev = pbb.set_chunk_keys(32)  # 128 CTAs per support: partials far beyond the fixed array
     try:
-        x = torch.zeros(16, dtype=torch.bfloat16, device=dev)  # never read: rejected before launch
-        o = torch.zeros(16, dtype=torch.float32, device=dev)
-        p = torch.zeros(16, dtype=torch.int32, device=dev)
-        rc = pbb.lib().pbb_decode_step_noalloc(x.data_ptr(), x.data_ptr(), x.data_ptr(), x.data_ptr(),
-                                               x.data_ptr(), p.data_ptr(), o.data_ptr(), batch, Hq,
+        q = torch.zeros((batch, Hq, d), dtype=torch.bfloat16, device=dev)
+        kn = torch.zeros((batch, Hkv, d), dtype=torch.bfloat16, device=dev)
+        vn = torch.zeros_like(kn)
+        kr = torch.zeros((batch, Hkv, B, d), dtype=torch.bfloat16, device=dev)
+        vr = torch.zeros_like(kr)
+        pos = torch.full((batch,), 3 * B // 2, dtype=torch.int32, device=dev)
+        out = torch.full((batch, Hq, d), -7.0, dtype=torch.float32, device=dev)
+        rc = pbb.lib().pbb_decode_step_noalloc(q.data_ptr(), kn.data_ptr(), vn.data_ptr(), kr.data_ptr(),
+                                               vr.data_ptr(), pos.data_ptr(), out.data_ptr(), batch, Hq,
                                                Hkv, d, B, None)
         assert rc == pbb.PBB_ERR_SCRATCH_LIMIT
         assert "scratch" in pbb.error_string(rc)
+        torch.cuda.synchronize()
+        assert bool((out == -7.0).all()), "a refused step must not write its output"
     finally:
         pbb.set_chunk_keys(prev)
