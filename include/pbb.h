@@ -104,21 +104,26 @@ int pbb_ring_prefill(const void* k_hist, const void* v_hist, const int32_t* pos,
                      cudaStream_t stream);
 
 /*
- * Make sure the library's workspace on the current device holds the split
- * partials of a step of this shape (and of every smaller batch). The
- * workspace (per device, owned by the library, freed at exit) holds the
- * per-split partial (max, sum, output) of Eq. (lse) and one counter per
- * (sequence, KV head); a decode step grows it on demand, which allocates, so
- * call this first when decode steps are to be captured in a CUDA graph.
- *   - Every decode step on a device (pbb_decode_step, _f32, _layers and
- *     pbb_swa_decode_step) uses this one workspace, including its work-queue
- *     head: steps whose execution overlaps on the GPU (different streams, or
- *     graphs replayed on different streams) race on it, and the caller must
- *     order them. Issuing calls from several host threads is safe: the library
- *     serialises its own bookkeeping, and a growth waits for the steps already
- *     launched before it frees the old buffers.
+ * Make sure the library's workspace of (current device, `stream`) holds the
+ * split partials of a step of this shape (and of every smaller batch). A
+ * workspace (owned by the library, freed at exit) holds the work-queue words,
+ * one counter per (sequence, KV head) and the per-split partial (max, sum,
+ * output) of Eq. (lse). Every decode step (pbb_decode_step, _f32, _layers and
+ * pbb_swa_decode_step) uses the workspace of the stream it is issued on and
+ * grows it on demand, which allocates and waits for the device; so call this
+ * first, on the capture stream, when decode steps are to be captured in a
+ * CUDA graph.
+ *   - Steps on different streams use different workspaces and may overlap on
+ *     the GPU. Steps on one stream run in order. A captured graph keeps the
+ *     workspace of the stream it was captured on: do not replay it while steps
+ *     (or replays of other graphs captured on that stream) run on other
+ *     streams, and do not let that stream's workspace grow after the capture
+ *     (growth frees the buffers the graph holds).
+ *   - Issuing calls from several host threads is safe: the library serialises
+ *     its own bookkeeping, and a growth waits for the steps already launched
+ *     before it frees the old buffers.
  */
-int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype, cudaStream_t stream);
 
 /*
  * One PBB decode step for every sequence (bf16 q/k/v/ring, fp32 out).
@@ -170,10 +175,13 @@ int pbb_decode_step_layers(const void* q, const void* k_new, const void* v_new, 
  * the current token included. Same ring contents and precondition: the step
  * writes k_new/v_new into slot t mod B, which holds position t-B, outside the
  * window. A ring can be switched between the two kinds of step at any
- * position. Runs on the CUDA-core kernel for every group size. Returns
+ * position. Runs on the same kernels as the PBB step (the tensor-core kernel
+ * for bf16 with Hq/Hkv in {4, 6, 8} and B a multiple of 64, under the same
+ * rules; its tiles start at slot multiples of 32 and mask the slots outside
+ * the window's run). Returns
  * PBB_ERR_INVALID_ARG for a window outside [1, B]. pbb_reserve_workspace
- * covers window steps with window = B; for a smaller window make one step
- * outside any stream capture first.
+ * covers window steps with window = B; for a smaller window make one step on
+ * the capture stream outside any stream capture first.
  */
 int pbb_swa_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
                         void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
@@ -300,10 +308,9 @@ int pbb_set_kernel(int kernel);
 
 /*
  * No counterpart in the paper: a library-usage variant for callers that cannot
- * allocate device memory while they decode (a runtime that owns all of HBM
- * through its own pool and forbids other allocations, code inside a CUDA
- * stream capture, loops that cannot afford cudaMalloc's implicit device
- * synchronisation).
+ * allocate device memory while they decode (a serving runtime that owns all of
+ * HBM through its own pool and forbids other allocations, or a loop that cannot
+ * afford the device-wide synchronisation a cudaMalloc can bring).
  *
  * Same arguments, layouts and result as pbb_decode_step (bf16), but the split
  * scratch (per-(sequence, KV head) arrival counters and split partials) lives
@@ -327,6 +334,19 @@ int pbb_set_kernel(int kernel);
 int pbb_decode_step_noalloc(const void* q, const void* k_new, const void* v_new, void* k_ring,
                             void* v_ring, const int32_t* pos, float* out, int batch, int Hq,
                             int Hkv, int d, int B, cudaStream_t stream);
+
+/*
+ * No counterpart in the paper: a measurement utility. Reads every byte of
+ * buf[0, bytes) once from device memory (streaming loads, one persistent grid of
+ * 4 CTAs per SM) and xor-folds the 32-bit words into *sink, so the bytes cannot
+ * be skipped. Timing it gives the read-only HBM bandwidth, the roof of a decode
+ * step (which reads its K/V support and writes almost nothing), next to the
+ * copy (read + write) bandwidth. buf: device pointer, 16-byte aligned, bytes a
+ * multiple of 16; sink: device pointer, 8-byte aligned, caller-owned (its value
+ * is only a checksum). Asynchronous on `stream`; PBB_ERR_INVALID_ARG on a
+ * null or misaligned argument, nothing launched for bytes = 0.
+ */
+int pbb_stream_read(const void* buf, size_t bytes, unsigned long long* sink, cudaStream_t stream);
 
 /* Static description of an error code. */
 const char* pbb_error_string(int code);

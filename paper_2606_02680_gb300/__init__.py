@@ -35,7 +35,8 @@ __all__ = [
     "PBB_ERR_SCRATCH_LIMIT", "PbbError",
     "lib", "lib_path", "set_kernel", "plan_forward", "ring_bytes", "ring_alloc", "Rings", "ring_prefill", "decode_step", "decode_step_layers", "swa_decode_step", "forward", "backward", "ring_from_sequence",
     "decode_step_host", "HostPipeline", "advance_positions", "get_device_status", "reserve_workspace",
-    "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "EXPORTS",
+    "set_wait_timeout_ns", "set_chunk_keys", "plan_chunk_keys", "plan_kernel", "error_string", "stream_read",
+    "EXPORTS",
 ]
 
 PBB_OK = 0
@@ -57,7 +58,7 @@ EXPORTS = {
     "pbb_ring_alloc": (_I, [ctypes.POINTER(_P), ctypes.POINTER(_P), _I, _I, _I, _I, _I, _P]),
     "pbb_ring_free": (_I, [_P, _P, _P]),
     "pbb_ring_prefill": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
-    "pbb_reserve_workspace": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_reserve_workspace": (_I, [_I, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_f32": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_decode_step_noalloc": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P]),
@@ -74,6 +75,7 @@ EXPORTS = {
     "pbb_set_kernel": (_I, [_I]),
     "pbb_plan_chunk_keys": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_plan_kernel": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_stream_read": (_I, [_P, _SZ, _P, _P]),
     "pbb_error_string": (ctypes.c_char_p, [_I]),
 }
 
@@ -446,13 +448,26 @@ def advance_positions(pos: torch.Tensor, stream=None) -> None:
            "pbb_advance_positions")
 
 
+def stream_read(buf: torch.Tensor, sink: torch.Tensor, stream=None) -> None:
+    """Read every byte of the contiguous device tensor `buf` once (pbb_stream_read), xor-folded
+    into the int64 device tensor `sink`: the read-only HBM bandwidth probe."""
+    if not buf.is_cuda or not buf.is_contiguous() or not sink.is_cuda or sink.dtype != torch.int64:
+        raise ValueError("buf must be a contiguous device tensor and sink an int64 device tensor")
+    _check(lib().pbb_stream_read(ctypes.c_void_p(buf.data_ptr()), buf.numel() * buf.element_size(),
+                                 ctypes.c_void_p(sink.data_ptr()), _stream(stream)), "pbb_stream_read")
+
+
 def get_device_status(stream=None) -> int:
     """Synchronise and return (and clear) the device status word (PBB_OK or a PBB_ERR_DEVICE_* code)."""
     return int(lib().pbb_get_device_status(_stream(stream)))
 
 
-def reserve_workspace(max_batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> None:
-    _check(lib().pbb_reserve_workspace(max_batch, Hq, Hkv, d, B, _dt(dtype)), "pbb_reserve_workspace")
+def reserve_workspace(max_batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16,
+                      stream=None) -> None:
+    """Grow the workspace of (current device, `stream`, default the current stream) for steps of
+    this shape, e.g. on the stream a CUDA graph will be captured on."""
+    _check(lib().pbb_reserve_workspace(max_batch, Hq, Hkv, d, B, _dt(dtype), _stream(stream)),
+           "pbb_reserve_workspace")
 
 
 def set_wait_timeout_ns(ns: int) -> None:

@@ -11,7 +11,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libpbb.so")
 OBJ_DIR = os.path.join(PKG, "_build")
-SOURCES = ("pbb_api.cu", "pbb_backward.cu", "pbb_decode.cu", "pbb_forward.cu", "pbb_noalloc.cu")
+SOURCES = ("pbb_api.cu", "pbb_backward.cu", "pbb_decode.cu", "pbb_forward.cu", "pbb_noalloc.cu",
+           "pbb_probe.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -5,7 +5,9 @@
 #include <atomic>
 #include <climits>
 #include <cstdint>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "pbb.h"
 #include "pbb_internal.h"
@@ -15,9 +17,11 @@ namespace {
 constexpr int kMaxDevices = 64;
 constexpr int kMaxBlock = 1 << 20;
 
-// Library-owned scratch of one device: the work-queue control words and one
-// counter per (sequence, KV head), all of which read zero between steps, and
-// the split partials.
+// Library-owned scratch of one (device, stream): the work-queue control words
+// and one counter per (sequence, KV head), all of which read zero between
+// steps, and the split partials. Steps issued on one stream run in order, so
+// they never use a workspace at the same time; steps on different streams get
+// different workspaces and may overlap on the GPU.
 struct Workspace {
     int* counters = nullptr;  // [0, 2): queue control; then one per (sequence, KV head)
     size_t counter_cap = 0;   // ints allocated
@@ -25,8 +29,10 @@ struct Workspace {
     size_t parts_bytes = 0;
 };
 
+using WsKey = std::pair<int, uintptr_t>;  // (device, stream handle)
+
 std::mutex g_mutex;
-Workspace g_ws[kMaxDevices];
+std::map<WsKey, Workspace> g_ws;  // guarded by g_mutex; entries are never erased
 int g_sms[kMaxDevices] = {};
 std::atomic<unsigned long long> g_timeout_ns{1000000000ull};
 std::atomic<int> g_chunk_override{0};
@@ -96,20 +102,29 @@ int sm_count(int dev)
     return g_sms[dev];
 }
 
-// The split plan. Whole supports are the cheapest work items (no cross-CTA
-// combine), but a batch of P supports on G resident CTAs leaves P mod G
-// supports for a last round; when that round would leave more than half the
-// CTAs idle, those last supports are split into about G / (P mod G) chunks
-// each, so the step ends on small items. A batch with fewer supports than CTAs
-// splits every support so that there are about G items. Chunks never hold less
-// than kMinChunkBytes of K+V (below that the combine costs more than the
-// parallel streaming saves). Measured on GB300 at 512 supports on 456 CTAs,
-// splitting every support into 2-4 chunks was 5-25 % slower than running them
-// whole, while splitting only the last round's supports paid for long supports
-// (see below); a positive pbb_set_chunk_keys override splits every support
-// into chunks of that many keys.
+// The split plan of the CUDA-core kernel. Whole supports are the cheapest work
+// items there (no cross-CTA combine), but a batch of P supports on G resident
+// CTAs leaves P mod G supports for a last round; when that round would leave
+// more than half the CTAs idle, those last supports are split into about
+// G / (P mod G) chunks each, so the step ends on small items. A batch with
+// fewer supports than CTAs splits every support so that there are about G
+// items. Chunks never hold less than kMinChunkBytes of K+V (below that the
+// combine costs more than the parallel streaming saves). Measured on GB300 at
+// 512 supports on 456 CTAs, splitting every support into 2-4 chunks was 5-25 %
+// slower than running them whole, while splitting only the last round's
+// supports paid for long supports (see below).
+//
+// The tensor-core kernel ends items on a separate epilogue warp, so a split
+// item costs its consumers nothing; its plan cuts every support into chunks
+// of about (supports x mean support) / (PBB_TC_ROUNDS x G) keys, so the
+// persistent grid balances on small items and the step does not end on a few
+// CTAs streaming long supports alone. A positive pbb_set_chunk_keys override
+// splits every support into chunks of that many keys, for either kernel.
 #ifndef PBB_MIN_CHUNK_KB
 #define PBB_MIN_CHUNK_KB 64
+#endif
+#ifndef PBB_TC_ROUNDS
+#define PBB_TC_ROUNDS 4
 #endif
 
 int min_split_keys(int d, int elem, int tile)
@@ -121,11 +136,6 @@ int min_split_keys(int d, int elem, int tile)
 
 }  // namespace
 
-// Whether the tensor-core kernel also splits a partly filled last round of long supports.
-#ifndef PBB_TC_SPLIT_LAST_ROUND
-#define PBB_TC_SPLIT_LAST_ROUND 0
-#endif
-
 namespace pbb {
 
 SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int window)
@@ -134,10 +144,47 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) dev = 0;
     const int tile = pbb::tile_keys(elem, d, group);
-    // ring keys of the longest support: B-1 for PBB (phase B-1), w-1 for a window of w
-    const int span = window > 0 ? window - 1 : B - 1;
+    const bool tc = pbb::tensor_core_shape(batch, Hkv, d, B, elem, group, window);
+    // keys of the longest support in the kernel's key space: B-1 for PBB (phase B-1), w-1 for a
+    // window of w; the tensor-core kernel counts a window's run from the tile-aligned slot below
+    // its start, up to tile-1 keys more
+    const int span = window > 0 ? window - 1 + (tc && window > 1 ? tile - 1 : 0) : B - 1;
     const int max_keys = span > 0 ? span : 1;
     const long long pairs = static_cast<long long>(batch) * Hkv;
+    const int over = g_chunk_override.load();
+    if (over > 0) {
+        sp.whole = 0;
+        int chunk = static_cast<int>(round_up(static_cast<size_t>(over), static_cast<size_t>(tile)));
+        sp.chunk = chunk;
+        sp.nchunk = (max_keys + chunk - 1) / chunk;
+        return sp;
+    }
+    auto whole_plan = [&]() {
+        sp.whole = static_cast<int>(pairs);
+        sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
+        sp.nchunk = 1;
+        return sp;
+    };
+    auto chunks_of = [&](long long chunk) {
+        const int min_keys = min_split_keys(d, elem, tile);
+        if (chunk < min_keys) chunk = min_keys;
+        chunk = static_cast<long long>(round_up(static_cast<size_t>(chunk), static_cast<size_t>(tile)));
+        if (chunk >= max_keys) return whole_plan();
+        sp.whole = 0;
+        sp.chunk = static_cast<int>(chunk);
+        sp.nchunk = (max_keys + sp.chunk - 1) / sp.chunk;
+        return sp;
+    };
+    int per_sm = pbb::decode_ctas_per_sm(batch, Hkv, elem, d, group, B, window);
+    if (per_sm <= 0) per_sm = 1;
+    const long long G = static_cast<long long>(sm_count(dev)) * per_sm;
+    if (tc) {
+        // mean ring keys of a support: (3h+1)/2 - 1 for PBB at a uniform phase (App. F.1), w-1
+        // for a window
+        const long long mean = window > 0 ? window - 1 : (3LL * B) / 4;
+        const long long want = static_cast<long long>(PBB_TC_ROUNDS) * G;
+        return chunks_of((pairs * (mean > 0 ? mean : 1) + want - 1) / want);
+    }
     auto finish = [&](long long split) {
         const long long max_split = (max_keys + min_split_keys(d, elem, tile) - 1) / min_split_keys(d, elem, tile);
         if (split > max_split) split = max_split;
@@ -151,30 +198,12 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
             sp.nchunk = 1;
         }
     };
-    const int over = g_chunk_override.load();
-    if (over > 0) {
-        sp.whole = 0;
-        int chunk = static_cast<int>(round_up(static_cast<size_t>(over), static_cast<size_t>(tile)));
-        sp.chunk = chunk;
-        sp.nchunk = (max_keys + chunk - 1) / chunk;
-        return sp;
-    }
-    int per_sm = pbb::decode_ctas_per_sm(batch, Hkv, elem, d, group, B, window);
-    if (per_sm <= 0) per_sm = 1;
-    const long long G = static_cast<long long>(sm_count(dev)) * per_sm;
     if (pairs >= G) {
         const long long R = pairs % G;
-        // Splitting the last round pays only for long supports on the CUDA-core kernel
-        // (measured: +29 % at B 4096 and +6 % at B 2048, but -12 to -15 % at B <= 1024 and
-        // -19 % for the tensor-core kernel, whose two consumer warps combine slowly).
-        const bool long_supports = max_keys >= 2047 && pbb::tile_keys(elem, d, group) == tile &&
-                                   (PBB_TC_SPLIT_LAST_ROUND || !pbb::tensor_core_shape(batch, Hkv, d, B, elem, group, window));
-        if (R == 0 || 2 * R > G || !long_supports) {  // no split
-            sp.whole = static_cast<int>(pairs);
-            sp.chunk = static_cast<int>(round_up(static_cast<size_t>(max_keys), static_cast<size_t>(tile)));
-            sp.nchunk = 1;
-            return sp;
-        }
+        // Splitting the last round pays only for long supports (measured: +29 % at B 4096 and
+        // +6 % at B 2048, but -12 to -15 % at B <= 1024).
+        const bool long_supports = max_keys >= 2047;
+        if (R == 0 || 2 * R > G || !long_supports) return whole_plan();
         sp.whole = static_cast<int>(pairs - R);
         finish((G + R - 1) / R);
     } else {
@@ -197,18 +226,20 @@ size_t parts_bytes(int batch, int Hkv, int d, int group, const pbb::SplitPlan& s
     return round_up(parts * d * sizeof(float), 256) + parts * 2 * sizeof(float);
 }
 
-// Make the workspace of device `dev` hold `pairs` counters and `pbytes` bytes
-// of partials. Allocating is refused while `stream` is being captured.
-// Caller holds g_mutex.
-int grow_workspace(int dev, size_t pairs, size_t pbytes, cudaStream_t stream, bool check_capture)
+// Make the workspace of (device `dev`, `stream`) hold `pairs` counters and
+// `pbytes` bytes of partials, and return it. Allocating is refused while
+// `stream` is being captured. Growth is rare (the first steps of a larger
+// shape, or pbb_reserve_workspace) and waits for the whole device, so that no
+// step still in flight, on any stream, can read a buffer it frees. Caller
+// holds g_mutex.
+int grow_workspace(int dev, cudaStream_t stream, size_t pairs, size_t pbytes, Workspace** out)
 {
-    Workspace& ws = g_ws[dev];
+    Workspace& ws = g_ws[WsKey(dev, reinterpret_cast<uintptr_t>(stream))];
+    *out = &ws;
     if (ws.counter_cap >= pairs && ws.parts_bytes >= pbytes) return PBB_OK;
-    if (check_capture) {
-        cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
-        if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess) return PBB_ERR_CUDA;
-        if (cap != cudaStreamCaptureStatusNone) return PBB_ERR_WORKSPACE;
-    }
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream, &cap) != cudaSuccess) return PBB_ERR_CUDA;
+    if (cap != cudaStreamCaptureStatusNone) return PBB_ERR_WORKSPACE;
     // Steps in flight may still use the old buffers.
     if (cudaDeviceSynchronize() != cudaSuccess) return PBB_ERR_CUDA;
     if (ws.counter_cap < pairs) {
@@ -281,18 +312,19 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     {
         const size_t pbytes = static_cast<size_t>(sp.whole) < pairs ? parts_bytes(batch, Hkv, d, group, sp) : 0;
         std::lock_guard<std::mutex> lock(g_mutex);
-        rc = grow_workspace(dev, pairs + 2, pbytes, stream, true);
+        Workspace* ws = nullptr;
+        rc = grow_workspace(dev, stream, pairs + 2, pbytes, &ws);
         if (rc != PBB_OK) return rc;
         const size_t parts = (pairs - static_cast<size_t>(sp.whole)) * a.nchunk * group;
-        a.ctl = g_ws[dev].counters;
-        a.counters = g_ws[dev].counters + 2;
+        a.ctl = ws->counters;
+        a.counters = ws->counters + 2;
         if (pbytes > 0) {
-            a.part_o = g_ws[dev].parts;
-            a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(g_ws[dev].parts) +
+            a.part_o = ws->parts;
+            a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(ws->parts) +
                                                  round_up(parts * d * sizeof(float), 256));
         }
-        // launched with the lock held: a call on another host thread that grows the workspace
-        // frees these buffers only after its cudaDeviceSynchronize, which waits for this launch
+        // launched with the lock held: a call on another host thread that grows a workspace
+        // frees the old buffers only after its cudaDeviceSynchronize, which waits for this launch
         return pbb::launch_decode(a, elem, stream) == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
     }
 }
@@ -361,7 +393,7 @@ int pbb_ring_prefill(const void* k_hist, const void* v_hist, const int32_t* pos,
                : PBB_ERR_CUDA;
 }
 
-int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
+int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype, cudaStream_t stream)
 {
     int rc = check_shape(max_batch, Hkv, d, B, dtype);
     if (rc != PBB_OK) return rc;
@@ -384,7 +416,8 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
         }
     }
     std::lock_guard<std::mutex> lock(g_mutex);
-    return grow_workspace(dev, static_cast<size_t>(max_batch) * Hkv + 2, need, nullptr, false);
+    Workspace* ws = nullptr;
+    return grow_workspace(dev, stream, static_cast<size_t>(max_batch) * Hkv + 2, need, &ws);
 }
 
 int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
@@ -558,13 +591,15 @@ int pbb_get_device_status(cudaStream_t stream)
         return PBB_ERR_DEVICE_TIMEOUT;  // forward and backward kernels only time out
     if (status == pbb::kDevOk) return PBB_OK;
     {
-        // An aborted step can leave split counters behind: zero them.
+        // An aborted step can leave split counters behind: zero them in every workspace of
+        // this device.
         std::lock_guard<std::mutex> lock(g_mutex);
-        Workspace& ws = g_ws[dev];
-        if (ws.counters) {
-            if (cudaMemset(ws.counters, 0, ws.counter_cap * sizeof(int)) != cudaSuccess) return PBB_ERR_CUDA;
-            if (cudaDeviceSynchronize() != cudaSuccess) return PBB_ERR_CUDA;
+        for (auto& kv : g_ws) {
+            if (kv.first.first != dev || !kv.second.counters) continue;
+            if (cudaMemset(kv.second.counters, 0, kv.second.counter_cap * sizeof(int)) != cudaSuccess)
+                return PBB_ERR_CUDA;
         }
+        if (cudaDeviceSynchronize() != cudaSuccess) return PBB_ERR_CUDA;
     }
     return status == pbb::kDevTimeout ? PBB_ERR_DEVICE_TIMEOUT : PBB_ERR_DEVICE_POSITION;
 }

@@ -100,7 +100,8 @@ enum : int { kFirst = 1, kLast = 2, kCurrent = 4, kEnd = 8 };
 // Descriptor of the tile in one stage, written by the producer before it arms the stage.
 struct __align__(16) TileMeta {
     int b, kvh, chunk, nk;  // item and ring keys in this tile
-    int nch, r, flags, pad; // chunks of the support, phase, kFirst/kLast/kCurrent/kEnd
+    int nch, r, flags, lo;  // chunks of the support, phase, kFirst/kLast/kCurrent/kEnd, and the
+                            // first tile row in the support (tensor-core kernel; rows < lo masked)
 };
 
 // ---------------------------------------------------------- elements ----
@@ -519,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                     mt.nch = nch;
                     mt.r = r;
                     mt.flags = (first ? kFirst : 0) | (it == ntiles - 1 ? kLast : 0) | (current ? kCurrent : 0);
-                    mt.pad = 0;
+                    mt.lo = 0;
                     meta_s[s] = mt;
                     unsigned char* st = dsmem + s * C::STAGE;
                     const uint32_t bytes = static_cast<uint32_t>(2 * nk * C::ROW + (first ? a.gq * C::ROW : 0) +
@@ -791,22 +792,33 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
 // S^T [16 keys x 8 heads] = K [16 x d] . Q^T [d x 8] is an mma.m16n8k16 chain
 // over d, and the output O^T [d x 8 heads] += V^T [d x 16 keys] . P^T
 // [16 keys x 8 heads] is one mma per 16 output dims. This kernel serves bf16
-// PBB steps with G = 8, or G = 4 and 6 with their query columns padded to 8 by
+// steps with G = 8, or G = 4 and 6 with their query columns padded to 8 by
 // zero rows (whose outputs are not written), and block sizes that are multiples
-// of twice the tile, so that no tile straddles the end of a ring. The step is
-// bound by HBM (each K/V byte feeds 2G flops), so the warp-level mma is enough to
-// keep up with the copies. It keeps the persistent producer /
-// consumer structure, work queue, merge and combine of decode_kernel; what
-// changes is how a consumer warp handles its 16 keys of a tile:
-//   - K and V tiles arrive by 2-D TMA copies with the 128-byte swizzle, one
-//     box per 64 columns, so ldmatrix reads them without bank conflicts;
-//   - A operands come from ldmatrix (K) and ldmatrix.trans (V^T), the Q^T
-//     operand from registers loaded once per item;
-//   - the scores (fp32) go through the same online softmax; the weights P are
-//     split into a bf16 high part and a bf16 low part (p = hi + lo to about
-//     2^-16) and both are multiplied, so P.V keeps fp32-level accuracy; the
-//     C fragment of S^T becomes the B fragment of P^T by an 8x8 movmatrix
-//     transpose.
+// of twice the tile. The step is bound by HBM (each K/V byte feeds 2G flops),
+// so the warp-level mma is enough to keep up with the copies. Work items, the
+// queue and the split are those of decode_kernel; per CTA:
+//   - a producer warp (one lane) streams tiles of TK ring slots by 2-D TMA
+//     copies with the 128-byte swizzle, one box per 64 columns. Tiles start at
+//     multiples of TK in slot order and B is a multiple of 2 TK, so no box
+//     crosses the end of a ring; a support whose run of slots starts or ends
+//     inside a tile (a sliding window's run starts at any slot) masks the
+//     tile's rows outside [lo, nk);
+//   - two consumer warps take 16 rows of every tile each: A operands from
+//     ldmatrix (K) and ldmatrix.trans (V^T), the Q^T operand from registers
+//     loaded once per item; the scores (fp32) go through the online softmax;
+//     the weights P are split into a bf16 high part and a bf16 low part
+//     (p = hi + lo to about 2^-16) and both are multiplied, so P.V keeps
+//     fp32-level accuracy; the C fragment of S^T becomes the B fragment of P^T
+//     by an 8x8 movmatrix transpose;
+//   - an epilogue warp ends the items. At an item's last tile the consumer
+//     warps leave their (max, sum, output) states in one of two shared-memory
+//     slots and go straight on to the next item's tiles; the epilogue warp
+//     merges the states (Eq. lse), writes `out` or the item's split partial
+//     and, for the last item of a split support to finish, fuses the partials
+//     in chunk order. The item ends (shared-memory merges, global writes and
+//     the L2 round trips of the split combine) thus overlap the streaming of
+//     the next item instead of stalling it, which is what makes splitting
+//     supports into chunks cheap enough to balance the persistent grid.
 #ifndef PBB_TC_CONSUMER_WARPS
 #define PBB_TC_CONSUMER_WARPS 2
 #endif
@@ -817,8 +829,11 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
 #define PBB_TC_MIN_CTAS 3
 #endif
 constexpr int kTcConsumers = PBB_TC_CONSUMER_WARPS;
-constexpr int kTcThreads = (kTcConsumers + 1) * 32;
+constexpr int kTcProducer = kTcConsumers;          // warp index of the producer
+constexpr int kTcEpilogue = kTcConsumers + 1;      // warp index of the epilogue warp
+constexpr int kTcThreads = (kTcConsumers + 2) * 32;
 constexpr int kTcStages = PBB_TC_STAGES;
+constexpr int kTcEpiSlots = 2;                     // item-end slots between consumers and epilogue
 
 template <int D>
 struct TcCfg {
@@ -833,13 +848,175 @@ struct TcCfg {
     static constexpr int KN_OFF = Q_OFF + G * ROW;         // k_new row (chunk 0)
     static constexpr int VN_OFF = KN_OFF + ROW;            // v_new row (chunk 0)
     static constexpr int STAGE = (VN_OFF + ROW + 1023) / 1024 * 1024;  // boxes stay 1024-aligned
-    static constexpr int MERGE = kTcConsumers * G * D * 4;
-    static constexpr int SMEM = kTcStages * STAGE + MERGE + 1024;      // + alignment slack
+    static constexpr int EPI_O = kTcConsumers * G * D * 4; // one slot: the consumer warps' outputs
+    static constexpr int SMEM = kTcStages * STAGE + kTcEpiSlots * EPI_O + 1024;  // + alignment slack
     static constexpr int KSTEPS = D / 16;                  // k-steps of the score chain
     static constexpr int MTILES = D / 16;                  // 16-dim tiles of the output
     static constexpr int PVD = D / 32;                     // dims per lane for the current token
     static_assert(BOX_BYTES % 1024 == 0, "swizzle atoms");
+    static_assert(D % 128 == 0 || D == 64, "head sizes");
 };
+
+// Wait for phase `parity` of `bar`, giving up when another warp of the CTA has aborted or after
+// kGuardNs. Returns false if it gave up.
+__device__ __forceinline__ bool mbar_wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag)
+{
+    if (mbar_test(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try(bar, parity)) {
+        if (*abort_flag) return false;
+        if (global_ns() - t0 > kGuardNs) return false;
+    }
+    return true;
+}
+
+// End of one work item, run by the 32 lanes of the epilogue warp: merge the NC consumer
+// warps' (max, sum, output) states of the item (Eq. lse), from ml [NC][G] and o [NC][G][D];
+// write `out` for an unsplit support, else the item's partial, and let the last item of the
+// (sequence, KV head) to finish fuse all partials in chunk order (so results do not depend on
+// scheduling). `o` serves as scratch for the combine weights afterwards.
+template <int G, int D, int NC>
+__device__ __forceinline__ void epilogue_item(const DecodeArgs& a, const TileMeta& mt, const float2* ml, float* o,
+                                              int lane)
+{
+    constexpr int V4 = D / 4;         // float4 per head row
+    constexpr int HPI = 32 / V4;      // head rows per warp iteration (1 at d = 128, 2 at d = 64)
+    const size_t head = static_cast<size_t>(mt.b) * a.Hkv + mt.kvh;
+    const bool split = mt.nch > 1;
+    const size_t part = split ? (head - a.whole) * a.nchunk + mt.chunk : 0;
+    const int c4 = lane % V4;
+    float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * a.gq) * D;
+#pragma unroll
+    for (int j0 = 0; j0 < G; j0 += HPI) {
+        const int j = j0 + lane / V4;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NC; ++w) M = fmaxf(M, ml[w * G + j].x);
+        float L = 0.f;
+        float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int w = 0; w < NC; ++w) {
+            const float2 mw = ml[w * G + j];
+            const float sc = exp2f(mw.x - M);
+            const float4 ow = reinterpret_cast<const float4*>(o + (w * G + j) * D)[c4];
+            L = fmaf(mw.y, sc, L);
+            O.x = fmaf(ow.x, sc, O.x);
+            O.y = fmaf(ow.y, sc, O.y);
+            O.z = fmaf(ow.z, sc, O.z);
+            O.w = fmaf(ow.w, sc, O.w);
+        }
+        if (!split) {
+            if (j < a.gq) {
+                const float inv = 1.f / L;
+                reinterpret_cast<float4*>(out_g + j * D)[c4] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+            }
+        } else {
+            reinterpret_cast<float4*>(a.part_o + (part * G + j) * D)[c4] = O;
+            if (c4 == 0) reinterpret_cast<float2*>(a.part_ml)[part * G + j] = make_float2(M, L);
+        }
+    }
+    if (!split) return;
+    // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
+    __threadfence();
+    __syncwarp();
+    int last = 0;
+    if (lane == 0) last = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
+    last = __shfl_sync(kFull, last, 0);
+    if (!last) return;
+    __threadfence();
+    const float* po = a.part_o + (head - a.whole) * a.nchunk * G * D;
+    const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + (head - a.whole) * a.nchunk * G;
+    const int nch = mt.nch;
+    if (nch * G <= NC * G * D) {
+        // weights e^(m_c - M) / L of every (chunk, head) into the slot's scratch: all (max, sum)
+        // pairs are loaded at once, then reduced across the lanes per head
+        float* wgt = o;  // [nch][G]
+        float Mh[G], Lh[G];
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            Mh[j] = -INFINITY;
+            Lh[j] = 0.f;
+        }
+        for (int c = lane; c < nch; c += 32) {
+#pragma unroll
+            for (int j = 0; j < G; ++j) Mh[j] = fmaxf(Mh[j], __ldcg(&pml[c * G + j]).x);
+        }
+#pragma unroll
+        for (int j = 0; j < G; ++j)
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) Mh[j] = fmaxf(Mh[j], __shfl_xor_sync(kFull, Mh[j], off));
+        for (int c = lane; c < nch; c += 32) {
+#pragma unroll
+            for (int j = 0; j < G; ++j) {
+                const float2 m2 = __ldcg(&pml[c * G + j]);
+                const float e = fast_exp2(m2.x - Mh[j]);
+                wgt[c * G + j] = e;
+                Lh[j] = fmaf(m2.y, e, Lh[j]);
+            }
+        }
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) Lh[j] += __shfl_xor_sync(kFull, Lh[j], off);
+            Lh[j] = 1.f / Lh[j];
+        }
+        __syncwarp();
+        // every lane owns float4 c4 of HPL head rows; per chunk, the loads of all its rows are in
+        // flight together (two chunks per iteration)
+        constexpr int HPL = G / HPI;
+        float4 acc[HPL];
+#pragma unroll
+        for (int x = 0; x < HPL; ++x) acc[x] = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int jl = lane / V4;  // head offset of this lane within a row group
+#pragma unroll 2
+        for (int c = 0; c < nch; ++c) {
+#pragma unroll
+            for (int x = 0; x < HPL; ++x) {
+                const int j = x * HPI + jl;
+                if (j < a.gq) {  // the real query heads
+                    const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
+                    const float w = wgt[c * G + j];
+                    acc[x].x = fmaf(p.x, w, acc[x].x);
+                    acc[x].y = fmaf(p.y, w, acc[x].y);
+                    acc[x].z = fmaf(p.z, w, acc[x].z);
+                    acc[x].w = fmaf(p.w, w, acc[x].w);
+                }
+            }
+        }
+#pragma unroll
+        for (int x = 0; x < HPL; ++x) {
+            const int j = x * HPI + jl;
+            if (j < a.gq) {
+                const float inv = (HPI == 1 || jl == 0) ? Lh[x * HPI] : Lh[x * HPI + HPI - 1];
+                reinterpret_cast<float4*>(out_g + j * D)[c4] =
+                    make_float4(acc[x].x * inv, acc[x].y * inv, acc[x].z * inv, acc[x].w * inv);
+            }
+        }
+    } else {
+        for (int j0 = 0; j0 < a.gq; j0 += HPI) {
+            const int j = j0 + lane / V4;
+            if (j < a.gq) {
+                float M = -INFINITY;
+                for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+                float L = 0.f;
+                float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int c = 0; c < nch; ++c) {
+                    const float2 m2 = __ldcg(&pml[c * G + j]);
+                    const float sc = fast_exp2(m2.x - M);
+                    const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
+                    L = fmaf(m2.y, sc, L);
+                    O.x = fmaf(p.x, sc, O.x);
+                    O.y = fmaf(p.y, sc, O.y);
+                    O.z = fmaf(p.z, sc, O.z);
+                    O.w = fmaf(p.w, sc, O.w);
+                }
+                const float inv = 1.f / L;
+                reinterpret_cast<float4*>(out_g + j * D)[c4] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+            }
+        }
+    }
+    if (lane == 0) a.counters[head] = 0;
+}
 
 template <int D>
 __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
@@ -848,18 +1025,20 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
 {
     using C = TcCfg<D>;
     constexpr int G = C::G;
+    constexpr int TK = C::TK;
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t full_bar[kTcStages];
     __shared__ __align__(8) uint64_t empty_bar[kTcStages];
+    __shared__ __align__(8) uint64_t epi_full[kTcEpiSlots];   // consumers -> epilogue (count kTcConsumers)
+    __shared__ __align__(8) uint64_t epi_empty[kTcEpiSlots];  // epilogue -> consumers (count 1)
     __shared__ TileMeta meta_s[kTcStages];
-    __shared__ float2 ml_s[kTcConsumers][G];
-    __shared__ unsigned sbar_count;
-    __shared__ volatile unsigned sbar_gen;
+    __shared__ TileMeta epi_meta[kTcEpiSlots];
+    __shared__ float2 epi_ml[kTcEpiSlots][kTcConsumers][G];
     __shared__ volatile int abort_s;
-    __shared__ int last_s;
     __shared__ int issued_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
         (reinterpret_cast<uintptr_t>(dsmem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+    float* epi_o = reinterpret_cast<float*>(dsmem + kTcStages * C::STAGE);  // [kTcEpiSlots][kTcConsumers][G][D]
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) {
@@ -868,9 +1047,12 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             mbar_init(&full_bar[s], 1);
             mbar_init(&empty_bar[s], kTcConsumers);
         }
+#pragma unroll
+        for (int s = 0; s < kTcEpiSlots; ++s) {
+            mbar_init(&epi_full[s], kTcConsumers);
+            mbar_init(&epi_empty[s], 1);
+        }
         fence_mbar_init();
-        sbar_count = 0;
-        sbar_gen = 0;
         abort_s = 0;
         issued_s = 0;
     }
@@ -883,7 +1065,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
     }
     __syncthreads();
 
-    if (warp == kTcConsumers) {
+    if (warp == kTcProducer) {
         // ================= producer: one lane =================
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&kmap)) : "memory");
@@ -908,20 +1090,22 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
                     continue;
                 }
-                const int B = a.B, h = B >> 1;
-                const int blk = t / B;
-                const int r = t - blk * B;
-                const bool bridge = (blk > 0) && (r < h);
-                const int n = bridge ? h + r : r;  // ring keys of the support (positions a(t) .. t-1)
-                const int base = bridge ? h : 0;   // slot of ring key 0
+                const int B = a.B;
+                int r, n, base;
+                support_keys(t, B, a.window, r, n, base);
+                // the run of n slots from `base`, in tile-aligned key space: tiles start at slot
+                // multiples of TK, the run occupies aligned keys [lo0, lo0 + n)
+                const int lo0 = n > 0 ? base % TK : 0;
+                const int tbase = base - lo0;         // slot of aligned key 0
+                const int span = lo0 + n;             // aligned keys up to the end of the run
                 const bool whole = pair < a.whole;
-                const int csize = whole ? max(n, 1) : a.chunk;  // keys per chunk of this support
-                const int nch = n > 0 ? (n + csize - 1) / csize : 1;
+                const int csize = whole ? max(span, 1) : a.chunk;  // aligned keys per chunk (tiles)
+                const int nch = span > 0 ? (span + csize - 1) / csize : 1;
                 if (chunk >= nch) continue;
                 const int i0 = chunk * csize;
-                const int i1 = min(i0 + csize, n);
+                const int i1 = min(i0 + csize, span);
                 const int nkeys = max(i1 - i0, 0);
-                const int ntiles = nkeys > 0 ? (nkeys + C::TK - 1) / C::TK : 1;
+                const int ntiles = nkeys > 0 ? (nkeys + TK - 1) / TK : 1;
                 const int head = b * a.Hkv + kvh;
                 for (int it = 0; it < ntiles; ++it, ++seq) {
                     const int s = seq % kTcStages;
@@ -934,8 +1118,9 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                         ok = false;
                         break;
                     }
-                    const int k0 = i0 + it * C::TK;
-                    const int nk = max(min(C::TK, i1 - k0), 0);
+                    const int k0 = i0 + it * TK;                  // aligned key of the tile's row 0
+                    const int nk = max(min(TK, i1 - k0), 0);      // rows [lo, nk) are in the run
+                    const int lo = min(max(lo0 - k0, 0), TK);
                     const bool first = it == 0;
                     const bool current = first && chunk == 0;
                     TileMeta mt;
@@ -946,17 +1131,18 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     mt.nch = nch;
                     mt.r = r;
                     mt.flags = (first ? kFirst : 0) | (it == ntiles - 1 ? kLast : 0) | (current ? kCurrent : 0);
-                    mt.pad = 0;
+                    mt.lo = lo;
                     meta_s[s] = mt;
                     unsigned char* st = dsmem + s * C::STAGE;
-                    const uint32_t bytes = static_cast<uint32_t>((nk > 0 ? 2 * C::BOXES * C::BOX_BYTES : 0) +
+                    const bool rows = nk > lo;
+                    const uint32_t bytes = static_cast<uint32_t>((rows ? 2 * C::BOXES * C::BOX_BYTES : 0) +
                                                                  (first ? a.gq * C::ROW : 0) + (current ? 2 * C::ROW : 0));
                     fence_proxy_async();
                     mbar_expect_tx(&full_bar[s], bytes);
-                    if (nk > 0) {
-                        // whole boxes of TK rows: the tile never crosses slot B-1 (B is a multiple of
-                        // 2*TK and tiles start at multiples of TK), rows past the support are masked
-                        int slot = base + k0;
+                    if (rows) {
+                        // whole boxes of TK rows at a slot multiple of TK: the box never crosses
+                        // slot B-1 (B is a multiple of 2*TK); rows outside [lo, nk) are masked
+                        int slot = tbase + k0;
                         if (slot >= B) slot -= B;
                         const int y = head * B + slot;
 #pragma unroll
@@ -997,15 +1183,32 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             }
             issued_s = seq;
         }
+    } else if (warp == kTcEpilogue) {
+        // ================= epilogue: ends the items the consumers hand over =================
+        for (int k = 0;; ++k) {
+            const int es = k % kTcEpiSlots;
+            if (!mbar_wait_or_abort(&epi_full[es], static_cast<uint32_t>((k / kTcEpiSlots) & 1), &abort_s)) {
+                if (!abort_s) {
+                    abort_s = 1;
+                    atomicCAS(&g_status, kDevOk, kDevTimeout);
+                }
+                break;
+            }
+            const TileMeta mt = epi_meta[es];
+            if (mt.flags & kEnd) break;
+            epilogue_item<G, D, kTcConsumers>(a, mt, &epi_ml[es][0][0], epi_o + es * (kTcConsumers * G * D), lane);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&epi_empty[es]);
+        }
     } else {
         // ================= consumers =================
         const int g = lane >> 2, tig = lane & 3;  // fragment row group and thread in group
         const float qscale = 1.4426950408889634f * rsqrtf(static_cast<float>(D));
-        float* merge_o = reinterpret_cast<float*>(dsmem + kTcStages * C::STAGE);  // [kTcConsumers][G][D]
         uint32_t qb[C::KSTEPS][2];  // Q^T B fragments: head g, dims 16kk + 2tig (+8)
         float o[C::MTILES][4];      // O^T C fragments: dims 16mt + g (+8), heads 2tig, 2tig+1
         float m0 = -INFINITY, m1 = -INFINITY;  // running max of heads 2tig, 2tig+1 (log2 domain)
         float l0 = 0.f, l1 = 0.f;               // this lane's share of their running sums
+        int epi_seq = 0;                         // items handed to the epilogue warp
 #pragma unroll
         for (int kk = 0; kk < C::KSTEPS; ++kk) qb[kk][0] = qb[kk][1] = 0u;
 #pragma unroll
@@ -1027,8 +1230,24 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                 break;
             }
             const TileMeta mt = meta_s[s];
-            if (mt.flags & kEnd) break;
             if (abort_s) break;
+            if (mt.flags & kEnd) {
+                // hand the end marker to the epilogue warp through the next slot
+                const int es = epi_seq % kTcEpiSlots;
+                if (epi_seq >= kTcEpiSlots &&
+                    !mbar_wait_or_abort(&epi_empty[es], static_cast<uint32_t>((epi_seq / kTcEpiSlots - 1) & 1),
+                                        &abort_s)) {
+                    if (!abort_s) {
+                        abort_s = 1;
+                        atomicCAS(&g_status, kDevOk, kDevTimeout);
+                    }
+                    break;
+                }
+                if (warp == 0 && lane == 0) epi_meta[es] = mt;
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&epi_full[es]);
+                break;
+            }
             const unsigned char* st = dsmem + s * C::STAGE;
             const size_t head = static_cast<size_t>(mt.b) * a.Hkv + mt.kvh;
 
@@ -1086,8 +1305,10 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                 }
             }
 
-            const int nkw = min(max(mt.nk - warp * 16, 0), 16);  // this warp's keys: rows 16*warp ..
-            if (nkw > 0) {
+            // this warp's rows 16*warp .. 16*warp+15 of the tile; rows outside [lo, nk) are masked
+            const int row0 = 16 * warp;
+            const int lo = mt.lo;
+            if (row0 + 16 > lo && row0 < mt.nk) {
                 const uint32_t kbase = smem_addr(st + C::K_OFF);
                 const uint32_t vbase = smem_addr(st + C::V_OFF);
                 // ---- scores S^T [16 keys x 8 heads]: two independent mma chains (even and odd
@@ -1097,7 +1318,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
 #pragma unroll
                 for (int kk = 0; kk < C::KSTEPS; ++kk) {
                     const int chunk16 = 2 * kk + chA;  // 16-byte chunk of the 256-byte (or 128-byte) row
-                    const int row = 16 * warp + rowA;
+                    const int row = row0 + rowA;
                     uint32_t af[4];
                     ldmatrix_x4(af, kbase + (chunk16 >> 3) * C::BOX_BYTES + swz(row, chunk16 & 7));
                     if (kk & 1)
@@ -1108,7 +1329,8 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
 #pragma unroll
                 for (int x = 0; x < 4; ++x) c[x] += c2[x];
                 // keys g and g+8 of this warp's block; heads 2tig and 2tig+1
-                const bool va = g < nkw, vb = g + 8 < nkw;
+                const bool va = (row0 + g >= lo) && (row0 + g < mt.nk);
+                const bool vb = (row0 + g + 8 >= lo) && (row0 + g + 8 < mt.nk);
                 const float z0 = va ? c[0] * qscale : -INFINITY;
                 const float z1 = va ? c[1] * qscale : -INFINITY;
                 const float z2 = vb ? c[2] * qscale : -INFINITY;
@@ -1148,7 +1370,7 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
 #pragma unroll
                 for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
                     const int chunk16 = 2 * mt_ + chV;
-                    const int row = 16 * warp + rowV;
+                    const int row = row0 + rowV;
                     uint32_t af[4];
                     ldmatrix_x4_trans(af, vbase + (chunk16 >> 3) * C::BOX_BYTES + swz(row, chunk16 & 7));
                     mma_bf16_16816(o[mt_], af, bh0, bh1);
@@ -1159,7 +1381,17 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             if (lane == 0) mbar_arrive(&empty_bar[s]);
             if (!(mt.flags & kLast)) continue;
 
-            // ---- end of the item: this warp's (max, sum, output) into the merge buffers
+            // ---- end of the item: this warp's (max, sum, output) into a free epilogue slot
+            const int es = epi_seq % kTcEpiSlots;
+            if (epi_seq >= kTcEpiSlots &&
+                !mbar_wait_or_abort(&epi_empty[es], static_cast<uint32_t>((epi_seq / kTcEpiSlots - 1) & 1),
+                                    &abort_s)) {
+                if (!abort_s) {
+                    abort_s = 1;
+                    atomicCAS(&g_status, kDevOk, kDevTimeout);
+                }
+                break;
+            }
             {
                 float s0 = l0, s1 = l1;
 #pragma unroll
@@ -1168,25 +1400,22 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     s1 += __shfl_xor_sync(kFull, s1, off);
                 }
                 if (g == 0) {
-                    ml_s[warp][2 * tig] = make_float2(m0, s0);
-                    ml_s[warp][2 * tig + 1] = make_float2(m1, s1);
+                    epi_ml[es][warp][2 * tig] = make_float2(m0, s0);
+                    epi_ml[es][warp][2 * tig + 1] = make_float2(m1, s1);
                 }
             }
+            float* ow = epi_o + es * (kTcConsumers * G * D) + (warp * G) * D;
 #pragma unroll
             for (int mt_ = 0; mt_ < C::MTILES; ++mt_) {
-                float* ow = merge_o + (warp * G) * D;
                 ow[(2 * tig) * D + 16 * mt_ + g] = o[mt_][0];
                 ow[(2 * tig + 1) * D + 16 * mt_ + g] = o[mt_][1];
                 ow[(2 * tig) * D + 16 * mt_ + g + 8] = o[mt_][2];
                 ow[(2 * tig + 1) * D + 16 * mt_ + g + 8] = o[mt_][3];
             }
-            const bool ok = finish_item<G, D, kTcConsumers>(a, mt, head, &ml_s[0][0], merge_o, &sbar_count,
-                                                            &sbar_gen, &last_s, tid, lane, warp);
-            if (!ok) {
-                abort_s = 1;
-                atomicCAS(&g_status, kDevOk, kDevTimeout);
-                break;
-            }
+            if (warp == 0 && lane == 0) epi_meta[es] = mt;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&epi_full[es]);
+            ++epi_seq;
         }
     }
     __syncthreads();
@@ -1383,19 +1612,23 @@ int device_sms()
 #ifndef PBB_TC_PAD_MIN_FILL
 #define PBB_TC_PAD_MIN_FILL 1
 #endif
+// Sliding-window steps on the tensor-core kernel (0 keeps them on the CUDA cores).
+#ifndef PBB_TC_WINDOWS
+#define PBB_TC_WINDOWS 1
+#endif
 
-// Whether a step of this shape runs the tensor-core kernel, before the chunk check: a bf16 PBB
-// step (its tiles start at multiples of the tile in slot order, slots 0 and h, as whole TMA
-// boxes need; a window's run starts at any slot), GQA group 8 (or 4 or 6, padded), d 64 or
-// 128, block a multiple of two tiles (no tile straddles the ring end), row coordinates within
-// int32.
+// Whether a step of this shape runs the tensor-core kernel, before the chunk check: a bf16 step
+// (PBB or window; tiles start at slot multiples of the tile, and rows of a tile outside the
+// support are masked), GQA group 8 (or 4 or 6, padded), d 64 or 128, block a multiple of two
+// tiles (no tile straddles the ring end), row coordinates within int32.
 std::atomic<int> g_kernel_choice{PBB_KERNEL_AUTO};
 
 bool tc_shape(int batch, int Hkv, int d, int B, int elem_bytes, int group, int window)
 {
     const int choice = g_kernel_choice.load();
     if (choice == PBB_KERNEL_CUDA_CORES) return false;
-    if (window != 0 || elem_bytes != 2 || !tc_group(group) || (d != 64 && d != 128)) return false;
+    if (elem_bytes != 2 || !tc_group(group) || (d != 64 && d != 128)) return false;
+    if (window != 0 && !PBB_TC_WINDOWS) return false;
     if (B % (32 * kTcConsumers) != 0 || tensor_map_encoder() == nullptr) return false;
     const unsigned long long rows = static_cast<unsigned long long>(batch) * Hkv * B;
     if (rows >= (1ull << 31)) return false;

@@ -235,10 +235,10 @@ def test_graph_capture_matches_eager(chunk_keys):
         pbb.advance_positions(pos)
     torch.cuda.synchronize()
 
-    pbb.reserve_workspace(w.batch, w.Hq, w.Hkv, w.d, w.B)
+    s = torch.cuda.Stream()
+    pbb.reserve_workspace(w.batch, w.Hq, w.Hkv, w.d, w.B, stream=s)  # the capture stream's workspace
     pos2, kr2, vr2 = fresh()
     out_g = torch.empty_like(out_e)
-    s = torch.cuda.Stream()
     torch.cuda.synchronize()
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=s):

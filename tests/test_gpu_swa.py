@@ -178,3 +178,54 @@ def test_full_size_window_B(batch, B):
     finally:
         pbb.set_chunk_keys(prev)
     assert pbb.get_device_status() == pbb.PBB_OK
+
+
+@pytest.fixture
+def tensor_cores():
+    prev = pbb.set_kernel("tensor_cores")
+    yield
+    pbb.set_kernel(prev)
+
+
+@pytest.mark.parametrize("group,d", [(4, 128), (8, 128), (6, 64), (8, 64)])
+@pytest.mark.parametrize("window", [1, 2, 33, 127, 128])
+def test_windows_on_tensor_cores(chunk_keys, tensor_cores, group, d, window):
+    """Window steps on the tensor-core kernel (B = 128, a multiple of two tiles). A window's
+    run of ring slots starts at any slot and may wrap past slot B-1, while tiles start at slot
+    multiples of 32: the first and last tiles of a run are masked outside it, and the slot
+    being written (position t-B, outside the window) is never read. Ragged prefilled rings
+    from positions near 0 (short runs in the first block) up to a few blocks; the library's
+    plan, then 32-key chunks (every support split, so the epilogue warp's combine runs)."""
+    w = inputs.Workload(f"swa_tc_g{group}_d{d}_w{window}", batch=3, Hq=2 * group, Hkv=2, d=d, B=128,
+                        dtype="bf16", steps=40, t0_lo=0, t0_hi=700, seed=400 + 7 * group + d + window)
+    chunk_keys(0)
+    run_and_check(w, window=window)
+    chunk_keys(32)
+    run_and_check(w, window=window, check_every=3)
+
+
+def test_window_on_both_kernels_against_the_oracle(chunk_keys):
+    """The same window step on both kernels (which round P differently: fp32 weights on the
+    CUDA cores, a bf16 high and low part on the tensor cores), each against the oracle."""
+    chunk_keys(0)
+    w = inputs.Workload("swa_tc_vs_cc", batch=6, Hq=32, Hkv=4, d=128, B=256, dtype="bf16", steps=1,
+                        t0_lo=0, t0_hi=3000, seed=77)
+    window = 200
+    dev = torch.device("cuda")
+    t0 = inputs.start_positions(w)
+    wk, wv = inputs.history_window(w, t0)
+    q, k, v = inputs.step_inputs(w, 0)
+    t = t0.numpy()
+    ref = oracle.attend_window(q, torch.cat([wk, k.unsqueeze(2)], 2), torch.cat([wv, v.unsqueeze(2)], 2),
+                               s0=t - w.B, t=t, w=window)
+    for kernel in ("tensor_cores", "cuda_cores"):
+        prev = pbb.set_kernel(kernel)
+        try:
+            pos = t0.to(torch.int32).to(dev)
+            kr = torch.zeros((w.batch, w.Hkv, w.B, w.d), dtype=torch.bfloat16, device=dev)
+            vr = torch.zeros_like(kr)
+            pbb.ring_prefill(wk.to(dev), wv.to(dev), pos, kr, vr)
+            out = pbb.swa_decode_step(q.to(dev), k.to(dev), v.to(dev), kr, vr, pos, window=window).cpu()
+        finally:
+            pbb.set_kernel(prev)
+        check_close(out, ref, "bf16", kernel)
