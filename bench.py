@@ -871,12 +871,10 @@ def run_ours(args):
         achieved = res["launch_bytes_mean"] / (res["kernel_ms_mean"] / 1e3) / 1e9
         key = w.name if window is None else f"{w.name}_swa"
         traffic = recorded_traffic(key, res["launch_bytes_mean"])
-        if window is None:
-            kernel = ("decode_kernel_tc<%d>" % w.d
-                      if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w)) == "tensor_cores"
-                      else "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group))
-        else:
-            kernel = "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group)
+        # window steps follow the same kernel choice as PBB steps of the shape
+        kernel = ("decode_kernel_tc<%d>" % w.d
+                  if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w)) == "tensor_cores"
+                  else "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group))
         line = {
             "metric": METRIC if window is None else METRIC_SWA, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,

@@ -115,16 +115,23 @@ int sm_count(int dev)
 // supports paid for long supports (see below).
 //
 // The tensor-core kernel ends items on a separate epilogue warp, so a split
-// item costs its consumers nothing; its plan cuts every support into chunks
-// of about (supports x mean support) / (PBB_TC_ROUNDS x G) keys, so the
-// persistent grid balances on small items and the step does not end on a few
-// CTAs streaming long supports alone. A positive pbb_set_chunk_keys override
-// splits every support into chunks of that many keys, for either kernel.
+// item costs its consumers little; its plan cuts every support into chunks of
+// about (supports x mean support) / (PBB_TC_ROUNDS x G) keys, and at least
+// PBB_TC_MIN_CHUNK_KB of K+V, so the persistent grid balances on small items and
+// the step does not end on a few CTAs streaming long supports alone. A positive
+// pbb_set_chunk_keys override splits every support into chunks of that many
+// keys, for either kernel.
 #ifndef PBB_MIN_CHUNK_KB
 #define PBB_MIN_CHUNK_KB 64
 #endif
 #ifndef PBB_TC_ROUNDS
 #define PBB_TC_ROUNDS 4
+#endif
+// Smallest chunk of the tensor-core plan, in KiB of K+V: smaller chunks cost more in item
+// starts and split combines than they gain in balance (measured on GB300 at batch 64: 448 keys
+// of d 128 beat 128-288 keys at B 512 and B 1024).
+#ifndef PBB_TC_MIN_CHUNK_KB
+#define PBB_TC_MIN_CHUNK_KB 224
 #endif
 
 int min_split_keys(int d, int elem, int tile)
@@ -166,7 +173,7 @@ SplitPlan plan_split(int batch, int Hkv, int d, int B, int elem, int group, int 
         return sp;
     };
     auto chunks_of = [&](long long chunk) {
-        const int min_keys = min_split_keys(d, elem, tile);
+        const int min_keys = tc ? (PBB_TC_MIN_CHUNK_KB * 1024) / (2 * d * elem) : min_split_keys(d, elem, tile);
         if (chunk < min_keys) chunk = min_keys;
         chunk = static_cast<long long>(round_up(static_cast<size_t>(chunk), static_cast<size_t>(tile)));
         if (chunk >= max_keys) return whole_plan();

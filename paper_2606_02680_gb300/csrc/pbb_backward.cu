@@ -20,9 +20,9 @@
 // (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion through
 // tcgen05.commit on mbarriers) and elementwise warpgroups; thread r of a warpgroup owns
 // TMEM lane r. The long shape runs one CTA per SM with two elementwise warpgroups that
-// take alternate tiles (the scores of tile g sit in TMEM buffer g % 2), so two tiles'
-// exponentials run at once; the short shape (short supports, d = 64) runs two CTAs per
-// SM with one warpgroup each, on half the TMEM. P, dS and their transposes are rounded
+// share every tile, each on half of its columns (the scores of tile g sit in TMEM buffer
+// g % 2, so tile g+1's products run while tile g's exponentials do); the short shape
+// (short supports, d = 64) runs two CTAs per SM with one warpgroup each, on half the TMEM. P, dS and their transposes are rounded
 // to bf16 and written back over the scores in tensor memory as the A operands of the
 // next products. Tiles with no masked entry take a packed path (two columns per
 // ffma2/fadd2/fmul2, rounded like the scalar operations, so the results are the same
@@ -105,13 +105,37 @@ __global__ void delta_kernel(const __nv_bfloat16* __restrict__ out, const __nv_b
 }
 
 // ------------------------------------------------------------------ dQ ----
-// Items of 128 query rows (G heads x QT positions), key tiles of NK. TMEM: S and dP,
-// two buffers each (dS is written back over S as bf16 pairs, the A operand of
-// dQ += dS K), and one or two dQ accumulators alternating between items.
+// Items of 128 query rows (G heads x QT positions), key tiles of NK. TMEM: S in two
+// buffers (dS is written back over S as bf16 pairs, the A operand of dQ += dS K), dP in
+// two buffers, or in one for 128-key tiles, and one or two dQ accumulators alternating
+// between items. With one dP buffer the elementwise warpgroups release it as soon as
+// they hold the tile's dP in registers (dp_free), and the MMA thread issues the next
+// tile's dP then; the next tile's S is issued earlier still.
 // Columns of S and dP the elementwise threads load before each wait (32 or 64).
 #ifndef PBB_BWD_Q_QC
 #define PBB_BWD_Q_QC 64
 #endif
+
+// With two elementwise warpgroups: both share every tile, warpgroup w taking columns
+// [w N/2, (w+1) N/2) of its N score columns (1), or they take alternate tiles (0). Sharing keeps
+// the tensor pipe busy: with alternate tiles, tile g+2's scores can only be issued after tile
+// g's gradient products, which wait for tile g's exponentials, so both warpgroups went idle
+// together while the pipe drained; with shared tiles, tile g+1's scores are ready when the
+// warpgroups finish tile g.
+#ifndef PBB_BWD_SPLIT_COLS
+#define PBB_BWD_SPLIT_COLS 1
+#endif
+
+// TMEM column of the bf16-pair (P, dS or their transposes) operand for k-step kk (16 rows of
+// the reduction) in a score buffer of N columns. Each warpgroup writes its pairs over the
+// first columns it read itself: with split columns, warpgroup w's N/4 pair columns start at
+// column w N/2; otherwise pairs of k-step kk sit at column 8 kk.
+template <int N, bool SPLIT>
+__host__ __device__ constexpr uint32_t pair_col(int kk)
+{
+    return SPLIT ? static_cast<uint32_t>((kk / (N / 32)) * (N / 2) + 8 * (kk % (N / 32)))
+                 : static_cast<uint32_t>(8 * kk);
+}
 
 // Tiles with no masked entry take a packed path (1) or the masked one (0): PBB_BWD_Q_INNER for
 // the dQ pass (every shape), PBB_BWD_KV_INNER for the dK/dV pass (one-CTA shapes; the two-CTA
@@ -138,9 +162,13 @@ struct BqCfg {
     static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - KV_OFF) / KV_STAGE;
     static constexpr int STAGES = STAGE_ROOM < 4 ? STAGE_ROOM : 4;
     static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
-    static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = 4 * NK;
+    static constexpr int DPBUF = NK == 128 ? 1 : 2;            // dP buffers
+    static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = T_DP + DPBUF * NK;
     static constexpr int OBUF = T_DQ + 2 * D <= TMEM_COLS ? 2 : 1;
     static constexpr bool INNER = PBB_BWD_Q_INNER;
+    static constexpr bool SPLIT = WGS == 2 && PBB_BWD_SPLIT_COLS;
+    static_assert(DPBUF == 2 || (PBB_BWD_Q_QC >= NK / (SPLIT ? 2 : 1)),
+                  "one dP buffer: each warpgroup loads its columns of a tile before one wait");
     static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_DQ + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
@@ -178,7 +206,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t q_full, q_empty, done_bar;
     __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
-    __shared__ __align__(8) uint64_t s_full[2], ds_full[2], item_done[2], o_free[2];
+    __shared__ __align__(8) uint64_t s_full[2], ds_full[2], item_done[2], o_free[2], dp_free;
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
@@ -197,10 +225,11 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&ds_full[b], 128);        // the warpgroup that owns buffer b
+            mbar_init(&ds_full[b], C::SPLIT ? 256 : 128);  // the warpgroups that handle buffer b
             mbar_init(&item_done[b], 1);
             mbar_init(&o_free[b], 128 * WGS);   // every warpgroup reads its share of the dQ row
         }
+        mbar_init(&dp_free, C::SPLIT ? 256 : 128);  // one dP buffer: the warpgroups of a tile hold it
         fence_mbar_init();
         abort_s = 0;
     }
@@ -272,18 +301,35 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             const uint32_t kv_base = smem_addr(dsmem + C::KV_OFF);
             uint32_t gt = 0, ic = 0;
             bool ok = true, issued_any = false;
-            auto issue_sdp = [&](uint32_t g) {  // S = Q K^T and dP = dO V^T into buffer g % 2
-                const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE, vb = kb + C::BOXES * C::KBOX;
+            // S = Q K^T into buffer g % 2, and dP = dO V^T into buffer g % DPBUF; the commit of
+            // s_full covers both
+            auto issue_s = [&](uint32_t g) {
+                const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * C::QBOX + (kk & 3) * 32;
                     const uint32_t koff = (kk >> 2) * C::KBOX + (kk & 3) * 32;
                     umma_bf16(tmem + C::T_S + (g & 1u) * NK, umma_desc_sw128(q_base + off, 16, 1024),
                               umma_desc_sw128(kb + koff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
-                    umma_bf16(tmem + C::T_DP + (g & 1u) * NK, umma_desc_sw128(do_base + off, 16, 1024),
+                }
+            };
+            auto issue_dp = [&](uint32_t g) {
+                const uint32_t vb = kv_base + (g % STAGES) * C::KV_STAGE + C::BOXES * C::KBOX;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * C::QBOX + (kk & 3) * 32;
+                    const uint32_t koff = (kk >> 2) * C::KBOX + (kk & 3) * 32;
+                    umma_bf16(tmem + C::T_DP + (g % C::DPBUF) * NK, umma_desc_sw128(do_base + off, 16, 1024),
                               umma_desc_sw128(vb + koff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
                 }
                 umma_commit(&s_full[g & 1u]);
+            };
+            // with one dP buffer, tile g's dP goes in once the warpgroups hold tile g-1's
+            auto dp_ready = [&](uint32_t g) {
+                if (C::DPBUF == 2 || g == 0) return true;
+                if (!mbar_wait(&dp_free, (g - 1) & 1u, limit)) return false;
+                tmem_fence_after();
+                return true;
             };
             for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
@@ -293,8 +339,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     break;
                 }
                 tmem_fence_after();
-                issue_sdp(gt);
+                issue_s(gt);
                 issued_any = true;
+                if (!dp_ready(gt)) {
+                    ok = false;
+                    break;
+                }
+                issue_dp(gt);
                 if (it.ntiles == 1) umma_commit(&q_empty);
                 for (int j = 0; j < it.ntiles; ++j) {
                     const uint32_t g = gt + j;
@@ -304,7 +355,12 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                             break;
                         }
                         tmem_fence_after();
-                        issue_sdp(g + 1);
+                        issue_s(g + 1);
+                        if (!dp_ready(g + 1)) {
+                            ok = false;
+                            break;
+                        }
+                        issue_dp(g + 1);
                         if (j + 2 == it.ntiles) umma_commit(&q_empty);  // the item's last read of Q and dO
                     }
                     if (!mbar_wait(&ds_full[g & 1u], (g >> 1) & 1u, limit) ||
@@ -317,7 +373,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
 #pragma unroll
                     for (int kk = 0; kk < NK / 16; ++kk)
-                        umma_bf16_tmem_a(tmem + C::T_DQ + ob * D, tmem + C::T_S + (g & 1u) * NK + 8 * kk,
+                        umma_bf16_tmem_a(tmem + C::T_DQ + ob * D, tmem + C::T_S + (g & 1u) * NK + pair_col<NK, C::SPLIT>(kk),
                                          umma_desc_sw128(kb + kk * 2048, C::KBOX, 1024), idesc_q,
                                          (j > 0 || kk > 0) ? 1u : 0u);
                     umma_commit(&kv_empty[g % STAGES]);
@@ -355,7 +411,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             const float l2 = valid ? a.lse[row] * kLog2e : 0.f, dr = valid ? a.delta[row] : 0.f;
             for (int j = 0; j < it.ntiles; ++j) {
                 const uint32_t g = gt + j;
-                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
+                if (WGS == 2 && !C::SPLIT && static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -366,21 +422,28 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 // every key of the tile in every valid row's support: the packed path
                 const bool inner = C::INNER && !edge && __all_sync(kFull, valid);
                 // QC columns at a time (all their loads before one wait): their dS (QC/2
-                // bf16-pair columns) goes over columns already read
-                constexpr int QC = PBB_BWD_Q_QC < NK ? PBB_BWD_Q_QC : NK;
+                // bf16-pair columns) goes over columns already read; with split columns this
+                // warpgroup takes columns [wg NK/2, (wg+1) NK/2)
+                constexpr int NW = C::SPLIT ? NK / 2 : NK;  // this warpgroup's columns of the tile
+                constexpr int QC = PBB_BWD_Q_QC < NW ? PBB_BWD_Q_QC : NW;
+                const int col0 = C::SPLIT ? wg * NW : 0;
 #pragma unroll
-                for (int c = 0; c < NK / QC; ++c) {
+                for (int c = 0; c < NW / QC; ++c) {
                     uint32_t v1[QC], v2[QC];
 #pragma unroll
                     for (int h32 = 0; h32 < QC / 32; ++h32) {
                         uint32_t* a1 = v1 + 32 * h32;
                         uint32_t* a2 = v2 + 32 * h32;
-                        tmem_ld32(lane_base + C::T_S + (g & 1u) * NK + QC * c + 32 * h32,
+                        tmem_ld32(lane_base + C::T_S + (g & 1u) * NK + col0 + QC * c + 32 * h32,
                                   *reinterpret_cast<uint32_t(*)[32]>(a1));
-                        tmem_ld32(lane_base + C::T_DP + (g & 1u) * NK + QC * c + 32 * h32,
+                        tmem_ld32(lane_base + C::T_DP + (g % C::DPBUF) * NK + col0 + QC * c + 32 * h32,
                                   *reinterpret_cast<uint32_t(*)[32]>(a2));
                     }
                     tmem_wait_ld();
+                    if constexpr (C::DPBUF == 1) {  // this warpgroup's dP of the tile is in registers
+                        tmem_fence_before();
+                        mbar_arrive(&dp_free);
+                    }
                     uint32_t pk[QC / 2];
                     if (inner) {
 #pragma unroll
@@ -400,7 +463,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                             float e[2];
 #pragma unroll
                             for (int y = 0; y < 2; ++y) {
-                                const int key = key0 + QC * c + 2 * x + y;
+                                const int key = key0 + col0 + QC * c + 2 * x + y;
                                 const bool vis = valid && (!edge || (key >= as && key <= t));
                                 const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[2 * x + y]), sc2, -l2)) : 0.f;
                                 e[y] = p * (__uint_as_float(v2[2 * x + y]) - dr);
@@ -410,7 +473,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     }
 #pragma unroll
                     for (int h16 = 0; h16 < QC / 32; ++h16)
-                        tmem_st16(lane_base + C::T_S + (g & 1u) * NK + (QC / 2) * c + 16 * h16,
+                        tmem_st16(lane_base + C::T_S + (g & 1u) * NK + col0 + (QC / 2) * c + 16 * h16,
                                   *reinterpret_cast<const uint32_t(*)[16]>(pk + 16 * h16));
                 }
                 tmem_wait_st();
@@ -477,6 +540,7 @@ struct BkvCfg {
     // per column (lse2, D, t, a(t)) as a float4 (one load per entry on the masked path); with
     // the packed path, (-lse2, -D) again as a float2 array (one load per column pair)
     static constexpr bool INNER = PBB_BWD_KV_INNER && CTAS == 1;
+    static constexpr bool SPLIT = WGS == 2 && PBB_BWD_SPLIT_COLS;
     static constexpr int META = NQ * (INNER ? 24 : 16);
     static constexpr int STAGE = (2 * BOXES * QBOX + META + 1023) / 1024 * 1024;  // Q, dO, metadata
     static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - RING_OFF) / STAGE;
@@ -543,7 +607,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
             mbar_init(&s_full[b], 1);
-            mbar_init(&p_full[b], 128);  // the warpgroup that owns buffer b
+            mbar_init(&p_full[b], C::SPLIT ? 256 : 128);  // the warpgroups that handle buffer b
         }
         fence_mbar_init();
         abort_s = 0;
@@ -689,9 +753,9 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
 #pragma unroll
                     for (int kk = 0; kk < NQ / 16; ++kk) {
                         const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
-                        umma_bf16_tmem_a(tmem + C::T_DV, tmem + C::T_ST + (g & 1u) * NQ + 8 * kk,
+                        umma_bf16_tmem_a(tmem + C::T_DV, tmem + C::T_ST + (g & 1u) * NQ + pair_col<NQ, C::SPLIT>(kk),
                                          umma_desc_sw128(db + kk * 2048, C::QBOX, 1024), idesc_o, acc);
-                        umma_bf16_tmem_a(tmem + C::T_DK, tmem + C::T_DPT + (g & 1u) * NQ + 8 * kk,
+                        umma_bf16_tmem_a(tmem + C::T_DK, tmem + C::T_DPT + (g & 1u) * NQ + pair_col<NQ, C::SPLIT>(kk),
                                          umma_desc_sw128(qb + kk * 2048, C::QBOX, 1024), idesc_o, acc);
                     }
                     umma_commit(&qd_empty[g % STAGES]);
@@ -724,7 +788,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             const bool kvalid = key < a.n;
             for (int i = 0; i < it.nqt; ++i) {
                 const uint32_t g = gt + i;
-                if (WGS == 2 && static_cast<int>(g & 1u) != wg) continue;
+                if (WGS == 2 && !C::SPLIT && static_cast<int>(g & 1u) != wg) continue;
                 if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
                     ok = false;
                     break;
@@ -739,17 +803,20 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 const bool inner =
                     C::INNER && __all_sync(kFull, kvalid && tql < a.n && key <= tq0 && key >= support_start(tql, h));
                 // KC columns at a time: their P^T and dS^T (KC/2 bf16-pair columns each) go over
-                // columns already read
-                constexpr int KC = PBB_BWD_KV_KC < NQ ? PBB_BWD_KV_KC : NQ;
+                // columns already read; with split columns this warpgroup takes columns
+                // [wg NQ/2, (wg+1) NQ/2)
+                constexpr int NW = C::SPLIT ? NQ / 2 : NQ;  // this warpgroup's columns of the tile
+                constexpr int KC = PBB_BWD_KV_KC < NW ? PBB_BWD_KV_KC : NW;
+                const int col0 = C::SPLIT ? wg * NW : 0;
 #pragma unroll
-                for (int c = 0; c < NQ / KC; ++c) {
+                for (int c = 0; c < NW / KC; ++c) {
                     uint32_t v1[KC], v2[KC];
                     if constexpr (KC == 32) {
-                        tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + KC * c, v1);
-                        tmem_ld32(lane_base + C::T_DPT + (g & 1u) * NQ + KC * c, v2);
+                        tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + col0 + KC * c, v1);
+                        tmem_ld32(lane_base + C::T_DPT + (g & 1u) * NQ + col0 + KC * c, v2);
                     } else {
-                        tmem_ld16(lane_base + C::T_ST + (g & 1u) * NQ + KC * c, v1);
-                        tmem_ld16(lane_base + C::T_DPT + (g & 1u) * NQ + KC * c, v2);
+                        tmem_ld16(lane_base + C::T_ST + (g & 1u) * NQ + col0 + KC * c, v1);
+                        tmem_ld16(lane_base + C::T_DPT + (g & 1u) * NQ + col0 + KC * c, v2);
                     }
                     tmem_wait_ld();
                     uint32_t pk[KC / 2], dk[KC / 2];
@@ -757,7 +824,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
 #pragma unroll
                         for (int x = 0; x < KC / 2; ++x) {
                             // (-lse2, -D) of columns cc and cc + 1
-                            const float4 m = *reinterpret_cast<const float4*>(meta_ld + KC * c + 2 * x);
+                            const float4 m = *reinterpret_cast<const float4*>(meta_ld + col0 + KC * c + 2 * x);
                             const float2 arg = __ffma2_rn(
                                 make_float2(__uint_as_float(v1[2 * x]), __uint_as_float(v1[2 * x + 1])),
                                 make_float2(sc2, sc2), make_float2(m.x, m.z));
@@ -774,7 +841,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                             float pe[2], de[2];
 #pragma unroll
                             for (int y = 0; y < 2; ++y) {
-                                const int cc = KC * c + 2 * x + y;
+                                const int cc = col0 + KC * c + 2 * x + y;
                                 const float4 m = meta[cc];  // (lse2, D, t, a(t)) of column cc; t = -1 past n
                                 const int t = __float_as_int(m.z), at = __float_as_int(m.w);
                                 const bool vis = kvalid && key <= t && key >= at;
@@ -787,11 +854,11 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                         }
                     }
                     if constexpr (KC == 32) {
-                        tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + 16 * c, pk);
-                        tmem_st16(lane_base + C::T_DPT + (g & 1u) * NQ + 16 * c, dk);
+                        tmem_st16(lane_base + C::T_ST + (g & 1u) * NQ + col0 + 16 * c, pk);
+                        tmem_st16(lane_base + C::T_DPT + (g & 1u) * NQ + col0 + 16 * c, dk);
                     } else {
-                        tmem_st8(lane_base + C::T_ST + (g & 1u) * NQ + 8 * c, pk);
-                        tmem_st8(lane_base + C::T_DPT + (g & 1u) * NQ + 8 * c, dk);
+                        tmem_st8(lane_base + C::T_ST + (g & 1u) * NQ + col0 + 8 * c, pk);
+                        tmem_st8(lane_base + C::T_DPT + (g & 1u) * NQ + col0 + 8 * c, dk);
                     }
                 }
                 tmem_wait_st();
@@ -910,6 +977,10 @@ cudaError_t launch_bwd_shape(const BackwardArgs& a, cudaStream_t stream)
 #ifndef PBB_BWD_SHORT_SHAPE
 #define PBB_BWD_SHORT_SHAPE 1
 #endif
+// Keys per tile of the dQ pass in the long shape: 128 (one dP buffer, released early) or 64 (two).
+#ifndef PBB_BWD_Q_NK
+#define PBB_BWD_Q_NK 128
+#endif
 
 template <int D, int G>
 cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
@@ -918,7 +989,7 @@ cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
         if (a.B < 512)
             return launch_bwd_shape<D, BqCfg<D, G, 32, 1, 2>, BkvCfg<D, G, 32, 1, 2>>(a, stream);
     }
-    return launch_bwd_shape<D, BqCfg<D, G, 64, 2, 1>, BkvCfg<D, G, 64, 2, 1>>(a, stream);
+    return launch_bwd_shape<D, BqCfg<D, G, PBB_BWD_Q_NK, 2, 1>, BkvCfg<D, G, 64, 2, 1>>(a, stream);
 }
 
 template <int D>

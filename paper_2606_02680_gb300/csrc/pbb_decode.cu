@@ -309,6 +309,16 @@ struct Cfg {
 
 // ----------------------------------------------------------- item end ----
 
+// atomicAdd with acquire-release semantics at GPU scope (one round trip: it publishes the
+// caller's earlier stores and sees the stores published before earlier updates).
+__device__ __forceinline__ int atomic_add_acq_rel_gpu(int* p, int v)
+{
+    int old;
+    asm volatile("atom.acq_rel.gpu.global.add.s32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+
 // End of a work item, run by all consumer threads: merge the consumer warps'
 // (max, sum, output) states of the item (Eq. lse) from ml_s [NC][G] and
 // merge_o [NC][G][D]; write `out` for an unsplit support, else the item's
@@ -344,13 +354,14 @@ __device__ __forceinline__ bool finish_item(const DecodeArgs& a, const TileMeta&
         }
     }
     if (ok && mt.nch > 1) {
-        // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
-        __threadfence();
+        // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials.
+        // The barrier orders every consumer thread's partial stores before thread 0's counter
+        // update, which releases them to the GPU and, for the last item, acquires the other
+        // items' partials (the semaphore pattern of a split-k reduction).
         ok = consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
-        if (ok && ctid == 0) *last_s = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
+        if (ok && ctid == 0) *last_s = (atomic_add_acq_rel_gpu(a.counters + head, 1) == mt.nch - 1);
         ok = ok && consumer_barrier<NC>(sbar_count, sbar_gen, lane, kGuardNs);
         if (ok && *last_s) {
-            __threadfence();
             const float* po = a.part_o + (head - a.whole) * a.nchunk * G * D;
             const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + (head - a.whole) * a.nchunk * G;
             float* out_g = a.out + (static_cast<size_t>(mt.b) * a.Hq + static_cast<size_t>(mt.kvh) * a.gq) * D;
@@ -857,6 +868,16 @@ struct TcCfg {
     static_assert(D % 128 == 0 || D == 64, "head sizes");
 };
 
+// Index into pos[] of work item `item`: items [0, whole) are whole supports, then nchunk
+// chunks of each later support; a support is (sequence, KV head), and the layers of a
+// multi-layer step share the positions of their sequences.
+__device__ __forceinline__ int tc_item_seq(const DecodeArgs& a, int item)
+{
+    const int pair = item < a.whole ? item : a.whole + (item - a.whole) / a.nchunk;
+    const int b = pair / a.Hkv;
+    return b < a.pos_batch ? b : b % a.pos_batch;
+}
+
 // Wait for phase `parity` of `bar`, giving up when another warp of the CTA has aborted or after
 // kGuardNs. Returns false if it gave up.
 __device__ __forceinline__ bool mbar_wait_or_abort(uint64_t* bar, uint32_t parity, volatile int* abort_flag)
@@ -916,104 +937,102 @@ __device__ __forceinline__ void epilogue_item(const DecodeArgs& a, const TileMet
         }
     }
     if (!split) return;
-    // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials
-    __threadfence();
+    // split combine (Eq. lse): the last item of this (sequence, KV head) fuses all partials.
+    // The partial stores of every lane are ordered before lane 0's counter update by the
+    // warp barrier, and the update releases them to the GPU (and, for the last item,
+    // acquires the other items' partials) in one atomic, the semaphore pattern of a
+    // split-k reduction; under a saturated memory system each L2 round trip costs
+    // microseconds, so the combine issues its loads in as few rounds as it can.
     __syncwarp();
     int last = 0;
-    if (lane == 0) last = (atomicAdd(a.counters + head, 1) == mt.nch - 1);
+    if (lane == 0) last = (atomic_add_acq_rel_gpu(a.counters + head, 1) == mt.nch - 1);
     last = __shfl_sync(kFull, last, 0);
     if (!last) return;
-    __threadfence();
     const float* po = a.part_o + (head - a.whole) * a.nchunk * G * D;
     const float2* pml = reinterpret_cast<const float2*>(a.part_ml) + (head - a.whole) * a.nchunk * G;
     const int nch = mt.nch;
-    if (nch * G <= NC * G * D) {
-        // weights e^(m_c - M) / L of every (chunk, head) into the slot's scratch: all (max, sum)
-        // pairs are loaded at once, then reduced across the lanes per head
-        float* wgt = o;  // [nch][G]
-        float Mh[G], Lh[G];
+    constexpr int HPL = G / HPI;  // head rows per lane: each lane owns float4 c4 of them
+    const int jl = lane / V4;     // head offset of this lane within a row group
+    float4 acc[HPL];
 #pragma unroll
-        for (int j = 0; j < G; ++j) {
-            Mh[j] = -INFINITY;
-            Lh[j] = 0.f;
-        }
-        for (int c = lane; c < nch; c += 32) {
-#pragma unroll
-            for (int j = 0; j < G; ++j) Mh[j] = fmaxf(Mh[j], __ldcg(&pml[c * G + j]).x);
-        }
+    for (int x = 0; x < HPL; ++x) acc[x] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (nch <= 32) {
+        // one round: every lane loads the (max, sum) pairs of chunk c = lane, and the
+        // partials of chunks 0 and 1 are requested at the same time
+        float2 m2[G];
 #pragma unroll
         for (int j = 0; j < G; ++j)
-#pragma unroll
-            for (int off = 16; off >= 1; off >>= 1) Mh[j] = fmaxf(Mh[j], __shfl_xor_sync(kFull, Mh[j], off));
-        for (int c = lane; c < nch; c += 32) {
-#pragma unroll
-            for (int j = 0; j < G; ++j) {
-                const float2 m2 = __ldcg(&pml[c * G + j]);
-                const float e = fast_exp2(m2.x - Mh[j]);
-                wgt[c * G + j] = e;
-                Lh[j] = fmaf(m2.y, e, Lh[j]);
-            }
-        }
-#pragma unroll
-        for (int j = 0; j < G; ++j) {
-#pragma unroll
-            for (int off = 16; off >= 1; off >>= 1) Lh[j] += __shfl_xor_sync(kFull, Lh[j], off);
-            Lh[j] = 1.f / Lh[j];
-        }
-        __syncwarp();
-        // every lane owns float4 c4 of HPL head rows; per chunk, the loads of all its rows are in
-        // flight together (two chunks per iteration)
-        constexpr int HPL = G / HPI;
-        float4 acc[HPL];
-#pragma unroll
-        for (int x = 0; x < HPL; ++x) acc[x] = make_float4(0.f, 0.f, 0.f, 0.f);
-        const int jl = lane / V4;  // head offset of this lane within a row group
-#pragma unroll 2
-        for (int c = 0; c < nch; ++c) {
-#pragma unroll
-            for (int x = 0; x < HPL; ++x) {
-                const int j = x * HPI + jl;
-                if (j < a.gq) {  // the real query heads
-                    const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
-                    const float w = wgt[c * G + j];
-                    acc[x].x = fmaf(p.x, w, acc[x].x);
-                    acc[x].y = fmaf(p.y, w, acc[x].y);
-                    acc[x].z = fmaf(p.z, w, acc[x].z);
-                    acc[x].w = fmaf(p.w, w, acc[x].w);
-                }
-            }
-        }
+            m2[j] = lane < nch ? __ldcg(&pml[lane * G + j]) : make_float2(-INFINITY, 0.f);
+        float4 p0[HPL], p1[HPL];
 #pragma unroll
         for (int x = 0; x < HPL; ++x) {
             const int j = x * HPI + jl;
-            if (j < a.gq) {
-                const float inv = (HPI == 1 || jl == 0) ? Lh[x * HPI] : Lh[x * HPI + HPI - 1];
-                reinterpret_cast<float4*>(out_g + j * D)[c4] =
-                    make_float4(acc[x].x * inv, acc[x].y * inv, acc[x].z * inv, acc[x].w * inv);
+            p0[x] = __ldcg(reinterpret_cast<const float4*>(po + j * D) + c4);
+            p1[x] = nch > 1 ? __ldcg(reinterpret_cast<const float4*>(po + (G + j) * D) + c4)
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+        // weights e^(m_c - M) / L per (chunk, head), into the slot's scratch o [nch][G]
+        float* wgt = o;
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            float M = m2[j].x;
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) M = fmaxf(M, __shfl_xor_sync(kFull, M, off));
+            const float e = lane < nch ? fast_exp2(m2[j].x - M) : 0.f;
+            float L = m2[j].y * e;
+#pragma unroll
+            for (int off = 16; off >= 1; off >>= 1) L += __shfl_xor_sync(kFull, L, off);
+            if (lane < nch) wgt[lane * G + j] = e / L;
+        }
+        __syncwarp();
+#pragma unroll
+        for (int x = 0; x < HPL; ++x) {
+            const int j = x * HPI + jl;
+            const float w0 = wgt[j], w1 = nch > 1 ? wgt[G + j] : 0.f;
+            acc[x].x = fmaf(p1[x].x, w1, p0[x].x * w0);
+            acc[x].y = fmaf(p1[x].y, w1, p0[x].y * w0);
+            acc[x].z = fmaf(p1[x].z, w1, p0[x].z * w0);
+            acc[x].w = fmaf(p1[x].w, w1, p0[x].w * w0);
+        }
+#pragma unroll 2
+        for (int c = 2; c < nch; ++c) {
+#pragma unroll
+            for (int x = 0; x < HPL; ++x) {
+                const int j = x * HPI + jl;
+                const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
+                const float w = wgt[c * G + j];
+                acc[x].x = fmaf(p.x, w, acc[x].x);
+                acc[x].y = fmaf(p.y, w, acc[x].y);
+                acc[x].z = fmaf(p.z, w, acc[x].z);
+                acc[x].w = fmaf(p.w, w, acc[x].w);
             }
         }
     } else {
-        for (int j0 = 0; j0 < a.gq; j0 += HPI) {
-            const int j = j0 + lane / V4;
-            if (j < a.gq) {
-                float M = -INFINITY;
-                for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
-                float L = 0.f;
-                float4 O = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int c = 0; c < nch; ++c) {
-                    const float2 m2 = __ldcg(&pml[c * G + j]);
-                    const float sc = fast_exp2(m2.x - M);
-                    const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
-                    L = fmaf(m2.y, sc, L);
-                    O.x = fmaf(p.x, sc, O.x);
-                    O.y = fmaf(p.y, sc, O.y);
-                    O.z = fmaf(p.z, sc, O.z);
-                    O.w = fmaf(p.w, sc, O.w);
-                }
-                const float inv = 1.f / L;
-                reinterpret_cast<float4*>(out_g + j * D)[c4] = make_float4(O.x * inv, O.y * inv, O.z * inv, O.w * inv);
+        // many chunks: per head, the max, the sum and the weighted outputs in three passes
+#pragma unroll
+        for (int x = 0; x < HPL; ++x) {
+            const int j = x * HPI + jl;
+            float M = -INFINITY;
+            for (int c = 0; c < nch; ++c) M = fmaxf(M, __ldcg(&pml[c * G + j]).x);
+            float L = 0.f;
+            for (int c = 0; c < nch; ++c) {
+                const float2 m = __ldcg(&pml[c * G + j]);
+                const float sc = fast_exp2(m.x - M);
+                const float4 p = __ldcg(reinterpret_cast<const float4*>(po + (c * G + j) * D) + c4);
+                L = fmaf(m.y, sc, L);
+                acc[x].x = fmaf(p.x, sc, acc[x].x);
+                acc[x].y = fmaf(p.y, sc, acc[x].y);
+                acc[x].z = fmaf(p.z, sc, acc[x].z);
+                acc[x].w = fmaf(p.w, sc, acc[x].w);
             }
+            const float inv = 1.f / L;
+            acc[x] = make_float4(acc[x].x * inv, acc[x].y * inv, acc[x].z * inv, acc[x].w * inv);
         }
+    }
+#pragma unroll
+    for (int x = 0; x < HPL; ++x) {
+        const int j = x * HPI + jl;
+        if (j < a.gq) reinterpret_cast<float4*>(out_g + j * D)[c4] = acc[x];  // the real query heads
     }
     if (lane == 0) a.counters[head] = 0;
 }
@@ -1072,8 +1091,13 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
             int seq = 0;
             bool ok = true;
-            for (int item = blockIdx.x; ok && item < a.total_items;
-                 item = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1)) {
+            // The next item's index (an atomic on the queue) and its position are fetched while
+            // the current item's last tiles are issued, so neither round trip to L2 sits between
+            // two items.
+            int item = blockIdx.x;
+            int t_item = item < a.total_items ? __ldg(a.pos + tc_item_seq(a, item)) : 0;
+            while (ok && item < a.total_items) {
+                int next = -1, t_next = 0;
                 // items [0, whole): whole supports; then nchunk chunks of each later support
                 int pair, chunk;
                 if (item < a.whole) {
@@ -1085,14 +1109,10 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                     chunk = j % a.nchunk;
                 }
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
-                const int t = __ldg(a.pos + (b < a.pos_batch ? b : b % a.pos_batch));  // layers share positions
-                if (t < 0) {
-                    if (chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
-                    continue;
-                }
+                const int t = t_item;
                 const int B = a.B;
-                int r, n, base;
-                support_keys(t, B, a.window, r, n, base);
+                int r = 0, n = 0, base = 0;
+                if (t >= 0) support_keys(t, B, a.window, r, n, base);
                 // the run of n slots from `base`, in tile-aligned key space: tiles start at slot
                 // multiples of TK, the run occupies aligned keys [lo0, lo0 + n)
                 const int lo0 = n > 0 ? base % TK : 0;
@@ -1101,13 +1121,19 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                 const bool whole = pair < a.whole;
                 const int csize = whole ? max(span, 1) : a.chunk;  // aligned keys per chunk (tiles)
                 const int nch = span > 0 ? (span + csize - 1) / csize : 1;
-                if (chunk >= nch) continue;
+                // a sequence with a negative position is skipped (and flagged once); so are the
+                // chunks past the end of a short support
+                const bool skip = t < 0 || chunk >= nch;
+                if (t < 0 && chunk == 0 && kvh == 0) atomicCAS(&g_status, kDevOk, kDevBadPosition);
                 const int i0 = chunk * csize;
                 const int i1 = min(i0 + csize, span);
                 const int nkeys = max(i1 - i0, 0);
-                const int ntiles = nkeys > 0 ? (nkeys + TK - 1) / TK : 1;
+                const int ntiles = skip ? 0 : (nkeys > 0 ? (nkeys + TK - 1) / TK : 1);
                 const int head = b * a.Hkv + kvh;
+                const int ahead = max(ntiles - 3, 0);  // tile at which the next index is fetched
                 for (int it = 0; it < ntiles; ++it, ++seq) {
+                    if (it == ahead) next = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1);
+                    if (it == ntiles - 1 && next < a.total_items) t_next = __ldg(a.pos + tc_item_seq(a, next));
                     const int s = seq % kTcStages;
                     if (seq >= kTcStages &&
                         !mbar_wait(&empty_bar[s], static_cast<uint32_t>((seq / kTcStages - 1) & 1), kGuardNs)) {
@@ -1163,6 +1189,11 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                                  C::ROW, &full_bar[s]);
                     }
                 }
+                if (!ok) break;
+                if (next < 0) next = static_cast<int>(gridDim.x) + atomicAdd(a.ctl, 1);  // a skipped item
+                if (ntiles == 0 && next < a.total_items) t_next = __ldg(a.pos + tc_item_seq(a, next));
+                item = next;
+                t_item = t_next;
             }
             if (ok) {  // end-of-work descriptor
                 const int s = seq % kTcStages;
