@@ -193,12 +193,14 @@ def read_roof(dev, gib: int = 4, reps: int = 10):
         pbb.stream_read(buf, sink)
         ev[2 * i + 1].record(stream)
     torch.cuda.synchronize()
+    if int(sink.item()) < 0:  # bit 63: a bounded wait on a copy ran out
+        raise RuntimeError("pbb_stream_read: a wait on a bulk copy ran out")
     ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(reps)]
     del buf
     torch.cuda.empty_cache()
     return {"gbs": nbytes / (min(ms) / 1e3) / 1e9, "gbs_median": nbytes / (statistics.median(ms) / 1e3) / 1e9,
-            "how": f"pbb_stream_read over {gib} GiB (streaming 16-byte loads, read once), best of {reps} "
-                   f"event-timed launches in this run"}
+            "how": f"pbb_stream_read over {gib} GiB (16 KiB bulk copies into shared memory, 8 in flight per "
+                   f"SM, read once), best of {reps} event-timed launches in this run"}
 
 
 def kernel_source_sha() -> str:

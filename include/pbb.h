@@ -337,14 +337,16 @@ int pbb_decode_step_noalloc(const void* q, const void* k_new, const void* v_new,
 
 /*
  * No counterpart in the paper: a measurement utility. Reads every byte of
- * buf[0, bytes) once from device memory (streaming loads, one persistent grid of
- * 4 CTAs per SM) and xor-folds the 32-bit words into *sink, so the bytes cannot
- * be skipped. Timing it gives the read-only HBM bandwidth, the roof of a decode
- * step (which reads its K/V support and writes almost nothing), next to the
- * copy (read + write) bandwidth. buf: device pointer, 16-byte aligned, bytes a
- * multiple of 16; sink: device pointer, 8-byte aligned, caller-owned (its value
- * is only a checksum). Asynchronous on `stream`; PBB_ERR_INVALID_ARG on a
- * null or misaligned argument, nothing launched for bytes = 0.
+ * buf[0, bytes) once from device memory the way the decode kernels do (16 KiB
+ * bulk copies into a shared-memory ring, 8 in flight, one CTA per SM; a tail
+ * under 16 KiB by plain loads). Timing it gives the read-only HBM bandwidth,
+ * the roof of a decode step (which reads its K/V support and writes almost
+ * nothing), next to the copy (read + write) bandwidth. buf: device pointer,
+ * 16-byte aligned, bytes a multiple of 16; sink: device pointer, 8-byte
+ * aligned, caller-owned: the tail's words are xor-folded into it, and bit 63
+ * is set if a bounded wait on a copy ran out. Asynchronous on `stream`;
+ * PBB_ERR_INVALID_ARG on a null or misaligned argument, nothing launched for
+ * bytes = 0.
  */
 int pbb_stream_read(const void* buf, size_t bytes, unsigned long long* sink, cudaStream_t stream);
 

@@ -868,12 +868,39 @@ struct TcCfg {
     static_assert(D % 128 == 0 || D == 64, "head sizes");
 };
 
-// Index into pos[] of work item `item`: items [0, whole) are whole supports, then nchunk
-// chunks of each later support; a support is (sequence, KV head), and the layers of a
-// multi-layer step share the positions of their sequences.
+// Work item -> (support, chunk) on the tensor-core kernel. Items [0, whole) are whole supports,
+// then the chunks of each later support together. PBB_TC_CHUNK_MAJOR = 1 orders the chunks
+// chunk-major instead (chunk 0 of every split support, then chunk 1, ...), so the queue ends on
+// the short remainders of the longest supports; measured on GB300 it lost 5 % at B 2048 (the
+// chunks past short supports, which the producer skips at two L2 round trips each, then pile up
+// at the end of the queue) and tied elsewhere. A support is (sequence, KV head).
+#ifndef PBB_TC_CHUNK_MAJOR
+#define PBB_TC_CHUNK_MAJOR 0
+#endif
+__device__ __forceinline__ void tc_item(const DecodeArgs& a, int item, int& pair, int& chunk)
+{
+    if (item < a.whole) {
+        pair = item;
+        chunk = 0;
+        return;
+    }
+    const int j = item - a.whole;
+    if (PBB_TC_CHUNK_MAJOR) {
+        const int split = a.batch * a.Hkv - a.whole;  // supports that are split
+        pair = a.whole + j % split;
+        chunk = j / split;
+    } else {
+        pair = a.whole + j / a.nchunk;
+        chunk = j % a.nchunk;
+    }
+}
+
+// Index into pos[] of work item `item` (the layers of a multi-layer step share the positions of
+// their sequences).
 __device__ __forceinline__ int tc_item_seq(const DecodeArgs& a, int item)
 {
-    const int pair = item < a.whole ? item : a.whole + (item - a.whole) / a.nchunk;
+    int pair, chunk;
+    tc_item(a, item, pair, chunk);
     const int b = pair / a.Hkv;
     return b < a.pos_batch ? b : b % a.pos_batch;
 }
@@ -1098,16 +1125,8 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
             int t_item = item < a.total_items ? __ldg(a.pos + tc_item_seq(a, item)) : 0;
             while (ok && item < a.total_items) {
                 int next = -1, t_next = 0;
-                // items [0, whole): whole supports; then nchunk chunks of each later support
                 int pair, chunk;
-                if (item < a.whole) {
-                    pair = item;
-                    chunk = 0;
-                } else {
-                    const int j = item - a.whole;
-                    pair = a.whole + j / a.nchunk;
-                    chunk = j % a.nchunk;
-                }
+                tc_item(a, item, pair, chunk);
                 const int kvh = pair % a.Hkv, b = pair / a.Hkv;
                 const int t = t_item;
                 const int B = a.B;

@@ -2,43 +2,64 @@
 // measured against next to the copy bandwidth.
 //
 // A decode step reads its K/V support and writes almost nothing (the fp32
-// output and one ring row per (sequence, KV head)), so its ceiling is the
-// DRAM read bandwidth, which is higher than the bandwidth of a copy (a copy
-// turns the bus around between reads and writes). This kernel reads every
-// 16-byte word of a buffer exactly once with streaming (evict-first) loads,
-// four independent loads in flight per thread, and folds the words into one
-// 64-bit xor so that no load can be dropped. No counterpart in the paper.
+// output and one ring row per (sequence, KV head)), so its ceiling is the DRAM
+// read bandwidth, which is higher than the bandwidth of a copy (a copy turns
+// the bus around between reads and writes). The probe reads the way the decode
+// kernels do: one lane per CTA streams the buffer in 16 KiB bulk copies
+// (cp.async.bulk) into an 8-stage shared-memory ring whose stages complete on
+// mbarriers, one CTA per SM, each CTA taking every gridDim-th chunk. The data is
+// never looked at; every wait is bounded, and a wait that runs out sets a bit
+// in *sink instead of hanging. A tail shorter than a chunk is read by plain
+// loads. No counterpart in the paper.
 #include <cuda_runtime.h>
 
 #include <cstdint>
 
 #include "pbb.h"
+#include "pbb_device.cuh"
 
 namespace {
 
-constexpr int kProbeThreads = 512;
-constexpr int kProbeCtasPerSm = 4;
+constexpr int kProbeChunk = 16384;                   // bytes per bulk copy
+constexpr int kProbeStages = 8;                      // copies in flight per CTA
+constexpr unsigned long long kProbeLimitNs = 1000000000ull;
 
-__global__ void __launch_bounds__(kProbeThreads) stream_read_kernel(const uint4* __restrict__ p, size_t n,
-                                                                    unsigned long long* sink)
+__global__ void __launch_bounds__(32) stream_read_kernel(const unsigned char* __restrict__ p, size_t bytes,
+                                                         unsigned long long* sink)
 {
-    const size_t stride = static_cast<size_t>(gridDim.x) * blockDim.x;
-    size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-    uint32_t acc = 0;
-    for (; i + 3 * stride < n; i += 4 * stride) {
-        const uint4 a = __ldcs(p + i);
-        const uint4 b = __ldcs(p + i + stride);
-        const uint4 c = __ldcs(p + i + 2 * stride);
-        const uint4 d = __ldcs(p + i + 3 * stride);
-        acc ^= a.x ^ a.y ^ a.z ^ a.w ^ b.x ^ b.y ^ b.z ^ b.w ^ c.x ^ c.y ^ c.z ^ c.w ^ d.x ^ d.y ^ d.z ^ d.w;
+    extern __shared__ __align__(128) unsigned char ring[];
+    __shared__ __align__(8) uint64_t full[kProbeStages];
+    const size_t chunks = bytes / kProbeChunk;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kProbeStages; ++s) pbb::mbar_init(&full[s], 1);
+        pbb::fence_mbar_init();
+        uint32_t k = 0;
+        bool ok = true;
+        for (size_t c = blockIdx.x; c < chunks; c += gridDim.x, ++k) {
+            const int s = k % kProbeStages;
+            if (k >= kProbeStages &&
+                !pbb::mbar_wait(&full[s], static_cast<uint32_t>(((k / kProbeStages) - 1) & 1u), kProbeLimitNs)) {
+                ok = false;
+                break;
+            }
+            pbb::mbar_expect_tx(&full[s], kProbeChunk);
+            pbb::bulk_g2s(ring + s * kProbeChunk, p + c * kProbeChunk, kProbeChunk, &full[s]);
+        }
+        // every copy lands before the CTA (and its shared memory) goes away
+        const uint32_t first = k > kProbeStages ? k - kProbeStages : 0;
+        for (uint32_t j = first; j < k; ++j)
+            if (!pbb::mbar_wait(&full[j % kProbeStages], static_cast<uint32_t>((j / kProbeStages) & 1u), kProbeLimitNs))
+                ok = false;
+        if (!ok) atomicOr(sink, 1ull << 63);
     }
-    for (; i < n; i += stride) {
-        const uint4 a = __ldcs(p + i);
-        acc ^= a.x ^ a.y ^ a.z ^ a.w;
+    if (blockIdx.x == 0) {  // the tail after the last whole chunk, 16 bytes per lane
+        uint32_t acc = 0;
+        for (size_t i = chunks * kProbeChunk + 16 * threadIdx.x; i < bytes; i += 16 * blockDim.x) {
+            const uint4 v = __ldcs(reinterpret_cast<const uint4*>(p + i));
+            acc ^= v.x ^ v.y ^ v.z ^ v.w;
+        }
+        if (acc != 0) atomicXor(sink, static_cast<unsigned long long>(acc));
     }
-#pragma unroll
-    for (int off = 16; off >= 1; off >>= 1) acc ^= __shfl_xor_sync(0xffffffffu, acc, off);
-    if ((threadIdx.x & 31) == 0 && acc != 0) atomicXor(sink, static_cast<unsigned long long>(acc));
 }
 
 }  // namespace
@@ -53,7 +74,9 @@ extern "C" int pbb_stream_read(const void* buf, size_t bytes, unsigned long long
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
         return PBB_ERR_CUDA;
-    stream_read_kernel<<<sms * kProbeCtasPerSm, kProbeThreads, 0, stream>>>(static_cast<const uint4*>(buf),
-                                                                           bytes / 16, sink);
+    constexpr int smem = kProbeChunk * kProbeStages;
+    if (cudaFuncSetAttribute(stream_read_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
+        return PBB_ERR_CUDA;
+    stream_read_kernel<<<sms, 32, smem, stream>>>(static_cast<const unsigned char*>(buf), bytes, sink);
     return cudaGetLastError() == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
