@@ -57,6 +57,7 @@
 
 #include <atomic>
 #include <mutex>
+#include <utility>
 
 #include "pbb.h"
 #include "pbb_device.cuh"
@@ -468,6 +469,10 @@ __global__ void __launch_bounds__(kThreads, Cfg<ELEM, D, G>::MIN_CTAS) decode_ke
                 reinterpret_cast<uint4*>(dsmem + s * C::STAGE + C::Q_OFF + a.gq * C::ROW)[x] = make_uint4(0u, 0u, 0u, 0u);
     }
     __syncthreads();
+    // the set-up above touches no global memory; everything below may read what the previous
+    // grid of the stream wrote (rings, positions, the queue words)
+    pdl_wait();
+    pdl_launch_dependents();
 
     if (warp == kConsumers) {
         // ================= producer: one lane =================
@@ -1110,6 +1115,10 @@ __global__ void __launch_bounds__(kTcThreads, PBB_TC_MIN_CTAS)
                 reinterpret_cast<uint4*>(dsmem + s * C::STAGE + C::Q_OFF + a.gq * C::ROW)[x] = make_uint4(0u, 0u, 0u, 0u);
     }
     __syncthreads();
+    // the set-up above touches no global memory; everything below may read what the previous
+    // grid of the stream wrote (rings, positions, the queue words)
+    pdl_wait();
+    pdl_launch_dependents();
 
     if (warp == kTcProducer) {
         // ================= producer: one lane =================
@@ -1497,6 +1506,8 @@ __global__ void prefill_kernel(const uint4* __restrict__ k_hist, const uint4* __
                                uint4* __restrict__ v_ring, int Hkv, int B, int row16,
                                long long total)
 {
+    pdl_wait();
+    pdl_launch_dependents();
     for (long long i = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; i < total;
          i += static_cast<long long>(gridDim.x) * blockDim.x) {
         const int x = static_cast<int>(i % row16);
@@ -1520,7 +1531,33 @@ __global__ void prefill_kernel(const uint4* __restrict__ k_hist, const uint4* __
 
 __global__ void advance_kernel(int32_t* pos, int batch)
 {
+    pdl_wait();
+    pdl_launch_dependents();
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < batch; i += gridDim.x * blockDim.x) pos[i] += 1;
+}
+
+// Launches of the decode-step kernels (decode, position advance, ring load) allow programmatic
+// dependent launch: a kernel may be scheduled while the previous kernel of the stream finishes,
+// so its launch and set-up overlap that kernel's tail; each of them calls pdl_wait before it
+// touches global memory, so it sees everything the previous kernel wrote, as with plain stream
+// order. PBB_PDL = 0 launches them plainly.
+#ifndef PBB_PDL
+#define PBB_PDL 1
+#endif
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), int grid, int block, size_t smem, cudaStream_t stream, Args&&... args)
+{
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(static_cast<unsigned>(grid));
+    cfg.blockDim = dim3(static_cast<unsigned>(block));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = PBB_PDL ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
 }
 
 // Opt the kernel in to its dynamic shared memory (above the 48 KiB default), once per device.
@@ -1569,8 +1606,7 @@ cudaError_t launch_t(const DecodeArgs& a, cudaStream_t stream)
     const long long ctas = static_cast<long long>(sms) * per_sm;
     const int grid = static_cast<int>(a.total_items < ctas ? a.total_items : ctas);
     if (grid < 1) return cudaSuccess;
-    decode_kernel<ELEM, D, G><<<grid, kThreads, C::SMEM, stream>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(decode_kernel<ELEM, D, G>, grid, kThreads, C::SMEM, stream, a);
 }
 
 // ---- tensor-core path: TMA tensor maps over the rings and the launch
@@ -1712,8 +1748,7 @@ cudaError_t launch_tc(const DecodeArgs& a, cudaStream_t stream)
     const long long ctas = static_cast<long long>(sms) * per_sm;
     const int grid = static_cast<int>(a.total_items < ctas ? a.total_items : ctas);
     if (grid < 1) return cudaSuccess;
-    decode_kernel_tc<D><<<grid, kTcThreads, C::SMEM, stream>>>(a, kmap, vmap);
-    return cudaGetLastError();
+    return launch_pdl(decode_kernel_tc<D>, grid, kTcThreads, C::SMEM, stream, a, kmap, vmap);
 }
 
 template <int ELEM, int D>
@@ -1807,19 +1842,16 @@ cudaError_t launch_prefill(const void* k_hist, const void* v_hist, const int32_t
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const long long want = (total + 255) / 256;
     const int blocks = static_cast<int>(want < sms * 16LL ? want : sms * 16LL);
-    prefill_kernel<<<blocks, 256, 0, stream>>>(static_cast<const uint4*>(k_hist),
-                                               static_cast<const uint4*>(v_hist), pos,
-                                               static_cast<uint4*>(k_ring),
-                                               static_cast<uint4*>(v_ring), Hkv, B, row16, total);
-    return cudaGetLastError();
+    return launch_pdl(prefill_kernel, blocks, 256, 0, stream, static_cast<const uint4*>(k_hist),
+                      static_cast<const uint4*>(v_hist), pos, static_cast<uint4*>(k_ring),
+                      static_cast<uint4*>(v_ring), Hkv, B, row16, total);
 }
 
 cudaError_t launch_advance(int32_t* pos, int batch, cudaStream_t stream)
 {
     if (batch == 0) return cudaSuccess;
     const int blocks = (batch + 255) / 256 < 64 ? (batch + 255) / 256 : 64;
-    advance_kernel<<<blocks, 256, 0, stream>>>(pos, batch);
-    return cudaGetLastError();
+    return launch_pdl(advance_kernel, blocks, 256, 0, stream, pos, batch);
 }
 
 bool rows_tensor_map(CUtensorMap* map, const void* base, unsigned long long rows, int d, int box_rows)

@@ -158,6 +158,13 @@ __device__ __forceinline__ float fast_exp2(float x)
     return y;
 }
 
+// Programmatic dependent launch. pdl_wait: block until the grids this one depends on in its
+// stream have completed and their memory is visible (a no-op for a launch without the
+// attribute). pdl_launch_dependents: let the next grid of the stream be scheduled now; it still
+// runs no further than its own pdl_wait until this grid completes.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar)
 {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
