@@ -91,6 +91,17 @@ def test_misaligned_pointers_rejected(pbb):
     assert rc == -1
 
 
+def test_stream_read_arguments_checked_on_the_host(pbb):
+    lib = pbb.lib()
+    p = 0x10000  # never dereferenced: every check below fails, or returns, before any launch
+    assert lib.pbb_stream_read(None, 1024, p, None) == -1
+    assert lib.pbb_stream_read(p + 8, 1024, p, None) == -1       # buffer not 16-byte aligned
+    assert lib.pbb_stream_read(p, 1000, p, None) == -1           # size not a multiple of 16
+    assert lib.pbb_stream_read(p, 1024, p + 4, None) == -1       # sink not 8-byte aligned
+    assert lib.pbb_stream_read(p, 1024, None, None) == -1
+    assert lib.pbb_stream_read(None, 0, None, None) == 0         # nothing to read: no launch
+
+
 def test_empty_batch_is_a_no_op(pbb):
     lib = pbb.lib()
     assert lib.pbb_decode_step(None, None, None, None, None, None, None, 0, 8, 2, 128, 128, None) == 0
