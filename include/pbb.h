@@ -38,7 +38,7 @@
  *     never synchronise. Sizes: batch >= 0, Hq % Hkv == 0 with
  *     Hq/Hkv in {1, 2, 4, 6, 8}, d in {64, 128}, B even and 2 <= B <= 2^20.
  *     A group of 6 (12 query heads on 2 KV heads, the paper's models of Sec. 5)
- *     runs on the group-8 CUDA-core kernel with two zero query rows that are
+ *     runs as a group of 8 (on either kernel) with two zero query rows that are
  *     computed and never written.
  *   - Return value: PBB_OK or a negative PBB_ERR_* code; nothing is launched
  *     when argument checking fails. Faults the device finds (a negative
@@ -287,10 +287,10 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
 /*
  * Which kernel a decode step of this shape runs on the current device:
  * PBB_KERNEL_CUDA_CORES (packed fp32 FMAs; every shape) or PBB_KERNEL_TENSOR_CORES
- * (bf16 PBB steps with Hq/Hkv = 8, where the scores of a 16-key block against the
+ * (bf16 steps with Hq/Hkv = 8, where the scores of a 16-key block against the
  * 8 query heads form a dense mma tile, or Hq/Hkv = 4 or 6 with the tile's other
- * columns zero; needs B a multiple of 64). Groups 4 and 6 take the tensor cores
- * only when batch*Hkv fills the resident CTAs. Negative on error.
+ * columns zero; needs B a multiple of 64). Window steps of the shape take the
+ * same kernel. Negative on error.
  */
 enum { PBB_KERNEL_AUTO = -1, PBB_KERNEL_CUDA_CORES = 0, PBB_KERNEL_TENSOR_CORES = 1 };
 int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);

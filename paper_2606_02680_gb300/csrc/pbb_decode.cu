@@ -1691,12 +1691,13 @@ int device_sms()
     });
 }
 
-// Padded groups (4 and 6 heads in the 8-column score tile) take the tensor cores only when the
-// supports at least fill the resident CTAs. With fewer supports every support is split, and
-// there the CUDA-core kernel, whose four consumer warps merge and combine the split partials
-// faster, wins (measured on GB300: 7-34 % at batch 1 to 32, Hq 32, Hkv 8).
+// PBB_TC_PAD_MIN_FILL = 1 keeps padded groups (4 and 6 heads in the 8-column score tile) on the
+// CUDA cores unless the supports fill the resident CTAs. That paid while the tensor-core kernel's
+// two consumer warps ended the items themselves; with the epilogue warp the tensor cores win at
+// small batches too (measured on GB300, Hq 32, Hkv 8: batch 8 / 32 at B 4096 25.4 / 74.5 against
+// 33.5 / 105.7 us per step, batch 32 at B 1024 9.7 against 12.2 us), so it is off.
 #ifndef PBB_TC_PAD_MIN_FILL
-#define PBB_TC_PAD_MIN_FILL 1
+#define PBB_TC_PAD_MIN_FILL 0
 #endif
 // Sliding-window steps on the tensor-core kernel (0 keeps them on the CUDA cores).
 #ifndef PBB_TC_WINDOWS

@@ -91,16 +91,15 @@ def test_group8_tensor_core_layers():
     run_layers(w, 2, 30)
 
 
-@pytest.mark.parametrize("kernel", ["auto", "tensor_cores"])
+@pytest.mark.parametrize("kernel", ["cuda_cores", "tensor_cores"])
 def test_group6_layers(kernel):
     """Two local layers of the paper's model shape (12 query heads on 2 KV heads, d 64), on
-    the library's choice (the CUDA cores at this batch) and on the tensor cores."""
+    both kernels (the library's choice is the tensor cores)."""
     w = inputs.Workload("layers_g6", batch=3, Hq=12, Hkv=2, d=64, B=128, dtype="bf16", steps=0,
                         t0_lo=0, t0_hi=2000, seed=304)
     prev = pbb.set_kernel(kernel)
     try:
-        assert pbb.plan_kernel(2 * w.batch, w.Hq, w.Hkv, w.d, w.B) == (
-            "cuda_cores" if kernel == "auto" else "tensor_cores")
+        assert pbb.plan_kernel(2 * w.batch, w.Hq, w.Hkv, w.d, w.B) == kernel
         run_layers(w, 2, 30)
     finally:
         pbb.set_kernel(prev)

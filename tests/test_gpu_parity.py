@@ -100,12 +100,12 @@ def test_ragged_prefilled(chunk_keys, group, d, dtype):
 def test_paper_model_shape_group6(chunk_keys, kernel, which):
     """The paper's models (Sec. 5): 12 query heads on 2 KV heads, head size 64, block 128.
     GQA group 6 runs on either kernel's 8 query columns with two zero query rows that are
-    never written (at batch 1 the library picks the CUDA cores): batch 1 from t = 0 across
+    never written (the library picks the tensor cores, B being a multiple of 64): batch 1 from t = 0 across
     5 block boundaries, every step, then ragged prefilled positions with every support
     split into 32-key chunks."""
     w = inputs.Workload("paper_g6", batch=1, Hq=12, Hkv=2, d=64, B=128, dtype="bf16",
                         steps=5 * 128 + 3, t0_lo=0, t0_hi=1, seed=612)
-    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "cuda_cores"
+    assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == "tensor_cores"
     kernel(which)
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B) == which
     run_and_check(w, chunk_keys, ring_every=128)
@@ -352,17 +352,16 @@ def test_bf16_tensor_core_ragged_outliers(chunk_keys, kernel, group, d):
 
 
 def test_kernel_choice(kernel):
-    """The library's choice: group 8 always on the tensor cores; groups 4 and 6 there once
-    the supports fill the resident CTAs (3 per SM), else on the CUDA cores; fp32, windows,
-    groups 1 and 2 and blocks that are not a multiple of 64 on the CUDA cores. pbb_set_kernel
-    overrides it within what each kernel supports."""
+    """The library's choice: bf16 groups 4, 6 and 8 with B a multiple of 64 on the tensor cores,
+    whatever the batch; fp32, groups 1 and 2 and blocks that are not a multiple of 64 on the
+    CUDA cores. pbb_set_kernel overrides it within what each kernel supports."""
     import torch as _t
     assert pbb.plan_kernel(1, 16, 2, 128, 4096) == "tensor_cores"
     assert pbb.plan_kernel(512, 32, 8, 128, 4096) == "tensor_cores"
-    assert pbb.plan_kernel(8, 32, 8, 128, 4096) == "cuda_cores"
-    assert pbb.plan_kernel(32, 16, 4, 128, 1024) == "cuda_cores"
+    assert pbb.plan_kernel(8, 32, 8, 128, 4096) == "tensor_cores"
+    assert pbb.plan_kernel(32, 16, 4, 128, 1024) == "tensor_cores"
     assert pbb.plan_kernel(512, 12, 2, 64, 128) == "tensor_cores"  # the paper's heads, 1,024 supports
-    assert pbb.plan_kernel(1, 12, 2, 64, 128) == "cuda_cores"
+    assert pbb.plan_kernel(1, 12, 2, 64, 128) == "tensor_cores"
     assert pbb.plan_kernel(512, 16, 2, 128, 96) == "cuda_cores"
     assert pbb.plan_kernel(512, 32, 8, 128, 4096, _t.float32) == "cuda_cores"
     assert pbb.plan_kernel(512, 16, 8, 128, 4096) == "cuda_cores"  # group 2

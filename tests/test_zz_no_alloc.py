@@ -46,7 +46,7 @@ def _state(pbb, w, t0, wk, wv, dev):
 
 
 @pytest.mark.parametrize("Hq,Hkv,d,kernel", [(16, 4, 128, "auto"), (12, 2, 64, "auto"), (8, 4, 128, "auto"),
-                                              (16, 4, 128, "tensor_cores"), (12, 2, 64, "tensor_cores")])
+                                              (16, 4, 128, "cuda_cores"), (12, 2, 64, "cuda_cores")])
 def test_noalloc_matches_decode_step_and_oracle_on_two_calls(lib, Hq, Hkv, d, kernel):
     pbb = lib
     from paper_2606_02680_gb300 import inputs
@@ -61,8 +61,8 @@ def test_noalloc_matches_decode_step_and_oracle_on_two_calls(lib, Hq, Hkv, d, ke
 def _noalloc_against_decode_step(pbb, inputs, Hq, Hkv, d):
     dev = torch.device("cuda", 0)
     # small batch: the plan splits every support across many CTAs, so the scratch is used;
-    # (12, 2, 64) is the paper's model shape, GQA group 6; at this batch the library keeps
-    # groups 4 and 6 on the CUDA cores, and the tensor-core cases force that kernel
+    # (12, 2, 64) is the paper's model shape, GQA group 6; the library runs groups 4 and 6 on
+    # the tensor cores and group 2 on the CUDA cores, and the cuda_cores cases force that kernel
     w = inputs.Workload("noalloc", batch=4, Hq=Hq, Hkv=Hkv, d=d, B=2048, dtype="bf16", steps=2,
                         t0_lo=2048, t0_hi=100000, seed=77 + Hq)
     assert pbb.plan_chunk_keys(w.batch, w.Hq, w.Hkv, w.d, w.B) < w.B - 1
