@@ -318,7 +318,7 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None, lay
         warmup += 3
         graph = "on" if e0.elapsed_time(e1) / 3 < 0.1 else "off"
     use_graph = graph == "on"
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
+    ev = [] if use_graph else [torch.cuda.Event(enable_timing=True) for _ in range(2 * steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     g = None
     if use_graph:
@@ -369,7 +369,6 @@ def time_device(w, dev, steps, warmup, dist=None, graph="auto", window=None, lay
         # around single launches (eager, or recorded as nodes inside a graph) add the launch
         # latency of these short kernels and read longer than the whole step.
         kern_ms = [total_ms / steps] * steps
-        first = warmup
     else:
         kern_ms = [ev[2 * i].elapsed_time(ev[2 * i + 1]) for i in range(steps)]
     launch_bytes = [layers * bytemodel.step_bytes(t_np + first + i, w.Hq, w.Hkv, w.d, w.B, w.elem_bytes, window)
