@@ -10,18 +10,20 @@
 // Three kernels, none with floating-point atomics (results are deterministic):
 //   delta_kernel       D for every row (dO . O);
 //   bwd_kv_tc_kernel   items of 128 keys of one (sequence, KV head): it streams the
-//                      query tiles (64 rows: the G heads of the group stacked) whose
-//                      supports hold any of its keys (positions s0 .. h(floor(s_last/h)+2)-1,
-//                      the keys' own half-block and the next one, bridge rows included)
-//                      and accumulates dK and dV in tensor memory;
+//                      query tiles (128 rows in the long shape, 32 in the short one: the
+//                      G heads of the group stacked) whose supports hold any of its keys
+//                      (positions s0 .. h(floor(s_last/h)+2)-1, the keys' own half-block
+//                      and the next one, bridge rows included) and accumulates dK and dV
+//                      in tensor memory;
 //   bwd_q_tc_kernel    items of 128 query rows: it streams the key tiles of [a(t0), t_last]
 //                      and accumulates dQ in tensor memory.
 // Both are persistent on the fifth-generation tensor cores: a TMA producer warp
 // (128-byte swizzle), one MMA-issuing lane (tcgen05.mma, completion through
 // tcgen05.commit on mbarriers) and elementwise warpgroups; thread r of a warpgroup owns
 // TMEM lane r. The long shape runs one CTA per SM with two elementwise warpgroups that
-// share every tile, each on half of its columns (the scores of tile g sit in TMEM buffer
-// g % 2, so tile g+1's products run while tile g's exponentials do); the short shape
+// share every tile, each on half of its columns (dQ pass: the scores of tile g sit in TMEM
+// buffer g % 2, so tile g+1's products run while tile g's exponentials do; dK/dV pass: one
+// buffer each for S^T and dP^T, the next dP^T issued once the warpgroups hold this one); the short shape
 // (short supports, d = 64) runs two CTAs per SM with one warpgroup each, on half the TMEM. P, dS and their transposes are rounded
 // to bf16 and written back over the scores in tensor memory as the A operands of the
 // next products. Tiles with no masked entry take a packed path (two columns per
@@ -516,13 +518,20 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 }
 
 // ------------------------------------------------------------- dK, dV ----
-// Items of 128 keys, query tiles of 64 rows (G heads x QT positions). TMEM: S^T and
-// dP^T, two buffers each (P^T and dS^T are written back over them as bf16 pairs, the
-// A operands of dV += P^T dO and dK += dS^T Q), then dV and dK. Per query tile the
-// producer warp also stages, for each of its 64 columns, the base-2 log-partition, D,
-// the position and its support start.
-// Shapes as for the dQ pass: NQ query rows per tile (64 or 32), WGS elementwise warpgroups,
-// CTAS CTAs per SM.
+// Items of 128 keys, query tiles of NQ rows (G heads x QT positions). Per query tile the
+// producer warp also stages, for each of its NQ columns, the base-2 log-partition, D, the
+// position and its support start. TMEM:
+//  - NQ = 64 or 32: S^T and dP^T, two buffers each (P^T and dS^T are written back over
+//    them as bf16 pairs, the A operands of dV += P^T dO and dK += dS^T Q), then dV and dK;
+//  - NQ = 128 (two elementwise warpgroups on split columns): S^T and dP^T one buffer each,
+//    then dV and dK (4 x 128 columns at d = 128). The warpgroups release the dP^T buffer once
+//    they hold the tile's dP^T in registers (dp_free), so the next tile's dP^T is issued
+//    while they compute; P^T and dS^T both go back over the S^T buffer, and the next tile's
+//    S^T follows the gradient products that read them. Every score product is an N = 128
+//    MMA: with both operands in shared memory, an N = 64 product runs at 2/3 of the tensor
+//    rate.
+// Shapes as for the dQ pass: NQ query rows per tile, WGS elementwise warpgroups, CTAS CTAs
+// per SM.
 // Columns of S^T and dP^T the elementwise threads load before each wait (16 or 32): fewer waits
 // per tile against more registers.
 #ifndef PBB_BWD_KV_KC
@@ -547,13 +556,24 @@ struct BkvCfg {
     static constexpr int STAGE_MAX = CTAS == 1 ? 3 : 4;
     static constexpr int STAGES = STAGE_ROOM < STAGE_MAX ? STAGE_ROOM : STAGE_MAX;
     static constexpr int SMEM = RING_OFF + STAGES * STAGE + 1024;
-    static constexpr int T_ST = 0, T_DPT = 2 * NQ, T_DV = 4 * NQ, T_DK = 4 * NQ + D;
+    static constexpr int SBUF = NQ == 128 ? 1 : 2;  // S^T and dP^T buffers
+    static constexpr int T_ST = 0, T_DPT = SBUF * NQ, T_DV = 2 * SBUF * NQ, T_DK = T_DV + D;
+    static_assert(SBUF == 2 || (SPLIT && CTAS == 1 && NQ == 128), "one score buffer: both warpgroups share every tile");
     static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_DK + D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
     static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
     static_assert(NQ % 32 == 0, "the producer warp stages NQ / 32 columns per lane");
 };
+
+// TMEM column of the P^T pairs for k-step kk (16 query rows) in the one-buffer dK/dV shape
+// (128-row tiles, split columns): warpgroup kk / 4 holds query columns [64 (kk / 4), +64),
+// and each 32-column half of them takes its 16 P^T pair columns, then its 16 dS^T pair
+// columns, over its own S^T columns. dS^T's pairs for kk sit 16 columns further on.
+__host__ __device__ constexpr uint32_t pds_col(int kk)
+{
+    return static_cast<uint32_t>(64 * (kk / 4) + 32 * ((kk % 4) / 2) + 8 * (kk % 2));
+}
 
 struct KItem {
     int pair, s0, tq0, nqt;
@@ -586,7 +606,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t kv_full, kv_empty, done_bar, item_done, o_free;
     __shared__ __align__(8) uint64_t qd_full[STAGES], qd_empty[STAGES];
-    __shared__ __align__(8) uint64_t s_full[2], p_full[2];
+    __shared__ __align__(8) uint64_t s_full[2], p_full[2], dp_free;
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
@@ -609,6 +629,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             mbar_init(&s_full[b], 1);
             mbar_init(&p_full[b], C::SPLIT ? 256 : 128);  // the warpgroups that handle buffer b
         }
+        mbar_init(&dp_free, C::SPLIT ? 256 : 128);  // one dP^T buffer: the warpgroups of a tile hold it
         fence_mbar_init();
         abort_s = 0;
     }
@@ -724,7 +745,84 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 umma_commit(&s_full[g & 1u]);
                 return true;
             };
-            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            auto qd_ready = [&](uint32_t g) {
+                if (!mbar_wait(&qd_full[g % STAGES], (g / STAGES) & 1u, limit)) return false;
+                tmem_fence_after();
+                return true;
+            };
+            if constexpr (C::SBUF == 1) {
+                // one score buffer per kind: tile g's dP^T goes in once the warpgroups hold tile
+                // g-1's, before tile g-1's gradient products; tile g's S^T after them
+                auto issue_one = [&](uint32_t g, bool dpt) {  // S^T = K Q^T, or dP^T = V dO^T
+                    const uint32_t qb = ring + (g % STAGES) * C::STAGE + (dpt ? C::BOXES * C::QBOX : 0);
+                    const uint32_t ab = dpt ? v_base : k_base;
+#pragma unroll
+                    for (int kk = 0; kk < D / 16; ++kk)
+                        umma_bf16(tmem + (dpt ? C::T_DPT : C::T_ST),
+                                  umma_desc_sw128(ab + (kk >> 2) * C::KBOX + (kk & 3) * 32, 16, 1024),
+                                  umma_desc_sw128(qb + (kk >> 2) * C::QBOX + (kk & 3) * 32, 16, 1024), idesc_s,
+                                  kk > 0 ? 1u : 0u);
+                };
+                auto dp_ready = [&](uint32_t g) {
+                    if (g == 0) return true;
+                    if (!mbar_wait(&dp_free, (g - 1) & 1u, limit)) return false;
+                    tmem_fence_after();
+                    return true;
+                };
+                for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                    const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
+                    if (!mbar_wait(&kv_full, ic & 1u, limit) || !qd_ready(gt)) {
+                        ok = false;
+                        break;
+                    }
+                    tmem_fence_after();
+                    issue_one(gt, false);
+                    issued_any = true;
+                    if (!dp_ready(gt)) {
+                        ok = false;
+                        break;
+                    }
+                    issue_one(gt, true);
+                    umma_commit(&s_full[0]);
+                    if (it.nqt == 1) umma_commit(&kv_empty);  // the item's last read of K and V
+                    for (int i = 0; i < it.nqt; ++i) {
+                        const uint32_t g = gt + i;
+                        const bool more = i + 1 < it.nqt;
+                        if (more && (!dp_ready(g + 1) || !qd_ready(g + 1))) {
+                            ok = false;
+                            break;
+                        }
+                        if (more) issue_one(g + 1, true);
+                        if (!mbar_wait(&p_full[0], g & 1u, limit) ||
+                            (i == 0 && ic >= 1 && !mbar_wait(&o_free, (ic - 1) & 1u, limit))) {
+                            ok = false;
+                            break;
+                        }
+                        tmem_fence_after();
+                        // dV (+)= P^T dO and dK (+)= dS^T Q: P^T and dS^T in the S^T buffer, B MN-major
+                        const uint32_t qb = ring + (g % STAGES) * C::STAGE, db = qb + C::BOXES * C::QBOX;
+#pragma unroll
+                        for (int kk = 0; kk < NQ / 16; ++kk) {
+                            const uint32_t acc = (i > 0 || kk > 0) ? 1u : 0u;
+                            const uint32_t pc = C::T_ST + pds_col(kk);
+                            umma_bf16_tmem_a(tmem + C::T_DV, tmem + pc, umma_desc_sw128(db + kk * 2048, C::QBOX, 1024),
+                                             idesc_o, acc);
+                            umma_bf16_tmem_a(tmem + C::T_DK, tmem + pc + 16,
+                                             umma_desc_sw128(qb + kk * 2048, C::QBOX, 1024), idesc_o, acc);
+                        }
+                        umma_commit(&qd_empty[g % STAGES]);
+                        if (more) {
+                            issue_one(g + 1, false);
+                            umma_commit(&s_full[0]);
+                            if (i + 2 == it.nqt) umma_commit(&kv_empty);
+                        }
+                    }
+                    if (!ok) break;
+                    umma_commit(&item_done);
+                    gt += it.nqt;
+                }
+            }
+            for (int idx = blockIdx.x; C::SBUF == 2 && ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
                 if (!mbar_wait(&kv_full, ic & 1u, limit)) {
                     ok = false;
@@ -789,11 +887,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             for (int i = 0; i < it.nqt; ++i) {
                 const uint32_t g = gt + i;
                 if (WGS == 2 && !C::SPLIT && static_cast<int>(g & 1u) != wg) continue;
-                if (!warp_wait(&s_full[g & 1u], (g >> 1) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
-                    ok = false;
-                    break;
-                }
-                tmem_fence_after();
+                const uint32_t sb = g % C::SBUF;
                 const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
                                                                      2 * C::BOXES * C::QBOX);
                 const float2* meta_ld = reinterpret_cast<const float2*>(meta + NQ);
@@ -802,14 +896,74 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 const int tq0 = it.tq0 + i * C::QT, tql = tq0 + C::QT - 1;
                 const bool inner =
                     C::INNER && __all_sync(kFull, kvalid && tql < a.n && key <= tq0 && key >= support_start(tql, h));
+                if (!warp_wait(&s_full[sb], (g / C::SBUF) & 1u, limit) || __any_sync(kFull, abort_s != 0)) {
+                    ok = false;
+                    break;
+                }
+                tmem_fence_after();
                 // KC columns at a time: their P^T and dS^T (KC/2 bf16-pair columns each) go over
                 // columns already read; with split columns this warpgroup takes columns
                 // [wg NQ/2, (wg+1) NQ/2)
                 constexpr int NW = C::SPLIT ? NQ / 2 : NQ;  // this warpgroup's columns of the tile
                 constexpr int KC = PBB_BWD_KV_KC < NW ? PBB_BWD_KV_KC : NW;
                 const int col0 = C::SPLIT ? wg * NW : 0;
+                if constexpr (C::SBUF == 1) {
+                    // 32 columns of S^T and dP^T at a time, before one wait; once the last
+                    // half's dP^T is in registers the dP^T buffer is free. Each half takes its own
+                    // P^T and dS^T pairs (16 columns each, pds_col) over its S^T columns
 #pragma unroll
-                for (int c = 0; c < NW / KC; ++c) {
+                    for (int hh = 0; hh < NW / 32; ++hh) {
+                        uint32_t v1[32], v2[32];
+                        tmem_ld32(lane_base + C::T_ST + col0 + 32 * hh, v1);
+                        tmem_ld32(lane_base + C::T_DPT + col0 + 32 * hh, v2);
+                        tmem_wait_ld();
+                        if (hh + 1 == NW / 32) {
+                            tmem_fence_before();
+                            mbar_arrive(&dp_free);
+                        }
+#pragma unroll
+                        for (int c2 = 0; c2 < 2; ++c2) {
+                            uint32_t pk[8], dk[8];
+                            if (inner) {
+#pragma unroll
+                                for (int x = 0; x < 8; ++x) {
+                                    const int j = 16 * c2 + 2 * x;
+                                    const float4 m = *reinterpret_cast<const float4*>(meta_ld + col0 + 32 * hh + j);
+                                    const float2 arg =
+                                        __ffma2_rn(make_float2(__uint_as_float(v1[j]), __uint_as_float(v1[j + 1])),
+                                                   make_float2(sc2, sc2), make_float2(m.x, m.z));
+                                    const float2 p = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                                    const float2 ds = __fmul2_rn(
+                                        p, __fadd2_rn(make_float2(__uint_as_float(v2[j]), __uint_as_float(v2[j + 1])),
+                                                      make_float2(m.y, m.w)));
+                                    pk[x] = pack_bf16x2(p.x, p.y);
+                                    dk[x] = pack_bf16x2(ds.x, ds.y);
+                                }
+                            } else {
+#pragma unroll
+                                for (int x = 0; x < 8; ++x) {
+                                    float pe[2], de[2];
+#pragma unroll
+                                    for (int y = 0; y < 2; ++y) {
+                                        const int j = 16 * c2 + 2 * x + y;
+                                        const float4 m = meta[col0 + 32 * hh + j];  // (lse2, D, t, a(t)); t = -1 past n
+                                        const int t = __float_as_int(m.z), at = __float_as_int(m.w);
+                                        const bool vis = kvalid && key <= t && key >= at;
+                                        const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[j]), sc2, -m.x)) : 0.f;
+                                        pe[y] = p;
+                                        de[y] = p * (__uint_as_float(v2[j]) - m.y);
+                                    }
+                                    pk[x] = pack_bf16x2(pe[0], pe[1]);
+                                    dk[x] = pack_bf16x2(de[0], de[1]);
+                                }
+                            }
+                            tmem_st8(lane_base + C::T_ST + col0 + 32 * hh + 8 * c2, pk);
+                            tmem_st8(lane_base + C::T_ST + col0 + 32 * hh + 16 + 8 * c2, dk);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int c = 0; C::SBUF == 2 && c < NW / KC; ++c) {
                     uint32_t v1[KC], v2[KC];
                     if constexpr (KC == 32) {
                         tmem_ld32(lane_base + C::T_ST + (g & 1u) * NQ + col0 + KC * c, v1);
@@ -863,7 +1017,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 }
                 tmem_wait_st();
                 tmem_fence_before();
-                mbar_arrive(&p_full[g & 1u]);
+                mbar_arrive(&p_full[sb]);
             }
             if (!ok) break;
             if (!warp_wait(&item_done, ic & 1u, limit)) {
@@ -981,6 +1135,11 @@ cudaError_t launch_bwd_shape(const BackwardArgs& a, cudaStream_t stream)
 #ifndef PBB_BWD_Q_NK
 #define PBB_BWD_Q_NK 128
 #endif
+// Query rows per tile of the dK/dV pass in the long shape: 128 (one S^T and one dP^T buffer) or 64
+// (two each).
+#ifndef PBB_BWD_KV_NQ
+#define PBB_BWD_KV_NQ 128
+#endif
 
 template <int D, int G>
 cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
@@ -989,7 +1148,7 @@ cudaError_t launch_bwd(const BackwardArgs& a, cudaStream_t stream)
         if (a.B < 512)
             return launch_bwd_shape<D, BqCfg<D, G, 32, 1, 2>, BkvCfg<D, G, 32, 1, 2>>(a, stream);
     }
-    return launch_bwd_shape<D, BqCfg<D, G, PBB_BWD_Q_NK, 2, 1>, BkvCfg<D, G, 64, 2, 1>>(a, stream);
+    return launch_bwd_shape<D, BqCfg<D, G, PBB_BWD_Q_NK, 2, 1>, BkvCfg<D, G, PBB_BWD_KV_NQ, 2, 1>>(a, stream);
 }
 
 template <int D>

@@ -95,6 +95,15 @@ def test_block_sizes(B):
     run_backward(w)
 
 
+@pytest.mark.parametrize("group", [2, 4])
+def test_long_shape_head_dim_64(group):
+    """d 64 with B = 1024: the one-CTA shape (128-row query tiles in the dK/dV pass, three
+    Q/dO stages at this head size) over ragged tiles and both half-blocks."""
+    w = inputs.SequenceWorkload(f"bwd_d64_B1024_g{group}", batch=1, Hq=2 * group, Hkv=2, d=64, B=1024, n=1500,
+                                seed=165 + group)
+    run_backward(w)
+
+
 @pytest.mark.parametrize("n", [1, 7, 65])
 def test_short_sequences(n):
     w = inputs.SequenceWorkload(f"bwd_n{n}", batch=2, Hq=4, Hkv=1, d=64, B=32, n=n, seed=170 + n)
