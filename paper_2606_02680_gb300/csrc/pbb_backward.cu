@@ -524,12 +524,15 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 //  - NQ = 64 or 32: S^T and dP^T, two buffers each (P^T and dS^T are written back over
 //    them as bf16 pairs, the A operands of dV += P^T dO and dK += dS^T Q), then dV and dK;
 //  - NQ = 128 (two elementwise warpgroups on split columns): S^T and dP^T one buffer each,
-//    then dV and dK (4 x 128 columns at d = 128). The warpgroups release the dP^T buffer once
-//    they hold the tile's dP^T in registers (dp_free), so the next tile's dP^T is issued
-//    while they compute; P^T and dS^T both go back over the S^T buffer, and the next tile's
-//    S^T follows the gradient products that read them. Every score product is an N = 128
-//    MMA: with both operands in shared memory, an N = 64 product runs at 2/3 of the tensor
-//    rate.
+//    then dV and dK (4 x 128 columns at d = 128). Every score product is an N = 128 MMA:
+//    with both operands in shared memory, an N = 64 product runs at 2/3 of the tensor rate.
+//    The score products end with one more K step, a column of ones against the tile's
+//    -lse2 / sc2 (S^T) or -D (dP^T) split into three bf16 terms, so the scores arrive with
+//    the per-column terms applied and the elementwise threads read no per-column data on
+//    unmasked tiles. P^T and dS^T both go back over the S^T buffer, and the next tile's S^T
+//    follows the gradient products that read them; its dP^T follows (dp_full), and the
+//    warpgroups compute a half's exponentials before they wait for it. They release the
+//    dP^T buffer once they hold the tile's dP^T (dp_free).
 // Shapes as for the dQ pass: NQ query rows per tile, WGS elementwise warpgroups, CTAS CTAs
 // per SM.
 // Columns of S^T and dP^T the elementwise threads load before each wait (16 or 32): fewer waits
@@ -545,20 +548,27 @@ struct BkvCfg {
     static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
     static constexpr int KBOX = M * 128, QBOX = NQ * 128;
     static constexpr int K_OFF = 0, V_OFF = BOXES * KBOX;
-    static constexpr int RING_OFF = 2 * BOXES * KBOX;
+    // one-buffer shape: the score products take -lse2 / sc2 and -D as one more K step against
+    // a column of ones (AUG): a 128 x 16 ones tile after K and V, and per stage the 16-wide
+    // extra K step of S^T and of dP^T (32-byte swizzle, 32 bytes a row)
+    static constexpr bool AUG = NQ == 128;
+    static constexpr int ONES_OFF = 2 * BOXES * KBOX, XROW = 32;
+    static constexpr int RING_OFF = ONES_OFF + (AUG ? M * XROW : 0);
     // per column (lse2, D, t, a(t)) as a float4 (one load per entry on the masked path); with
     // the packed path, (-lse2, -D) again as a float2 array (one load per column pair)
     static constexpr bool INNER = PBB_BWD_KV_INNER && CTAS == 1;
     static constexpr bool SPLIT = WGS == 2 && PBB_BWD_SPLIT_COLS;
     static constexpr int META = NQ * (INNER ? 24 : 16);
-    static constexpr int STAGE = (2 * BOXES * QBOX + META + 1023) / 1024 * 1024;  // Q, dO, metadata
+    static constexpr int META_OFF = 2 * BOXES * QBOX;
+    static constexpr int XS_OFF = (META_OFF + META + 255) / 256 * 256, XD_OFF = XS_OFF + NQ * XROW;
+    static constexpr int STAGE = ((AUG ? XD_OFF + NQ * XROW : META_OFF + META) + 1023) / 1024 * 1024;  // Q, dO, metadata (+ extra K steps)
     static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - RING_OFF) / STAGE;
     static constexpr int STAGE_MAX = CTAS == 1 ? 3 : 4;
     static constexpr int STAGES = STAGE_ROOM < STAGE_MAX ? STAGE_ROOM : STAGE_MAX;
     static constexpr int SMEM = RING_OFF + STAGES * STAGE + 1024;
     static constexpr int SBUF = NQ == 128 ? 1 : 2;  // S^T and dP^T buffers
     static constexpr int T_ST = 0, T_DPT = SBUF * NQ, T_DV = 2 * SBUF * NQ, T_DK = T_DV + D;
-    static_assert(SBUF == 2 || (SPLIT && CTAS == 1 && NQ == 128), "one score buffer: both warpgroups share every tile");
+    static_assert(SBUF == 2 || (SPLIT && CTAS == 1 && NQ == 128 && AUG), "one score buffer: both warpgroups share every tile");
     static_assert(STAGES >= 2, "shared memory budget");
     static_assert(T_DK + D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
@@ -573,6 +583,16 @@ struct BkvCfg {
 __host__ __device__ constexpr uint32_t pds_col(int kk)
 {
     return static_cast<uint32_t>(64 * (kk / 4) + 32 * ((kk % 4) / 2) + 8 * (kk % 2));
+}
+
+// The first 16-byte half of a 16-element bf16 K-step row holding x as three bf16 terms
+// (hi, mid, lo: x to about 24 bits, summed exactly by the fp32 accumulation), then zeros.
+__device__ __forceinline__ uint4 bf16_split3_row(float x)
+{
+    const float hi = __bfloat162float(__float2bfloat16_rn(x));
+    const float mid = __bfloat162float(__float2bfloat16_rn(x - hi));
+    const float lo = __bfloat162float(__float2bfloat16_rn(x - hi - mid));
+    return make_uint4(pack_bf16x2(hi, mid), pack_bf16x2(lo, 0.f), 0u, 0u);
 }
 
 struct KItem {
@@ -606,7 +626,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t kv_full, kv_empty, done_bar, item_done, o_free;
     __shared__ __align__(8) uint64_t qd_full[STAGES], qd_empty[STAGES];
-    __shared__ __align__(8) uint64_t s_full[2], p_full[2], dp_free;
+    __shared__ __align__(8) uint64_t s_full[2], p_full[2], dp_free, dp_full;
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
     unsigned char* dsmem = reinterpret_cast<unsigned char*>(
@@ -630,8 +650,14 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
             mbar_init(&p_full[b], C::SPLIT ? 256 : 128);  // the warpgroups that handle buffer b
         }
         mbar_init(&dp_free, C::SPLIT ? 256 : 128);  // one dP^T buffer: the warpgroups of a tile hold it
+        mbar_init(&dp_full, 1);                     // one dP^T buffer: its product is complete
         fence_mbar_init();
         abort_s = 0;
+    }
+    if constexpr (C::AUG) {  // the ones operand of the extra K step (bf16 1.0 everywhere, so unswizzled)
+        for (int i = tid; i < C::M * C::XROW / 16; i += C::THREADS)
+            reinterpret_cast<uint4*>(dsmem + C::ONES_OFF)[i] = make_uint4(0x3F803F80u, 0x3F803F80u, 0x3F803F80u, 0x3F803F80u);
+        fence_proxy_async();
     }
     if (warp == 0) tmem_alloc<C::TMEM_COLS>(&tmem_base_s);
     tmem_fence_before();
@@ -685,14 +711,25 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     break;
                 }
                 unsigned char* st = dsmem + C::RING_OFF + s * C::STAGE;
-                float4* meta = reinterpret_cast<float4*>(st + 2 * C::BOXES * C::QBOX);
+                float4* meta = reinterpret_cast<float4*>(st + C::META_OFF);
 #pragma unroll
                 for (int e = 0; e < MV; ++e) {
+                    const int c = lane + 32 * e;
                     mv[e].x *= kLog2e;
-                    meta[lane + 32 * e] = mv[e];
-                    if constexpr (C::INNER)
-                        reinterpret_cast<float2*>(meta + NQ)[lane + 32 * e] = make_float2(-mv[e].x, -mv[e].y);
+                    meta[c] = mv[e];
+                    if constexpr (C::INNER && !C::AUG)
+                        reinterpret_cast<float2*>(meta + NQ)[c] = make_float2(-mv[e].x, -mv[e].y);
+                    if constexpr (C::AUG) {
+                        // row c of the extra K steps: -lse2 / sc2 for S^T (so that sc2 S^T is the
+                        // exponent) and -D for dP^T, as bf16 hi/mid/lo; the second half zero
+                        const float sc2 = kLog2e * rsqrtf(static_cast<float>(D));
+                        *reinterpret_cast<uint4*>(st + C::XS_OFF + swz32(c, 0)) = bf16_split3_row(-mv[e].x / sc2);
+                        *reinterpret_cast<uint4*>(st + C::XS_OFF + swz32(c, 1)) = make_uint4(0u, 0u, 0u, 0u);
+                        *reinterpret_cast<uint4*>(st + C::XD_OFF + swz32(c, 0)) = bf16_split3_row(-mv[e].y);
+                        *reinterpret_cast<uint4*>(st + C::XD_OFF + swz32(c, 1)) = make_uint4(0u, 0u, 0u, 0u);
+                    }
                 }
+                if constexpr (C::AUG) fence_proxy_async();  // the MMAs read the extra K steps
                 __threadfence_block();
                 __syncwarp();
                 if (lane == 0) {
@@ -751,17 +788,23 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 return true;
             };
             if constexpr (C::SBUF == 1) {
-                // one score buffer per kind: tile g's dP^T goes in once the warpgroups hold tile
-                // g-1's, before tile g-1's gradient products; tile g's S^T after them
-                auto issue_one = [&](uint32_t g, bool dpt) {  // S^T = K Q^T, or dP^T = V dO^T
-                    const uint32_t qb = ring + (g % STAGES) * C::STAGE + (dpt ? C::BOXES * C::QBOX : 0);
+                // one score buffer per kind: tile g's S^T goes in after tile g-1's gradient
+                // products (they read P^T and dS^T from the S^T buffer), then its dP^T (once the
+                // warpgroups hold tile g-1's). S^T = K Q^T - (lse2 / sc2) 1^T and
+                // dP^T = V dO^T - D 1^T: the last K step is the ones tile against the stage's row
+                // of -lse2 / sc2 (or -D) terms
+                const uint32_t ones = smem_addr(dsmem + C::ONES_OFF);
+                auto issue_one = [&](uint32_t g, bool dpt) {
+                    const uint32_t sbase = ring + (g % STAGES) * C::STAGE;
+                    const uint32_t qb = sbase + (dpt ? C::BOXES * C::QBOX : 0);
                     const uint32_t ab = dpt ? v_base : k_base;
+                    const uint32_t dst = tmem + (dpt ? C::T_DPT : C::T_ST);
 #pragma unroll
                     for (int kk = 0; kk < D / 16; ++kk)
-                        umma_bf16(tmem + (dpt ? C::T_DPT : C::T_ST),
-                                  umma_desc_sw128(ab + (kk >> 2) * C::KBOX + (kk & 3) * 32, 16, 1024),
+                        umma_bf16(dst, umma_desc_sw128(ab + (kk >> 2) * C::KBOX + (kk & 3) * 32, 16, 1024),
                                   umma_desc_sw128(qb + (kk >> 2) * C::QBOX + (kk & 3) * 32, 16, 1024), idesc_s,
                                   kk > 0 ? 1u : 0u);
+                    umma_bf16(dst, umma_desc_sw32(ones), umma_desc_sw32(sbase + (dpt ? C::XD_OFF : C::XS_OFF)), idesc_s, 1u);
                 };
                 auto dp_ready = [&](uint32_t g) {
                     if (g == 0) return true;
@@ -777,22 +820,35 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     }
                     tmem_fence_after();
                     issue_one(gt, false);
+                    umma_commit(&s_full[0]);
                     issued_any = true;
                     if (!dp_ready(gt)) {
                         ok = false;
                         break;
                     }
                     issue_one(gt, true);
-                    umma_commit(&s_full[0]);
+                    umma_commit(&dp_full);
                     if (it.nqt == 1) umma_commit(&kv_empty);  // the item's last read of K and V
                     for (int i = 0; i < it.nqt; ++i) {
                         const uint32_t g = gt + i;
                         const bool more = i + 1 < it.nqt;
-                        if (more && (!dp_ready(g + 1) || !qd_ready(g + 1))) {
-                            ok = false;
-                            break;
+                        // the next tile's dP^T goes ahead of this tile's gradient products if its
+                        // Q/dO stage has landed; else after its S^T, so that waiting for the copy
+                        // does not hold back the products whose completion frees the other stage
+                        // (the warpgroups compute the exponentials of S^T before they need dP^T)
+                        bool dp_early = false;
+                        if (more) {
+                            if (!dp_ready(g + 1)) {
+                                ok = false;
+                                break;
+                            }
+                            dp_early = mbar_test(&qd_full[(g + 1) % STAGES], ((g + 1) / STAGES) & 1u);
+                            if (dp_early) {
+                                tmem_fence_after();
+                                issue_one(g + 1, true);
+                                umma_commit(&dp_full);
+                            }
                         }
-                        if (more) issue_one(g + 1, true);
                         if (!mbar_wait(&p_full[0], g & 1u, limit) ||
                             (i == 0 && ic >= 1 && !mbar_wait(&o_free, (ic - 1) & 1u, limit))) {
                             ok = false;
@@ -812,8 +868,16 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                         }
                         umma_commit(&qd_empty[g % STAGES]);
                         if (more) {
+                            if (!dp_early && !qd_ready(g + 1)) {
+                                ok = false;
+                                break;
+                            }
                             issue_one(g + 1, false);
                             umma_commit(&s_full[0]);
+                            if (!dp_early) {
+                                issue_one(g + 1, true);
+                                umma_commit(&dp_full);
+                            }
                             if (i + 2 == it.nqt) umma_commit(&kv_empty);
                         }
                     }
@@ -888,8 +952,8 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 const uint32_t g = gt + i;
                 if (WGS == 2 && !C::SPLIT && static_cast<int>(g & 1u) != wg) continue;
                 const uint32_t sb = g % C::SBUF;
-                const float4* meta = reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE +
-                                                                     2 * C::BOXES * C::QBOX);
+                const float4* meta =
+                    reinterpret_cast<const float4*>(dsmem + C::RING_OFF + (g % STAGES) * C::STAGE + C::META_OFF);
                 const float2* meta_ld = reinterpret_cast<const float2*>(meta + NQ);
                 // a tile whose every query sees every key of the warp's rows needs no mask: the
                 // packed path (bit-identical arithmetic, half the instructions)
@@ -908,13 +972,40 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 constexpr int KC = PBB_BWD_KV_KC < NW ? PBB_BWD_KV_KC : NW;
                 const int col0 = C::SPLIT ? wg * NW : 0;
                 if constexpr (C::SBUF == 1) {
-                    // 32 columns of S^T and dP^T at a time, before one wait; once the last
-                    // half's dP^T is in registers the dP^T buffer is free. Each half takes its own
-                    // P^T and dS^T pairs (16 columns each, pds_col) over its S^T columns
+                    // 32 columns at a time: S^T and its exponentials first, then (once its product
+                    // is complete) dP^T; after the last half's dP^T loads the dP^T buffer is free.
+                    // Each half takes its own P^T and dS^T pairs (16 columns each, pds_col) over
+                    // its S^T columns. The scores already hold -lse2 / sc2 and -D (the extra K
+                    // step), so the packed path reads no per-column data: P = 2^(sc2 S^T),
+                    // dS = P dP^T
 #pragma unroll
                     for (int hh = 0; hh < NW / 32; ++hh) {
                         uint32_t v1[32], v2[32];
                         tmem_ld32(lane_base + C::T_ST + col0 + 32 * hh, v1);
+                        tmem_wait_ld();
+                        float pr[32];
+                        if (inner) {
+#pragma unroll
+                            for (int x = 0; x < 16; ++x) {
+                                const float2 arg = __fmul2_rn(
+                                    make_float2(__uint_as_float(v1[2 * x]), __uint_as_float(v1[2 * x + 1])), make_float2(sc2, sc2));
+                                pr[2 * x] = fast_exp2(arg.x);
+                                pr[2 * x + 1] = fast_exp2(arg.y);
+                            }
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) {
+                                const float4 m = meta[col0 + 32 * hh + j];  // (lse2, D, t, a(t)); t = -1 past n
+                                const int t = __float_as_int(m.z), at = __float_as_int(m.w);
+                                const bool vis = kvalid && key <= t && key >= at;
+                                pr[j] = vis ? fast_exp2(__uint_as_float(v1[j]) * sc2) : 0.f;
+                            }
+                        }
+                        if (hh == 0 && !warp_wait(&dp_full, g & 1u, limit)) {
+                            ok = false;
+                            break;
+                        }
+                        if (hh == 0) tmem_fence_after();
                         tmem_ld32(lane_base + C::T_DPT + col0 + 32 * hh, v2);
                         tmem_wait_ld();
                         if (hh + 1 == NW / 32) {
@@ -924,43 +1015,19 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
 #pragma unroll
                         for (int c2 = 0; c2 < 2; ++c2) {
                             uint32_t pk[8], dk[8];
-                            if (inner) {
 #pragma unroll
-                                for (int x = 0; x < 8; ++x) {
-                                    const int j = 16 * c2 + 2 * x;
-                                    const float4 m = *reinterpret_cast<const float4*>(meta_ld + col0 + 32 * hh + j);
-                                    const float2 arg =
-                                        __ffma2_rn(make_float2(__uint_as_float(v1[j]), __uint_as_float(v1[j + 1])),
-                                                   make_float2(sc2, sc2), make_float2(m.x, m.z));
-                                    const float2 p = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
-                                    const float2 ds = __fmul2_rn(
-                                        p, __fadd2_rn(make_float2(__uint_as_float(v2[j]), __uint_as_float(v2[j + 1])),
-                                                      make_float2(m.y, m.w)));
-                                    pk[x] = pack_bf16x2(p.x, p.y);
-                                    dk[x] = pack_bf16x2(ds.x, ds.y);
-                                }
-                            } else {
-#pragma unroll
-                                for (int x = 0; x < 8; ++x) {
-                                    float pe[2], de[2];
-#pragma unroll
-                                    for (int y = 0; y < 2; ++y) {
-                                        const int j = 16 * c2 + 2 * x + y;
-                                        const float4 m = meta[col0 + 32 * hh + j];  // (lse2, D, t, a(t)); t = -1 past n
-                                        const int t = __float_as_int(m.z), at = __float_as_int(m.w);
-                                        const bool vis = kvalid && key <= t && key >= at;
-                                        const float p = vis ? fast_exp2(fmaf(__uint_as_float(v1[j]), sc2, -m.x)) : 0.f;
-                                        pe[y] = p;
-                                        de[y] = p * (__uint_as_float(v2[j]) - m.y);
-                                    }
-                                    pk[x] = pack_bf16x2(pe[0], pe[1]);
-                                    dk[x] = pack_bf16x2(de[0], de[1]);
-                                }
+                            for (int x = 0; x < 8; ++x) {
+                                const int j = 16 * c2 + 2 * x;
+                                const float2 p = make_float2(pr[j], pr[j + 1]);
+                                const float2 ds = __fmul2_rn(p, make_float2(__uint_as_float(v2[j]), __uint_as_float(v2[j + 1])));
+                                pk[x] = pack_bf16x2(p.x, p.y);
+                                dk[x] = pack_bf16x2(ds.x, ds.y);
                             }
                             tmem_st8(lane_base + C::T_ST + col0 + 32 * hh + 8 * c2, pk);
                             tmem_st8(lane_base + C::T_ST + col0 + 32 * hh + 16 + 8 * c2, dk);
                         }
                     }
+                    if (!ok) break;
                 }
 #pragma unroll
                 for (int c = 0; C::SBUF == 2 && c < NW / KC; ++c) {

@@ -108,6 +108,14 @@ __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, i
         : "memory");
 }
 
+// Prefetch one tensor-map box into L2 (no shared memory written, no barrier).
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap* map, int x, int y)
+{
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
+
 __device__ __forceinline__ void ldmatrix_x4(uint32_t (&r)[4], uint32_t addr)
 {
     asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
@@ -191,6 +199,25 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr, uint32_t lbo
     d |= 1ull << 46;
     d |= 2ull << 61;
     return d;
+}
+
+// Shared-memory matrix descriptor of a K-major operand one 16-element bf16 K step wide in the
+// 32-byte swizzle layout (layout type 6): rows of 32 bytes, 8-row atoms of 256 bytes, the two
+// 16-byte halves of row r swapped when bit 2 of r is set.
+__device__ __forceinline__ uint64_t umma_desc_sw32(uint32_t saddr)
+{
+    uint64_t d = static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+    d |= static_cast<uint64_t>(16u >> 4) << 16;
+    d |= static_cast<uint64_t>(256u >> 4) << 32;
+    d |= 1ull << 46;
+    d |= 6ull << 61;
+    return d;
+}
+
+// Byte offset of 16-byte half `c` of row `r` in a 32-byte-swizzled tile.
+__host__ __device__ constexpr uint32_t swz32(int r, int c)
+{
+    return static_cast<uint32_t>(r * 32 + ((c ^ ((r >> 2) & 1)) << 4));
 }
 
 // Instruction descriptor of kind::f16 with bf16 A and B, fp32 accumulation, A K-major,
