@@ -159,11 +159,16 @@ struct BqCfg {
     static constexpr int TMEM_COLS = CTAS == 1 ? 512 : 256;
     static constexpr int QBOX = M * 128, KBOX = NK * 128;
     static constexpr int Q_OFF = 0, DO_OFF = BOXES * QBOX;
+    // K and V in rings of their own: V is read by the dP product alone and its stage is free
+    // again long before K's, which the dQ product reads too; K takes the odd stage (3 K + 2 V
+    // at d = 128 in the long shape, where 2 + 2 left the MMA thread waiting for K)
     static constexpr int KV_OFF = 2 * BOXES * QBOX;
-    static constexpr int KV_STAGE = 2 * BOXES * KBOX;
-    static constexpr int STAGE_ROOM = (227 * 1024 / CTAS - 2048 - KV_OFF) / KV_STAGE;
-    static constexpr int STAGES = STAGE_ROOM < 4 ? STAGE_ROOM : 4;
-    static constexpr int SMEM = KV_OFF + STAGES * KV_STAGE + 1024;
+    static constexpr int K_STAGE = BOXES * KBOX;  // = V's
+    static constexpr int ROOM = (227 * 1024 / CTAS - 2048 - KV_OFF) / K_STAGE;
+    static constexpr int UNITS = ROOM < 8 ? ROOM : 8;
+    static constexpr int KST = (UNITS + 1) / 2, VST = UNITS / 2;
+    static constexpr int V_OFF = KV_OFF + KST * K_STAGE;
+    static constexpr int SMEM = V_OFF + VST * K_STAGE + 1024;
     static constexpr int DPBUF = NK == 128 ? 1 : 2;            // dP buffers
     static constexpr int T_S = 0, T_DP = 2 * NK, T_DQ = T_DP + DPBUF * NK;
     static constexpr int OBUF = T_DQ + 2 * D <= TMEM_COLS ? 2 : 1;
@@ -171,7 +176,7 @@ struct BqCfg {
     static constexpr bool SPLIT = WGS == 2 && PBB_BWD_SPLIT_COLS;
     static_assert(DPBUF == 2 || (PBB_BWD_Q_QC >= NK / (SPLIT ? 2 : 1)),
                   "one dP buffer: each warpgroup loads its columns of a tile before one wait");
-    static_assert(STAGES >= 2, "shared memory budget");
+    static_assert(VST >= 2, "shared memory budget");
     static_assert(T_DQ + OBUF * D <= TMEM_COLS, "TMEM budget");
     static_assert(CTAS * (SMEM + 1024) <= 227 * 1024, "shared memory budget");
     static_assert(QT % 8 == 0, "a head's rows must start on a swizzle atom");
@@ -204,10 +209,10 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 const BackwardArgs a)
 {
     using C = BqCfg<D, G, NK_, WGS_, CTAS_>;
-    constexpr int STAGES = C::STAGES, NK = C::NK, WGS = C::WGS, OBUF = C::OBUF;
+    constexpr int KST = C::KST, VST = C::VST, NK = C::NK, WGS = C::WGS, OBUF = C::OBUF;
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t q_full, q_empty, done_bar;
-    __shared__ __align__(8) uint64_t kv_full[STAGES], kv_empty[STAGES];
+    __shared__ __align__(8) uint64_t k_full[KST], k_empty[KST], v_full[VST], v_empty[VST];
     __shared__ __align__(8) uint64_t s_full[2], ds_full[2], item_done[2], o_free[2], dp_free;
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
@@ -220,9 +225,14 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         mbar_init(&q_empty, 1);
         mbar_init(&done_bar, 1);
 #pragma unroll
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&kv_full[s], 1);
-            mbar_init(&kv_empty[s], 1);
+        for (int s = 0; s < KST; ++s) {
+            mbar_init(&k_full[s], 1);
+            mbar_init(&k_empty[s], 1);
+        }
+#pragma unroll
+        for (int s = 0; s < VST; ++s) {
+            mbar_init(&v_full[s], 1);
+            mbar_init(&v_empty[s], 1);
         }
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
@@ -244,7 +254,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
 
     if (warp == C::PRODUCER) {
         if (lane == 0) {
-            uint32_t gt = 0, ic = 0, q_issued = 0;
+            uint32_t gt = 0, ic = 0, q_issued = 0, k_issued = 0, v_issued = 0;
             bool ok = true;
             for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
@@ -266,8 +276,8 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 ++q_issued;
                 const int krow0 = it.pair * a.n + it.lo;
                 for (int j = 0; j < it.ntiles; ++j, ++gt) {
-                    const int s = gt % STAGES;
-                    if (gt >= STAGES && !mbar_wait(&kv_empty[s], ((gt / STAGES) - 1) & 1u, limit)) {
+                    const int sk = gt % KST, sv = gt % VST;
+                    if (gt >= KST && !mbar_wait(&k_empty[sk], ((gt / KST) - 1) & 1u, limit)) {
                         ok = false;
                         break;
                     }
@@ -275,13 +285,22 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                         ok = false;
                         break;
                     }
-                    unsigned char* st = dsmem + C::KV_OFF + s * C::KV_STAGE;
-                    mbar_expect_tx(&kv_full[s], static_cast<uint32_t>(C::KV_STAGE));
+                    unsigned char* kst = dsmem + C::KV_OFF + sk * C::K_STAGE;
+                    mbar_expect_tx(&k_full[sk], static_cast<uint32_t>(C::K_STAGE));
 #pragma unroll
-                    for (int bx = 0; bx < C::BOXES; ++bx) {
-                        tma_load_2d(st + bx * C::KBOX, &kmap, bx * 64, krow0 + j * NK, &kv_full[s]);
-                        tma_load_2d(st + (C::BOXES + bx) * C::KBOX, &vmap, bx * 64, krow0 + j * NK, &kv_full[s]);
+                    for (int bx = 0; bx < C::BOXES; ++bx)
+                        tma_load_2d(kst + bx * C::KBOX, &kmap, bx * 64, krow0 + j * NK, &k_full[sk]);
+                    ++k_issued;
+                    if (gt >= VST && !mbar_wait(&v_empty[sv], ((gt / VST) - 1) & 1u, limit)) {
+                        ok = false;
+                        break;
                     }
+                    unsigned char* vst = dsmem + C::V_OFF + sv * C::K_STAGE;
+                    mbar_expect_tx(&v_full[sv], static_cast<uint32_t>(C::K_STAGE));
+#pragma unroll
+                    for (int bx = 0; bx < C::BOXES; ++bx)
+                        tma_load_2d(vst + bx * C::KBOX, &vmap, bx * 64, krow0 + j * NK, &v_full[sv]);
+                    ++v_issued;
                 }
             }
             if (!ok) {
@@ -290,9 +309,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             }
             // drain: the last copies into Q/dO and into each stage land before shared memory goes away
             if (q_issued > 0) mbar_wait(&q_full, (q_issued - 1) & 1u, kGuardNs);
-            for (uint32_t s = 0; s < STAGES && s < gt; ++s) {
-                const uint32_t j = s + STAGES * ((gt - 1 - s) / STAGES);
-                mbar_wait(&kv_full[s], (j / STAGES) & 1u, kGuardNs);
+            for (uint32_t s = 0; s < KST && s < k_issued; ++s) {
+                const uint32_t j = s + KST * ((k_issued - 1 - s) / KST);
+                mbar_wait(&k_full[s], (j / KST) & 1u, kGuardNs);
+            }
+            for (uint32_t s = 0; s < VST && s < v_issued; ++s) {
+                const uint32_t j = s + VST * ((v_issued - 1 - s) / VST);
+                mbar_wait(&v_full[s], (j / VST) & 1u, kGuardNs);
             }
         }
     } else if (warp == C::MMA) {
@@ -300,13 +323,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             constexpr uint32_t idesc_s = umma_idesc_bf16(C::M, NK, 0);
             constexpr uint32_t idesc_q = umma_idesc_bf16(C::M, D, 1);
             const uint32_t q_base = smem_addr(dsmem + C::Q_OFF), do_base = smem_addr(dsmem + C::DO_OFF);
-            const uint32_t kv_base = smem_addr(dsmem + C::KV_OFF);
+            const uint32_t k_base = smem_addr(dsmem + C::KV_OFF), v_base = smem_addr(dsmem + C::V_OFF);
             uint32_t gt = 0, ic = 0;
             bool ok = true, issued_any = false;
             // S = Q K^T into buffer g % 2, and dP = dO V^T into buffer g % DPBUF; the commit of
-            // s_full covers both
+            // s_full covers both, and dP's own commit frees V's stage
             auto issue_s = [&](uint32_t g) {
-                const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
+                const uint32_t kb = k_base + (g % KST) * C::K_STAGE;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * C::QBOX + (kk & 3) * 32;
@@ -316,7 +339,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 }
             };
             auto issue_dp = [&](uint32_t g) {
-                const uint32_t vb = kv_base + (g % STAGES) * C::KV_STAGE + C::BOXES * C::KBOX;
+                const uint32_t vb = v_base + (g % VST) * C::K_STAGE;
 #pragma unroll
                 for (int kk = 0; kk < D / 16; ++kk) {
                     const uint32_t off = (kk >> 2) * C::QBOX + (kk & 3) * 32;
@@ -324,7 +347,14 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     umma_bf16(tmem + C::T_DP + (g % C::DPBUF) * NK, umma_desc_sw128(do_base + off, 16, 1024),
                               umma_desc_sw128(vb + koff, 16, 1024), idesc_s, kk > 0 ? 1u : 0u);
                 }
+                umma_commit(&v_empty[g % VST]);
                 umma_commit(&s_full[g & 1u]);
+            };
+            auto k_ready = [&](uint32_t g) { return mbar_wait(&k_full[g % KST], (g / KST) & 1u, limit); };
+            auto v_ready = [&](uint32_t g) {
+                if (!mbar_wait(&v_full[g % VST], (g / VST) & 1u, limit)) return false;
+                tmem_fence_after();
+                return true;
             };
             // with one dP buffer, tile g's dP goes in once the warpgroups hold tile g-1's
             auto dp_ready = [&](uint32_t g) {
@@ -336,14 +366,14 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
             for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
                 const uint32_t ob = ic % OBUF;
-                if (!mbar_wait(&q_full, ic & 1u, limit) || !mbar_wait(&kv_full[gt % STAGES], (gt / STAGES) & 1u, limit)) {
+                if (!mbar_wait(&q_full, ic & 1u, limit) || !k_ready(gt)) {
                     ok = false;
                     break;
                 }
                 tmem_fence_after();
                 issue_s(gt);
                 issued_any = true;
-                if (!dp_ready(gt)) {
+                if (!dp_ready(gt) || !v_ready(gt)) {
                     ok = false;
                     break;
                 }
@@ -352,13 +382,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 for (int j = 0; j < it.ntiles; ++j) {
                     const uint32_t g = gt + j;
                     if (j + 1 < it.ntiles) {
-                        if (!mbar_wait(&kv_full[(g + 1) % STAGES], ((g + 1) / STAGES) & 1u, limit)) {
+                        if (!k_ready(g + 1)) {
                             ok = false;
                             break;
                         }
                         tmem_fence_after();
                         issue_s(g + 1);
-                        if (!dp_ready(g + 1)) {
+                        if (!dp_ready(g + 1) || !v_ready(g + 1)) {
                             ok = false;
                             break;
                         }
@@ -372,13 +402,13 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                     }
                     tmem_fence_after();
                     // dQ (+)= dS K: dS from TMEM (over S buffer g % 2), K MN-major
-                    const uint32_t kb = kv_base + (g % STAGES) * C::KV_STAGE;
+                    const uint32_t kb = k_base + (g % KST) * C::K_STAGE;
 #pragma unroll
                     for (int kk = 0; kk < NK / 16; ++kk)
                         umma_bf16_tmem_a(tmem + C::T_DQ + ob * D, tmem + C::T_S + (g & 1u) * NK + pair_col<NK, C::SPLIT>(kk),
                                          umma_desc_sw128(kb + kk * 2048, C::KBOX, 1024), idesc_q,
                                          (j > 0 || kk > 0) ? 1u : 0u);
-                    umma_commit(&kv_empty[g % STAGES]);
+                    umma_commit(&k_empty[g % KST]);
                 }
                 if (!ok) break;
                 umma_commit(&item_done[ob]);
