@@ -55,6 +55,16 @@ __device__ __forceinline__ int support_start(int t, int h)
     return m > 0 ? h * (m - 1) : 0;
 }
 
+// Work item of round r for this CTA of a persistent grid: round r covers items
+// [r G, (r + 1) G) (G = grid size), and the CTA's slot in it turns by one each round. Item
+// lengths repeat along the index (a key item's length depends on its place in its
+// half-block), so a fixed slot gave some CTAs only the longest items: at B 4096 the busiest
+// CTA of the dK/dV pass had 17.5 % more query tiles than the mean, 6.3 % with the turn.
+__device__ __forceinline__ int rotated_item(int r)
+{
+    return r * static_cast<int>(gridDim.x) + static_cast<int>((blockIdx.x + static_cast<unsigned>(r)) % gridDim.x);
+}
+
 // A bounded wait whose outcome is the same in every lane of the warp (warp-collective
 // tcgen05 loads and stores follow it).
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)
@@ -256,7 +266,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         if (lane == 0) {
             uint32_t gt = 0, ic = 0, q_issued = 0, k_issued = 0, v_issued = 0;
             bool ok = true;
-            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
                 const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
                 if (ic > 0 && !mbar_wait(&q_empty, (ic - 1) & 1u, limit)) {
@@ -363,7 +373,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 tmem_fence_after();
                 return true;
             };
-            for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
                 const uint32_t ob = ic % OBUF;
                 if (!mbar_wait(&q_full, ic & 1u, limit) || !k_ready(gt)) {
@@ -433,7 +443,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         const int gi = r / C::QT, rp = r - gi * C::QT;
         uint32_t gt = 0, ic = 0;
         bool ok = true;
-        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
             const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
             const uint32_t ob = ic % OBUF;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
@@ -701,7 +711,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         // the whole warp: lane 0 issues the copies, every lane stages two columns' metadata
         uint32_t gt = 0, ic = 0, kv_issued = 0;
         bool ok = true;
-        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
             const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
             if (ic > 0 && !warp_wait(&kv_empty, (ic - 1) & 1u, limit)) {
@@ -842,7 +852,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     tmem_fence_after();
                     return true;
                 };
-                for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+                for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
                     const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
                     if (!mbar_wait(&kv_full, ic & 1u, limit) || !qd_ready(gt)) {
                         ok = false;
@@ -916,7 +926,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     gt += it.nqt;
                 }
             }
-            for (int idx = blockIdx.x; C::SBUF == 2 && ok && idx < n_items; idx += gridDim.x, ++ic) {
+            for (int rd = 0, idx = rotated_item(0); C::SBUF == 2 && ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
                 const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
                 if (!mbar_wait(&kv_full, ic & 1u, limit)) {
                     ok = false;
@@ -974,7 +984,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
         uint32_t gt = 0, ic = 0;
         bool ok = true;
-        for (int idx = blockIdx.x; ok && idx < n_items; idx += gridDim.x, ++ic) {
+        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
             const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
             const int key = it.s0 + r;
             const bool kvalid = key < a.n;
