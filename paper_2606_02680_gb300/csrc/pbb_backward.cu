@@ -55,16 +55,6 @@ __device__ __forceinline__ int support_start(int t, int h)
     return m > 0 ? h * (m - 1) : 0;
 }
 
-// Work item of round r for this CTA of a persistent grid: round r covers items
-// [r G, (r + 1) G) (G = grid size), and the CTA's slot in it turns by one each round. Item
-// lengths repeat along the index (a key item's length depends on its place in its
-// half-block), so a fixed slot gave some CTAs only the longest items: at B 4096 the busiest
-// CTA of the dK/dV pass had 17.5 % more query tiles than the mean, 6.3 % with the turn.
-__device__ __forceinline__ int rotated_item(int r)
-{
-    return r * static_cast<int>(gridDim.x) + static_cast<int>((blockIdx.x + static_cast<unsigned>(r)) % gridDim.x);
-}
-
 // A bounded wait whose outcome is the same in every lane of the warp (warp-collective
 // tcgen05 loads and stores follow it).
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsigned long long limit)

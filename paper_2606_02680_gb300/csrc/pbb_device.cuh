@@ -201,6 +201,17 @@ __device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr, uint32_t lbo
     return d;
 }
 
+// Work item of round r for this CTA of a persistent grid: round r covers items
+// [r G, (r + 1) G) (G = grid size), and the CTA's slot in it turns by one each round. Item
+// lengths repeat along the index (a key item's length depends on its place in its
+// half-block, a query item's support on its position), so a fixed slot gave some CTAs only
+// the longest items: at B 4096 the busiest CTA of the backward's dK/dV pass had 17.5 % more
+// work than the mean (6.3 % with the turn), of the paired forward 7.7 % (3.0 %).
+__device__ __forceinline__ int rotated_item(int r)
+{
+    return r * static_cast<int>(gridDim.x) + static_cast<int>((blockIdx.x + static_cast<unsigned>(r)) % gridDim.x);
+}
+
 // Shared-memory matrix descriptor of a K-major operand one 16-element bf16 K step wide in the
 // 32-byte swizzle layout (layout type 6): rows of 32 bytes, 8-row atoms of 256 bytes, the two
 // 16-byte halves of row r swapped when bit 2 of r is set.
