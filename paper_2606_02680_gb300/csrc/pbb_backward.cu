@@ -256,7 +256,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         if (lane == 0) {
             uint32_t gt = 0, ic = 0, q_issued = 0, k_issued = 0, v_issued = 0;
             bool ok = true;
-            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+            for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
                 const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
                 if (ic > 0 && !mbar_wait(&q_empty, (ic - 1) & 1u, limit)) {
@@ -363,7 +363,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 tmem_fence_after();
                 return true;
             };
-            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+            for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
                 const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
                 const uint32_t ob = ic % OBUF;
                 if (!mbar_wait(&q_full, ic & 1u, limit) || !k_ready(gt)) {
@@ -433,7 +433,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
         const int gi = r / C::QT, rp = r - gi * C::QT;
         uint32_t gt = 0, ic = 0;
         bool ok = true;
-        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+        for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
             const QItem it = make_qitem<C::QT, NK>(idx, a.n, a.B);
             const uint32_t ob = ic % OBUF;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
@@ -701,7 +701,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         // the whole warp: lane 0 issues the copies, every lane stages two columns' metadata
         uint32_t gt = 0, ic = 0, kv_issued = 0;
         bool ok = true;
-        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+        for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
             const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
             if (ic > 0 && !warp_wait(&kv_empty, (ic - 1) & 1u, limit)) {
@@ -842,7 +842,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     tmem_fence_after();
                     return true;
                 };
-                for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+                for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
                     const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
                     if (!mbar_wait(&kv_full, ic & 1u, limit) || !qd_ready(gt)) {
                         ok = false;
@@ -916,7 +916,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                     gt += it.nqt;
                 }
             }
-            for (int rd = 0, idx = rotated_item(0); C::SBUF == 2 && ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+            for (int rd = 0, idx = item_turned(0); C::SBUF == 2 && ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
                 const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
                 if (!mbar_wait(&kv_full, ic & 1u, limit)) {
                     ok = false;
@@ -974,7 +974,7 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
         const float sc2 = kLog2e * rsqrtf(static_cast<float>(D)), sc = rsqrtf(static_cast<float>(D));
         uint32_t gt = 0, ic = 0;
         bool ok = true;
-        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+        for (int rd = 0, idx = item_turned(0); ok && idx < n_items; ++rd, idx = item_turned(rd), ++ic) {
             const KItem it = make_kitem<C::QT>(idx, a.n, a.B);
             const int key = it.s0 + r;
             const bool kvalid = key < a.n;

@@ -230,7 +230,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&vmap)) : "memory");
             uint32_t gt = 0, ic = 0, q_issued = 0;  // tiles, items and Q loads issued
             bool ok = true;
-            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+            for (int rd = 0, idx = item_mirrored(0); ok && idx < n_items; ++rd, idx = item_mirrored(rd), ++ic) {
                 const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
                 const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
                 const uint32_t qb = ic % QBUF;
@@ -302,7 +302,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 }
                 umma_commit(&s_full[g & 1u]);
             };
-            for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+            for (int rd = 0, idx = item_mirrored(0); ok && idx < n_items; ++rd, idx = item_mirrored(rd), ++ic) {
                 const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
                 const uint32_t ob = ic % C::OBUF;
                 const uint32_t qb = ic % QBUF;
@@ -376,7 +376,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
         const int gi = r / C::QT, rp = r - gi * C::QT;
         uint32_t gt = 0, ic = 0;
         bool ok = true;
-        for (int rd = 0, idx = rotated_item(0); ok && idx < n_items; ++rd, idx = rotated_item(rd), ++ic) {
+        for (int rd = 0, idx = item_mirrored(0); ok && idx < n_items; ++rd, idx = item_mirrored(rd), ++ic) {
             const Item it = make_item<C::QT, C::NK>(idx, a.n, a.B);
             const uint32_t ob = ic % C::OBUF;
             const uint32_t o_col = C::T_O + ob * D + wg * OC;  // this thread's output columns
@@ -721,7 +721,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 if (qk) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
                 uint32_t gt = 0, issued = 0, ic[2] = {0, 0}, q_issued[2] = {0, 0};
                 bool ok = true;
-                for (int rd = 0, sidx = rotated_item(0); ok && sidx < n_sitems; ++rd, sidx = rotated_item(rd)) {
+                for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
                     const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
                     const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
                     if (qk) {
@@ -789,7 +789,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 uint32_t gk = 0, gv = 0;                  // K and V tiles consumed
                 uint32_t ic[2] = {0, 0}, gp[2] = {0, 0};  // items and P tiles consumed, per item slot
                 bool ok = true, issued_any = false;
-                for (int rd = 0, sidx = rotated_item(0); ok && sidx < n_sitems; ++rd, sidx = rotated_item(rd)) {
+                for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
                     const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
                     const int jb[2] = {0, it.hasB ? it.jB0 : it.nt};  // first and end tile of each item
                     const int je[2] = {it.ntA, it.nt};
@@ -876,7 +876,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
         const int gi = r / C::QT, rp = r - gi * C::QT;
         uint32_t g = 0, ic = 0;  // this item slot's tiles and items so far
         bool ok = true;
-        for (int rd = 0, sidx = rotated_item(0); ok && sidx < n_sitems; ++rd, sidx = rotated_item(rd)) {
+        for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
             const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
             if (x == 1 && !it.hasB) continue;
             const int t0 = it.t0 + x * C::QT, tl = x == 0 ? it.tlA : it.tlB;
