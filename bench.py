@@ -874,6 +874,11 @@ def run_ours(args):
         kernel = ("decode_kernel_tc<%d>" % w.d
                   if pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, inputs.torch_dtype(w)) == "tensor_cores"
                   else "decode_kernel<%d,%d,%d>" % (w.elem_bytes, w.d, w.group))
+        # a decode call of this batch sorts its sequences by support length first (one more launch)
+        call_batch = w.batch * (args.layers if args.layer_launches == "one" else 1)
+        ordered = int(pbb.plan_support_order(call_batch, w.Hq, w.Hkv, w.d, w.B, window or 0, inputs.torch_dtype(w)))
+        if ordered:
+            kernel += " after support_order_kernel"
         line = {
             "metric": METRIC if window is None else METRIC_SWA, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_s * 1e3 / args.steps,
@@ -897,7 +902,7 @@ def run_ours(args):
                          "kernel_ms_median": res["kernel_ms_median"]},
             "clocks": res["clocks"],
             "timing": res["timing"],
-            "gpu_launches": 2 * args.steps,
+            "gpu_launches": (2 + ordered) * args.steps,
         }
         if not args.sweep and args.layers == 1 and w.batch * w.Hkv * w.B * w.d * w.elem_bytes * 2 > L2_BYTES:
             rr = read_roof(dev)
@@ -912,7 +917,8 @@ def run_ours(args):
             line["config"]["layers"] = args.layers
             line["config"]["layer_launches"] = ("one multi-layer launch per step" if args.layer_launches == "one"
                                                 else "one decode launch per layer")
-            line["gpu_launches"] = (2 if args.layer_launches == "one" else args.layers + 1) * args.steps
+            line["gpu_launches"] = ((2 + ordered) if args.layer_launches == "one"
+                                    else args.layers * (1 + ordered) + 1) * args.steps
         if rank == 0 and world == 1 and not args.no_cpu_baseline and not args.sweep and window is None and \
                 args.layers == 1:
             line["cpu_baseline"] = oracle_sample(w, args.cpu_seconds)

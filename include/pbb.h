@@ -107,8 +107,9 @@ int pbb_ring_prefill(const void* k_hist, const void* v_hist, const int32_t* pos,
  * Make sure the library's workspace of (current device, `stream`) holds the
  * split partials of a step of this shape (and of every smaller batch). A
  * workspace (owned by the library, freed at exit) holds the work-queue words,
- * one counter per (sequence, KV head) and the per-split partial (max, sum,
- * output) of Eq. (lse). Every decode step (pbb_decode_step, _f32, _layers and
+ * one counter per (sequence, KV head), the order of the sequences for a
+ * longest-first step (pbb_plan_support_order) and the per-split partial (max,
+ * sum, output) of Eq. (lse). Every decode step (pbb_decode_step, _f32, _layers and
  * pbb_swa_decode_step) uses the workspace of the stream it is issued on and
  * grows it on demand, which allocates and waits for the device; so call this
  * first, on the capture stream, when decode steps are to be captured in a
@@ -294,6 +295,18 @@ int pbb_plan_chunk_keys(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtyp
  */
 enum { PBB_KERNEL_AUTO = -1, PBB_KERNEL_CUDA_CORES = 0, PBB_KERNEL_TENSOR_CORES = 1 };
 int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype);
+
+/*
+ * Whether a decode step of this shape (window = 0 for PBB, else the window size
+ * of pbb_swa_decode_step) launches the support-ordering kernel before the decode
+ * kernel on the current device: 1 or 0, negative on error. No counterpart in the
+ * paper. A step on the tensor-core kernel whose supports are all whole work items,
+ * with at least four of them per resident CTA, first sorts its sequences by
+ * support length (one small kernel, into the stream's workspace) and then takes
+ * the supports longest first, so that its CTAs finish together. The order changes
+ * no result: every support is an independent work item.
+ */
+int pbb_plan_support_order(int batch, int Hq, int Hkv, int d, int B, int window, pbb_dtype dtype);
 
 /*
  * Kernel choice for the decode steps that follow (process-wide, like

@@ -75,6 +75,7 @@ EXPORTS = {
     "pbb_set_kernel": (_I, [_I]),
     "pbb_plan_chunk_keys": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_plan_kernel": (_I, [_I, _I, _I, _I, _I, _I]),
+    "pbb_plan_support_order": (_I, [_I, _I, _I, _I, _I, _I, _I]),
     "pbb_stream_read": (_I, [_P, _SZ, _P, _P]),
     "pbb_error_string": (ctypes.c_char_p, [_I]),
 }
@@ -511,6 +512,15 @@ def set_kernel(kernel: str) -> str:
     if prev < PBB_KERNEL_AUTO:
         raise PbbError(prev, "pbb_set_kernel")
     return {v: k for k, v in _KERNEL_NAMES.items()}[prev]
+
+
+def plan_support_order(batch: int, Hq: int, Hkv: int, d: int, B: int, window: int = 0,
+                       dtype=torch.bfloat16) -> bool:
+    """Whether a step of this shape first sorts its sequences by support length (one more kernel)."""
+    rc = int(lib().pbb_plan_support_order(batch, Hq, Hkv, d, B, window, _dt(dtype)))
+    if rc < 0:
+        raise PbbError(rc, "pbb_plan_support_order")
+    return rc == 1
 
 
 def plan_kernel(batch: int, Hq: int, Hkv: int, d: int, B: int, dtype=torch.bfloat16) -> str:

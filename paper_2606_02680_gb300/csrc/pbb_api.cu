@@ -270,6 +270,20 @@ int grow_workspace(int dev, cudaStream_t stream, size_t pairs, size_t pbytes, Wo
     return cudaDeviceSynchronize() == cudaSuccess ? PBB_OK : PBB_ERR_CUDA;
 }
 
+// Longest-first order of whole supports (DecodeArgs::order): on the tensor-core kernel, when every
+// support is one work item and the step gives each resident CTA at least PBB_TC_ORDER_ROUNDS of
+// them. A step of fewer rounds is latency-bound, and the ordering kernel would add a launch to it.
+#ifndef PBB_TC_ORDER_ROUNDS
+#define PBB_TC_ORDER_ROUNDS 4
+#endif
+bool support_order_pays(const pbb::DecodeArgs& a, int elem, size_t pairs, int dev)
+{
+    if (PBB_TC_ORDER_ROUNDS <= 0 || static_cast<size_t>(a.whole) != pairs || !pbb::use_tensor_cores(a, elem)) return false;
+    const int per_sm = pbb::decode_ctas_per_sm(a.batch, a.Hkv, elem, a.d, a.gq, a.B, a.window);
+    const size_t resident = static_cast<size_t>(sm_count(dev)) * (per_sm > 0 ? per_sm : 1);
+    return pairs >= static_cast<size_t>(PBB_TC_ORDER_ROUNDS) * resident;
+}
+
 int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_ring, void* v_ring,
                 const int32_t* pos, float* out, int batch, int Hq, int Hkv, int d, int B,
                 int window, pbb_dtype dt, cudaStream_t stream, int pos_batch = 0)
@@ -316,11 +330,12 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
     if (items > static_cast<size_t>(INT_MAX)) return PBB_ERR_UNSUPPORTED;
     a.total_items = static_cast<int>(items);
     const int group = kernel_group(a, elem);
+    const bool order = support_order_pays(a, elem, pairs, dev);
     {
         const size_t pbytes = static_cast<size_t>(sp.whole) < pairs ? parts_bytes(batch, Hkv, d, group, sp) : 0;
         std::lock_guard<std::mutex> lock(g_mutex);
         Workspace* ws = nullptr;
-        rc = grow_workspace(dev, stream, pairs + 2, pbytes, &ws);
+        rc = grow_workspace(dev, stream, pairs + 2 + (order ? static_cast<size_t>(batch) : 0), pbytes, &ws);
         if (rc != PBB_OK) return rc;
         const size_t parts = (pairs - static_cast<size_t>(sp.whole)) * a.nchunk * group;
         a.ctl = ws->counters;
@@ -329,6 +344,11 @@ int decode_impl(const void* q, const void* k_new, const void* v_new, void* k_rin
             a.part_o = ws->parts;
             a.part_ml = reinterpret_cast<float*>(reinterpret_cast<char*>(ws->parts) +
                                                  round_up(parts * d * sizeof(float), 256));
+        }
+        if (order) {  // the sequences, longest support first, after the per-support counters
+            int* ord = ws->counters + 2 + pairs;
+            if (pbb::launch_support_order(a, ord, stream) != cudaSuccess) return PBB_ERR_CUDA;
+            a.order = ord;
         }
         // launched with the lock held: a call on another host thread that grows a workspace
         // frees the old buffers only after its cudaDeviceSynchronize, which waits for this launch
@@ -424,7 +444,9 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
     }
     std::lock_guard<std::mutex> lock(g_mutex);
     Workspace* ws = nullptr;
-    return grow_workspace(dev, stream, static_cast<size_t>(max_batch) * Hkv + 2, need, &ws);
+    // per-support counters, the queue words and the longest-first order of the sequences
+    return grow_workspace(dev, stream, static_cast<size_t>(max_batch) * Hkv + 2 + static_cast<size_t>(max_batch), need,
+                          &ws);
 }
 
 int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
@@ -657,6 +679,32 @@ int pbb_plan_kernel(int batch, int Hq, int Hkv, int d, int B, pbb_dtype dtype)
     const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem_size(dtype), Hq / Hkv, 0);
     a.chunk = sp.chunk;
     return pbb::use_tensor_cores(a, elem_size(dtype)) ? PBB_KERNEL_TENSOR_CORES : PBB_KERNEL_CUDA_CORES;
+}
+
+int pbb_plan_support_order(int batch, int Hq, int Hkv, int d, int B, int window, pbb_dtype dtype)
+{
+    int rc = check_shape(batch, Hkv, d, B, dtype);
+    if (rc != PBB_OK) return rc;
+    rc = check_group(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    if (window < 0 || window > B) return PBB_ERR_INVALID_ARG;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    const int elem = elem_size(dtype);
+    pbb::DecodeArgs a{};
+    a.batch = batch;
+    a.gq = Hq / Hkv;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.d = d;
+    a.B = B;
+    a.window = window;
+    const pbb::SplitPlan sp = pbb::plan_split(batch, Hkv, d, B, elem, Hq / Hkv, window);
+    a.whole = sp.whole;
+    a.chunk = sp.chunk;
+    a.nchunk = sp.nchunk;
+    return support_order_pays(a, elem, static_cast<size_t>(batch) * Hkv, dev) ? 1 : 0;
 }
 
 const char* pbb_error_string(int code)

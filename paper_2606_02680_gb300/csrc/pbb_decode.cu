@@ -885,7 +885,8 @@ struct TcCfg {
 __device__ __forceinline__ void tc_item(const DecodeArgs& a, int item, int& pair, int& chunk)
 {
     if (item < a.whole) {
-        pair = item;
+        // whole supports, longest first when the host ordered them (every support whole)
+        pair = a.order ? __ldg(a.order + item / a.Hkv) * a.Hkv + item % a.Hkv : item;
         chunk = 0;
         return;
     }
@@ -1536,6 +1537,53 @@ __global__ void advance_kernel(int32_t* pos, int batch)
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < batch; i += gridDim.x * blockDim.x) pos[i] += 1;
 }
 
+// The step's sequences by descending number of ring keys in their supports (support_keys' n):
+// a counting sort on 256 length classes, largest first, by one block. When every support is a
+// whole work item and the step runs several rounds of them per CTA, the tensor-core kernel takes
+// them in this order, so the step ends on short supports and its CTAs finish together
+// (longest processing time first). The order within a class is unspecified; the supports are
+// independent work items, so no result depends on it.
+__global__ void __launch_bounds__(1024) support_order_kernel(const int32_t* __restrict__ pos, int pos_batch,
+                                                             int batch, int B, int window, int* __restrict__ order)
+{
+    __shared__ int cnt[256];
+    pdl_wait();
+    pdl_launch_dependents();
+    for (int i = threadIdx.x; i < 256; i += blockDim.x) cnt[i] = 0;
+    __syncthreads();
+    auto cls = [&](int b) {  // class 0 holds the longest supports
+        int r, n, base;
+        support_keys(__ldg(pos + (b < pos_batch ? b : b % pos_batch)), B, window, r, n, base);
+        const long long c = 255 - static_cast<long long>(n) * 256 / B;
+        return static_cast<int>(c < 0 ? 0 : (c > 255 ? 255 : c));
+    };
+    for (int b = threadIdx.x; b < batch; b += blockDim.x) atomicAdd(&cnt[cls(b)], 1);
+    __syncthreads();
+    if (threadIdx.x < 32) {  // exclusive prefix sum over the classes, 8 a lane
+        const int l = static_cast<int>(threadIdx.x);
+        int v[8], sum = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            v[i] = cnt[8 * l + i];
+            sum += v[i];
+        }
+        int incl = sum;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+            const int o = __shfl_up_sync(kFull, incl, off);
+            if (l >= off) incl += o;
+        }
+        int run = incl - sum;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            cnt[8 * l + i] = run;
+            run += v[i];
+        }
+    }
+    __syncthreads();
+    for (int b = threadIdx.x; b < batch; b += blockDim.x) order[atomicAdd(&cnt[cls(b)], 1)] = b;
+}
+
 // Launches of the decode-step kernels (decode, position advance, ring load) allow programmatic
 // dependent launch: a kernel may be scheduled while the previous kernel of the stream finishes,
 // so its launch and set-up overlap that kernel's tail; each of them calls pdl_wait before it
@@ -1846,6 +1894,11 @@ cudaError_t launch_prefill(const void* k_hist, const void* v_hist, const int32_t
     return launch_pdl(prefill_kernel, blocks, 256, 0, stream, static_cast<const uint4*>(k_hist),
                       static_cast<const uint4*>(v_hist), pos, static_cast<uint4*>(k_ring),
                       static_cast<uint4*>(v_ring), Hkv, B, row16, total);
+}
+
+cudaError_t launch_support_order(const DecodeArgs& a, int* order, cudaStream_t stream)
+{
+    return launch_pdl(support_order_kernel, 1, 1024, 0, stream, a.pos, a.pos_batch, a.batch, a.B, a.window, order);
 }
 
 cudaError_t launch_advance(int32_t* pos, int batch, cudaStream_t stream)

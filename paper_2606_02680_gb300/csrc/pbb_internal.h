@@ -35,6 +35,8 @@ struct DecodeArgs {
     int chunk;           // ring keys per work item of the later supports (a multiple of the tile)
     int nchunk;          // work items per later support = ceil((B-1)/chunk)
     int total_items;     // whole + (batch * Hkv - whole) * nchunk
+    const int* order;    // null, or (whole == batch * Hkv, tensor-core kernel) the sequences in the order
+                         // their supports are taken: longest first (launch_support_order)
     unsigned long long timeout_ns;
 };
 
@@ -77,6 +79,10 @@ bool use_tensor_cores(const DecodeArgs& a, int elem_bytes);
 // Launch the fused append + attention + combine kernel (persistent grid of at
 // most SMs x resident CTAs). elem_bytes: 2 (bf16) or 4 (fp32).
 cudaError_t launch_decode(const DecodeArgs& a, int elem_bytes, cudaStream_t stream);
+// Writes the step's sequences into order[0, batch) by descending number of ring keys in their
+// supports (one block; a counting sort on 256 length classes, the order within a class
+// unspecified), for DecodeArgs::order.
+cudaError_t launch_support_order(const DecodeArgs& a, int* order, cudaStream_t stream);
 
 cudaError_t launch_prefill(const void* k_hist, const void* v_hist, const int32_t* pos, void* k_ring,
                            void* v_ring, int batch, int Hkv, int B, int row_bytes,

@@ -129,6 +129,8 @@ def test_headline_every_sequence_at_edge_phases():
     simulator."""
     w = inputs.sweep_workload(512, 4096, steps=2)
     assert pbb.plan_kernel(w.batch, w.Hq, w.Hkv, w.d, w.B, torch.bfloat16) == "tensor_cores"
+    # whole supports, several rounds per CTA: the step takes them longest first
+    assert pbb.plan_support_order(w.batch, w.Hq, w.Hkv, w.d, w.B)
     dev = torch.device("cuda", 0)
     t0 = _edge_start_positions(w.batch, w.B, seed=23)
     pos = t0.to(torch.int32).to(dev)
@@ -164,3 +166,15 @@ def test_headline_every_sequence_at_edge_phases():
             sim.append(new_k[i][sl], new_v[i][sl], (t0[sl] + i).numpy())
         assert np.array_equal(ring_bytes_np(k_ring[sl]), sim.k), f"K rings {lo}..{lo + chunk - 1}"
         assert np.array_equal(ring_bytes_np(v_ring[sl]), sim.v), f"V rings {lo}..{lo + chunk - 1}"
+
+
+def test_support_order_plan():
+    """Longest-first order only where every support is one work item on the tensor-core kernel
+    and each resident CTA gets several: not for chunked plans, small batches or the CUDA cores."""
+    assert pbb.plan_support_order(512, 32, 8, 128, 4096)             # the timed shape
+    assert pbb.plan_support_order(512, 32, 8, 128, 4096, window=4096)  # its window control
+    assert not pbb.plan_support_order(64, 32, 8, 128, 4096)          # chunked supports
+    assert not pbb.plan_support_order(8, 32, 8, 128, 4096)           # latency-bound
+    assert not pbb.plan_support_order(512, 32, 8, 128, 4096, dtype=torch.float32)  # CUDA cores
+    with pytest.raises(pbb.PbbError):
+        pbb.plan_support_order(512, 32, 8, 128, 4096, window=4097)
