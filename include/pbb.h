@@ -136,6 +136,8 @@ int pbb_reserve_workspace(int max_batch, int Hq, int Hkv, int d, int B, pbb_dtyp
  * after pbb_ring_prefill at t, or after steps at t-1, t-2, ... starting from a
  * zeroed ring at t = 0. pos is read on the device and never by the host.
  * Deterministic: the same inputs give bitwise the same out and rings.
+ * A step with many whole supports first launches a small kernel that sorts its
+ * sequences by support length (pbb_plan_support_order); it changes no result.
  */
 int pbb_decode_step(const void* q, const void* k_new, const void* v_new, void* k_ring,
                     void* v_ring, const int32_t* pos, float* out, int batch, int Hq, int Hkv,
