@@ -593,8 +593,8 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
 // union once. Warps 0-3 run the softmax of A, warps 4-7 that of B, each over its own S and
 // output in TMEM, so one warpgroup's softmax runs while the tensor pipe works on the other's
 // products, and the issuing thread queues four groups (S and P.V of both) per K/V tile. The
-// softmax warpgroups take 216 registers a thread (setmaxnreg) from the warpgroup of the producer,
-// MMA and spare warps.
+// softmax warpgroups take 216 registers a thread (setmaxnreg) from the warpgroup of the Q, K and
+// V producers and the MMA issuer.
 template <int D, int G>
 struct PairCfg {
     static constexpr int NK = 128, M = 128, QT = M / G, BOXES = D / 64;
@@ -611,12 +611,12 @@ struct PairCfg {
     static constexpr int V_OFF = K_OFF + KSTAGES * TILE;
     static constexpr int SMEM = V_OFF + VSTAGES * TILE + 1024;
     static constexpr int T_S = 0, T_O = 2 * NK;            // S of A and B, then the outputs
-    // warps 0-7 softmax, 8 Q and K producer, 9 V producer, 10 MMA issuer, 11 spare; at launch
+    // warps 0-7 softmax, 8 K producer, 9 V producer, 10 MMA issuer, 11 Q producer; at launch
     // 168 registers each (12 warps, three per SMSP). setmaxnreg is uniform per warpgroup and
     // the register file is split between the SMSPs, so each SMSP's three warps (two softmax,
     // one of warpgroup 2) must fit their launch share: 2 x 216 + 72 = 3 x 168, and over the
     // CTA 256 x 216 + 128 x 72 = 384 x 168
-    static constexpr int THREADS = 384, W_QK = 8, W_V = 9, W_MMA = 10;
+    static constexpr int THREADS = 384, W_K = 8, W_V = 9, W_MMA = 10, W_Q = 11;
     static constexpr int LAUNCH_REGS = 168;
     static constexpr int SOFTMAX_REGS = 216, OTHER_REGS = 72;
     static_assert(2 * SOFTMAX_REGS + OTHER_REGS <= 3 * LAUNCH_REGS, "register split per SMSP");
@@ -713,18 +713,22 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
     // each warpgroup's four warps run one setmaxnreg, at one place, ahead of its roles
     if (warp >= 8) {
         regs_dec_others();
-        if (warp == C::W_QK || warp == C::W_V) {
-            // ================= TMA producers: Q of both items and K tiles; V tiles =================
-            const bool qk = warp == C::W_QK;
+        if (warp == C::W_K || warp == C::W_V || warp == C::W_Q) {
+            // ================= TMA producers: Q of both items, K tiles, V tiles =================
+            // (Q on a warp of its own, so that the K tiles of the next item need not wait for the
+            // Q buffers, which free only after the current item's last S)
+            const bool qk = warp == C::W_K;
+            const bool q_role = warp == C::W_Q;
+            const bool tiles = !q_role;
             if (lane == 0) {
-                asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(qk ? &kmap : &vmap)) : "memory");
-                if (qk) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
+                if (tiles) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(qk ? &kmap : &vmap)) : "memory");
+                if (q_role) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
                 uint32_t gt = 0, issued = 0, ic[2] = {0, 0}, q_issued[2] = {0, 0};
                 bool ok = true;
                 for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
                     const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
                     const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
-                    if (qk) {
+                    if (q_role) {
                         for (int x = 0; x < (it.hasB ? 2 : 1); ++x) {
                             if (ic[x] >= 1 && !mbar_wait(&q_empty[x], (ic[x] - 1) & 1u, limit)) {
                                 ok = false;
@@ -745,7 +749,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                         if (!ok) break;
                     }
                     const int row0 = it.pair * a.n + it.loA;
-                    for (int j = 0; j < it.nt; ++j, ++gt) {
+                    for (int j = 0; tiles && j < it.nt; ++j, ++gt) {
                         if (abort_s) {
                             ok = false;
                             break;
@@ -851,8 +855,8 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                             issued_any = true;
                         }
                         if (!ok) break;
-                        if (need_k) umma_commit(&k_empty[gk++ % KS]);
-                        if (need_v) umma_commit(&v_empty[gv++ % VS]);
+                        gk += need_k;  // the softmax warpgroups release the K and V stages
+                        gv += need_v;
                     }
                 }
                 if (!ok) {
@@ -864,7 +868,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                     mbar_wait(&done_bar, 0u, kGuardNs);
                 }
             }
-        }  // warp 11 has no role: its registers went to the softmax warpgroups
+        }
     } else {
         regs_inc_softmax();
         // ================= softmax of item x (warps 4x .. 4x + 3) =================
@@ -875,10 +879,22 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
         const int h = a.B >> 1;
         const int gi = r / C::QT, rp = r - gi * C::QT;
         uint32_t g = 0, ic = 0;  // this item slot's tiles and items so far
+        uint32_t gkv = 0;        // K (and V) tiles of the items before this one
         bool ok = true;
         for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
             const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
+            const uint32_t gk0 = gkv;
+            gkv += it.nt;
             if (x == 1 && !it.hasB) continue;
+            // K/V stages are freed here rather than by commits of the issuing thread, whose every
+            // barrier operation delays its next products. Its last commit of iteration j (after S
+            // of both items on K_j and P.V of both on V_{j-1}) is item B's s_full where B has tile
+            // j, else item A's (A owns the iterations below jB0, all of them without B); iteration
+            // nt, the last P.V, ends with pv_last of B, or of A without B. The owner's first thread
+            // frees K_j and V_{j-1} once it has seen that commit: K_j sits in stage (gk0 + j) mod
+            // KS, V_j in (gk0 + j) mod VS.
+            const int jown = x == 1 ? 0 : (it.hasB ? it.jB0 : it.nt + 1);
+            const bool releaser = (tid & 127) == 0;
             const int t0 = it.t0 + x * C::QT, tl = x == 0 ? it.tlA : it.tlB;
             const int amax = x == 0 ? it.amaxA : it.amaxB;
             const int jb = x == 0 ? 0 : it.jB0, je = x == 0 ? it.ntA : it.nt;
@@ -889,6 +905,10 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 if (!warp_wait(&s_full[x], g & 1u, limit) || __any_sync(0xffffffffu, abort_s != 0)) {
                     ok = false;
                     break;
+                }
+                if (releaser && (x == 1 || j < jown)) {
+                    mbar_arrive(&k_empty[(gk0 + j) % KS]);
+                    if (j >= 1) mbar_arrive(&v_empty[(gk0 + j - 1) % VS]);
                 }
                 tmem_fence_after();
                 float z[NK];  // raw scores q.k of this row: every load issued, one wait
@@ -911,19 +931,48 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
 #pragma unroll
                     for (int c = 0; c < NK; ++c) z[c] = c >= lo ? z[c] : -INFINITY;
                 }
-                float mx0 = -INFINITY, mx1 = -INFINITY;
+                // P = exp2(z * scale - m) as bf16 pairs over the first half of this row's S
+                // columns, one 64-key half at a time; the arguments and the row sum in packed
+                // two-lane FMA and add
+                const float2 sc2 = make_float2(qscale, qscale);
+                auto write_p = [&](int c, float m) {
+                    const float nb = m == -INFINITY ? 0.f : -m;
+                    const float2 nb2 = make_float2(nb, nb);
+                    float2 la = make_float2(0.f, 0.f), lb = la;
+                    uint32_t pk[32];
 #pragma unroll
-                for (int c = 0; c < NK; c += 4) {
+                    for (int y = 0; y < 32; ++y) {
+                        const float2 arg = __ffma2_rn(make_float2(z[64 * c + 2 * y], z[64 * c + 2 * y + 1]), sc2, nb2);
+                        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
+                        if (y & 1) lb = __fadd2_rn(lb, e);
+                        else la = __fadd2_rn(la, e);
+                        pk[y] = pack_bf16x2(e.x, e.y);
+                    }
+                    tmem_st32(s_row + 32 * c, pk);
+                    return __fadd2_rn(la, lb);
+                };
+                // after the item's first tile the reference maximum seldom moves, so the first
+                // half of P is formed against it while the row maximum is found, and formed again
+                // only if it moved
+                const bool first = j == jb;
+                float2 l0 = make_float2(0.f, 0.f);
+                if (!first) l0 = write_p(0, m_used);
+                float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
+#pragma unroll
+                for (int c = 0; c < NK; c += 8) {
                     mx0 = fmax3(mx0, z[c], z[c + 1]);
                     mx1 = fmax3(mx1, z[c + 2], z[c + 3]);
+                    mx2 = fmax3(mx2, z[c + 4], z[c + 5]);
+                    mx3 = fmax3(mx3, z[c + 6], z[c + 7]);
                 }
-                const float mx = fmaxf(mx0, mx1) * qscale;
+                const float mx = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * qscale;
                 // the reference maximum moves only when the row maximum exceeds it by 2^8
                 // (see forward_kernel); s_full of this tile also covers P.V of the previous one,
                 // so O holds every earlier tile when it is rescaled
                 const bool grow = mx > m_used + 8.f;
                 const float m_new = grow ? mx : m_used;
-                if (__any_sync(0xffffffffu, grow)) {
+                const bool moved = __any_sync(0xffffffffu, grow);
+                if (moved) {
                     const float f = grow ? (m_used == -INFINITY ? 0.f : fast_exp2(m_used - m_new)) : 1.f;
                     l *= f;
                     if (j > jb) {
@@ -940,22 +989,12 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                     }
                     m_used = m_new;
                 }
-                const float nbase = m_used == -INFINITY ? 0.f : -m_used;
-                const float2 sc2 = make_float2(qscale, qscale), nb2 = make_float2(nbase, nbase);
-                float2 lacc = make_float2(0.f, 0.f);
-#pragma unroll
-                for (int c = 0; c < NK / 64; ++c) {
-                    uint32_t pk[32];
-#pragma unroll
-                    for (int y = 0; y < 32; ++y) {
-                        const float2 arg = __ffma2_rn(make_float2(z[64 * c + 2 * y], z[64 * c + 2 * y + 1]), sc2, nb2);
-                        const float2 e = make_float2(fast_exp2(arg.x), fast_exp2(arg.y));
-                        lacc = __fadd2_rn(lacc, e);
-                        pk[y] = pack_bf16x2(e.x, e.y);
-                    }
-                    tmem_st32(s_row + 32 * c, pk);
+                if (first || moved) {
+                    if (!first) tmem_wait_st();  // the first P's stores land before they are replaced
+                    l0 = write_p(0, m_used);
                 }
-                l += lacc.x + lacc.y;
+                const float2 l1 = write_p(1, m_used);
+                l += (l0.x + l0.y) + (l1.x + l1.y);
                 tmem_wait_st();
                 tmem_fence_before();
                 mbar_arrive(&p_full[x]);
@@ -966,6 +1005,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 ok = false;
                 break;
             }
+            if (releaser && (x == 1 || !it.hasB)) mbar_arrive(&v_empty[(gk0 + it.nt - 1) % VS]);
             tmem_fence_after();
             const bool valid = t < a.n && t <= tl;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
