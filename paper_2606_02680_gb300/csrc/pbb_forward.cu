@@ -611,6 +611,12 @@ struct PairCfg {
     static constexpr int V_OFF = K_OFF + KSTAGES * TILE;
     static constexpr int SMEM = V_OFF + VSTAGES * TILE + 1024;
     static constexpr int T_S = 0, T_O = 2 * NK;            // S of A and B, then the outputs
+    // Iteration i of the issuing thread (K_j for S, V_{j-1} for P.V) waits on kv_full[i mod KVR],
+    // which the K and the V producer each arrive on once per iteration, with their copy's bytes
+    // or without a copy. A producer arrives for iteration i + KVR only after a stage wait that
+    // follows the issuing thread's iteration i: with one extra iteration per item, a producer
+    // runs at most 2 KSTAGES + 1 iterations ahead, so KVR = 8 keeps the phases apart.
+    static constexpr int KVR = 8;
     // warps 0-7 softmax, 8 K producer, 9 V producer, 10 MMA issuer, 11 Q producer; at launch
     // 168 registers each (12 warps, three per SMSP). setmaxnreg is uniform per warpgroup and
     // the register file is split between the SMSPs, so each SMSP's three warps (two softmax,
@@ -669,7 +675,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
     constexpr int NK = C::NK, KS = C::KSTAGES, VS = C::VSTAGES;
     extern __shared__ unsigned char dsmem_raw[];
     __shared__ __align__(8) uint64_t q_full[2], q_empty[2], done_bar;
-    __shared__ __align__(8) uint64_t k_full[KS], k_empty[KS], v_full[VS], v_empty[VS];
+    __shared__ __align__(8) uint64_t kv_full[C::KVR], k_empty[KS], v_empty[VS];
     __shared__ __align__(8) uint64_t s_full[2], p_full[2], pv_last[2], o_free[2];  // per item (A, B)
     __shared__ uint32_t tmem_base_s;
     __shared__ volatile int abort_s;
@@ -691,15 +697,11 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
         }
         mbar_init(&done_bar, 1);
 #pragma unroll
-        for (int s = 0; s < KS; ++s) {
-            mbar_init(&k_full[s], 1);
-            mbar_init(&k_empty[s], 1);
-        }
+        for (int s = 0; s < C::KVR; ++s) mbar_init(&kv_full[s], 2);  // the K and the V producer
 #pragma unroll
-        for (int s = 0; s < VS; ++s) {
-            mbar_init(&v_full[s], 1);
-            mbar_init(&v_empty[s], 1);
-        }
+        for (int s = 0; s < KS; ++s) mbar_init(&k_empty[s], 1);
+#pragma unroll
+        for (int s = 0; s < VS; ++s) mbar_init(&v_empty[s], 1);
         fence_mbar_init();
         abort_s = 0;
     }
@@ -723,7 +725,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
             if (lane == 0) {
                 if (tiles) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(qk ? &kmap : &vmap)) : "memory");
                 if (q_role) asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&qmap)) : "memory");
-                uint32_t gt = 0, issued = 0, ic[2] = {0, 0}, q_issued[2] = {0, 0};
+                uint32_t gt = 0, gi = 0, armed = 0, ic[2] = {0, 0}, q_issued[2] = {0, 0};
                 bool ok = true;
                 for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
                     const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
@@ -749,25 +751,32 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                         if (!ok) break;
                     }
                     const int row0 = it.pair * a.n + it.loA;
-                    for (int j = 0; tiles && j < it.nt; ++j, ++gt) {
+                    // iterations j = 0 .. nt: K_j for j < nt, V_{j-1} for j >= 1
+                    for (int j = 0; tiles && j <= it.nt; ++j, ++gi) {
                         if (abort_s) {
                             ok = false;
                             break;
                         }
+                        uint64_t* fullb = &kv_full[gi % C::KVR];
+                        if (qk ? j == it.nt : j == 0) {
+                            mbar_arrive(fullb);
+                            continue;
+                        }
                         const int ns = qk ? KS : VS;
                         const int s = gt % ns;
-                        uint64_t* fullb = qk ? &k_full[s] : &v_full[s];
                         uint64_t* emptyb = qk ? &k_empty[s] : &v_empty[s];
                         if (gt >= static_cast<uint32_t>(ns) && !mbar_wait(emptyb, ((gt / ns) - 1) & 1u, limit)) {
                             ok = false;
                             break;
                         }
                         unsigned char* st = dsmem + (qk ? C::K_OFF : C::V_OFF) + s * C::TILE;
+                        const int tile = qk ? j : j - 1;
                         mbar_expect_tx(fullb, static_cast<uint32_t>(C::TILE));
 #pragma unroll
                         for (int bx = 0; bx < C::BOXES; ++bx)
-                            tma_load_2d(st + bx * C::KBOX, qk ? &kmap : &vmap, bx * 64, row0 + j * NK, fullb);
-                        issued = gt + 1;
+                            tma_load_2d(st + bx * C::KBOX, qk ? &kmap : &vmap, bx * 64, row0 + tile * NK, fullb);
+                        ++gt;
+                        armed = gi + 1;
                     }
                 }
                 if (!ok) {
@@ -777,11 +786,8 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 // drain the copies still in flight before shared memory goes away
                 for (int x = 0; x < 2; ++x)
                     if (q_issued[x] > 0) mbar_wait(&q_full[x], (q_issued[x] - 1) & 1u, kGuardNs);
-                const uint32_t ns = qk ? KS : VS;
-                for (uint32_t s = 0; s < ns && s < issued; ++s) {
-                    const uint32_t jj = s + ns * ((issued - 1 - s) / ns);
-                    mbar_wait(qk ? &k_full[s] : &v_full[s], (jj / ns) & 1u, kGuardNs);
-                }
+                for (uint32_t i = armed > C::KVR ? armed - C::KVR : 0; i < armed; ++i)
+                    mbar_wait(&kv_full[i % C::KVR], (i / C::KVR) & 1u, kGuardNs);
             }
         } else if (warp == C::W_MMA) {
             // ================= MMA issuer =================
@@ -790,22 +796,16 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 constexpr uint32_t idesc_o = umma_idesc_bf16(C::M, D, 1);
                 const uint32_t q_base = smem_addr(dsmem + C::Q_OFF);
                 const uint32_t k_base = smem_addr(dsmem + C::K_OFF), v_base = smem_addr(dsmem + C::V_OFF);
-                uint32_t gk = 0, gv = 0;                  // K and V tiles consumed
+                uint32_t gk = 0, gv = 0, gi = 0;          // K and V tiles consumed, iterations
                 uint32_t ic[2] = {0, 0}, gp[2] = {0, 0};  // items and P tiles consumed, per item slot
                 bool ok = true, issued_any = false;
                 for (int rd = 0, sidx = item_mirrored(0); ok && sidx < n_sitems; ++rd, sidx = item_mirrored(rd)) {
                     const PItem it = make_pitem<C::QT, NK>(sidx, a.n, a.B);
                     const int jb[2] = {0, it.hasB ? it.jB0 : it.nt};  // first and end tile of each item
                     const int je[2] = {it.ntA, it.nt};
-                    for (int j = 0; ok && j <= it.nt; ++j) {
-                        bool need_k = false, need_v = false;
-#pragma unroll
-                        for (int x = 0; x < 2; ++x) {
-                            need_k |= j >= jb[x] && j < je[x];
-                            need_v |= j >= jb[x] + 1 && j - 1 < je[x];
-                        }
-                        if ((need_k && !mbar_wait(&k_full[gk % KS], (gk / KS) & 1u, limit)) ||
-                            (need_v && !mbar_wait(&v_full[gv % VS], (gv / VS) & 1u, limit))) {
+                    for (int j = 0; ok && j <= it.nt; ++j, ++gi) {
+                        const bool need_k = j < it.nt, need_v = j >= 1;  // K_j, V_{j-1}
+                        if (!mbar_wait(&kv_full[gi % C::KVR], (gi / C::KVR) & 1u, limit)) {
                             ok = false;
                             break;
                         }
