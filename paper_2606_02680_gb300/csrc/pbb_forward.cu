@@ -893,8 +893,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
             // nt, the last P.V, ends with pv_last of B, or of A without B. The owner's first thread
             // frees K_j and V_{j-1} once it has seen that commit: K_j sits in stage (gk0 + j) mod
             // KS, V_j in (gk0 + j) mod VS.
-            const int jown = x == 1 ? 0 : (it.hasB ? it.jB0 : it.nt + 1);
-            const bool releaser = (tid & 127) == 0;
+            const int jown = (tid & 127) != 0 ? -1 : x == 1 ? it.nt : (it.hasB ? it.jB0 : it.nt);
             const int t0 = it.t0 + x * C::QT, tl = x == 0 ? it.tlA : it.tlB;
             const int amax = x == 0 ? it.amaxA : it.amaxB;
             const int jb = x == 0 ? 0 : it.jB0, je = x == 0 ? it.ntA : it.nt;
@@ -906,7 +905,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                     ok = false;
                     break;
                 }
-                if (releaser && (x == 1 || j < jown)) {
+                if (j < jown) {
                     mbar_arrive(&k_empty[(gk0 + j) % KS]);
                     if (j >= 1) mbar_arrive(&v_empty[(gk0 + j - 1) % VS]);
                 }
@@ -1005,7 +1004,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 ok = false;
                 break;
             }
-            if (releaser && (x == 1 || !it.hasB)) mbar_arrive(&v_empty[(gk0 + it.nt - 1) % VS]);
+            if ((tid & 127) == 0 && (x == 1 || !it.hasB)) mbar_arrive(&v_empty[(gk0 + it.nt - 1) % VS]);
             tmem_fence_after();
             const bool valid = t < a.n && t <= tl;
             const int b = it.pair / a.Hkv, kvh = it.pair - b * a.Hkv;
