@@ -147,6 +147,44 @@ __device__ __forceinline__ float fmax3(float a, float b, float c)
     return d;
 }
 
+// Writes EC consecutive outputs o of one row, starting at element e0 of `out` (bf16, or fp32
+// with f32). A thread's row is 256 or 128 bytes from its neighbours', so each store instruction
+// of a warp touches 32 lines: 32-byte stores halve those instructions where the output base is
+// 32-byte aligned (every chunk is then too); other bases take 16-byte stores.
+template <int EC>
+__device__ __forceinline__ void store_chunk(void* out, bool f32, size_t e0, const float (&o)[EC], bool wide)
+{
+    if (f32) {
+        float* dst = static_cast<float*>(out) + e0;
+        if (wide) {
+#pragma unroll
+            for (int y = 0; y < EC / 8; ++y) {
+                uint32_t w[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) w[i] = __float_as_uint(o[8 * y + i]);
+                st_global_v8(dst + 8 * y, w);
+            }
+        } else {
+#pragma unroll
+            for (int y = 0; y < EC / 4; ++y)
+                reinterpret_cast<float4*>(dst)[y] = make_float4(o[4 * y], o[4 * y + 1], o[4 * y + 2], o[4 * y + 3]);
+        }
+    } else {
+        uint32_t pk[EC / 2];
+#pragma unroll
+        for (int y = 0; y < EC / 2; ++y) pk[y] = pack_bf16x2(o[2 * y], o[2 * y + 1]);
+        __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(out) + e0;
+        if (wide) {
+#pragma unroll
+            for (int y = 0; y < EC / 16; ++y) st_global_v8(dst + 16 * y, pk + 8 * y);
+        } else {
+#pragma unroll
+            for (int y = 0; y < EC / 8; ++y)
+                reinterpret_cast<uint4*>(dst)[y] = make_uint4(pk[4 * y], pk[4 * y + 1], pk[4 * y + 2], pk[4 * y + 3]);
+        }
+    }
+}
+
 // One work item: (sequence, KV head) pair, first position, keys and tiles.
 struct Item {
     int pair, t0, tl, lo, a_max, ntiles;
@@ -221,6 +259,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
     tmem_fence_after();
     const uint32_t tmem = tmem_base_s;
     const unsigned long long limit = a.timeout_ns;
+    const bool wide_out = (reinterpret_cast<uintptr_t>(a.out) & 31u) == 0;  // 32-byte output stores
 
     if (warp == C::PRODUCER_WARP) {
         // ================= TMA producer =================
@@ -547,25 +586,7 @@ forward_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__
                 float o[EC];
 #pragma unroll
                 for (int x = 0; x < EC; ++x) o[x] = __uint_as_float(v[x]) * inv;
-                if (valid) {
-                    const size_t e0 = row * D + wg * OC + EC * c;  // first output element of the chunk
-                    if (a.out_f32) {
-                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + e0);
-#pragma unroll
-                        for (int x = 0; x < EC / 4; ++x) dst[x] = make_float4(o[4 * x], o[4 * x + 1], o[4 * x + 2], o[4 * x + 3]);
-                    } else {
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + e0);
-#pragma unroll
-                        for (int x = 0; x < EC / 8; ++x) {
-                            uint4 pk;
-                            pk.x = pack_bf16x2(o[8 * x], o[8 * x + 1]);
-                            pk.y = pack_bf16x2(o[8 * x + 2], o[8 * x + 3]);
-                            pk.z = pack_bf16x2(o[8 * x + 4], o[8 * x + 5]);
-                            pk.w = pack_bf16x2(o[8 * x + 6], o[8 * x + 7]);
-                            dst[x] = pk;
-                        }
-                    }
-                }
+                if (valid) store_chunk<EC>(a.out, a.out_f32, row * D + wg * OC + EC * c, o, wide_out);
             }
             tmem_fence_before();
             mbar_arrive(&o_free[ob]);  // the next item may overwrite the output buffer
@@ -711,6 +732,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
     tmem_fence_after();
     const uint32_t tmem = tmem_base_s;
     const unsigned long long limit = a.timeout_ns;
+    const bool wide_out = (reinterpret_cast<uintptr_t>(a.out) & 31u) == 0;  // 32-byte output stores
     // warpgroup 2 (producers, MMA issuer, spare) gives registers to warpgroups 0 and 1 (softmax):
     // each warpgroup's four warps run one setmaxnreg, at one place, ahead of its roles
     if (warp >= 8) {
@@ -1018,24 +1040,7 @@ forward_pair_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_const
                 float o[32];
 #pragma unroll
                 for (int y = 0; y < 32; ++y) o[y] = __uint_as_float(v[y]) * inv;
-                if (valid) {
-                    if (a.out_f32) {
-                        float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.out) + row * D + 32 * c);
-#pragma unroll
-                        for (int y = 0; y < 8; ++y) dst[y] = make_float4(o[4 * y], o[4 * y + 1], o[4 * y + 2], o[4 * y + 3]);
-                    } else {
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(a.out) + row * D + 32 * c);
-#pragma unroll
-                        for (int y = 0; y < 4; ++y) {
-                            uint4 pk;
-                            pk.x = pack_bf16x2(o[8 * y], o[8 * y + 1]);
-                            pk.y = pack_bf16x2(o[8 * y + 2], o[8 * y + 3]);
-                            pk.z = pack_bf16x2(o[8 * y + 4], o[8 * y + 5]);
-                            pk.w = pack_bf16x2(o[8 * y + 6], o[8 * y + 7]);
-                            dst[y] = pk;
-                        }
-                    }
-                }
+                if (valid) store_chunk<32>(a.out, a.out_f32, row * D + 32 * c, o, wide_out);
             }
             tmem_fence_before();
             mbar_arrive(&o_free[x]);  // the next item of this slot may overwrite the output

@@ -129,6 +129,27 @@ def test_deterministic():
     assert torch.equal(o1.view(torch.int16), o2.view(torch.int16)) and torch.equal(l1, l2)
 
 
+@pytest.mark.parametrize("B,d", [(512, 128), (128, 64)])  # the paired and the one-item kernel
+@pytest.mark.parametrize("out_dtype", [torch.bfloat16, torch.float32])
+def test_output_alignment(B, d, out_dtype):
+    """An output 32-byte aligned takes 32-byte stores, one only 16-byte aligned 16-byte stores:
+    both hold the same bits."""
+    w = inputs.SequenceWorkload("fwd_align", batch=2, Hq=8, Hkv=2, d=d, B=B, n=1100, seed=84)
+    q, k, v = (x.cuda() for x in inputs.sequence_inputs(w))
+    shape = (w.batch, w.Hq, w.n, w.d)
+    numel = w.batch * w.Hq * w.n * w.d
+    step = 16 // torch.tensor([], dtype=out_dtype).element_size()  # elements in 16 bytes
+    buf = torch.empty(numel + 4 * step, dtype=out_dtype, device="cuda")
+    base = (-buf.data_ptr() % 32) // buf.element_size()  # first 32-byte aligned element
+    outs = []
+    for off in (base, base + step):  # 32-byte aligned, then 16-byte only
+        out = buf[off:off + numel].view(shape)
+        assert out.data_ptr() % 32 == (0 if off == base else 16)
+        outs.append(pbb.forward(q, k, v, w.B, out=out, out_dtype=out_dtype)[0].clone())
+    bits = torch.int16 if out_dtype == torch.bfloat16 else torch.int32
+    assert torch.equal(outs[0].view(bits), outs[1].view(bits))
+
+
 def sampled_rows(w, count, rng):
     bi = rng.integers(0, w.batch, count)
     j = rng.integers(0, w.Hq, count)
