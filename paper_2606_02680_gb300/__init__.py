@@ -404,9 +404,11 @@ def forward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, B: int, out: torc
 
 
 def backward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tensor, dout: torch.Tensor,
-             lse: torch.Tensor, B: int, stream=None):
+             lse: torch.Tensor, B: int, stream=None, dq: torch.Tensor | None = None,
+             dk: torch.Tensor | None = None, dv: torch.Tensor | None = None):
     """Gradients (dq, dk, dv), fp32, of pbb_forward (pbb_backward). out and lse are the
-    forward's outputs for q, k, v; dout is the upstream gradient (bf16, shaped like out)."""
+    forward's outputs for q, k, v; dout is the upstream gradient (bf16, shaped like out).
+    dq, dk, dv: buffers to receive the gradients (allocated when None)."""
     batch, Hq, n, d = q.shape
     Hkv = k.shape[1]
     for name, t, shape in (("k", k, (batch, Hkv, n, d)), ("v", v, (batch, Hkv, n, d)),
@@ -416,9 +418,15 @@ def backward(q: torch.Tensor, k: torch.Tensor, v: torch.Tensor, out: torch.Tenso
             raise ValueError(f"{name} must have shape {shape}")
     dev = q.device
     delta = torch.empty((batch, Hq, n), dtype=torch.float32, device=dev)
-    dq = torch.empty((batch, Hq, n, d), dtype=torch.float32, device=dev)
-    dk = torch.empty((batch, Hkv, n, d), dtype=torch.float32, device=dev)
-    dv = torch.empty((batch, Hkv, n, d), dtype=torch.float32, device=dev)
+    grads = []
+    for name, t, shape in (("dq", dq, (batch, Hq, n, d)), ("dk", dk, (batch, Hkv, n, d)),
+                           ("dv", dv, (batch, Hkv, n, d))):
+        if t is None:
+            t = torch.empty(shape, dtype=torch.float32, device=dev)
+        elif tuple(t.shape) != shape:
+            raise ValueError(f"{name} must have shape {shape}")
+        grads.append(t)
+    dq, dk, dv = grads
     bf = torch.bfloat16
     _check(lib().pbb_backward(_dev(q, "q", bf), _dev(k, "k", bf), _dev(v, "v", bf), _dev(out, "out", bf),
                               _dev(dout, "dout", bf), _dev(lse, "lse", torch.float32),

@@ -62,6 +62,28 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, unsign
     return __all_sync(kFull, mbar_wait(bar, parity, limit));
 }
 
+// 32 fp32 gradients of one row, v scaled by f, to dst. A thread writes its own row, so each
+// store instruction of a warp touches 32 lines: 32-byte stores halve those instructions where
+// the gradient's base is 32-byte aligned (every 32-column chunk is then too); other bases take
+// 16-byte stores.
+__device__ __forceinline__ void store_row32(float* dst, const uint32_t (&v)[32], float f, bool wide)
+{
+    if (wide) {
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+            uint32_t w[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) w[i] = __float_as_uint(__uint_as_float(v[8 * x + i]) * f);
+            st_global_v8(dst + 8 * x, w);
+        }
+    } else {
+#pragma unroll
+        for (int x = 0; x < 8; ++x)
+            reinterpret_cast<float4*>(dst)[x] = make_float4(__uint_as_float(v[4 * x]) * f, __uint_as_float(v[4 * x + 1]) * f,
+                                                            __uint_as_float(v[4 * x + 2]) * f, __uint_as_float(v[4 * x + 3]) * f);
+    }
+}
+
 // 16 consecutive fp32 columns of this thread's TMEM lane, and 8 columns stored.
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
 {
@@ -528,13 +550,7 @@ bwd_q_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant_
                 uint32_t v[32];
                 tmem_ld32(lane_base + C::T_DQ + ob * D + col, v);
                 tmem_wait_ld();
-                if (valid) {
-                    float4* dst = reinterpret_cast<float4*>(a.dq + row * D + col);
-#pragma unroll
-                    for (int x = 0; x < 8; ++x)
-                        dst[x] = make_float4(__uint_as_float(v[4 * x]) * sc, __uint_as_float(v[4 * x + 1]) * sc,
-                                             __uint_as_float(v[4 * x + 2]) * sc, __uint_as_float(v[4 * x + 3]) * sc);
-                }
+                if (valid) store_row32(a.dq + row * D + col, v, sc, (reinterpret_cast<uintptr_t>(a.dq) & 31u) == 0);
             }
             tmem_fence_before();
             mbar_arrive(&o_free[ob]);
@@ -1133,19 +1149,14 @@ bwd_kv_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant
                 if (WGS == 2 && o != wg) continue;
                 const float f = o == 0 ? 1.f : sc;
                 float* dst_row = (o == 0 ? a.dv : a.dk) + row * D;
+                const bool wide = (reinterpret_cast<uintptr_t>(o == 0 ? a.dv : a.dk) & 31u) == 0;
                 const uint32_t src = lane_base + (o == 0 ? C::T_DV : C::T_DK);
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {
                     uint32_t v[32];
                     tmem_ld32(src + 32 * c, v);
                     tmem_wait_ld();
-                    if (kvalid) {
-                        float4* dst = reinterpret_cast<float4*>(dst_row + 32 * c);
-#pragma unroll
-                        for (int x = 0; x < 8; ++x)
-                            dst[x] = make_float4(__uint_as_float(v[4 * x]) * f, __uint_as_float(v[4 * x + 1]) * f,
-                                                 __uint_as_float(v[4 * x + 2]) * f, __uint_as_float(v[4 * x + 3]) * f);
-                    }
+                    if (kvalid) store_row32(dst_row + 32 * c, v, f, wide);
                 }
             }
             tmem_fence_before();

@@ -137,6 +137,28 @@ def test_deterministic():
         assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("B,d", [(128, 64), (1024, 128)])  # the short and the long shape
+def test_gradient_alignment(B, d):
+    """Gradients 32-byte aligned take 32-byte stores, ones only 16-byte aligned 16-byte stores:
+    both hold the same bits."""
+    w = inputs.SequenceWorkload("bwd_align", batch=1, Hq=8, Hkv=2, d=d, B=B, n=1500, seed=195)
+    dev = torch.device("cuda")
+    q, k, v = (x.to(dev) for x in inputs.sequence_inputs(w))
+    do = upstream(w, dev)
+    out, lse = pbb.forward(q, k, v, w.B)
+    g1 = pbb.backward(q, k, v, out, do, lse, w.B)
+    bufs = []
+    for g in g1:
+        buf = torch.empty(g.numel() + 16, dtype=torch.float32, device=dev)
+        base = (-buf.data_ptr() % 32) // 4 + 4  # 16 bytes past a 32-byte boundary
+        t = buf[base:base + g.numel()].view(g.shape)
+        assert t.data_ptr() % 32 == 16
+        bufs.append(t)
+    g2 = pbb.backward(q, k, v, out, do, lse, w.B, dq=bufs[0], dk=bufs[1], dv=bufs[2])
+    for a, b in zip(g1, g2):
+        assert a.data_ptr() % 32 == 0 and torch.equal(a, b)
+
+
 @pytest.mark.parametrize("name", ["fwd_b16_n8192_B128"])
 def test_full_size(name):
     """The benchmark's B = 128 workload at full size (batch 16, Hq 8, Hkv 2, d 64, n 8192), every gradient."""
