@@ -716,6 +716,16 @@ def oracle_forward_sample(w, seconds: float, rows_per_call: int = 64):
                       f"force over every position up to t (includes widening the slice to fp64)"}
 
 
+def fwd_kernel_label(w):
+    """The forward kernel a workload runs, with its launch shape."""
+    import paper_2606_02680_gb300 as pbb
+
+    nk, ctas = pbb.plan_forward(w.batch, w.Hq, w.Hkv, w.n, w.d, w.B)
+    if pbb.plan_forward_query_tiles(w.batch, w.Hq, w.Hkv, w.n, w.d, w.B) == 2:
+        return "forward_pair_kernel<%d,%d,%d keys,2 query tiles per CTA>" % (w.d, w.group, nk)
+    return "forward_kernel<%d,%d,%d keys,%d CTAs/SM>" % (w.d, w.group, nk, ctas)
+
+
 def run_forward(args, dist, rank, world, dev):
     import torch
 
@@ -745,8 +755,7 @@ def run_forward(args, dist, rank, world, dev):
         roof.update({"traffic": None,
                      "kernel": ("bwd_kv_tc_kernel<%d,%d> + bwd_q_tc_kernel<%d,%d> + delta_kernel<%d> (one call)"
                                 % (w.d, w.group, w.d, w.group, w.d)) if bwd else
-                               "forward_kernel<%d,%d,%d keys,%d CTAs/SM>" % ((w.d, w.group) + pbb.plan_forward(
-                                   w.batch, w.Hq, w.Hkv, w.n, w.d, w.B)),
+                               fwd_kernel_label(w),
                      "algorithmic_flops_per_launch": flops, "algorithmic_bytes_per_launch": bytes_,
                      "hbm_gbs": bytes_ / kern_s / 1e9, "tflops": flops / kern_s / 1e12,
                      "kernel_ms_mean": res["kernel_ms_mean"], "kernel_ms_median": res["kernel_ms_median"]})

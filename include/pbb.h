@@ -225,6 +225,16 @@ int pbb_forward(const void* q, const void* k, const void* v, void* out, float* l
 int pbb_plan_forward(int batch, int Hq, int Hkv, int n, int d, int B, int* keys_per_tile, int* ctas_per_sm);
 
 /*
+ * The query tiles (128 rows of the GQA group's heads) one persistent CTA of
+ * pbb_forward works on at once for these sizes on the current device: 2 where
+ * long supports with B a multiple of 256 take the paired-item kernel (two
+ * consecutive query tiles of one sequence and KV head stream their union of keys
+ * once, their softmaxes alternating on the tensor pipe), else 1. Negative on
+ * error, with pbb_plan_forward's shape rules. Nothing is launched.
+ */
+int pbb_plan_forward_query_tiles(int batch, int Hq, int Hkv, int n, int d, int B);
+
+/*
  * Gradients of pbb_forward (the backward pass of the paper's fused training
  * kernel, Sec. 3: bridge gradients flow into the previous half-block's K and V).
  * With P_ts = exp(q_t.k_s/sqrt(d) - lse_t) on A(t) and D_t = dO_t . o_t:

@@ -66,6 +66,7 @@ EXPORTS = {
     "pbb_decode_step_layers": (_I, [_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_forward": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_plan_forward": (_I, [_I, _I, _I, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+    "pbb_plan_forward_query_tiles": (_I, [_I, _I, _I, _I, _I, _I]),
     "pbb_ring_from_sequence": (_I, [_P, _P, _I, _P, _P, _I, _I, _I, _I, _I, _P]),
     "pbb_backward": (_I, [_P, _P, _P, _P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _P]),
     "pbb_advance_positions": (_I, [_P, _I, _P]),
@@ -520,6 +521,15 @@ def set_kernel(kernel: str) -> str:
     if prev < PBB_KERNEL_AUTO:
         raise PbbError(prev, "pbb_set_kernel")
     return {v: k for k, v in _KERNEL_NAMES.items()}[prev]
+
+
+def plan_forward_query_tiles(batch: int, Hq: int, Hkv: int, n: int, d: int, B: int) -> int:
+    """Query tiles one CTA of pbb_forward works on at once for these sizes: 2 for the paired
+    kernel, else 1 (pbb_plan_forward_query_tiles)."""
+    rc = int(lib().pbb_plan_forward_query_tiles(batch, Hq, Hkv, n, d, B))
+    if rc < 0:
+        raise PbbError(rc, "pbb_plan_forward_query_tiles")
+    return rc
 
 
 def plan_support_order(batch: int, Hq: int, Hkv: int, d: int, B: int, window: int = 0,

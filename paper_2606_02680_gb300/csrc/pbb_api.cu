@@ -10,6 +10,7 @@
 #include <utility>
 
 #include "pbb.h"
+#include "pbb_forward_plan.h"
 #include "pbb_internal.h"
 
 namespace {
@@ -542,6 +543,28 @@ int pbb_plan_forward(int batch, int Hq, int Hkv, int n, int d, int B, int* keys_
     *keys_per_tile = plan.keys_per_tile;
     *ctas_per_sm = plan.ctas_per_sm;
     return PBB_OK;
+}
+
+int pbb_plan_forward_query_tiles(int batch, int Hq, int Hkv, int n, int d, int B)
+{
+    int rc = check_shape(batch, Hkv, d, B, PBB_BF16);
+    if (rc != PBB_OK) return rc;
+    rc = check_group_sequence(Hq, Hkv);
+    if (rc != PBB_OK) return rc;
+    if (n < 0) return PBB_ERR_INVALID_ARG;
+    int dev = 0;
+    rc = current_device(&dev);
+    if (rc != PBB_OK) return rc;
+    pbb::ForwardArgs a{};
+    a.batch = batch;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.n = n;
+    a.d = d;
+    a.B = B;
+    int tiles = 0;
+    if (pbb::plan_forward_query_tiles(a, &tiles) != cudaSuccess) return PBB_ERR_CUDA;
+    return tiles;
 }
 
 int pbb_backward(const void* q, const void* k, const void* v, const void* out, const void* dout, const float* lse,

@@ -38,6 +38,7 @@
 
 #include "pbb_device.cuh"
 #include "pbb_internal.h"
+#include "pbb_store.cuh"
 
 namespace pbb {
 

@@ -166,14 +166,6 @@ __device__ __forceinline__ float fast_exp2(float x)
     return y;
 }
 
-// One 32-byte global store (sm_100 and later); p must be 32-byte aligned.
-__device__ __forceinline__ void st_global_v8(void* p, const uint32_t* w)
-{
-    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]),
-                 "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
-                 : "memory");
-}
-
 // Programmatic dependent launch. pdl_wait: block until the grids this one depends on in its
 // stream have completed and their memory is visible (a no-op for a launch without the
 // attribute). pdl_launch_dependents: let the next grid of the stream be scheduled now; it still

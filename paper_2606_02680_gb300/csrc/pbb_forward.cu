@@ -58,7 +58,9 @@
 #include <stdint.h>
 
 #include "pbb_device.cuh"
+#include "pbb_forward_plan.h"
 #include "pbb_internal.h"
+#include "pbb_store.cuh"
 
 namespace pbb {
 
@@ -1148,6 +1150,26 @@ cudaError_t launch_fwd(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* p
 #define PBB_FWD_PAIR 1
 #endif
 
+// 1: the paired kernel is usable on device dev; 2: its register split does not hold; 0: a
+// runtime error (in *err). setmaxnreg moves registers within the block's launch allocation, so
+// the split is only valid if the kernel launches with LAUNCH_REGS per thread (else an increase
+// would wait forever); anything else falls back to the one-item kernel.
+template <int D, int G>
+int pair_kernel_usable(int dev, cudaError_t* err)
+{
+    using C = PairCfg<D, G>;
+    auto kernel = forward_pair_kernel<D, G>;
+    static std::atomic<int> state[kMaxCachedDevices] = {};
+    return cached_per_device(state, dev, [&] {
+        *err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+        if (*err != cudaSuccess) return 0;
+        cudaFuncAttributes fa{};
+        *err = cudaFuncGetAttributes(&fa, kernel);
+        if (*err != cudaSuccess) return 0;
+        return fa.numRegs == C::LAUNCH_REGS ? 1 : 2;
+    });
+}
+
 template <int D, int G>
 cudaError_t launch_fwd_pair(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
@@ -1156,19 +1178,7 @@ cudaError_t launch_fwd_pair(const ForwardArgs& a, cudaStream_t stream, ForwardPl
     int dev = 0;
     cudaError_t err = cudaGetDevice(&dev);
     if (err != cudaSuccess) return err;
-    // 1: usable; 2: the register split does not hold. setmaxnreg moves registers within the
-    // block's launch allocation, so the split is only valid if the kernel launches with
-    // LAUNCH_REGS per thread (else an increase would wait forever); anything else falls back to
-    // the one-item kernel
-    static std::atomic<int> state[kMaxCachedDevices] = {};
-    const int usable = cached_per_device(state, dev, [&] {
-        err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
-        if (err != cudaSuccess) return 0;
-        cudaFuncAttributes fa{};
-        err = cudaFuncGetAttributes(&fa, kernel);
-        if (err != cudaSuccess) return 0;
-        return fa.numRegs == C::LAUNCH_REGS ? 1 : 2;
-    });
+    const int usable = pair_kernel_usable<D, G>(dev, &err);
     if (usable < 1) return err;
     if (usable != 1) return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
     const long long nq = (a.n + C::QT - 1) / C::QT;
@@ -1202,6 +1212,13 @@ cudaError_t launch_fwd_pair(const ForwardArgs& a, cudaStream_t stream, ForwardPl
 #define PBB_FWD_SHORT_MAX_B 512
 #endif
 
+// Whether a call of these sizes takes the paired-item kernel's shape (which still falls back to
+// the one-item kernel where its register split does not hold).
+bool pair_shape(const ForwardArgs& a)
+{
+    return PBB_FWD_LONG_SHAPE != 1 && PBB_FWD_PAIR && a.B >= PBB_FWD_SHORT_MAX_B && (a.B / 2) % 128 == 0;
+}
+
 template <int D, int G>
 cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream, ForwardPlan* plan)
 {
@@ -1213,9 +1230,30 @@ cudaError_t launch_fwd_shape(const ForwardArgs& a, cudaStream_t stream, ForwardP
 #if PBB_FWD_LONG_SHAPE == 1
     return launch_fwd<D, G, 128, 2, 1>(a, stream, plan);
 #else
-    if (PBB_FWD_PAIR && (a.B / 2) % 128 == 0) return launch_fwd_pair<D, G>(a, stream, plan);
+    if (pair_shape(a)) return launch_fwd_pair<D, G>(a, stream, plan);
     return launch_fwd<D, G, 128, 1, 1>(a, stream, plan);
 #endif
+}
+
+template <int D>
+cudaError_t query_tiles_d(const ForwardArgs& a, int* query_tiles)
+{
+    *query_tiles = 1;
+    if (!pair_shape(a)) return cudaSuccess;
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return err;
+    int usable = 0;
+    switch (a.Hq / a.Hkv) {
+        case 1: usable = pair_kernel_usable<D, 1>(dev, &err); break;
+        case 2: usable = pair_kernel_usable<D, 2>(dev, &err); break;
+        case 4: usable = pair_kernel_usable<D, 4>(dev, &err); break;
+        case 8: usable = pair_kernel_usable<D, 8>(dev, &err); break;
+        default: return cudaErrorInvalidValue;
+    }
+    if (usable < 1) return err;
+    if (usable == 1) *query_tiles = 2;
+    return cudaSuccess;
 }
 
 template <int D>
@@ -1242,6 +1280,13 @@ cudaError_t forward_dispatch(const ForwardArgs& a, cudaStream_t stream, ForwardP
 cudaError_t launch_forward(const ForwardArgs& a, cudaStream_t stream) { return forward_dispatch(a, stream, nullptr); }
 
 cudaError_t plan_forward(const ForwardArgs& a, ForwardPlan* plan) { return forward_dispatch(a, nullptr, plan); }
+
+cudaError_t plan_forward_query_tiles(const ForwardArgs& a, int* query_tiles)
+{
+    if (a.d == 64) return query_tiles_d<64>(a, query_tiles);
+    if (a.d == 128) return query_tiles_d<128>(a, query_tiles);
+    return cudaErrorInvalidValue;
+}
 
 cudaError_t launch_seq_ring(const void* k, const void* v, void* k_ring, void* v_ring, int batch, int Hkv,
                             int n, int B, int row_bytes, cudaStream_t stream)

@@ -51,3 +51,19 @@ def test_traffic_record_scales_with_algorithmic_bytes(bench, monkeypatch):
         monkeypatch.setattr(bench, "kernel_source_sha", lambda: "another source")
         assert bench.recorded_traffic(key, 1e9) is None
     assert bench.recorded_traffic("no_such_workload", 1e9) is None
+
+
+def test_forward_kernel_label(bench, monkeypatch):
+    """The forward line names the kernel that runs: the paired-item kernel where pbb_forward
+    takes two query tiles per CTA, else the one-item kernel with its CTAs per SM."""
+    import paper_2606_02680_gb300 as pbb
+    from paper_2606_02680_gb300 import inputs
+
+    w = inputs.FORWARD_WORKLOADS["fwd_b2_n32768_B4096"]
+    monkeypatch.setattr(pbb, "plan_forward", lambda *a: (128, 1))
+    monkeypatch.setattr(pbb, "plan_forward_query_tiles", lambda *a: 2)
+    assert bench.fwd_kernel_label(w) == "forward_pair_kernel<128,4,128 keys,2 query tiles per CTA>"
+    monkeypatch.setattr(pbb, "plan_forward", lambda *a: (32, 3))
+    monkeypatch.setattr(pbb, "plan_forward_query_tiles", lambda *a: 1)
+    w = inputs.FORWARD_WORKLOADS["fwd_b16_n8192_B128"]
+    assert bench.fwd_kernel_label(w) == "forward_kernel<64,4,32 keys,3 CTAs/SM>"

@@ -228,4 +228,11 @@ def test_launch_shapes():
     assert pbb.plan_forward(16, 8, 2, 8192, 64, 128) == (32, 3)
     assert pbb.plan_forward(16, 8, 2, 8192, 128, 128) == (64, 2)
     assert pbb.plan_forward(1, 8, 2, 0, 64, 128)[1] == 0  # no work
+    # two query tiles per CTA where B is a multiple of 256 and the supports are long
+    assert pbb.plan_forward_query_tiles(2, 32, 8, 32768, 128, 4096) == 2
+    assert pbb.plan_forward_query_tiles(2, 32, 8, 4000, 64, 512) == 2
+    assert pbb.plan_forward_query_tiles(1, 8, 2, 3000, 128, 640) == 1  # 640 / 2 not a multiple of 128
+    assert pbb.plan_forward_query_tiles(16, 8, 2, 8192, 64, 128) == 1
+    with pytest.raises(pbb.PbbError):
+        pbb.plan_forward_query_tiles(1, 6, 4, 100, 64, 128)  # Hq not a multiple of Hkv
 
