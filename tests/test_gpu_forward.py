@@ -94,6 +94,18 @@ def test_long_blocks_groups_and_dims(group, d):
     run_full(w)
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_paired_kernel_one_tile_items(d):
+    """Many short sequences under a long block (n = 100, B = 512): every paired item has one
+    K/V tile, so each CTA runs ten such items back to back, one extra iteration each. Its K and
+    V producers then run furthest ahead of the issuing thread on the per-iteration barrier ring
+    (2 x stages + 1 iterations: 9 at d = 64), which the ring must outlast."""
+    w = inputs.SequenceWorkload(f"fwd_one_tile_d{d}", batch=384, Hq=8, Hkv=2, d=d, B=512, n=100,
+                                seed=96 + d)
+    assert pbb.plan_forward_query_tiles(w.batch, w.Hq, w.Hkv, w.n, w.d, w.B) == 2
+    run_full(w)
+
+
 @pytest.mark.parametrize("n", [1, 7, 8, 63, 64, 65])
 def test_short_sequences(n):
     w = inputs.SequenceWorkload(f"fwd_n{n}", batch=3, Hq=4, Hkv=1, d=64, B=32, n=n, seed=70 + n)
