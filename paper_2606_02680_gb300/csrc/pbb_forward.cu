@@ -637,14 +637,15 @@ struct PairCfg {
     // Iteration i of the issuing thread (K_j for S, V_{j-1} for P.V) waits on kv_full[i mod KVR],
     // which the K and the V producer each arrive on once per iteration, with their copy's bytes
     // or without a copy. Before copying tile t into a ring of S stages, a producer waits for tile
-    // t - S to be freed, which follows the issuing thread's iteration of that tile. Those S tiles
-    // span at most 2 S iterations (one extra iteration per item, when every item has one tile),
-    // and a copy may be followed by one arrival without a copy: a producer runs at most 2 S + 1
-    // iterations ahead of the issuing thread. A slot is safe to reuse once the issuing thread has
-    // passed its previous iteration, so KVR must exceed that lead: 8 at d = 128 (3 K and 2 V
+    // t - S to be freed, which happens after the issuing thread has passed that tile's
+    // iteration. Those S tiles span at most 2 S iterations (one extra iteration per item, when
+    // every item has one tile), and a copy may be followed by one arrival without a copy: a
+    // producer arrives for iterations at most 2 S past the last one the issuing thread has
+    // passed. A slot may take the arrivals of iteration i once the issuing thread has passed
+    // i - KVR, so KVR >= 2 S + 1 suffices; it keeps one slot more: 8 at d = 128 (3 K and 2 V
     // stages), 10 at d = 64 (4 and 4).
     static constexpr int KVR = 2 * (KSTAGES > VSTAGES ? KSTAGES : VSTAGES) + 2;
-    static_assert(KVR > 2 * KSTAGES + 1 && KVR > 2 * VSTAGES + 1, "kv_full ring shorter than a producer's lead");
+    static_assert(KVR > 2 * KSTAGES && KVR > 2 * VSTAGES, "kv_full ring shorter than a producer's lead");
     // warps 0-7 softmax, 8 K producer, 9 V producer, 10 MMA issuer, 11 Q producer; at launch
     // 168 registers each (12 warps, three per SMSP). setmaxnreg is uniform per warpgroup and
     // the register file is split between the SMSPs, so each SMSP's three warps (two softmax,
