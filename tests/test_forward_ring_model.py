@@ -1,4 +1,5 @@
-"""A model, on the CPU, of the paired forward kernel's per-iteration K/V barrier ring.
+"""Models, on the CPU, of two synchronisation rules of the paired forward kernel: its
+per-iteration K/V barrier ring, and which softmax warpgroup frees each K/V stage.
 
 Iteration i of the issuing thread (S on K_j, P.V on V_{j-1}; j = 0 .. nt per item) waits on
 slot i mod R of a ring of mbarriers. The K and the V producer each arrive on that slot once per
@@ -111,3 +112,74 @@ def test_the_model_finds_the_overlap_of_a_short_ring():
     rng = random.Random(7)
     assert sum(simulate([1] * 40, 4, 4, 8, rng) for _ in range(300)) > 0
     assert sum(simulate([1] * 40, 4, 4, 9, rng) for _ in range(300)) == 0
+
+
+# ---- who frees the K/V stages ------------------------------------------------------------
+# The paired kernel's softmax warpgroups free the K and V stages: the first thread of item x's
+# warpgroup frees K_j and V_{j-1} after seeing x's s_full of tile j when x owns iteration j
+# (item B owns its tiles, item A the iterations below B's first tile, all of them without B),
+# and V_{nt-1} after x's pv_last when x owns the last iteration. A stage freed twice would let a
+# copy overwrite a tile still being read; one never freed stalls the producer. The geometry is
+# the kernel's make_pitem, restated.
+
+def support_start(t, h):
+    m = t // h
+    return h * (m - 1) if m > 0 else 0
+
+
+def make_pitem(sidx, n, B, QT, NK=128):
+    nq = (n + QT - 1) // QT
+    nsp = (nq + 1) // 2
+    pair = sidx // nsp
+    t0 = (sidx - pair * nsp) * 2 * QT
+    tlA = min(t0 + QT, n) - 1
+    hasB = t0 + QT < n
+    tlB = min(t0 + 2 * QT, n) - 1 if hasB else tlA
+    h = B // 2
+    loA = support_start(t0, h)
+    loB = support_start(t0 + QT, h) if hasB else loA
+    return {"hasB": hasB, "nt": (tlB - loA + NK) // NK, "ntA": (tlA - loA + NK) // NK,
+            "jB0": (loB - loA) // NK}
+
+
+def check_item_releases(it):
+    nt, hasB = it["nt"], it["hasB"]
+    jb = [0, it["jB0"] if hasB else nt]
+    je = [it["ntA"], nt]
+    # the issuing thread's commits, in order, per iteration j = 0 .. nt
+    last_commit = {}
+    for j in range(nt + 1):
+        for x in (0, 1):
+            sk = jb[x] <= j < je[x]
+            pv = j >= jb[x] + 1 and j - 1 < je[x]
+            if sk:
+                last_commit[j] = ("s_full", x)
+            elif pv:
+                last_commit[j] = ("pv_last", x)
+    assert set(last_commit) == set(range(nt + 1)), "an iteration without products"
+    freed = {"k": [], "v": []}
+    for x in (0, 1):
+        if x == 1 and not hasB:
+            continue
+        jown = nt if x == 1 else (it["jB0"] if hasB else nt)
+        for j in range(jb[x], je[x]):
+            if j < jown:  # after x's s_full of tile j
+                assert last_commit[j] == ("s_full", x), (it, j, x)
+                freed["k"].append(j)
+                if j >= 1:
+                    freed["v"].append(j - 1)
+        if x == 1 or not hasB:  # after x's pv_last, the item's last P.V
+            assert last_commit[nt] == ("pv_last", x), (it, x)
+            freed["v"].append(nt - 1)
+    assert sorted(freed["k"]) == list(range(nt)), (it, freed)
+    assert sorted(freed["v"]) == list(range(nt)), (it, freed)
+
+
+@pytest.mark.parametrize("B", [512, 768, 1024, 2048, 4096])
+@pytest.mark.parametrize("group", [1, 2, 4, 8])
+def test_every_stage_is_freed_once_by_the_last_reader(B, group):
+    QT = 128 // group
+    for n in (1, 31, 32, 33, 63, 64, 65, 100, 777, 2 * B + 5, 3 * B):
+        nq = (n + QT - 1) // QT
+        for sidx in range((nq + 1) // 2):  # one (sequence, KV head): the items repeat per pair
+            check_item_releases(make_pitem(sidx, n, B, QT))
